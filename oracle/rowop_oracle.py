@@ -1,0 +1,214 @@
+"""Python face of the double-precision CPU oracle (``rowop_oracle.c``).
+
+TEST INFRASTRUCTURE ONLY.  This module is the checker the CUDA library is
+compared against.  Only the test suite, ``__graft_entry__.smoke()`` and the
+benchmark's CPU-baseline / reference leg may import it; the product path
+(``paper_2607_23089_gb300``) never does, and this module never imports the
+product.  Inputs arrive here as exact float64 copies of whatever the GPU saw
+(bf16 and fp32 values convert to double without rounding), outputs leave as
+float64.
+
+Definitions (textbook / PyTorch convention; the paper names the family only
+through its running-example kernel names in §2.1 and writes no formula):
+
+* softmax     ``y = exp(x - max x) / sum exp(x - max x)``
+* log-softmax ``y = (x - max x) - log(sum exp(x - max x))``
+* LayerNorm   ``y = (x - mu) / sqrt(var + eps) * gamma + beta`` with the biased
+  (population) variance
+* RMSNorm     ``y = x / sqrt(mean(x^2) + eps) * gamma``
+* ragged      row ``i`` is ``x[off[i]:off[i+1]]``; gamma/beta are indexed by the
+  column inside the row.
+
+``eps`` is passed as the float32 value the GPU uses, widened to double.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "rowop_oracle.c")
+_BUILD_DIR = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD_DIR, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+SMALL, MEDIUM, LARGE = 0, 1, 2
+
+
+def build(force: bool = False) -> str:
+    """Compile ``rowop_oracle.c`` with gcc (-O2, no fast-math) into a shared
+    library next to it.  OpenMP is used when the compiler offers it; without
+    it the row loop simply runs on one thread."""
+    os.makedirs(_BUILD_DIR, exist_ok=True)
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    base = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fno-fast-math",
+            "-ffp-contract=off", _SRC, "-o", tmp, "-lm"]
+    try:
+        subprocess.run(base[:1] + ["-fopenmp"] + base[1:], check=True,
+                       capture_output=True)
+    except subprocess.CalledProcessError:
+        subprocess.run(base, check=True, capture_output=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        lib = ctypes.CDLL(build())
+        d, i64, ci = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
+        dbl = ctypes.c_double
+        lib.oracle_softmax.argtypes = [d, d, i64, i64, ci]
+        lib.oracle_logsoftmax.argtypes = [d, d, i64, i64, ci]
+        lib.oracle_layernorm.argtypes = [d, d, d, d, i64, i64, dbl, ci]
+        lib.oracle_rmsnorm.argtypes = [d, d, d, i64, i64, dbl, ci]
+        lib.oracle_softmax_ragged.argtypes = [d, d, d, i64, ci]
+        lib.oracle_logsoftmax_ragged.argtypes = [d, d, d, i64, ci]
+        lib.oracle_layernorm_ragged.argtypes = [d, d, d, d, d, i64, dbl, ci]
+        lib.oracle_rmsnorm_ragged.argtypes = [d, d, d, d, i64, dbl, ci]
+        lib.oracle_bucket.argtypes = [i64, i64]
+        lib.oracle_bucket.restype = ci
+        for name in ("oracle_softmax", "oracle_logsoftmax", "oracle_layernorm",
+                     "oracle_rmsnorm", "oracle_softmax_ragged",
+                     "oracle_logsoftmax_ragged", "oracle_layernorm_ragged",
+                     "oracle_rmsnorm_ragged"):
+            getattr(lib, name).restype = None
+        _lib = lib
+        return lib
+
+
+def _f64(a) -> np.ndarray:
+    a = np.asarray(a, dtype=np.float64)
+    return np.ascontiguousarray(a)
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _threads(nthreads):
+    return int(nthreads) if nthreads else 1
+
+
+def _as_eps(eps: float) -> float:
+    # The GPU adds eps as a float32; the oracle uses that same value.
+    return float(np.float32(eps))
+
+
+def _dense(name, x, nthreads, *extra_arrays, eps=None):
+    x = _f64(x)
+    if x.ndim != 2:
+        raise ValueError("dense oracle wants a 2-D rows x cols array")
+    rows, cols = x.shape
+    y = np.empty_like(x)
+    lib = _load()
+    args = [_ptr(x), _ptr(y)] + [_ptr(a) for a in extra_arrays]
+    args += [rows, cols]
+    if eps is not None:
+        args.append(_as_eps(eps))
+    args.append(_threads(nthreads))
+    getattr(lib, name)(*args)
+    return y
+
+
+def _vec(v, n, fill):
+    if v is None:
+        return np.full(n, fill, dtype=np.float64)
+    v = _f64(v).reshape(-1)
+    if v.shape[0] < n:
+        raise ValueError("gamma/beta shorter than the row length")
+    return v
+
+
+def softmax(x, nthreads=1):
+    return _dense("oracle_softmax", x, nthreads)
+
+
+def logsoftmax(x, nthreads=1):
+    return _dense("oracle_logsoftmax", x, nthreads)
+
+
+def layernorm(x, gamma=None, beta=None, eps=1e-5, nthreads=1):
+    x = _f64(x)
+    n = x.shape[1]
+    return _dense("oracle_layernorm", x, nthreads, _vec(gamma, n, 1.0),
+                  _vec(beta, n, 0.0), eps=eps)
+
+
+def rmsnorm(x, gamma=None, eps=1e-6, nthreads=1):
+    x = _f64(x)
+    n = x.shape[1]
+    return _dense("oracle_rmsnorm", x, nthreads, _vec(gamma, n, 1.0), eps=eps)
+
+
+def _offsets(offsets):
+    off = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
+    if off.ndim != 1 or off.shape[0] < 1:
+        raise ValueError("offsets must be a 1-D array of rows+1 entries")
+    if off[0] != 0 or np.any(np.diff(off) < 0):
+        raise ValueError("offsets must start at 0 and never decrease")
+    return off
+
+
+def _ragged(name, x, offsets, nthreads, *extra_arrays, eps=None):
+    x = _f64(x).reshape(-1)
+    off = _offsets(offsets)
+    rows = off.shape[0] - 1
+    if off[-1] > x.shape[0]:
+        raise ValueError("offsets run past the packed buffer")
+    y = np.zeros_like(x)
+    lib = _load()
+    args = [_ptr(x), _ptr(y)] + [_ptr(a) for a in extra_arrays]
+    args += [_ptr(off), rows]
+    if eps is not None:
+        args.append(_as_eps(eps))
+    args.append(_threads(nthreads))
+    getattr(lib, name)(*args)
+    return y
+
+
+def _max_len(off):
+    return int(np.max(np.diff(off))) if off.shape[0] > 1 else 0
+
+
+def softmax_ragged(x, offsets, nthreads=1):
+    return _ragged("oracle_softmax_ragged", x, offsets, nthreads)
+
+
+def logsoftmax_ragged(x, offsets, nthreads=1):
+    return _ragged("oracle_logsoftmax_ragged", x, offsets, nthreads)
+
+
+def layernorm_ragged(x, offsets, gamma=None, beta=None, eps=1e-5, nthreads=1):
+    off = _offsets(offsets)
+    n = max(_max_len(off), 1)
+    return _ragged("oracle_layernorm_ragged", x, off, nthreads,
+                   _vec(gamma, n, 1.0), _vec(beta, n, 0.0), eps=eps)
+
+
+def rmsnorm_ragged(x, offsets, gamma=None, eps=1e-6, nthreads=1):
+    off = _offsets(offsets)
+    n = max(_max_len(off), 1)
+    return _ragged("oracle_rmsnorm_ragged", x, off, nthreads,
+                   _vec(gamma, n, 1.0), eps=eps)
+
+
+def bucket(length: int, esize: int) -> int:
+    """Row-length dispatch rule: 0 SMALL (<= 4 KiB), 1 MEDIUM (<= 32 KiB),
+    2 LARGE, by the row's byte size."""
+    return int(_load().oracle_bucket(int(length), int(esize)))
+
+
+__all__ = ["build", "softmax", "logsoftmax", "layernorm", "rmsnorm",
+           "softmax_ragged", "logsoftmax_ragged", "layernorm_ragged",
+           "rmsnorm_ragged", "bucket", "SMALL", "MEDIUM", "LARGE"]

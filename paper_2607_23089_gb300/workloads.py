@@ -1,0 +1,165 @@
+"""Seeded synthetic inputs for the row-op workloads.
+
+This module only draws random numbers; it holds none of the operators'
+arithmetic, and both the CUDA path's tests/benchmark and the CPU oracle take
+their inputs from it.  Every draw uses ``torch.Generator('cpu')`` seeded per
+workload, in float32, in a fixed order: row lengths (ragged) -> x -> outlier
+mask / sign -> per-row scale -> gamma -> beta.  bf16 tensors are made from the
+float32 draws by round-to-nearest-even (``.to(torch.bfloat16)``).
+
+The five workloads (rows x cols, dtype, distribution, seed):
+
+1. ``softmax_1k``    fp32 softmax, 1024 x 1000, x = 4*N(0,1), seed 0.
+2. ``short_rows``    fp32 softmax and log-softmax, 32768 x C for C in
+   {64, 128, 256, 512}, x = 4*N(0,1), seed 1 (one generator per C).
+3. ``medium_norm``   bf16 RMSNorm (eps 1e-6) and LayerNorm (eps 1e-5),
+   8192 x 4096, x = N(0,1) * U(0.1, 10) per row, gamma = 1 + 0.1*N(0,1),
+   beta = 0.1*N(0,1) per column, seed 2.
+4. ``long_rows``     fp32 log-softmax, 256 x 262144, x = N(0,1) with each
+   entry independently (p = 0.001) replaced by +80 or -80 (p = 1/2 each),
+   seed 3.
+5. ``ragged_ln``     bf16 LayerNorm (eps 1e-5) over 16384 ragged rows with
+   lengths uniform on {1..32768} as int64 CSR offsets into one packed buffer,
+   x = N(0,1) * U(0.1, 10) per row, gamma/beta of length 32768 drawn as in
+   workload 3, seed 4.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from typing import Optional
+
+import torch
+
+ESIZE = {torch.float32: 4, torch.bfloat16: 2}
+
+
+@dataclass
+class Case:
+    """One operator call on one synthetic input (host tensors)."""
+    name: str
+    op: str                      # softmax | logsoftmax | layernorm | rmsnorm
+    x: torch.Tensor              # dense: rows x cols; ragged: packed 1-D
+    dtype: torch.dtype
+    offsets: Optional[torch.Tensor] = None   # int64 [rows+1] when ragged
+    gamma: Optional[torch.Tensor] = None
+    beta: Optional[torch.Tensor] = None
+    eps: float = 0.0
+    max_len: int = 0
+    meta: dict = field(default_factory=dict)
+
+    @property
+    def ragged(self) -> bool:
+        return self.offsets is not None
+
+    @property
+    def rows(self) -> int:
+        return (self.offsets.numel() - 1) if self.ragged else self.x.shape[0]
+
+    @property
+    def elements(self) -> int:
+        return int(self.offsets[-1]) if self.ragged else self.x.numel()
+
+    def algorithmic_bytes(self) -> int:
+        """Bytes the operator must move: read x once, write y once, read
+        gamma/beta once, read the offsets once."""
+        es = ESIZE[self.dtype]
+        b = 2 * self.elements * es
+        ncol = self.max_len if self.ragged else self.x.shape[1]
+        if self.gamma is not None:
+            b += ncol * es
+        if self.beta is not None:
+            b += ncol * es
+        if self.ragged:
+            b += self.offsets.numel() * 8
+        return b
+
+
+def _gen(seed: int) -> torch.Generator:
+    return torch.Generator("cpu").manual_seed(seed)
+
+
+def _affine(g: torch.Generator, n: int, dtype):
+    gamma = (1.0 + 0.1 * torch.randn(n, generator=g)).to(dtype)
+    beta = (0.1 * torch.randn(n, generator=g)).to(dtype)
+    return gamma, beta
+
+
+def softmax_1k(rows: int = 1024, cols: int = 1000) -> Case:
+    g = _gen(0)
+    x = 4.0 * torch.randn(rows, cols, generator=g)
+    return Case("softmax_1k", "softmax", x, torch.float32)
+
+
+def short_rows(cols: int, op: str = "softmax", rows: int = 32768) -> Case:
+    g = _gen(1)
+    x = 4.0 * torch.randn(rows, cols, generator=g)
+    return Case(f"short_rows_{op}_{cols}", op, x, torch.float32,
+                meta={"cols": cols})
+
+
+def medium_norm(op: str, rows: int = 8192, cols: int = 4096) -> Case:
+    g = _gen(2)
+    x = torch.randn(rows, cols, generator=g)
+    scale = 0.1 + 9.9 * torch.rand(rows, 1, generator=g)
+    x = (x * scale).to(torch.bfloat16)
+    gamma, beta = _affine(g, cols, torch.bfloat16)
+    if op == "rmsnorm":
+        return Case(f"medium_norm_{op}", op, x, torch.bfloat16, gamma=gamma,
+                    eps=1e-6)
+    return Case(f"medium_norm_{op}", op, x, torch.bfloat16, gamma=gamma,
+                beta=beta, eps=1e-5)
+
+
+def long_rows(rows: int = 256, cols: int = 262144, op: str = "logsoftmax",
+              p_outlier: float = 0.001, outlier: float = 80.0) -> Case:
+    g = _gen(3)
+    x = torch.randn(rows, cols, generator=g)
+    mask = torch.rand(rows, cols, generator=g) < p_outlier
+    sign = torch.rand(rows, cols, generator=g) < 0.5
+    spike = torch.where(sign, torch.tensor(outlier), torch.tensor(-outlier))
+    x = torch.where(mask, spike, x)
+    return Case(f"long_rows_{op}", op, x, torch.float32)
+
+
+def ragged_lengths(rows: int, max_len: int, g: torch.Generator,
+                   min_len: int = 1) -> torch.Tensor:
+    return torch.randint(min_len, max_len + 1, (rows,), generator=g,
+                         dtype=torch.int64)
+
+
+def offsets_from_lengths(lengths: torch.Tensor) -> torch.Tensor:
+    off = torch.zeros(lengths.numel() + 1, dtype=torch.int64)
+    off[1:] = torch.cumsum(lengths, 0)
+    return off
+
+
+def ragged_ln(rows: int = 16384, max_len: int = 32768, op: str = "layernorm",
+              dtype=torch.bfloat16, seed: int = 4) -> Case:
+    g = _gen(seed)
+    lengths = ragged_lengths(rows, max_len, g)
+    off = offsets_from_lengths(lengths)
+    total = int(off[-1])
+    x = torch.randn(total, generator=g)
+    scale = 0.1 + 9.9 * torch.rand(rows, generator=g)
+    x = (x * torch.repeat_interleave(scale, lengths)).to(dtype)
+    gamma, beta = _affine(g, max_len, dtype)
+    eps = {"layernorm": 1e-5, "rmsnorm": 1e-6}.get(op, 0.0)
+    return Case(f"ragged_{op}", op, x, dtype, offsets=off,
+                gamma=gamma if op in ("layernorm", "rmsnorm") else None,
+                beta=beta if op == "layernorm" else None,
+                eps=eps, max_len=max_len)
+
+
+def all_cases(scale_down: int = 1):
+    """The five workloads as a flat list of cases.  ``scale_down`` > 1 divides
+    every row count (not the row lengths) for quicker runs."""
+    s = max(1, int(scale_down))
+    out = [softmax_1k(rows=max(1, 1024 // s))]
+    for c in (64, 128, 256, 512):
+        for op in ("softmax", "logsoftmax"):
+            out.append(short_rows(c, op, rows=max(1, 32768 // s)))
+    for op in ("rmsnorm", "layernorm"):
+        out.append(medium_norm(op, rows=max(1, 8192 // s)))
+    out.append(long_rows(rows=max(1, 256 // s)))
+    out.append(ragged_ln(rows=max(1, 16384 // s)))
+    return out

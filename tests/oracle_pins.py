@@ -1,0 +1,258 @@
+"""Pins for the CPU oracle: checks that tie it to the mathematics rather than
+to itself.  Each ``pin_*`` function takes an oracle module (the real one, or a
+deliberately broken copy in the mutation tests) and raises AssertionError when
+the oracle disagrees with
+
+* closed forms derived by hand (``tests/golden/hand_cases.json``),
+* invariants that any correct implementation satisfies,
+* an independent brute-force restatement using ``math.fsum``,
+* PyTorch's float64 CPU routines (a library, used only here),
+* the row-length dispatch thresholds stated in the library's interface.
+"""
+from __future__ import annotations
+
+import json
+import math
+import os
+
+import numpy as np
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+_EXPR_NAMES = {"ln": math.log, "exp": math.exp, "sqrt": math.sqrt,
+               "inf": math.inf}
+
+
+def _ev(s: str) -> float:
+    return float(eval(s, {"__builtins__": {}}, _EXPR_NAMES))  # noqa: S307
+
+
+def _close(a, b, rtol=1e-13, atol=1e-14):
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    assert a.shape == b.shape, (a.shape, b.shape)
+    ok = np.isclose(a, b, rtol=rtol, atol=atol, equal_nan=True)
+    if not ok.all():
+        d = np.where(ok, 0.0, np.abs(np.nan_to_num(a - b, nan=np.inf)))
+        raise AssertionError(f"max |diff| {d.max()}\n{a}\n{b}")
+
+
+def _call(orc, op, x, gamma=None, beta=None, eps=0.0):
+    if op == "softmax":
+        return orc.softmax(x)
+    if op == "logsoftmax":
+        return orc.logsoftmax(x)
+    if op == "layernorm":
+        return orc.layernorm(x, gamma, beta, eps=eps)
+    if op == "rmsnorm":
+        return orc.rmsnorm(x, gamma, eps=eps)
+    raise ValueError(op)
+
+
+def _call_ragged(orc, op, x, off, gamma=None, beta=None, eps=0.0):
+    if op == "softmax":
+        return orc.softmax_ragged(x, off)
+    if op == "logsoftmax":
+        return orc.logsoftmax_ragged(x, off)
+    if op == "layernorm":
+        return orc.layernorm_ragged(x, off, gamma, beta, eps=eps)
+    if op == "rmsnorm":
+        return orc.rmsnorm_ragged(x, off, gamma, eps=eps)
+    raise ValueError(op)
+
+
+OPS = ("softmax", "logsoftmax", "layernorm", "rmsnorm")
+
+
+# --------------------------------------------------------------------------
+def pin_hand_cases(orc):
+    with open(os.path.join(GOLDEN, "hand_cases.json")) as f:
+        cases = json.load(f)["cases"]
+    for c in cases:
+        x = np.array([[_ev(v) for v in row] for row in c["x"]])
+        exp = np.array([[_ev(v) for v in row] for row in c["expected"]])
+        g = np.array([_ev(v) for v in c["gamma"]]) if "gamma" in c else None
+        b = np.array([_ev(v) for v in c["beta"]]) if "beta" in c else None
+        got = _call(orc, c["op"], x, g, b, c.get("eps", 0.0))
+        _close(got, exp, rtol=1e-14, atol=1e-15)
+        # The same rows as a ragged batch give the same answer.
+        off = np.arange(0, x.size + 1, x.shape[1], dtype=np.int64)
+        got_r = _call_ragged(orc, c["op"], x.reshape(-1), off, g, b,
+                             c.get("eps", 0.0))
+        _close(got_r.reshape(x.shape), exp, rtol=1e-14, atol=1e-15)
+
+
+def pin_softmax_invariants(orc):
+    rng = np.random.default_rng(11)
+    x = rng.normal(0, 4, size=(17, 61))
+    p = orc.softmax(x)
+    _close(p.sum(axis=1), np.ones(17), rtol=0, atol=1e-13)
+    assert (p > 0).all() and (p < 1).all()
+    # Order is preserved: argmax of softmax is argmax of x.
+    assert (p.argmax(axis=1) == x.argmax(axis=1)).all()
+    # Shift invariance.
+    _close(orc.softmax(x + 123.25), p, rtol=1e-12, atol=1e-16)
+    # log(softmax) == log-softmax, and log-softmax is shift invariant.
+    ls = orc.logsoftmax(x)
+    _close(np.log(p), ls, rtol=1e-12, atol=1e-13)
+    _close(orc.logsoftmax(x - 77.5), ls, rtol=1e-12, atol=1e-12)
+    # Ratios: p_i / p_j = exp(x_i - x_j).
+    _close(p[:, 3] / p[:, 5], np.exp(x[:, 3] - x[:, 5]), rtol=1e-12)
+    # Large entries (the long-row workload's +-80 spikes) do not overflow.
+    z = np.zeros((1, 9))
+    z[0, 2] = 80.0
+    z[0, 7] = -80.0
+    q = orc.softmax(z)
+    assert np.isfinite(q).all()
+    _close(q[0, 2], 1.0 / (1.0 + 7.0 * math.exp(-80.0) + math.exp(-160.0)),
+           rtol=1e-14)
+
+
+def pin_layernorm_invariants(orc):
+    rng = np.random.default_rng(12)
+    x = rng.normal(3, 2, size=(9, 47))
+    y = orc.layernorm(x, eps=0.0)
+    _close(y.mean(axis=1), np.zeros(9), rtol=0, atol=1e-13)
+    _close(y.var(axis=1), np.ones(9), rtol=1e-12)
+    # Affine invariance at eps = 0: LN(a x + b) == LN(x) for a > 0, and a
+    # negative scale flips the sign.
+    _close(orc.layernorm(2.5 * x - 40.0, eps=0.0), y, rtol=1e-10, atol=1e-12)
+    _close(orc.layernorm(-0.5 * x, eps=0.0), -y, rtol=1e-10, atol=1e-12)
+    # With eps > 0 the output variance is var/(var + eps).
+    eps = 0.75
+    ye = orc.layernorm(x, eps=eps)
+    v = x.var(axis=1)
+    _close(ye.var(axis=1), v / (v + np.float64(np.float32(eps))), rtol=1e-12)
+    _close(ye.mean(axis=1), np.zeros(9), rtol=0, atol=1e-13)
+    # Two distinct values normalise to -1, +1.
+    _close(orc.layernorm(np.array([[4.0, 10.0]]), eps=0.0), [[-1.0, 1.0]])
+    # gamma/beta act per column after normalising.
+    g = rng.normal(1, 0.1, 47)
+    b = rng.normal(0, 0.1, 47)
+    _close(orc.layernorm(x, g, b, eps=0.0), y * g + b, rtol=1e-12, atol=1e-13)
+
+
+def pin_rmsnorm_invariants(orc):
+    rng = np.random.default_rng(13)
+    x = rng.normal(0, 3, size=(8, 33))
+    y = orc.rmsnorm(x, eps=0.0)
+    # Unit root-mean-square at eps = 0, and scale invariance.
+    _close(np.sqrt((y * y).mean(axis=1)), np.ones(8), rtol=1e-13)
+    _close(orc.rmsnorm(17.0 * x, eps=0.0), y, rtol=1e-12)
+    _close(orc.rmsnorm(-x, eps=0.0), -y, rtol=1e-12)
+    # No mean subtraction: a constant row c gives c/sqrt(c^2 + eps) * gamma,
+    # i.e. sign(c) * gamma at eps = 0.
+    g = rng.normal(1, 0.1, 33)
+    for c in (-2.5, 0.125, 9.0):
+        row = np.full((1, 33), c)
+        _close(orc.rmsnorm(row, g, eps=0.0), (np.sign(c) * g)[None],
+               rtol=1e-14)
+        eps = 0.5
+        _close(orc.rmsnorm(row, g, eps=eps),
+               (c / math.sqrt(c * c + eps) * g)[None], rtol=1e-14)
+    # gamma acts per column.
+    _close(orc.rmsnorm(x, g, eps=0.0), y * g, rtol=1e-12)
+
+
+# --------------------------------------------------------------------------
+def _brute_row(op, x, gamma, beta, eps):
+    n = len(x)
+    if op in ("softmax", "logsoftmax"):
+        m = max(x)
+        e = [math.exp(v - m) for v in x]
+        s = math.fsum(e)
+        if op == "softmax":
+            return [v / s for v in e]
+        return [(v - m) - math.log(s) for v in x]
+    if op == "layernorm":
+        mu = math.fsum(x) / n
+        var = math.fsum([(v - mu) ** 2 for v in x]) / n
+        d = math.sqrt(var + eps)
+        return [(v - mu) / d * gamma[j] + beta[j] for j, v in enumerate(x)]
+    if op == "rmsnorm":
+        d = math.sqrt(math.fsum([v * v for v in x]) / n + eps)
+        return [v / d * gamma[j] for j, v in enumerate(x)]
+    raise ValueError(op)
+
+
+def pin_brute_force(orc):
+    rng = np.random.default_rng(14)
+    for trial in range(40):
+        rows = int(rng.integers(1, 9))
+        cols = int(rng.integers(1, 34))
+        op = OPS[trial % 4]
+        x = rng.normal(0, 1 + trial % 5, size=(rows, cols))
+        g = rng.normal(1, 0.2, cols)
+        b = rng.normal(0, 0.2, cols)
+        eps = float(np.float32([0.0, 1e-5, 1e-6, 0.1][trial % 4]))
+        got = _call(orc, op, x, g, b, eps)
+        exp = np.array([_brute_row(op, list(r), g, b, eps) for r in x])
+        _close(got, exp, rtol=1e-11, atol=1e-12)
+
+
+def pin_torch_float64(orc):
+    import torch
+    import torch.nn.functional as F
+    rng = np.random.default_rng(15)
+    x = rng.normal(0, 4, size=(6, 130))
+    g = rng.normal(1, 0.1, 130)
+    b = rng.normal(0, 0.1, 130)
+    t = torch.from_numpy(x)
+    _close(orc.softmax(x), torch.softmax(t, dim=1).numpy(), rtol=1e-12,
+           atol=1e-15)
+    _close(orc.logsoftmax(x), torch.log_softmax(t, dim=1).numpy(),
+           rtol=1e-12, atol=1e-13)
+    eps = float(np.float32(1e-5))
+    _close(orc.layernorm(x, g, b, eps=eps),
+           F.layer_norm(t, (130,), torch.from_numpy(g), torch.from_numpy(b),
+                        eps=eps).numpy(), rtol=1e-11, atol=1e-12)
+    if hasattr(F, "rms_norm"):
+        eps = float(np.float32(1e-6))
+        _close(orc.rmsnorm(x, g, eps=eps),
+               F.rms_norm(t, (130,), torch.from_numpy(g), eps=eps).numpy(),
+               rtol=1e-11, atol=1e-12)
+
+
+def pin_ragged(orc):
+    rng = np.random.default_rng(16)
+    lens = np.array([5, 0, 1, 33, 2, 0, 17], dtype=np.int64)
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    x = rng.normal(0, 2, int(off[-1]))
+    g = rng.normal(1, 0.1, int(lens.max()))
+    b = rng.normal(0, 0.1, int(lens.max()))
+    for op in OPS:
+        eps = 1e-5 if op in ("layernorm", "rmsnorm") else 0.0
+        y = _call_ragged(orc, op, x, off, g, b, eps)
+        for i, n in enumerate(lens):
+            seg = slice(off[i], off[i + 1])
+            if n == 0:
+                continue
+            ref = _call(orc, op, x[seg][None, :], g[:n], b[:n], eps)[0]
+            _close(y[seg], ref, rtol=0, atol=0)
+        # gamma/beta are indexed by the column inside the row: a row of 2
+        # sees gamma[0:2], not gamma[off:off+2].
+    # Length-1 rows.
+    one = np.arange(0, 4, dtype=np.int64)
+    xs = np.array([3.0, -2.0, 0.5])
+    _close(orc.softmax_ragged(xs, one), np.ones(3))
+    _close(orc.logsoftmax_ragged(xs, one), np.zeros(3))
+    _close(orc.layernorm_ragged(xs, one, np.array([2.0]), np.array([0.5]),
+                                eps=1e-5), np.full(3, 0.5))
+
+
+def pin_bucket_rule(orc):
+    # Thresholds by row bytes: <= 4096 SMALL, <= 32768 MEDIUM, else LARGE.
+    for esize in (2, 4):
+        s_max = 4096 // esize
+        m_max = 32768 // esize
+        assert orc.bucket(1, esize) == 0
+        assert orc.bucket(s_max, esize) == 0
+        assert orc.bucket(s_max + 1, esize) == 1
+        assert orc.bucket(m_max, esize) == 1
+        assert orc.bucket(m_max + 1, esize) == 2
+        assert orc.bucket(1 << 20, esize) == 2
+
+
+ALL_PINS = [pin_hand_cases, pin_softmax_invariants, pin_layernorm_invariants,
+            pin_rmsnorm_invariants, pin_brute_force, pin_torch_float64,
+            pin_ragged, pin_bucket_rule]

@@ -1,0 +1,86 @@
+"""Plant plausible mistakes in a copy of the oracle (on the CPU) and check
+that the pin suite catches every one.  The real oracle is never modified:
+each mutant is compiled from an edited copy of the C source in a temporary
+directory and loaded through a fresh copy of the Python wrapper."""
+import importlib.util
+import os
+import re
+
+import pytest
+
+from tests.oracle_pins import ALL_PINS
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "rowop_oracle.c")
+WRAPPER = os.path.join(ROOT, "oracle", "rowop_oracle.py")
+
+# (function whose body is edited, text, replacement, what the mistake is)
+MUTANTS = [
+    ("softmax_row", "s += exp(x[j] - m);", "s += exp(x[j]);",
+     "sum without the max shift"),
+    ("softmax_row", "y[j] = exp(x[j] - m) / s;", "y[j] = exp(x[j] - m) * s;",
+     "multiply instead of divide"),
+    ("softmax_row", "if (x[j] > m)", "if (x[j] < m)", "min instead of max"),
+    ("logsoftmax_row", "(x[j] - m) - log_s", "(x[j] - m) + log_s",
+     "wrong sign of log-sum"),
+    ("logsoftmax_row", "(x[j] - m) - log_s", "x[j] - log_s",
+     "dropped max term"),
+    ("layernorm_row", "sq / (double)n", "sq / (double)(n - 1)",
+     "unbiased variance"),
+    ("layernorm_row", "sqrt(var + eps)", "(sqrt(var) + eps)",
+     "eps outside the root"),
+    ("layernorm_row", "* gamma[j] + beta[j]", "* gamma[j]", "dropped beta"),
+    ("layernorm_row", "gamma[j]", "gamma[0]", "gamma index"),
+    ("layernorm_row", "(x[j] - mu) / den", "(x[j] - mu) * den",
+     "inverted scale"),
+    ("rmsnorm_row", "sq / (double)n", "sq", "sum instead of mean of squares"),
+    ("rmsnorm_row", "sqrt(ms + eps)", "sqrt(ms)", "dropped eps"),
+    ("rmsnorm_row", "* gamma[j]", "", "dropped gamma"),
+    ("oracle_softmax_ragged", "off[r + 1] - off[r]", "off[r + 1] - off[r] - 1",
+     "ragged row length off by one"),
+    ("oracle_layernorm_ragged", "gamma, beta,", "gamma + off[r], beta,",
+     "gamma indexed by packed offset"),
+    ("oracle_bucket", "bytes <= 4096", "bytes < 4096",
+     "SMALL threshold off by one"),
+    ("oracle_bucket", "bytes <= 32768", "bytes <= 65536",
+     "MEDIUM threshold"),
+]
+
+
+def _mutate(src: str, func: str, old: str, new: str) -> str:
+    m = re.search(r"\n[a-z ]*\b" + re.escape(func) + r"\(", src)
+    assert m, func
+    start = m.start()
+    end = src.index("\n}\n", start)
+    body = src[start:end]
+    assert old in body, (func, old)
+    return src[:start] + body.replace(old, new, 1) + src[end:]
+
+
+def _load_mutant(tmp_path, text):
+    d = tmp_path / "mut"
+    d.mkdir()
+    (d / "rowop_oracle.c").write_text(text)
+    spec = importlib.util.spec_from_file_location("oracle_mutant", WRAPPER)
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    mod._SRC = str(d / "rowop_oracle.c")
+    mod._BUILD_DIR = str(d / "_build")
+    mod._LIB_PATH = str(d / "_build" / "liboracle.so")
+    mod._lib = None
+    return mod
+
+
+@pytest.mark.parametrize("func,old,new,what", MUTANTS,
+                         ids=[m[3].replace(" ", "_") for m in MUTANTS])
+def test_pins_catch_mutant(tmp_path, func, old, new, what):
+    with open(SRC) as f:
+        src = f.read()
+    mod = _load_mutant(tmp_path, _mutate(src, func, old, new))
+    caught = []
+    for pin in ALL_PINS:
+        try:
+            pin(mod)
+        except (AssertionError, ValueError, FloatingPointError) as e:
+            caught.append(pin.__name__)
+    assert caught, f"no pin caught the planted mistake: {what}"
