@@ -1,0 +1,456 @@
+#!/usr/bin/env python3
+"""Benchmark of librowop on one or more GB300s.
+
+Headline workload (a "step" = one pass of the whole hot path): ragged bf16
+LayerNorm over 16384 rows with lengths uniform on {1..32768} (int64 CSR
+offsets into one packed buffer, gamma/beta per column), eps 1e-5, seed 4 --
+one classify launch plus one fused launch that serves all three row buckets
+(SMALL warp groups, MEDIUM CTA-per-row, LARGE cluster split).  Inputs and
+outputs (0.54 GB each) are larger than L2, so no flush is needed between
+steps.
+
+Metric: effective HBM GB/s = algorithmic bytes (read x once, write y once,
+gamma/beta once, offsets once) / time.  Also reported in the same JSON line:
+every workload's own figure (`per_config`, L2 flushed between timed calls
+where its footprint is within 2x L2), the roofline of the dominant kernel, an
+end-to-end figure through the C ABI with pinned host buffers, clocks sampled
+during the timed region, and the CPU oracle as a baseline.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+Under torchrun each rank runs the same workload on its own GPU (weak
+scaling, no collective on the data path); rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "effective HBM GB/s (bytes read+written) and % of GB300 peak per row-op config"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing (one process per GPU; only barriers and a max-reduce)
+# ---------------------------------------------------------------------------
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if args.impl != "reference" else "gloo"
+        dist.init_process_group(backend)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(v, world, device):
+    if world == 1:
+        return v
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([v], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+        return False
+
+    def summary(self):
+        rows = []
+        for line in (self.out or "").splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"],
+                    "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i, v in enumerate(r)
+                          if v.lower().startswith("active")})
+        return {"sm_mhz": statistics.median(r[0] for r in rows),
+                "sm_max_mhz": max(r[1] for r in rows), "reasons": reasons,
+                "samples": len(rows)}
+
+
+# ---------------------------------------------------------------------------
+# GPU timing helpers
+# ---------------------------------------------------------------------------
+class L2Flusher:
+    def __init__(self, torch, device):
+        l2 = torch.cuda.get_device_properties(device).L2_cache_size
+        self.buf = torch.empty(max(2 * l2, 256 << 20) // 4, dtype=torch.int32,
+                               device=device)
+
+    def __call__(self):
+        self.buf.fill_(1)
+
+
+def time_calls(torch, fn, steps, warmup, flush=None):
+    """Per-call device time (ms) with CUDA events on the current stream; an
+    L2 flush, when given, runs before each call outside the timed span."""
+    for _ in range(warmup):
+        if flush:
+            flush()
+        fn()
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(steps):
+        if flush:
+            flush()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record()
+        fn()
+        b.record()
+        b.synchronize()
+        times.append(a.elapsed_time(b))
+    return times
+
+
+def per_config(torch, rw, wl, device, peak, steps):
+    """Every workload of the suite, each timed on its own."""
+    flush = L2Flusher(torch, device)
+    l2 = torch.cuda.get_device_properties(device).L2_cache_size
+    out = []
+    for case in wl.all_cases():
+        x = case.x.to(device)
+        g = case.gamma.to(device) if case.gamma is not None else None
+        b = case.beta.to(device) if case.beta is not None else None
+        if case.ragged:
+            off = case.offsets.to(device)
+            y = torch.empty_like(x)
+            ws = rw.ragged_workspace(case.rows, device)
+            fn = lambda: rw.run(case.op, x, offsets=off, max_len=case.max_len,  # noqa: E731
+                                gamma=g, beta=b, eps=case.eps, out=y, ws=ws)
+        else:
+            y = torch.empty_like(x)
+            fn = lambda: rw.run(case.op, x, gamma=g, beta=b, eps=case.eps, out=y)  # noqa: E731
+        nbytes = case.algorithmic_bytes()
+        use_flush = nbytes <= 2 * l2  # footprint within 2x L2
+        ts = time_calls(torch, fn, steps, 3, flush if use_flush else None)
+        st = rw.check_status()
+        if st != 0:
+            raise RuntimeError(f"{case.name}: device status {rw.STATUS.get(st, st)}")
+        med = statistics.median(ts)
+        best = min(ts)
+        gbs = nbytes / (med * 1e-3) / 1e9
+        out.append({
+            "name": case.name, "op": case.op,
+            "dtype": "bf16" if case.dtype == torch.bfloat16 else "f32",
+            "shape": ([case.rows, "ragged", case.max_len] if case.ragged
+                      else list(case.x.shape)),
+            "bytes": nbytes, "ms_median": round(med, 5), "ms_best": round(best, 5),
+            "gbs_median": round(gbs, 1),
+            "gbs_best": round(nbytes / (best * 1e-3) / 1e9, 1),
+            "pct_of_8TBs": round(100 * gbs / NOMINAL_HBM_GBS, 1),
+            "pct_of_measured": round(100 * gbs / peak, 1),
+            "rows_per_s": round(case.rows / (med * 1e-3), 1),
+            "l2": "flushed" if use_flush else "inputs larger than L2",
+        })
+        del x, y, g, b
+    return out
+
+
+def profile_traffic():
+    """DRAM traffic per launch of the dominant kernel from the committed ncu
+    summary, if it was taken on the current kernel sources."""
+    from paper_2607_23089_gb300 import build as bld
+    p = os.path.join(ROOT, "profiles", "fused_ragged_layernorm_traffic.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+    except Exception:
+        return None
+    if d.get("source_stamp") != bld._stamp(()):
+        return None
+    return d.get("traffic_bytes_per_launch")
+
+
+def cpu_oracle_baseline(case, max_elems):
+    """The double-precision oracle on a bounded sample of the workload (its
+    first rows), on all host cores."""
+    import numpy as np
+    from oracle import rowop_oracle as orc
+    off = case.offsets.numpy()
+    rows = int(np.searchsorted(off, max_elems, side="right") - 1)
+    rows = max(1, min(case.rows, rows))
+    n = int(off[rows])
+    x = case.x[:n].double().numpy()
+    g = case.gamma.double().numpy()
+    b = case.beta.double().numpy()
+    cores = os.cpu_count() or 1
+    t0 = time.perf_counter()
+    orc.layernorm_ragged(x, off[:rows + 1], g, b, eps=case.eps, nthreads=cores)
+    dt = time.perf_counter() - t0
+    nbytes = 2 * n * 2 + 2 * case.max_len * 2 + (rows + 1) * 8
+    return {"value": round(nbytes / dt / 1e9, 3), "unit": "GB/s", "cores": cores,
+            "kind": "oracle", "seconds": round(dt, 3),
+            "sample": f"first {rows} of {case.rows} rows ({n} of {case.elements} elements), "
+                      "float64 C oracle, OpenMP over rows"}
+
+
+# ---------------------------------------------------------------------------
+def run_reference(args, rank, world):
+    """The CPU oracle as the reference arm, on host cores, rank 0 only."""
+    if rank != 0:
+        return 0
+    from paper_2607_23089_gb300 import workloads as wl
+    from oracle import rowop_oracle as orc
+    orc.build()
+    case = wl.ragged_ln()
+    import numpy as np
+    off = case.offsets.numpy()
+    max_elems = int(os.environ.get("ROWOP_REF_SAMPLE_ELEMS", 16_000_000))
+    rows = max(1, int(np.searchsorted(off, max_elems, side="right") - 1))
+    n = int(off[rows])
+    x = case.x[:n].double().numpy()
+    g = case.gamma.double().numpy()
+    b = case.beta.double().numpy()
+    cores = os.cpu_count() or 1
+    sub = off[:rows + 1]
+    for _ in range(args.warmup):
+        orc.layernorm_ragged(x, sub, g, b, eps=case.eps, nthreads=cores)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        orc.layernorm_ragged(x, sub, g, b, eps=case.eps, nthreads=cores)
+        times.append(time.perf_counter() - t0)
+    nbytes = 2 * n * 2 + 2 * case.max_len * 2 + (rows + 1) * 8
+    tot = sum(times)
+    value = nbytes * len(times) / tot / 1e9
+    sample = (f"first {rows} of {case.rows} rows ({n} of {case.elements} elements) of the "
+              "ragged bf16 LayerNorm workload, float64 C oracle, OpenMP over rows")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": "GB/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(1e3 * tot / len(times), 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": "ragged_ln (sample)", "rows": rows, "elements": n},
+        "cpu_baseline": {"value": round(value, 3), "unit": "GB/s", "cores": cores,
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 3), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_rowop(args, rank, world, local):
+    import torch
+    from paper_2607_23089_gb300 import build as bld
+    from paper_2607_23089_gb300 import rowop as rw
+    from paper_2607_23089_gb300 import workloads as wl
+
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA device")
+    bld.build()
+    rw.load()
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    peak, peak_src = peaks()
+
+    case = wl.ragged_ln()
+    nbytes = case.algorithmic_bytes()
+    x = case.x.to(device)
+    off = case.offsets.to(device)
+    g = case.gamma.to(device)
+    b = case.beta.to(device)
+    y = torch.empty_like(x)
+    ws = rw.ragged_workspace(case.rows, device)
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+    code = rw.dtype_code(case.dtype)
+
+    def step():
+        st = rw.rowop_layernorm_ragged(x.data_ptr(), y.data_ptr(), g.data_ptr(), b.data_ptr(),
+                                       off.data_ptr(), case.rows, case.max_len, code, case.eps,
+                                       ws.data_ptr(), ws.numel(), sp)
+        if st != 0:
+            raise RuntimeError(rw.STATUS.get(st, st))
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        start.record(stream)
+        for _ in range(args.steps):
+            step()
+        end.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
+    ms = start.elapsed_time(end)
+    st = rw.check_status()
+    if st != 0:
+        raise RuntimeError(f"device status {rw.STATUS.get(st, st)}")
+    ms = max_over_ranks(ms, world, device)
+    ms_step = ms / args.steps
+    value = world * nbytes * args.steps / (ms * 1e-3) / 1e9
+
+    # dominant kernel alone: the fused launch (plan reused, no classify pass)
+    st = rw.rowop_ragged_plan(off.data_ptr(), case.rows, case.max_len, code, ws.data_ptr(),
+                              ws.numel(), sp)
+    assert st == 0
+
+    def fused():
+        rw.rowop_layernorm_ragged_planned(x.data_ptr(), y.data_ptr(), g.data_ptr(),
+                                          b.data_ptr(), off.data_ptr(), case.rows,
+                                          case.max_len, code, case.eps, ws.data_ptr(),
+                                          ws.numel(), sp)
+    fused_ms = statistics.mean(time_calls(torch, fused, max(args.steps, 10), 3))
+    achieved = nbytes / (fused_ms * 1e-3) / 1e9
+
+    # end to end through the C ABI with pinned host buffers
+    hx = case.x.pin_memory()
+    hoff = case.offsets.pin_memory()
+    hg = case.gamma.pin_memory()
+    hb = case.beta.pin_memory()
+    hy = torch.empty_like(case.x).pin_memory()
+
+    def e2e_step():
+        x.copy_(hx, non_blocking=True)
+        off.copy_(hoff, non_blocking=True)
+        g.copy_(hg, non_blocking=True)
+        b.copy_(hb, non_blocking=True)
+        step()
+        hy.copy_(y, non_blocking=True)
+    e2e_steps = max(3, min(args.steps, 10))
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    a = torch.cuda.Event(enable_timing=True)
+    z = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    z.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(a.elapsed_time(z) / e2e_steps, world, device)
+    h2d = (hx.numel() * hx.element_size() + hoff.numel() * 8 +
+           hg.numel() * hg.element_size() + hb.numel() * hb.element_size())
+    d2h = hy.numel() * hy.element_size()
+
+    result = {
+        "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": "ragged_ln: bf16 LayerNorm, 16384 ragged rows, "
+                               "len ~ U{1..32768}, int64 CSR offsets, eps 1e-5, seed 4",
+                   "rows": case.rows, "elements": case.elements, "max_len": case.max_len,
+                   "algorithmic_bytes_per_step": nbytes,
+                   "l2": "inputs larger than L2 (no flush needed)",
+                   "parallelism": f"replicas x{world} (rows are independent)",
+                   "pct_of_8TBs": round(100 * value / world / NOMINAL_HBM_GBS, 1)},
+        "gpu_launches": 2 * args.steps,
+        "clocks": clk.summary(),
+        "e2e": {"value": round(world * nbytes / (e2e_ms * 1e-3) / 1e9, 1), "unit": "GB/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": round(e2e_ms, 4)},
+        "roofline": {"bound": "hbm", "kernel": "tile_row_kernel<LayerNorm,bf16,ragged,cluster>",
+                     "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "peak_source": peak_src,
+                     "traffic": profile_traffic(),
+                     "algorithmic_bytes_per_launch": nbytes,
+                     "launch_ms": round(fused_ms, 5)},
+    }
+    if rank == 0 and not args.no_per_config:
+        result["per_config"] = per_config(torch, rw, wl, device, peak, args.config_steps)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_oracle_baseline(case, args.cpu_sample_elems)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="rowop", choices=["rowop", "reference"])
+    ap.add_argument("--config-steps", type=int, default=20)
+    ap.add_argument("--cpu-sample-elems", type=int, default=270_000_000)
+    ap.add_argument("--no-per-config", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    rank, world, local = dist_setup(args)
+    try:
+        if args.impl == "reference":
+            return run_reference(args, rank, world)
+        return run_rowop(args, rank, world, local)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    sys.exit(main())

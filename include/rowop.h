@@ -1,0 +1,220 @@
+/*
+ * rowop.h -- C ABI of librowop: row-wise reduce-then-normalise operators
+ * (softmax, log-softmax, LayerNorm, RMSNorm) on one NVIDIA GB300 (sm_103a).
+ *
+ * The operator family is the one whose row-length dispatch the paper's
+ * running example names (small_row_kernel, medium_row_kernel,
+ * large_row_kernel chosen by launch_by_rows, tiled by BLOCK_ROWS; §2.1 "A
+ * Running Example").  The paper gives the kernel names only, so the
+ * operators follow the textbook / PyTorch definitions:
+ *
+ *   softmax      y_j = exp(x_j - m) / s,   m = max_j x_j, s = sum_j exp(x_j - m)
+ *   log-softmax  y_j = (x_j - m) - log(s)
+ *   LayerNorm    y_j = (x_j - mu) / sqrt(var + eps) * gamma_j + beta_j
+ *                (mu = mean, var = biased variance of the row)
+ *   RMSNorm      y_j = x_j / sqrt(mean_j(x_j^2) + eps) * gamma_j
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - All pointers are DEVICE pointers owned by the caller; the library never
+ *   allocates device memory on a call and keeps no pointer after it returns.
+ * - Element type is rowop_dtype_t: float32, or bfloat16 with float32
+ *   arithmetic inside and round-to-nearest-even on output.  gamma and beta
+ *   have the element type of the data.  gamma == NULL means all ones and
+ *   beta == NULL all zeros.
+ * - Dense layout: row r starts at element r*ld of `in` and of `out`; ld is in
+ *   elements, ld >= cols, and is shared by in and out.  Any element-aligned
+ *   pointer and any ld are accepted: 16-byte aligned rows take the vector
+ *   path, other rows take per-element loads and stores at the row edges.
+ * - Ragged layout: row i is elements [offsets[i], offsets[i+1]) of one packed
+ *   buffer (the same offsets index `in` and `out`); offsets is a DEVICE
+ *   int64 array of rows+1 non-decreasing entries; gamma_j / beta_j are
+ *   indexed by the column j inside the row, so gamma/beta hold max_len
+ *   entries.  Rows whose length is negative (decreasing offsets) or larger
+ *   than max_len are skipped and flagged (see rowop_check_status).
+ * - in == out (exact in-place) is allowed; partial overlap is undefined.
+ * - Calls are asynchronous with respect to the host and ordered on `stream`
+ *   (NULL = legacy default stream), like cuBLAS.  Argument errors are found
+ *   before anything is launched and are returned synchronously.  A launch
+ *   failure returns ROWOP_ERR_CUDA.  Device-side conditions (a bounded wait
+ *   that ran out, rejected ragged rows) are recorded in a device status word
+ *   that rowop_check_status() reads.
+ * - rows == 0 is a valid no-op.  Results are deterministic: the same call on
+ *   the same data gives bitwise the same output, and a row's result depends
+ *   only on its values, its length and its start address modulo 16 bytes
+ *   (so a ragged row equals a dense call on the same row at the same
+ *   alignment, bit for bit).
+ */
+#ifndef ROWOP_H
+#define ROWOP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifndef __DRIVER_TYPES_H__
+typedef struct CUstream_st *cudaStream_t;
+#endif
+
+#if defined(__GNUC__)
+#define ROWOP_API __attribute__((visibility("default")))
+#else
+#define ROWOP_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum rowop_dtype {
+    ROWOP_F32 = 0,  /* float32 in, float32 out                         */
+    ROWOP_BF16 = 1  /* bfloat16 in/out, float32 arithmetic, RNE output */
+} rowop_dtype_t;
+
+typedef enum rowop_status {
+    ROWOP_OK = 0,
+    ROWOP_ERR_INVALID_ARG = 1,        /* NULL / misaligned pointer, bad size, ld < cols, eps < 0 */
+    ROWOP_ERR_UNSUPPORTED_DTYPE = 2,  /* dtype is not ROWOP_F32 or ROWOP_BF16 */
+    ROWOP_ERR_WORKSPACE = 3,          /* ragged workspace NULL, misaligned or too small */
+    ROWOP_ERR_CUDA = 4,               /* a CUDA runtime call or launch failed */
+    ROWOP_ERR_TIMEOUT = 5,            /* a bounded device wait ran out (see rowop_check_status) */
+    ROWOP_ERR_BAD_OFFSETS = 6,        /* ragged rows were skipped: decreasing offsets or len > max_len */
+    ROWOP_ERR_TOO_LONG = 7            /* row longer than rowop_max_row_len() */
+} rowop_status_t;
+
+/* Row-length buckets of launch_by_rows (§2.1): the kernel design a row goes to. */
+typedef enum rowop_bucket {
+    ROWOP_SMALL = 0,   /* row bytes <= 4096: a group of <= 32 lanes per row, registers   */
+    ROWOP_MEDIUM = 1,  /* row bytes <= 32768: one CTA per row, row staged by TMA bulk copy */
+    ROWOP_LARGE = 2    /* longer: a thread-block cluster splits the row, partials via DSMEM */
+} rowop_bucket_t;
+
+/* ---- dense rows x cols ---------------------------------------------------
+ * in    : rows x cols elements of dtype, row stride ld (elements)
+ * out   : same layout and ld as in; written in full for every row
+ * Returns ROWOP_OK or an error code; nothing is launched on error.        */
+
+/* Softmax along each row. */
+ROWOP_API int rowop_softmax(const void *in, void *out, int64_t rows, int64_t cols,
+                  int64_t ld, rowop_dtype_t dtype, cudaStream_t stream);
+
+/* Log-softmax along each row, computed as (x - max) - log(sum). */
+ROWOP_API int rowop_logsoftmax(const void *in, void *out, int64_t rows, int64_t cols,
+                     int64_t ld, rowop_dtype_t dtype, cudaStream_t stream);
+
+/* LayerNorm along each row (biased variance, eps inside the square root);
+ * gamma/beta: cols elements each, or NULL.  eps >= 0. */
+ROWOP_API int rowop_layernorm(const void *in, void *out, const void *gamma,
+                    const void *beta, int64_t rows, int64_t cols, int64_t ld,
+                    rowop_dtype_t dtype, float eps, cudaStream_t stream);
+
+/* RMSNorm along each row (no mean subtraction, no beta); gamma: cols
+ * elements, or NULL.  eps >= 0. */
+ROWOP_API int rowop_rmsnorm(const void *in, void *out, const void *gamma, int64_t rows,
+                  int64_t cols, int64_t ld, rowop_dtype_t dtype, float eps,
+                  cudaStream_t stream);
+
+/* ---- ragged rows (int64 CSR offsets into one packed buffer) ---------------
+ * offsets : device int64[rows + 1], non-decreasing
+ * max_len : an upper bound on every row's length (>= 0); sizes the on-chip
+ *           staging and bounds gamma/beta, which hold max_len elements
+ * ws      : device workspace of at least rowop_ragged_workspace_size(rows)
+ *           bytes, 256-byte aligned, owned by the caller.  It must not be
+ *           used by another call that may run at the same time.  After the
+ *           call (once the stream reaches it) byte ws[256 + i] holds the
+ *           bucket row i was dispatched to (255 = row rejected), and the
+ *           uint32 at ws[0] holds this call's device status bits.
+ * All buckets are handled in one pass over the rows (a classify launch, then
+ * one fused launch that serves all three buckets).                         */
+
+ROWOP_API size_t rowop_ragged_workspace_size(int64_t rows);
+
+ROWOP_API int rowop_softmax_ragged(const void *in, void *out, const int64_t *offsets,
+                         int64_t rows, int64_t max_len, rowop_dtype_t dtype,
+                         void *ws, size_t ws_bytes, cudaStream_t stream);
+
+ROWOP_API int rowop_logsoftmax_ragged(const void *in, void *out,
+                            const int64_t *offsets, int64_t rows,
+                            int64_t max_len, rowop_dtype_t dtype, void *ws,
+                            size_t ws_bytes, cudaStream_t stream);
+
+ROWOP_API int rowop_layernorm_ragged(const void *in, void *out, const void *gamma,
+                           const void *beta, const int64_t *offsets,
+                           int64_t rows, int64_t max_len, rowop_dtype_t dtype,
+                           float eps, void *ws, size_t ws_bytes,
+                           cudaStream_t stream);
+
+ROWOP_API int rowop_rmsnorm_ragged(const void *in, void *out, const void *gamma,
+                         const int64_t *offsets, int64_t rows,
+                         int64_t max_len, rowop_dtype_t dtype, float eps,
+                         void *ws, size_t ws_bytes, cudaStream_t stream);
+
+/* ---- ragged plans: classify once, run many operators ---------------------
+ * rowop_ragged_plan runs only the classify pass of launch_by_rows (bucket per
+ * row and the three row lists) into ws.  A *_ragged_planned call then skips
+ * that pass and reuses the plan: it must get the same offsets (unchanged
+ * contents), rows, max_len, dtype and ws as the plan, on the same stream or
+ * after it.  Each planned call leaves the plan reusable for the next one.
+ * The plain *_ragged calls above are plan + planned call in one.          */
+
+ROWOP_API int rowop_ragged_plan(const int64_t *offsets, int64_t rows,
+                                int64_t max_len, rowop_dtype_t dtype, void *ws,
+                                size_t ws_bytes, cudaStream_t stream);
+
+ROWOP_API int rowop_softmax_ragged_planned(const void *in, void *out,
+                                           const int64_t *offsets, int64_t rows,
+                                           int64_t max_len, rowop_dtype_t dtype,
+                                           void *ws, size_t ws_bytes,
+                                           cudaStream_t stream);
+
+ROWOP_API int rowop_logsoftmax_ragged_planned(const void *in, void *out,
+                                              const int64_t *offsets,
+                                              int64_t rows, int64_t max_len,
+                                              rowop_dtype_t dtype, void *ws,
+                                              size_t ws_bytes,
+                                              cudaStream_t stream);
+
+ROWOP_API int rowop_layernorm_ragged_planned(const void *in, void *out,
+                                             const void *gamma, const void *beta,
+                                             const int64_t *offsets, int64_t rows,
+                                             int64_t max_len, rowop_dtype_t dtype,
+                                             float eps, void *ws, size_t ws_bytes,
+                                             cudaStream_t stream);
+
+ROWOP_API int rowop_rmsnorm_ragged_planned(const void *in, void *out,
+                                           const void *gamma,
+                                           const int64_t *offsets, int64_t rows,
+                                           int64_t max_len, rowop_dtype_t dtype,
+                                           float eps, void *ws, size_t ws_bytes,
+                                           cudaStream_t stream);
+
+/* ---- dispatch rule, limits, status ---------------------------------------- */
+
+/* launch_by_rows (§2.1): the bucket for a row of len elements (len >= 0):
+ * SMALL if len*esize <= 4096, MEDIUM if <= 32768, else LARGE.
+ * Returns -1 for len < 0 or an unknown dtype.  Pure host function. */
+ROWOP_API int rowop_select_bucket(int64_t len, rowop_dtype_t dtype);
+
+/* Longest row (elements) the library accepts for dtype, dense or ragged. */
+ROWOP_API int64_t rowop_max_row_len(rowop_dtype_t dtype);
+
+/* Human-readable name of a status code (static storage, never NULL). */
+ROWOP_API const char *rowop_status_string(int status);
+
+/* Synchronises `stream`, then reads and clears the device status word of the
+ * current device: returns ROWOP_OK, ROWOP_ERR_TIMEOUT if any bounded device
+ * wait ran out, ROWOP_ERR_BAD_OFFSETS if ragged rows were rejected (timeout
+ * wins when both are set), or ROWOP_ERR_CUDA if the synchronisation failed. */
+ROWOP_API int rowop_check_status(cudaStream_t stream);
+
+/* Test hook for the bounded-wait path, launching one tiny kernel that waits
+ * on an on-chip barrier nothing will complete, for at most limit_ns
+ * nanoseconds (1 .. 10^9), then records a timeout in the status word and
+ * returns.  No memory traffic is in flight while it waits.  Returns
+ * ROWOP_ERR_INVALID_ARG for an out-of-range limit. */
+ROWOP_API int rowop_debug_wait_timeout(int64_t limit_ns, cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ROWOP_H */

@@ -1,0 +1,87 @@
+// dispatch.h -- internal host interface between the C ABI (rowop_api.cu) and
+// the per-operator launch code (ops_*.cu).  Not part of the public ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace rowop {
+
+struct DeviceInfo {
+  int device;
+  int sm_count;
+  int max_smem_optin;      // bytes of dynamic shared memory a CTA may opt into
+  unsigned int *status;    // device status word of this device
+};
+
+struct DenseCall {
+  int dtype;  // 0 fp32, 1 bf16
+  const void *in;
+  void *out;
+  const void *gamma;
+  const void *beta;
+  int64_t rows, cols, ld;
+  float eps;
+  cudaStream_t stream;
+};
+
+struct RaggedCall {
+  int dtype;
+  const void *in;
+  void *out;
+  const void *gamma;
+  const void *beta;
+  const int64_t *offsets;
+  int64_t rows, max_len;
+  float eps;
+  void *ws;
+  cudaStream_t stream;
+  bool classify;  // run the classify pass first (false: reuse a plan in ws)
+};
+
+// Ragged workspace layout (bytes): [0,4) status bits of the call, [64,76)
+// int32 counts per bucket, [128,140) uint32 work counters, [256, 256+rows)
+// uint8 bucket per row, then three int32 row lists of `rows` entries each
+// starting at ragged_lists_offset(rows).
+constexpr size_t kWsStatus = 0;
+constexpr size_t kWsCounts = 64;
+constexpr size_t kWsCounters = 128;
+constexpr size_t kWsBuckets = 256;
+inline size_t ragged_lists_offset(int64_t rows) {
+  return (kWsBuckets + static_cast<size_t>(rows) + 255) & ~static_cast<size_t>(255);
+}
+inline size_t ragged_ws_bytes(int64_t rows) {
+  return ragged_lists_offset(rows) + 3 * 4 * static_cast<size_t>(rows) + 256;
+}
+
+// Tile budget of one CTA portion: the longest row the resident split-row
+// design takes is this many 1 KiB tiles per CTA times the largest cluster.
+constexpr int kMaxPortionTiles = 192;
+constexpr int kMaxCluster = 16;
+inline int64_t max_row_len_elems(int esize) {
+  const int64_t e = 16 / esize;
+  return static_cast<int64_t>(kMaxPortionTiles) * kMaxCluster * 64 * e - (e - 1);
+}
+
+// Test-and-tuning knobs read from the environment (never change results):
+//   ROWOP_FORCE_BUCKET  0/1/2 -> dense rows use that design when it can hold
+//                       the row (SMALL only for rows of <= 288 chunks)
+//   ROWOP_CLUSTER       cluster size for split rows (1, 2, 4, 8, 16)
+//   ROWOP_STAGES        stage-ring depth of the tile kernel
+struct Knobs {
+  int force_bucket = -1;
+  int cluster = 0;
+  int stages = 0;
+};
+Knobs read_knobs();
+
+// Ragged classify pass into the workspace (defined in rowop_api.cu).
+cudaError_t launch_classify(const RaggedCall &c, const DeviceInfo &d);
+
+template <int OP>
+cudaError_t launch_dense(const DenseCall &c, const DeviceInfo &d);
+template <int OP>
+cudaError_t launch_ragged(const RaggedCall &c, const DeviceInfo &d);
+
+}  // namespace rowop

@@ -1,0 +1,297 @@
+// launchers.cuh -- host side of launch_by_rows (§2.1): picks the bucket design
+// for a call, sizes the stage ring, the cluster and the persistent grid, and
+// launches.  Included by one translation unit per operator (ops_*.cu), which
+// instantiates launch_dense<OP> and launch_ragged<OP>.
+#pragma once
+
+#include <algorithm>
+#include <map>
+#include <mutex>
+#include <tuple>
+
+#include "dispatch.h"
+#include "small_row.cuh"
+#include "tile_row.cuh"
+
+namespace rowop {
+
+constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s per bounded wait
+
+inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline bool congruent16(const void *a, const void *b) {
+  return ((reinterpret_cast<uintptr_t>(a) ^ reinterpret_cast<uintptr_t>(b)) & 15u) == 0;
+}
+inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+// Occupancy answers are cached per (kernel, shared memory, cluster size).
+inline int cached_occupancy(const void *kernel, size_t smem, int cluster,
+                            const cudaLaunchConfig_t *cfg) {
+  static std::mutex mu;
+  static std::map<std::tuple<const void *, size_t, int, int>, int> cache;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const auto key = std::make_tuple(kernel, smem, cluster, dev);
+  {
+    std::lock_guard<std::mutex> lk(mu);
+    auto it = cache.find(key);
+    if (it != cache.end()) return it->second;
+  }
+  int n = 0;
+  cudaError_t e;
+  if (cluster > 1) {
+    e = cudaOccupancyMaxActiveClusters(&n, kernel, cfg);
+  } else {
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel, kCtaThreads, smem);
+  }
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    n = 0;
+  }
+  std::lock_guard<std::mutex> lk(mu);
+  cache[key] = n;
+  return n;
+}
+
+// Kernel attributes are raised once per kernel and device.
+inline cudaError_t prepare_kernel(const void *kernel, const DeviceInfo &d, bool big_cluster) {
+  static std::mutex mu;
+  static std::map<std::pair<const void *, int>, bool> done;
+  std::lock_guard<std::mutex> lk(mu);
+  const auto key = std::make_pair(kernel, d.device);
+  if (done.count(key)) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       d.max_smem_optin);
+  if (e != cudaSuccess) return e;
+  if (big_cluster) {
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+  }
+  done[key] = true;
+  return cudaSuccess;
+}
+
+// ---------------------------------------------------------------------------
+// SMALL: register-resident rows, G lanes per row
+// ---------------------------------------------------------------------------
+template <int OP, typename T, int CPL, bool EXACT>
+cudaError_t launch_small_k(const SmallParams &p, const DeviceInfo &d, cudaStream_t stream) {
+  auto kern = small_row_kernel<OP, T, CPL, EXACT>;
+  const int bps = cached_occupancy(reinterpret_cast<const void *>(kern), 0, 1, nullptr);
+  const int64_t rows_per_cta = static_cast<int64_t>(kCtaWarps) * (32 / p.G);
+  const int64_t want = ceil_div(p.rows, rows_per_cta);
+  const int64_t cap = static_cast<int64_t>(std::max(bps, 1)) * d.sm_count;
+  const int grid = static_cast<int>(std::max<int64_t>(1, std::min(want, cap)));
+  kern<<<grid, kCtaThreads, 0, stream>>>(p);
+  return cudaGetLastError();
+}
+
+template <int OP, typename T>
+cudaError_t launch_small(const DenseCall &c, const DeviceInfo &d, bool exact, bool out_vec,
+                         bool gvec) {
+  constexpr int SZ = sizeof(T);
+  constexpr int E = 16 / SZ;
+  SmallParams p;
+  p.in = c.in;
+  p.out = c.out;
+  p.rows = c.rows;
+  p.cols = c.cols;
+  p.ld = c.ld;
+  p.G = small_group_lanes(c.cols, SZ);
+  p.a.gamma = c.gamma;
+  p.a.beta = c.beta;
+  p.a.glen = c.cols;
+  p.a.eps = c.eps;
+  p.a.gvec = gvec;
+  p.a.out_vec = out_vec;
+  const int64_t max_chunks = ceil_div(c.cols, E) + (exact ? 0 : 1);
+  const int cpl = small_cpl_class(max_chunks, p.G);
+  if (exact) {
+    if (cpl == 4) return launch_small_k<OP, T, 4, true>(p, d, c.stream);
+    if (cpl == 8) return launch_small_k<OP, T, 8, true>(p, d, c.stream);
+    return launch_small_k<OP, T, 9, true>(p, d, c.stream);
+  }
+  if (cpl == 4) return launch_small_k<OP, T, 4, false>(p, d, c.stream);
+  if (cpl == 8) return launch_small_k<OP, T, 8, false>(p, d, c.stream);
+  return launch_small_k<OP, T, 9, false>(p, d, c.stream);
+}
+
+// ---------------------------------------------------------------------------
+// MEDIUM / LARGE / ragged: the tile kernel
+// ---------------------------------------------------------------------------
+template <int OP, typename T, bool EXACT, bool CLUSTER, bool RAGGED>
+cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int64_t items,
+                          const DeviceInfo &d, cudaStream_t stream) {
+  auto kern = tile_row_kernel<OP, T, EXACT, CLUSTER, RAGGED>;
+  const void *kp = reinterpret_cast<const void *>(kern);
+  p.stage_bytes = static_cast<uint32_t>(stage_tiles) * kTileBytes;
+  p.max_tiles = stage_tiles;
+  // as many of the wanted stages as fit in the CTA's shared memory
+  while (stages > 1 &&
+         TileSmemLayout(p.stage_bytes, stages, stage_tiles).total >
+             static_cast<uint32_t>(d.max_smem_optin))
+    --stages;
+  p.stages = stages;
+  const TileSmemLayout L(p.stage_bytes, stages, stage_tiles);
+  const size_t smem = L.total;
+  if (smem > static_cast<size_t>(d.max_smem_optin)) return cudaErrorInvalidConfiguration;
+  cudaError_t e = prepare_kernel(kp, d, CLUSTER && cs > 8);
+  if (e != cudaSuccess) return e;
+
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  cfg.blockDim = dim3(kCtaThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  int grid;
+  if (CLUSTER) {
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cfg.gridDim = dim3(cs * std::max(1, d.sm_count / cs), 1, 1);
+    int ncl = cached_occupancy(kp, smem, cs, &cfg);
+    if (ncl < 1) ncl = 1;
+    grid = static_cast<int>(cs * std::max<int64_t>(1, std::min<int64_t>(items, ncl)));
+  } else {
+    const int bps = std::max(1, cached_occupancy(kp, smem, 1, nullptr));
+    grid = static_cast<int>(std::max<int64_t>(
+        1, std::min<int64_t>(items, static_cast<int64_t>(bps) * d.sm_count)));
+  }
+  cfg.gridDim = dim3(grid, 1, 1);
+  e = cudaLaunchKernelEx(&cfg, kern, p);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+inline int pick_stages(int stage_tiles, int knob) {
+  if (knob > 0) return std::min(knob, 16);
+  // about 48 KiB of stages per CTA, at least 2 so loads overlap compute
+  return std::max(2, std::min(8, 48 / std::max(1, stage_tiles)));
+}
+
+// Smallest cluster (power of two, >= 2) whose portions of a K-tile row hold
+// at most `cap` tiles; 16 if none does.
+inline int pick_cluster(int64_t K, int64_t cap, int knob) {
+  if (knob == 1 || knob == 2 || knob == 4 || knob == 8 || knob == 16) return knob;
+  int cs = 2;
+  while (cs < kMaxCluster && ceil_div(K, cs) > cap) cs <<= 1;
+  return cs;
+}
+
+template <int OP, typename T>
+cudaError_t launch_dense_t(const DenseCall &c, const DeviceInfo &d) {
+  constexpr int SZ = sizeof(T);
+  constexpr int E = 16 / SZ;
+  const Knobs kn = read_knobs();
+  const bool exact = aligned16(c.in) && aligned16(c.out) && ((c.ld * SZ) % 16 == 0) &&
+                     (c.cols % E == 0);
+  const bool out_vec = congruent16(c.in, c.out);
+  const bool gvec = (!c.gamma || aligned16(c.gamma)) && (!c.beta || aligned16(c.beta));
+  int bucket = bucket_of(c.cols, SZ);
+  const int64_t nc_max = ceil_div(c.cols + (exact ? 0 : E - 1), E);
+  const int64_t K = ceil_div(nc_max, kTileChunks);
+  if (kn.force_bucket == kSmall && nc_max <= 9 * 32) bucket = kSmall;
+  if (kn.force_bucket == kMedium && K <= kMaxPortionTiles) bucket = kMedium;
+  if (kn.force_bucket == kLarge) bucket = kLarge;
+  if (bucket == kMedium && K > kMaxPortionTiles) bucket = kLarge;
+
+  if (bucket == kSmall) return launch_small<OP, T>(c, d, exact, out_vec, gvec);
+
+  TileParams p = {};
+  p.in = c.in;
+  p.out = c.out;
+  p.gamma = c.gamma;
+  p.beta = c.beta;
+  p.glen = c.cols;
+  p.rows = c.rows;
+  p.cols = c.cols;
+  p.ld = c.ld;
+  p.eps = c.eps;
+  p.out_vec = out_vec;
+  p.gvec = gvec;
+  p.timeout_ns = kWaitLimitNs;
+  p.status = d.status;
+  if (bucket == kMedium) {
+    const int st = static_cast<int>(K);
+    const int S = pick_stages(st, kn.stages);
+    if (exact) return launch_tile_k<OP, T, true, false, false>(p, 1, S, st, c.rows, d, c.stream);
+    return launch_tile_k<OP, T, false, false, false>(p, 1, S, st, c.rows, d, c.stream);
+  }
+  const int cs = pick_cluster(K, 64, kn.cluster);
+  const int st = static_cast<int>(ceil_div(K, cs));
+  if (st > kMaxPortionTiles) return cudaErrorInvalidValue;
+  const int S = kn.stages > 0 ? std::min(kn.stages, 16) : (st >= 32 ? 1 : 2);
+  if (cs == 1) {
+    if (exact) return launch_tile_k<OP, T, true, false, false>(p, 1, S, st, c.rows, d, c.stream);
+    return launch_tile_k<OP, T, false, false, false>(p, 1, S, st, c.rows, d, c.stream);
+  }
+  if (exact) return launch_tile_k<OP, T, true, true, false>(p, cs, S, st, c.rows, d, c.stream);
+  return launch_tile_k<OP, T, false, true, false>(p, cs, S, st, c.rows, d, c.stream);
+}
+
+template <int OP>
+cudaError_t launch_dense(const DenseCall &c, const DeviceInfo &d) {
+  if (c.dtype == 0) return launch_dense_t<OP, float>(c, d);
+  return launch_dense_t<OP, __nv_bfloat16>(c, d);
+}
+
+template <int OP, typename T>
+cudaError_t launch_ragged_t(const RaggedCall &c, const DeviceInfo &d) {
+  constexpr int SZ = sizeof(T);
+  constexpr int E = 16 / SZ;
+  const Knobs kn = read_knobs();
+  unsigned char *ws = static_cast<unsigned char *>(c.ws);
+  const size_t lists = ragged_lists_offset(c.rows);
+  int32_t *list0 = reinterpret_cast<int32_t *>(ws + lists);
+  if (c.classify) {
+    const cudaError_t e = launch_classify(c, d);
+    if (e != cudaSuccess) return e;
+  }
+  if (c.max_len == 0) return cudaSuccess;
+
+  TileParams p = {};
+  p.in = c.in;
+  p.out = c.out;
+  p.gamma = c.gamma;
+  p.beta = c.beta;
+  p.glen = c.max_len;
+  p.eps = c.eps;
+  p.out_vec = congruent16(c.in, c.out);
+  p.gvec = (!c.gamma || aligned16(c.gamma)) && (!c.beta || aligned16(c.beta));
+  p.timeout_ns = kWaitLimitNs;
+  p.status = d.status;
+  p.offsets = c.offsets;
+  p.list_small = list0;
+  p.list_medium = list0 + c.rows;
+  p.list_large = list0 + 2 * c.rows;
+  p.counts = reinterpret_cast<const int32_t *>(ws + kWsCounts);
+  p.counters = reinterpret_cast<unsigned int *>(ws + kWsCounters);
+
+  const int64_t kmax = ceil_div(ceil_div(c.max_len + E - 1, E), kTileChunks);
+  const int64_t med_len = std::min<int64_t>(c.max_len, kMediumMaxBytes / SZ);
+  const int64_t kmed = ceil_div(ceil_div(med_len + E - 1, E), kTileChunks);
+  const bool has_large = bucket_of(c.max_len, SZ) == kLarge;
+  int cs = 1;
+  int64_t st = std::max<int64_t>(1, kmed);
+  if (has_large) {
+    cs = pick_cluster(kmax, std::max<int64_t>(kmed, 64), kn.cluster);
+    st = std::max<int64_t>(st, ceil_div(kmax, cs));
+  }
+  if (st > kMaxPortionTiles) return cudaErrorInvalidValue;
+  const int S = pick_stages(static_cast<int>(st), kn.stages);
+  if (cs > 1)
+    return launch_tile_k<OP, T, false, true, true>(p, cs, S, static_cast<int>(st), c.rows, d,
+                                                   c.stream);
+  return launch_tile_k<OP, T, false, false, true>(p, 1, S, static_cast<int>(st), c.rows, d,
+                                                  c.stream);
+}
+
+template <int OP>
+cudaError_t launch_ragged(const RaggedCall &c, const DeviceInfo &d) {
+  if (c.dtype == 0) return launch_ragged_t<OP, float>(c, d);
+  return launch_ragged_t<OP, __nv_bfloat16>(c, d);
+}
+
+}  // namespace rowop

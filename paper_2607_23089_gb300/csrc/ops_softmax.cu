@@ -1,0 +1,9 @@
+// ops_softmax.cu -- instantiates the dense and ragged launch paths (all three
+// bucket designs, fp32 and bf16) for the softmax operator.  One operator per
+// translation unit so the library compiles in parallel.
+#include "launchers.cuh"
+
+namespace rowop {
+template cudaError_t launch_dense<kSoftmax>(const DenseCall &, const DeviceInfo &);
+template cudaError_t launch_ragged<kSoftmax>(const RaggedCall &, const DeviceInfo &);
+}  // namespace rowop

@@ -1,0 +1,363 @@
+// rowop_api.cu -- the C ABI of librowop (declared in include/rowop.h):
+// synchronous argument validation, the per-device status word, and the hand
+// off to the per-operator launch paths (launch_by_rows, §2.1).
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+
+#include "classify.cuh"
+#include "common.cuh"
+#include "dispatch.h"
+#include "rowop.h"
+
+namespace rowop {
+
+extern template cudaError_t launch_dense<kSoftmax>(const DenseCall &, const DeviceInfo &);
+extern template cudaError_t launch_dense<kLogSoftmax>(const DenseCall &, const DeviceInfo &);
+extern template cudaError_t launch_dense<kLayerNorm>(const DenseCall &, const DeviceInfo &);
+extern template cudaError_t launch_dense<kRmsNorm>(const DenseCall &, const DeviceInfo &);
+extern template cudaError_t launch_ragged<kSoftmax>(const RaggedCall &, const DeviceInfo &);
+extern template cudaError_t launch_ragged<kLogSoftmax>(const RaggedCall &, const DeviceInfo &);
+extern template cudaError_t launch_ragged<kLayerNorm>(const RaggedCall &, const DeviceInfo &);
+extern template cudaError_t launch_ragged<kRmsNorm>(const RaggedCall &, const DeviceInfo &);
+
+// Device-side status bits (kStatusTimeout, kStatusBadOffsets), one word per
+// device; kernels receive its address.
+static __device__ unsigned int g_status_word;
+
+static int env_int(const char *name, int dflt) {
+  const char *v = std::getenv(name);
+  if (!v || !*v) return dflt;
+  return std::atoi(v);
+}
+
+Knobs read_knobs() {
+  Knobs k;
+  k.force_bucket = env_int("ROWOP_FORCE_BUCKET", -1);
+  k.cluster = env_int("ROWOP_CLUSTER", 0);
+  k.stages = env_int("ROWOP_STAGES", 0);
+  return k;
+}
+
+cudaError_t launch_classify(const RaggedCall &c, const DeviceInfo &d) {
+  unsigned char *ws = static_cast<unsigned char *>(c.ws);
+  int32_t *list0 = reinterpret_cast<int32_t *>(ws + ragged_lists_offset(c.rows));
+  ClassifyParams cp;
+  cp.offsets = c.offsets;
+  cp.rows = c.rows;
+  cp.max_len = c.max_len;
+  cp.esize = c.dtype == 0 ? 4 : 2;
+  cp.bucket = ws + kWsBuckets;
+  cp.list[0] = list0;
+  cp.list[1] = list0 + c.rows;
+  cp.list[2] = list0 + 2 * c.rows;
+  cp.counts = reinterpret_cast<int32_t *>(ws + kWsCounts);
+  cp.counters = reinterpret_cast<unsigned int *>(ws + kWsCounters);
+  cp.ws_status = reinterpret_cast<unsigned int *>(ws + kWsStatus);
+  cp.status = d.status;
+  ragged_classify_kernel<<<1, kClassifyThreads, 0, c.stream>>>(cp);
+  return cudaGetLastError();
+}
+
+static int device_info(DeviceInfo *out) {
+  static std::mutex mu;
+  static DeviceInfo cache[64];
+  static bool have[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    cudaGetLastError();
+    return ROWOP_ERR_CUDA;
+  }
+  std::lock_guard<std::mutex> lk(mu);
+  if (!have[dev]) {
+    DeviceInfo d;
+    d.device = dev;
+    void *status = nullptr;
+    if (cudaDeviceGetAttribute(&d.sm_count, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&d.max_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin,
+                               dev) != cudaSuccess ||
+        cudaGetSymbolAddress(&status, g_status_word) != cudaSuccess) {
+      cudaGetLastError();
+      return ROWOP_ERR_CUDA;
+    }
+    d.status = static_cast<unsigned int *>(status);
+    cache[dev] = d;
+    have[dev] = true;
+  }
+  *out = cache[dev];
+  return ROWOP_OK;
+}
+
+static int esize_of(int dtype) { return dtype == ROWOP_F32 ? 4 : (dtype == ROWOP_BF16 ? 2 : 0); }
+
+static bool elem_aligned(const void *p, int esize) {
+  return (reinterpret_cast<uintptr_t>(p) % static_cast<uintptr_t>(esize)) == 0;
+}
+
+static bool eps_ok(float eps) { return std::isfinite(eps) && eps >= 0.f; }
+
+static int from_cuda(cudaError_t e) {
+  if (e == cudaSuccess) return ROWOP_OK;
+  cudaGetLastError();
+  return ROWOP_ERR_CUDA;
+}
+
+// 0 = go on, 1 = valid no-op, else an error code (returned negated)
+static int check_dense(const void *in, const void *out, const void *gamma, const void *beta,
+                       int64_t rows, int64_t cols, int64_t ld, int dtype, float eps, bool norm) {
+  const int es = esize_of(dtype);
+  if (es == 0) return -ROWOP_ERR_UNSUPPORTED_DTYPE;
+  if (rows < 0) return -ROWOP_ERR_INVALID_ARG;
+  if (norm && !eps_ok(eps)) return -ROWOP_ERR_INVALID_ARG;
+  if (rows == 0) return 1;
+  if (cols <= 0 || ld < cols) return -ROWOP_ERR_INVALID_ARG;
+  if (!in || !out) return -ROWOP_ERR_INVALID_ARG;
+  if (!elem_aligned(in, es) || !elem_aligned(out, es)) return -ROWOP_ERR_INVALID_ARG;
+  if ((gamma && !elem_aligned(gamma, es)) || (beta && !elem_aligned(beta, es)))
+    return -ROWOP_ERR_INVALID_ARG;
+  if (ld > INT64_MAX / es / rows) return -ROWOP_ERR_INVALID_ARG;
+  if (cols > max_row_len_elems(es)) return -ROWOP_ERR_TOO_LONG;
+  return 0;
+}
+
+static int run_dense(int op, const void *in, void *out, const void *gamma, const void *beta,
+                     int64_t rows, int64_t cols, int64_t ld, rowop_dtype_t dtype, float eps,
+                     cudaStream_t stream) {
+  const bool norm = (op == kLayerNorm || op == kRmsNorm);
+  const int chk = check_dense(in, out, gamma, beta, rows, cols, ld, dtype, eps, norm);
+  if (chk < 0) return -chk;
+  if (chk == 1) return ROWOP_OK;
+  DeviceInfo d;
+  const int st = device_info(&d);
+  if (st != ROWOP_OK) return st;
+  DenseCall c;
+  c.dtype = dtype;
+  c.in = in;
+  c.out = out;
+  c.gamma = gamma;
+  c.beta = beta;
+  c.rows = rows;
+  c.cols = cols;
+  c.ld = ld;
+  c.eps = eps;
+  c.stream = stream;
+  switch (op) {
+    case kSoftmax: return from_cuda(launch_dense<kSoftmax>(c, d));
+    case kLogSoftmax: return from_cuda(launch_dense<kLogSoftmax>(c, d));
+    case kLayerNorm: return from_cuda(launch_dense<kLayerNorm>(c, d));
+    default: return from_cuda(launch_dense<kRmsNorm>(c, d));
+  }
+}
+
+// op < 0: only the classify pass (rowop_ragged_plan)
+static int run_ragged(int op, const void *in, void *out, const void *gamma, const void *beta,
+                      const int64_t *offsets, int64_t rows, int64_t max_len,
+                      rowop_dtype_t dtype, float eps, void *ws, size_t ws_bytes,
+                      cudaStream_t stream, bool classify) {
+  const int es = esize_of(dtype);
+  const bool norm = (op == kLayerNorm || op == kRmsNorm);
+  if (es == 0) return ROWOP_ERR_UNSUPPORTED_DTYPE;
+  if (rows < 0 || rows > INT32_MAX - 1 || max_len < 0) return ROWOP_ERR_INVALID_ARG;
+  if (norm && !eps_ok(eps)) return ROWOP_ERR_INVALID_ARG;
+  if (rows == 0) return ROWOP_OK;
+  if (!offsets || !elem_aligned(offsets, 8)) return ROWOP_ERR_INVALID_ARG;
+  if (op >= 0 && (!in || !out || !elem_aligned(in, es) || !elem_aligned(out, es)))
+    return ROWOP_ERR_INVALID_ARG;
+  if ((gamma && !elem_aligned(gamma, es)) || (beta && !elem_aligned(beta, es)))
+    return ROWOP_ERR_INVALID_ARG;
+  if (max_len > max_row_len_elems(es)) return ROWOP_ERR_TOO_LONG;
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 ||
+      ws_bytes < ragged_ws_bytes(rows))
+    return ROWOP_ERR_WORKSPACE;
+  DeviceInfo d;
+  const int st = device_info(&d);
+  if (st != ROWOP_OK) return st;
+  RaggedCall c;
+  c.dtype = dtype;
+  c.in = in;
+  c.out = out;
+  c.gamma = gamma;
+  c.beta = beta;
+  c.offsets = offsets;
+  c.rows = rows;
+  c.max_len = max_len;
+  c.eps = eps;
+  c.ws = ws;
+  c.stream = stream;
+  c.classify = classify;
+  if (op < 0) return from_cuda(launch_classify(c, d));
+  switch (op) {
+    case kSoftmax: return from_cuda(launch_ragged<kSoftmax>(c, d));
+    case kLogSoftmax: return from_cuda(launch_ragged<kLogSoftmax>(c, d));
+    case kLayerNorm: return from_cuda(launch_ragged<kLayerNorm>(c, d));
+    default: return from_cuda(launch_ragged<kRmsNorm>(c, d));
+  }
+}
+
+// Waits on a barrier phase that only half of its expected arrivals reach, so
+// the bounded wait must run out; records the timeout and returns.
+__global__ void debug_wait_timeout_kernel(uint64_t limit_ns, unsigned int *status) {
+  __shared__ __align__(8) uint64_t bar;
+  const uint32_t b = smem_addr(&bar);
+  if (threadIdx.x == 0) {
+    mbar_init(b, 2);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) mbar_arrive(b);
+  const bool ok = mbar_wait_bounded(b, 0, limit_ns);
+  if (!ok && threadIdx.x == 0) atomicOr(status, kStatusTimeout);
+  __syncthreads();
+  if (threadIdx.x == 0) asm volatile("mbarrier.inval.shared::cta.b64 [%0];" ::"r"(b) : "memory");
+}
+
+}  // namespace rowop
+
+using namespace rowop;
+
+extern "C" {
+
+int rowop_softmax(const void *in, void *out, int64_t rows, int64_t cols, int64_t ld,
+                  rowop_dtype_t dtype, cudaStream_t stream) {
+  return run_dense(kSoftmax, in, out, nullptr, nullptr, rows, cols, ld, dtype, 0.f, stream);
+}
+
+int rowop_logsoftmax(const void *in, void *out, int64_t rows, int64_t cols, int64_t ld,
+                     rowop_dtype_t dtype, cudaStream_t stream) {
+  return run_dense(kLogSoftmax, in, out, nullptr, nullptr, rows, cols, ld, dtype, 0.f, stream);
+}
+
+int rowop_layernorm(const void *in, void *out, const void *gamma, const void *beta,
+                    int64_t rows, int64_t cols, int64_t ld, rowop_dtype_t dtype, float eps,
+                    cudaStream_t stream) {
+  return run_dense(kLayerNorm, in, out, gamma, beta, rows, cols, ld, dtype, eps, stream);
+}
+
+int rowop_rmsnorm(const void *in, void *out, const void *gamma, int64_t rows, int64_t cols,
+                  int64_t ld, rowop_dtype_t dtype, float eps, cudaStream_t stream) {
+  return run_dense(kRmsNorm, in, out, gamma, nullptr, rows, cols, ld, dtype, eps, stream);
+}
+
+size_t rowop_ragged_workspace_size(int64_t rows) {
+  return rows <= 0 ? 256 : ragged_ws_bytes(rows);
+}
+
+int rowop_softmax_ragged(const void *in, void *out, const int64_t *offsets, int64_t rows,
+                         int64_t max_len, rowop_dtype_t dtype, void *ws, size_t ws_bytes,
+                         cudaStream_t stream) {
+  return run_ragged(kSoftmax, in, out, nullptr, nullptr, offsets, rows, max_len, dtype, 0.f, ws,
+                    ws_bytes, stream, true);
+}
+
+int rowop_logsoftmax_ragged(const void *in, void *out, const int64_t *offsets, int64_t rows,
+                            int64_t max_len, rowop_dtype_t dtype, void *ws, size_t ws_bytes,
+                            cudaStream_t stream) {
+  return run_ragged(kLogSoftmax, in, out, nullptr, nullptr, offsets, rows, max_len, dtype, 0.f,
+                    ws, ws_bytes, stream, true);
+}
+
+int rowop_layernorm_ragged(const void *in, void *out, const void *gamma, const void *beta,
+                           const int64_t *offsets, int64_t rows, int64_t max_len,
+                           rowop_dtype_t dtype, float eps, void *ws, size_t ws_bytes,
+                           cudaStream_t stream) {
+  return run_ragged(kLayerNorm, in, out, gamma, beta, offsets, rows, max_len, dtype, eps, ws,
+                    ws_bytes, stream, true);
+}
+
+int rowop_rmsnorm_ragged(const void *in, void *out, const void *gamma, const int64_t *offsets,
+                         int64_t rows, int64_t max_len, rowop_dtype_t dtype, float eps,
+                         void *ws, size_t ws_bytes, cudaStream_t stream) {
+  return run_ragged(kRmsNorm, in, out, gamma, nullptr, offsets, rows, max_len, dtype, eps, ws,
+                    ws_bytes, stream, true);
+}
+
+int rowop_ragged_plan(const int64_t *offsets, int64_t rows, int64_t max_len,
+                      rowop_dtype_t dtype, void *ws, size_t ws_bytes, cudaStream_t stream) {
+  return run_ragged(-1, nullptr, nullptr, nullptr, nullptr, offsets, rows, max_len, dtype, 0.f,
+                    ws, ws_bytes, stream, true);
+}
+
+int rowop_softmax_ragged_planned(const void *in, void *out, const int64_t *offsets,
+                                 int64_t rows, int64_t max_len, rowop_dtype_t dtype, void *ws,
+                                 size_t ws_bytes, cudaStream_t stream) {
+  return run_ragged(kSoftmax, in, out, nullptr, nullptr, offsets, rows, max_len, dtype, 0.f, ws,
+                    ws_bytes, stream, false);
+}
+
+int rowop_logsoftmax_ragged_planned(const void *in, void *out, const int64_t *offsets,
+                                    int64_t rows, int64_t max_len, rowop_dtype_t dtype,
+                                    void *ws, size_t ws_bytes, cudaStream_t stream) {
+  return run_ragged(kLogSoftmax, in, out, nullptr, nullptr, offsets, rows, max_len, dtype, 0.f,
+                    ws, ws_bytes, stream, false);
+}
+
+int rowop_layernorm_ragged_planned(const void *in, void *out, const void *gamma,
+                                   const void *beta, const int64_t *offsets, int64_t rows,
+                                   int64_t max_len, rowop_dtype_t dtype, float eps, void *ws,
+                                   size_t ws_bytes, cudaStream_t stream) {
+  return run_ragged(kLayerNorm, in, out, gamma, beta, offsets, rows, max_len, dtype, eps, ws,
+                    ws_bytes, stream, false);
+}
+
+int rowop_rmsnorm_ragged_planned(const void *in, void *out, const void *gamma,
+                                 const int64_t *offsets, int64_t rows, int64_t max_len,
+                                 rowop_dtype_t dtype, float eps, void *ws, size_t ws_bytes,
+                                 cudaStream_t stream) {
+  return run_ragged(kRmsNorm, in, out, gamma, nullptr, offsets, rows, max_len, dtype, eps, ws,
+                    ws_bytes, stream, false);
+}
+
+int rowop_select_bucket(int64_t len, rowop_dtype_t dtype) {
+  const int es = esize_of(dtype);
+  if (es == 0 || len < 0) return -1;
+  return bucket_of(len, es);
+}
+
+int64_t rowop_max_row_len(rowop_dtype_t dtype) {
+  const int es = esize_of(dtype);
+  return es == 0 ? 0 : max_row_len_elems(es);
+}
+
+const char *rowop_status_string(int status) {
+  switch (status) {
+    case ROWOP_OK: return "ROWOP_OK";
+    case ROWOP_ERR_INVALID_ARG: return "ROWOP_ERR_INVALID_ARG: invalid argument";
+    case ROWOP_ERR_UNSUPPORTED_DTYPE: return "ROWOP_ERR_UNSUPPORTED_DTYPE: unsupported dtype";
+    case ROWOP_ERR_WORKSPACE: return "ROWOP_ERR_WORKSPACE: workspace missing, misaligned or too small";
+    case ROWOP_ERR_CUDA: return "ROWOP_ERR_CUDA: a CUDA call or launch failed";
+    case ROWOP_ERR_TIMEOUT: return "ROWOP_ERR_TIMEOUT: a bounded device wait ran out";
+    case ROWOP_ERR_BAD_OFFSETS: return "ROWOP_ERR_BAD_OFFSETS: ragged rows rejected (decreasing offsets or len > max_len)";
+    case ROWOP_ERR_TOO_LONG: return "ROWOP_ERR_TOO_LONG: row longer than rowop_max_row_len()";
+    default: return "ROWOP: unknown status";
+  }
+}
+
+int rowop_check_status(cudaStream_t stream) {
+  DeviceInfo d;
+  const int st = device_info(&d);
+  if (st != ROWOP_OK) return st;
+  unsigned int word = 0;
+  if (cudaStreamSynchronize(stream) != cudaSuccess ||
+      cudaMemcpyAsync(&word, d.status, sizeof(word), cudaMemcpyDeviceToHost, stream) !=
+          cudaSuccess ||
+      cudaMemsetAsync(d.status, 0, sizeof(word), stream) != cudaSuccess ||
+      cudaStreamSynchronize(stream) != cudaSuccess) {
+    cudaGetLastError();
+    return ROWOP_ERR_CUDA;
+  }
+  if (word & kStatusTimeout) return ROWOP_ERR_TIMEOUT;
+  if (word & kStatusBadOffsets) return ROWOP_ERR_BAD_OFFSETS;
+  return ROWOP_OK;
+}
+
+int rowop_debug_wait_timeout(int64_t limit_ns, cudaStream_t stream) {
+  if (limit_ns < 1 || limit_ns > 1000000000LL) return ROWOP_ERR_INVALID_ARG;
+  DeviceInfo d;
+  const int st = device_info(&d);
+  if (st != ROWOP_OK) return st;
+  debug_wait_timeout_kernel<<<1, 32, 0, stream>>>(static_cast<uint64_t>(limit_ns), d.status);
+  return from_cuda(cudaGetLastError());
+}
+
+}  // extern "C"

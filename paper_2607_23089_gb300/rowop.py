@@ -1,0 +1,293 @@
+"""ctypes binding of librowop (``include/rowop.h``).
+
+Two layers, both argument marshalling only -- every step of the computation
+runs in the CUDA library:
+
+* ``rowop_*`` functions with the C names and C arguments (integers for
+  pointers and streams), returning the C status code;
+* tensor helpers (``softmax``, ``layernorm_ragged``, ...) that take CUDA torch
+  tensors, allocate outputs / workspace with torch, pass
+  ``data_ptr()`` and the current stream, and raise ``RowopError`` on a
+  non-OK status.
+
+There is no fallback: if the shared library has not been built the first
+call raises, and a tensor that is not on a CUDA device is rejected.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "_build", "librowop.so")
+
+ROWOP_F32, ROWOP_BF16 = 0, 1
+SMALL, MEDIUM, LARGE = 0, 1, 2
+STATUS = {
+    0: "ROWOP_OK", 1: "ROWOP_ERR_INVALID_ARG", 2: "ROWOP_ERR_UNSUPPORTED_DTYPE",
+    3: "ROWOP_ERR_WORKSPACE", 4: "ROWOP_ERR_CUDA", 5: "ROWOP_ERR_TIMEOUT",
+    6: "ROWOP_ERR_BAD_OFFSETS", 7: "ROWOP_ERR_TOO_LONG",
+}
+globals().update({v: k for k, v in STATUS.items()})
+
+_lock = threading.Lock()
+_lib = None
+
+_P = ctypes.c_void_p
+_I64 = ctypes.c_int64
+_I = ctypes.c_int
+_F = ctypes.c_float
+_SZ = ctypes.c_size_t
+
+# C signatures (argument types, return type), in header order.
+SIGNATURES = {
+    "rowop_softmax": ([_P, _P, _I64, _I64, _I64, _I, _P], _I),
+    "rowop_logsoftmax": ([_P, _P, _I64, _I64, _I64, _I, _P], _I),
+    "rowop_layernorm": ([_P, _P, _P, _P, _I64, _I64, _I64, _I, _F, _P], _I),
+    "rowop_rmsnorm": ([_P, _P, _P, _I64, _I64, _I64, _I, _F, _P], _I),
+    "rowop_ragged_workspace_size": ([_I64], _SZ),
+    "rowop_softmax_ragged": ([_P, _P, _P, _I64, _I64, _I, _P, _SZ, _P], _I),
+    "rowop_logsoftmax_ragged": ([_P, _P, _P, _I64, _I64, _I, _P, _SZ, _P], _I),
+    "rowop_layernorm_ragged": ([_P, _P, _P, _P, _P, _I64, _I64, _I, _F, _P, _SZ, _P], _I),
+    "rowop_rmsnorm_ragged": ([_P, _P, _P, _P, _I64, _I64, _I, _F, _P, _SZ, _P], _I),
+    "rowop_ragged_plan": ([_P, _I64, _I64, _I, _P, _SZ, _P], _I),
+    "rowop_softmax_ragged_planned": ([_P, _P, _P, _I64, _I64, _I, _P, _SZ, _P], _I),
+    "rowop_logsoftmax_ragged_planned": ([_P, _P, _P, _I64, _I64, _I, _P, _SZ, _P], _I),
+    "rowop_layernorm_ragged_planned": ([_P, _P, _P, _P, _P, _I64, _I64, _I, _F, _P, _SZ,
+                                        _P], _I),
+    "rowop_rmsnorm_ragged_planned": ([_P, _P, _P, _P, _I64, _I64, _I, _F, _P, _SZ, _P], _I),
+    "rowop_select_bucket": ([_I64, _I], _I),
+    "rowop_max_row_len": ([_I], _I64),
+    "rowop_status_string": ([_I], ctypes.c_char_p),
+    "rowop_check_status": ([_P], _I),
+    "rowop_debug_wait_timeout": ([_I64, _P], _I),
+}
+
+
+class RowopError(RuntimeError):
+    def __init__(self, status: int, what: str = ""):
+        self.status = status
+        super().__init__(f"{what}: {STATUS.get(status, status)}" if what else
+                         STATUS.get(status, str(status)))
+
+
+def load(path: str | None = None) -> ctypes.CDLL:
+    """Loads librowop.so (built by ``build.build()``); raises if it is missing."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        p = path or LIB_PATH
+        if not os.path.exists(p):
+            raise RuntimeError(
+                f"librowop is not built ({p} missing): run "
+                "paper_2607_23089_gb300.build.build() first")
+        lib = ctypes.CDLL(p)
+        for name, (argtypes, restype) in SIGNATURES.items():
+            fn = getattr(lib, name)
+            fn.argtypes = argtypes
+            fn.restype = restype
+        _lib = lib
+        return lib
+
+
+def _c(name):
+    def call(*args):
+        return getattr(load(), name)(*args)
+    call.__name__ = name
+    call.__doc__ = f"Direct call of the C function {name} (see include/rowop.h)."
+    return call
+
+
+for _name in SIGNATURES:
+    globals()[_name] = _c(_name)
+
+
+# ---------------------------------------------------------------------------
+# torch tensor helpers
+# ---------------------------------------------------------------------------
+def _torch():
+    import torch
+    return torch
+
+
+def dtype_code(dtype) -> int:
+    torch = _torch()
+    if dtype == torch.float32:
+        return ROWOP_F32
+    if dtype == torch.bfloat16:
+        return ROWOP_BF16
+    raise TypeError(f"librowop supports float32 and bfloat16, not {dtype}")
+
+
+def _stream(stream):
+    if stream is None:
+        return _torch().cuda.current_stream().cuda_stream
+    return getattr(stream, "cuda_stream", stream)
+
+
+def _ptr(t):
+    return None if t is None else t.data_ptr()
+
+
+def _check_cuda(*ts):
+    for t in ts:
+        if t is not None and not t.is_cuda:
+            raise ValueError("librowop operates on CUDA tensors only")
+
+
+def _ok(st, what):
+    if st != 0:
+        raise RowopError(st, what)
+
+
+def _dense_layout(x):
+    if x.dim() != 2:
+        raise ValueError("dense ops take a 2-D rows x cols tensor")
+    rows, cols = x.shape
+    if cols > 1 and x.stride(1) != 1:
+        raise ValueError("rows must be contiguous (stride(1) == 1)")
+    ld = x.stride(0) if rows > 1 else cols
+    return rows, cols, max(ld, cols)
+
+
+def _out_like(x, out):
+    if out is None:
+        out = _torch().empty_strided(x.shape, x.stride(), dtype=x.dtype, device=x.device)
+    elif out.shape != x.shape or out.stride() != x.stride() or out.dtype != x.dtype:
+        raise ValueError("out must match x in shape, strides and dtype")
+    return out
+
+
+def softmax(x, out=None, stream=None):
+    _check_cuda(x, out)
+    rows, cols, ld = _dense_layout(x)
+    out = _out_like(x, out)
+    _ok(rowop_softmax(x.data_ptr(), out.data_ptr(), rows, cols, ld,  # noqa: F821
+                      dtype_code(x.dtype), _stream(stream)), "rowop_softmax")
+    return out
+
+
+def logsoftmax(x, out=None, stream=None):
+    _check_cuda(x, out)
+    rows, cols, ld = _dense_layout(x)
+    out = _out_like(x, out)
+    _ok(rowop_logsoftmax(x.data_ptr(), out.data_ptr(), rows, cols, ld,  # noqa: F821
+                         dtype_code(x.dtype), _stream(stream)), "rowop_logsoftmax")
+    return out
+
+
+def layernorm(x, gamma=None, beta=None, eps=1e-5, out=None, stream=None):
+    _check_cuda(x, gamma, beta, out)
+    rows, cols, ld = _dense_layout(x)
+    out = _out_like(x, out)
+    _ok(rowop_layernorm(x.data_ptr(), out.data_ptr(), _ptr(gamma), _ptr(beta),  # noqa: F821
+                        rows, cols, ld, dtype_code(x.dtype), float(eps),
+                        _stream(stream)), "rowop_layernorm")
+    return out
+
+
+def rmsnorm(x, gamma=None, eps=1e-6, out=None, stream=None):
+    _check_cuda(x, gamma, out)
+    rows, cols, ld = _dense_layout(x)
+    out = _out_like(x, out)
+    _ok(rowop_rmsnorm(x.data_ptr(), out.data_ptr(), _ptr(gamma), rows, cols,  # noqa: F821
+                      ld, dtype_code(x.dtype), float(eps), _stream(stream)),
+        "rowop_rmsnorm")
+    return out
+
+
+def ragged_workspace(rows: int, device="cuda"):
+    """A workspace tensor for a ragged call over ``rows`` rows."""
+    n = rowop_ragged_workspace_size(int(rows))  # noqa: F821
+    return _torch().empty(int(n), dtype=_torch().uint8, device=device)
+
+
+def _ragged_args(x, offsets, ws, out):
+    _check_cuda(x, offsets, ws, out)
+    torch = _torch()
+    if offsets.dtype != torch.int64 or offsets.dim() != 1:
+        raise ValueError("offsets must be a 1-D int64 tensor")
+    rows = offsets.numel() - 1
+    if out is None:
+        out = torch.empty_like(x)
+    if ws is None:
+        ws = ragged_workspace(rows, x.device)
+    return rows, out, ws
+
+
+def softmax_ragged(x, offsets, max_len, out=None, ws=None, stream=None):
+    rows, out, ws = _ragged_args(x, offsets, ws, out)
+    _ok(rowop_softmax_ragged(x.data_ptr(), out.data_ptr(), offsets.data_ptr(),  # noqa: F821
+                             rows, int(max_len), dtype_code(x.dtype), ws.data_ptr(),
+                             ws.numel(), _stream(stream)), "rowop_softmax_ragged")
+    return out
+
+
+def logsoftmax_ragged(x, offsets, max_len, out=None, ws=None, stream=None):
+    rows, out, ws = _ragged_args(x, offsets, ws, out)
+    _ok(rowop_logsoftmax_ragged(x.data_ptr(), out.data_ptr(),  # noqa: F821
+                                offsets.data_ptr(), rows, int(max_len),
+                                dtype_code(x.dtype), ws.data_ptr(), ws.numel(),
+                                _stream(stream)), "rowop_logsoftmax_ragged")
+    return out
+
+
+def layernorm_ragged(x, offsets, max_len, gamma=None, beta=None, eps=1e-5,
+                     out=None, ws=None, stream=None):
+    _check_cuda(gamma, beta)
+    rows, out, ws = _ragged_args(x, offsets, ws, out)
+    _ok(rowop_layernorm_ragged(x.data_ptr(), out.data_ptr(), _ptr(gamma),  # noqa: F821
+                               _ptr(beta), offsets.data_ptr(), rows, int(max_len),
+                               dtype_code(x.dtype), float(eps), ws.data_ptr(),
+                               ws.numel(), _stream(stream)), "rowop_layernorm_ragged")
+    return out
+
+
+def rmsnorm_ragged(x, offsets, max_len, gamma=None, eps=1e-6, out=None, ws=None,
+                   stream=None):
+    _check_cuda(gamma)
+    rows, out, ws = _ragged_args(x, offsets, ws, out)
+    _ok(rowop_rmsnorm_ragged(x.data_ptr(), out.data_ptr(), _ptr(gamma),  # noqa: F821
+                             offsets.data_ptr(), rows, int(max_len),
+                             dtype_code(x.dtype), float(eps), ws.data_ptr(),
+                             ws.numel(), _stream(stream)), "rowop_rmsnorm_ragged")
+    return out
+
+
+def check_status(stream=None) -> int:
+    """Synchronises the stream and returns (and clears) the device status."""
+    return rowop_check_status(_stream(stream))  # noqa: F821
+
+
+def select_bucket(length: int, dtype) -> int:
+    code = dtype if isinstance(dtype, int) else dtype_code(dtype)
+    return rowop_select_bucket(int(length), code)  # noqa: F821
+
+
+def run(op: str, x, *, offsets=None, max_len=None, gamma=None, beta=None,
+        eps=None, out=None, ws=None, stream=None):
+    """One call of ``op`` on dense or ragged input (ragged when offsets is
+    given); returns the output tensor."""
+    if offsets is None:
+        if op == "softmax":
+            return softmax(x, out, stream)
+        if op == "logsoftmax":
+            return logsoftmax(x, out, stream)
+        if op == "layernorm":
+            return layernorm(x, gamma, beta, 1e-5 if eps is None else eps, out, stream)
+        if op == "rmsnorm":
+            return rmsnorm(x, gamma, 1e-6 if eps is None else eps, out, stream)
+    else:
+        if op == "softmax":
+            return softmax_ragged(x, offsets, max_len, out, ws, stream)
+        if op == "logsoftmax":
+            return logsoftmax_ragged(x, offsets, max_len, out, ws, stream)
+        if op == "layernorm":
+            return layernorm_ragged(x, offsets, max_len, gamma, beta,
+                                    1e-5 if eps is None else eps, out, ws, stream)
+        if op == "rmsnorm":
+            return rmsnorm_ragged(x, offsets, max_len, gamma,
+                                  1e-6 if eps is None else eps, out, ws, stream)
+    raise ValueError(f"unknown op {op}")

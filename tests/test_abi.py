@@ -1,0 +1,127 @@
+"""C-ABI checks that need no GPU: the library builds and loads, exports every
+function include/rowop.h declares, applies the row-length dispatch rule
+exactly as the oracle states it, and rejects bad arguments synchronously
+(before touching the device)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from oracle import rowop_oracle as orc
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "rowop.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2607_23089_gb300 import build, rowop
+    build.build()
+    return rowop
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return re.findall(r"ROWOP_API\s+[\w\s\*]+?\b(rowop_\w+)\s*\(", text)
+
+
+def test_header_declares_the_abi():
+    names = declared_functions()
+    for n in ("rowop_softmax", "rowop_logsoftmax", "rowop_layernorm", "rowop_rmsnorm",
+              "rowop_softmax_ragged", "rowop_logsoftmax_ragged", "rowop_layernorm_ragged",
+              "rowop_rmsnorm_ragged", "rowop_ragged_workspace_size",
+              "rowop_select_bucket", "rowop_status_string", "rowop_check_status"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    raw = ctypes.CDLL(lib.LIB_PATH)
+    names = declared_functions()
+    assert names
+    for n in names:
+        assert hasattr(raw, n), n
+        assert n in lib.SIGNATURES, n
+
+
+def test_select_bucket_matches_the_rule(lib):
+    for dtype, es in ((lib.ROWOP_F32, 4), (lib.ROWOP_BF16, 2)):
+        lens = set(range(0, 70)) | {1023, 1024, 1025, 2047, 2048, 2049, 8191, 8192,
+                                    8193, 16383, 16384, 16385, 262144, 1 << 22}
+        for n in sorted(lens):
+            assert lib.rowop_select_bucket(n, dtype) == orc.bucket(n, es), (n, es)
+    assert lib.rowop_select_bucket(-1, lib.ROWOP_F32) == -1
+    assert lib.rowop_select_bucket(10, 9) == -1
+
+
+def test_limits_and_strings(lib):
+    assert lib.rowop_max_row_len(lib.ROWOP_F32) >= 262144
+    assert lib.rowop_max_row_len(lib.ROWOP_BF16) >= 2 * 262144 - 8
+    assert lib.rowop_max_row_len(5) == 0
+    for code in range(8):
+        s = lib.rowop_status_string(code).decode()
+        assert s.startswith(lib.STATUS[code])
+    assert b"unknown" in lib.rowop_status_string(99)
+    assert lib.rowop_ragged_workspace_size(0) >= 256
+    n = 16384
+    ws = lib.rowop_ragged_workspace_size(n)
+    assert ws >= 256 + n + 3 * 4 * n
+
+
+FAKE = 1 << 20  # a non-NULL, 16-byte aligned address that is never touched
+
+
+def test_dense_validation(lib):
+    F32, BF16 = lib.ROWOP_F32, lib.ROWOP_BF16
+    sm = lib.rowop_softmax
+    assert sm(FAKE, FAKE, 4, 8, 8, 7, None) == lib.ROWOP_ERR_UNSUPPORTED_DTYPE
+    assert sm(FAKE, FAKE, -1, 8, 8, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert sm(None, None, 0, 8, 8, F32, None) == lib.ROWOP_OK  # empty batch: no-op
+    assert sm(FAKE, FAKE, 4, 0, 8, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert sm(FAKE, FAKE, 4, 8, 7, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert sm(None, FAKE, 4, 8, 8, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert sm(FAKE, None, 4, 8, 8, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert sm(FAKE + 2, FAKE, 4, 8, 8, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert sm(FAKE + 1, FAKE, 4, 8, 8, BF16, None) == lib.ROWOP_ERR_INVALID_ARG
+    too_long = lib.rowop_max_row_len(F32) + 1
+    assert sm(FAKE, FAKE, 1, too_long, too_long, F32, None) == lib.ROWOP_ERR_TOO_LONG
+    assert sm(FAKE, FAKE, 1 << 40, 1 << 30, 1 << 30, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    ln = lib.rowop_layernorm
+    assert ln(FAKE, FAKE, None, None, 4, 8, 8, F32, -1.0, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert ln(FAKE, FAKE, None, None, 4, 8, 8, F32, float("nan"), None) == lib.ROWOP_ERR_INVALID_ARG
+    assert ln(FAKE, FAKE, FAKE + 2, None, 4, 8, 8, F32, 1e-5, None) == lib.ROWOP_ERR_INVALID_ARG
+    rms = lib.rowop_rmsnorm
+    assert rms(FAKE, FAKE, None, 4, 8, 8, F32, float("inf"), None) == lib.ROWOP_ERR_INVALID_ARG
+    assert rms(FAKE, FAKE, None, 0, 8, 8, F32, 1e-6, None) == lib.ROWOP_OK
+
+
+def test_ragged_validation(lib):
+    F32 = lib.ROWOP_F32
+    ws_need = lib.rowop_ragged_workspace_size(10)
+    r = lib.rowop_softmax_ragged
+    assert r(FAKE, FAKE, FAKE, 10, 64, 3, FAKE, ws_need, None) == lib.ROWOP_ERR_UNSUPPORTED_DTYPE
+    assert r(FAKE, FAKE, FAKE, -1, 64, F32, FAKE, ws_need, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert r(FAKE, FAKE, FAKE, 0, 64, F32, None, 0, None) == lib.ROWOP_OK
+    assert r(FAKE, FAKE, FAKE, 10, -1, F32, FAKE, ws_need, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert r(FAKE, FAKE, None, 10, 64, F32, FAKE, ws_need, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert r(FAKE, FAKE, FAKE + 4, 10, 64, F32, FAKE, ws_need, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert r(FAKE, FAKE, FAKE, 10, 64, F32, None, ws_need, None) == lib.ROWOP_ERR_WORKSPACE
+    assert r(FAKE, FAKE, FAKE, 10, 64, F32, FAKE + 16, ws_need, None) == lib.ROWOP_ERR_WORKSPACE
+    assert r(FAKE, FAKE, FAKE, 10, 64, F32, FAKE, ws_need - 1, None) == lib.ROWOP_ERR_WORKSPACE
+    assert r(FAKE, FAKE, FAKE, 1 << 31, 64, F32, FAKE, 1 << 40, None) == lib.ROWOP_ERR_INVALID_ARG
+    too_long = lib.rowop_max_row_len(F32) + 1
+    assert r(FAKE, FAKE, FAKE, 10, too_long, F32, FAKE, ws_need, None) == lib.ROWOP_ERR_TOO_LONG
+    ln = lib.rowop_layernorm_ragged
+    assert ln(FAKE, FAKE, None, None, FAKE, 10, 64, F32, -0.5, FAKE, ws_need,
+              None) == lib.ROWOP_ERR_INVALID_ARG
+
+
+def test_debug_timeout_rejects_bad_limits(lib):
+    assert lib.rowop_debug_wait_timeout(0, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert lib.rowop_debug_wait_timeout(2 * 10**9, None) == lib.ROWOP_ERR_INVALID_ARG
+
+
+def test_binding_refuses_cpu_tensors(lib):
+    import torch
+    with pytest.raises(ValueError):
+        lib.softmax(torch.zeros(4, 8))

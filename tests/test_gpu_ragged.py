@@ -1,0 +1,206 @@
+"""GPU parity of the ragged (CSR-offset) entry points, through the C ABI.
+
+One call mixes rows of every bucket (empty, length 1, SMALL, MEDIUM and
+cluster-split LARGE rows).  Checks: values against the oracle; the bucket
+every row was dispatched to (read back from the workspace) equals the
+dispatch rule exactly; a ragged row equals, bit for bit, a dense call on the
+same row at the same 16-byte alignment; rejected rows (decreasing offsets,
+len > max_len) are left untouched and flagged; in-place calls.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import rowop_oracle as orc
+from tests.gpu_util import (ALL_OPS, DTYPES, ESIZE, assert_close, canary_tensor,
+                            eps_for, gen_affine, is_canary, oracle_ragged, to_f64)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def rw():
+    from paper_2607_23089_gb300 import build, rowop
+    build.build()
+    rowop.load()
+    torch.cuda.set_device(0)
+    return rowop
+
+
+def mixed_lengths(dtype, rows, seed, max_len):
+    """Lengths spread over all buckets, with empty and length-1 rows."""
+    es = ESIZE[dtype]
+    g = np.random.default_rng(seed)
+    small = 4096 // es
+    med = 32768 // es
+    pools = [(0, 2), (1, 64), (65, small), (small + 1, med), (med + 1, max_len)]
+    lens = []
+    for i in range(rows):
+        lo, hi = pools[i % len(pools)]
+        hi = max(lo, min(hi, max_len))
+        lens.append(int(g.integers(lo, hi + 1)))
+    lens = np.array(lens, dtype=np.int64)
+    g.shuffle(lens)
+    return lens
+
+
+def call_ragged(rw, op, x, y, off, rows, max_len, g, b, dtype, eps, ws):
+    code = rw.dtype_code(dtype)
+    s = torch.cuda.current_stream().cuda_stream
+    gp = None if g is None else g.data_ptr()
+    bp = None if b is None else b.data_ptr()
+    if op == "softmax":
+        return rw.rowop_softmax_ragged(x, y, off, rows, max_len, code, ws.data_ptr(),
+                                       ws.numel(), s)
+    if op == "logsoftmax":
+        return rw.rowop_logsoftmax_ragged(x, y, off, rows, max_len, code, ws.data_ptr(),
+                                          ws.numel(), s)
+    if op == "layernorm":
+        return rw.rowop_layernorm_ragged(x, y, gp, bp, off, rows, max_len, code, eps,
+                                         ws.data_ptr(), ws.numel(), s)
+    return rw.rowop_rmsnorm_ragged(x, y, gp, off, rows, max_len, code, eps,
+                                   ws.data_ptr(), ws.numel(), s)
+
+
+def run_ragged(rw, op, dtype, lens, max_len, seed, base_off=0, inplace=False,
+               offsets=None):
+    off = offsets if offsets is not None else \
+        np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    total = max(int(off.max()), 1)
+    rows = off.shape[0] - 1
+    gx = torch.Generator("cpu").manual_seed(seed)
+    x = (3.0 * torch.randn(total, generator=gx)).to(dtype)
+    gam, bet = gen_affine(max(max_len, 1), dtype, seed)
+    G = 256
+    xbuf = canary_tensor(G + base_off + total + G, dtype)
+    xbuf[G + base_off:G + base_off + total] = x.cuda()
+    ybuf = xbuf if inplace else canary_tensor(G + base_off + total + G, dtype)
+    es = ESIZE[dtype]
+    xp = xbuf.data_ptr() + (G + base_off) * es
+    yp = ybuf.data_ptr() + (G + base_off) * es
+    offd = torch.from_numpy(off).cuda()
+    ws = rw.ragged_workspace(rows)
+    gd = gam.cuda() if op in ("layernorm", "rmsnorm") else None
+    bd = bet.cuda() if op == "layernorm" else None
+    eps = eps_for(op)
+    st = call_ragged(rw, op, xp, yp, offd.data_ptr(), rows, max_len, gd, bd, dtype, eps, ws)
+    assert st == 0, rw.STATUS.get(st, st)
+    torch.cuda.synchronize()
+    y = ybuf[G + base_off:G + base_off + total]
+    return dict(x=x, y=y, ybuf=ybuf, off=off, ws=ws, gam=gam, bet=bet, eps=eps,
+                G=G, base_off=base_off, total=total)
+
+
+@pytest.mark.parametrize("dtype", DTYPES, ids=["f32", "bf16"])
+@pytest.mark.parametrize("op", ALL_OPS)
+@pytest.mark.parametrize("base_off", [0, 3])
+def test_ragged_parity(rw, op, dtype, base_off):
+    max_len = 70000 if dtype == torch.float32 else 40000
+    lens = mixed_lengths(dtype, 160, seed=5 + base_off, max_len=max_len)
+    r = run_ragged(rw, op, dtype, lens, max_len, seed=17 + base_off, base_off=base_off)
+    assert rw.check_status() == 0
+    ref = oracle_ragged(op, r["x"].double().numpy(), r["off"],
+                        r["gam"].double().numpy(), r["bet"].double().numpy(), r["eps"])
+    assert_close(to_f64(r["y"]), ref, dtype, f"ragged {op} {dtype}")
+    G, b = r["G"], r["base_off"]
+    assert is_canary(r["ybuf"][:G + b]).all()
+    assert is_canary(r["ybuf"][G + b + r["total"]:]).all()
+    # dispatch: the bucket byte of every row equals the rule, bit for bit
+    rows = len(lens)
+    buckets = r["ws"][256:256 + rows].cpu().numpy()
+    want = np.array([orc.bucket(int(n), ESIZE[dtype]) for n in lens], dtype=np.uint8)
+    assert (buckets == want).all()
+    assert r["ws"][:4].view(torch.int32).item() == 0
+
+
+@pytest.mark.parametrize("dtype", DTYPES, ids=["f32", "bf16"])
+@pytest.mark.parametrize("op", ALL_OPS)
+def test_ragged_row_equals_dense_row(rw, op, dtype):
+    """A ragged row and a dense call on the same row at the same 16-byte
+    alignment give identical bits."""
+    max_len = 50000 if dtype == torch.float32 else 30000
+    lens = mixed_lengths(dtype, 40, seed=9, max_len=max_len)
+    r = run_ragged(rw, op, dtype, lens, max_len, seed=23, base_off=1)
+    es = ESIZE[dtype]
+    code = rw.dtype_code(dtype)
+    s = torch.cuda.current_stream().cuda_stream
+    gd = r["gam"].cuda()
+    bd = r["bet"].cuda()
+    for i in range(len(lens)):
+        n = int(lens[i])
+        if n == 0:
+            continue
+        start = int(r["off"][i]) + r["base_off"]  # element index in the guarded buffer
+        h = (start * es) % 16 // es
+        buf = canary_tensor(64 + h + n + 64, dtype)
+        buf[64 + h:64 + h + n] = r["x"][r["off"][i]:r["off"][i] + n].cuda()
+        out = canary_tensor(64 + h + n + 64, dtype)
+        xp = buf.data_ptr() + (64 + h) * es
+        yp = out.data_ptr() + (64 + h) * es
+        if op == "softmax":
+            st = rw.rowop_softmax(xp, yp, 1, n, n, code, s)
+        elif op == "logsoftmax":
+            st = rw.rowop_logsoftmax(xp, yp, 1, n, n, code, s)
+        elif op == "layernorm":
+            st = rw.rowop_layernorm(xp, yp, gd.data_ptr(), bd.data_ptr(), 1, n, n, code,
+                                    r["eps"], s)
+        else:
+            st = rw.rowop_rmsnorm(xp, yp, gd.data_ptr(), 1, n, n, code, r["eps"], s)
+        assert st == 0
+        dense = out[64 + h:64 + h + n]
+        rag = r["y"][r["off"][i]:r["off"][i] + n]
+        bits = (lambda t: t.view(torch.int32)) if dtype == torch.float32 else \
+            (lambda t: t.view(torch.int16))
+        assert torch.equal(bits(dense), bits(rag)), f"row {i} len {n}"
+
+
+@pytest.mark.parametrize("op", ALL_OPS)
+def test_ragged_inplace(rw, op):
+    dtype = torch.bfloat16
+    lens = mixed_lengths(dtype, 50, seed=31, max_len=30000)
+    x0 = None
+    r = run_ragged(rw, op, dtype, lens, 30000, seed=41, base_off=5, inplace=True)
+    ref = oracle_ragged(op, r["x"].double().numpy(), r["off"], r["gam"].double().numpy(),
+                        r["bet"].double().numpy(), r["eps"])
+    assert_close(to_f64(r["y"]), ref, dtype, f"ragged in-place {op}")
+    del x0
+
+
+def test_ragged_rejects_bad_rows(rw):
+    dtype = torch.float32
+    # row 0 runs backwards (negative length), row 6 is longer than max_len;
+    # the legal rows in between do not overlap anything.
+    off = np.array([50, 10, 60, 360, 9360, 9380, 9480, 9480 + 9500], dtype=np.int64)
+    max_len = 9100
+    r = run_ragged(rw, "softmax", dtype, None, max_len, seed=3, offsets=off)
+    st = rw.check_status()
+    assert st == rw.ROWOP_ERR_BAD_OFFSETS
+    assert rw.check_status() == 0  # the status word was cleared
+    rows = off.shape[0] - 1
+    buckets = r["ws"][256:256 + rows].cpu().numpy()
+    lens_eff = np.diff(off)
+    for i in range(rows):
+        n = int(lens_eff[i])
+        seg = r["y"][int(off[i]):int(off[i]) + max(n, 0)]
+        if n < 0 or n > max_len:
+            assert buckets[i] == 255
+            if n > 0:
+                assert is_canary(seg).all()
+        else:
+            assert buckets[i] == orc.bucket(n, 4)
+            ref = orc.softmax(r["x"][int(off[i]):int(off[i]) + n].double().numpy()[None])[0]
+            assert_close(to_f64(seg), ref, dtype, f"row {i}")
+    assert r["ws"][:4].view(torch.int32).item() == 2
+
+
+def test_ragged_all_empty_and_tiny(rw):
+    for lens in ([0, 0, 0], [1], [1, 0, 1, 2]):
+        lens = np.array(lens, dtype=np.int64)
+        r = run_ragged(rw, "logsoftmax", torch.float32, lens, 4, seed=1)
+        assert rw.check_status() == 0
+        covered = int(r["off"][-1])
+        if covered == 0:
+            assert is_canary(r["y"]).all()  # nothing to write
+            continue
+        ref = oracle_ragged("logsoftmax", r["x"][:covered].double().numpy(), r["off"])
+        assert_close(to_f64(r["y"][:covered]), ref, torch.float32, "tiny")
