@@ -428,8 +428,44 @@ def run_rowop(args, rank, world, local):
     return 0
 
 
+def run_only(args, local):
+    """One workload (by case name), `warmup` + `steps` calls, nothing else:
+    the small, fixed command that profiler captures run."""
+    import torch
+    from paper_2607_23089_gb300 import build as bld
+    from paper_2607_23089_gb300 import rowop as rw
+    from paper_2607_23089_gb300 import workloads as wl
+    bld.build()
+    rw.load()
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    try:
+        case = wl.by_name(args.only)
+    except (KeyError, ValueError):
+        raise SystemExit(f"unknown workload {args.only}")
+    x = case.x.to(device)
+    y = torch.empty_like(x)
+    g = case.gamma.to(device) if case.gamma is not None else None
+    b = case.beta.to(device) if case.beta is not None else None
+    kw = dict(gamma=g, beta=b, eps=case.eps, out=y)
+    if case.ragged:
+        kw.update(offsets=case.offsets.to(device), max_len=case.max_len,
+                  ws=rw.ragged_workspace(case.rows, device))
+    ts = time_calls(torch, lambda: rw.run(case.op, x, **kw), args.steps, args.warmup)
+    st = rw.check_status()
+    if st != 0:
+        raise RuntimeError(rw.STATUS.get(st, st))
+    ms = statistics.median(ts)
+    print(json.dumps({"workload": case.name, "ms_median": round(ms, 5),
+                      "gbs": round(case.algorithmic_bytes() / (ms * 1e-3) / 1e9, 1)}))
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--only", default=None,
+                    help="run one workload by case name (e.g. medium_norm_rmsnorm, "
+                         "long_rows_logsoftmax, ragged_layernorm) and nothing else")
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
@@ -441,6 +477,8 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
+    if args.only:
+        return run_only(args, int(os.environ.get("LOCAL_RANK", "0")))
     rank, world, local = dist_setup(args)
     try:
         if args.impl == "reference":

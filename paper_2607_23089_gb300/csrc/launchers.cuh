@@ -53,7 +53,7 @@ inline int cached_occupancy(const void *kernel, size_t smem, int cluster,
 }
 
 // Kernel attributes are raised once per kernel and device.
-inline cudaError_t prepare_kernel(const void *kernel, const DeviceInfo &d, bool big_cluster) {
+inline cudaError_t prepare_kernel(const void *kernel, const DeviceInfo &d, bool cluster) {
   static std::mutex mu;
   static std::map<std::pair<const void *, int>, bool> done;
   std::lock_guard<std::mutex> lk(mu);
@@ -62,7 +62,7 @@ inline cudaError_t prepare_kernel(const void *kernel, const DeviceInfo &d, bool 
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        d.max_smem_optin);
   if (e != cudaSuccess) return e;
-  if (big_cluster) {
+  if (cluster) {  // clusters of up to 16 CTAs
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
   }
@@ -134,7 +134,7 @@ cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int
   const TileSmemLayout L(p.stage_bytes, stages, stage_tiles);
   const size_t smem = L.total;
   if (smem > static_cast<size_t>(d.max_smem_optin)) return cudaErrorInvalidConfiguration;
-  cudaError_t e = prepare_kernel(kp, d, CLUSTER && cs > 8);
+  cudaError_t e = prepare_kernel(kp, d, CLUSTER);
   if (e != cudaSuccess) return e;
 
   cudaLaunchConfig_t cfg = {};

@@ -163,3 +163,19 @@ def all_cases(scale_down: int = 1):
     out.append(long_rows(rows=max(1, 256 // s)))
     out.append(ragged_ln(rows=max(1, 16384 // s)))
     return out
+
+
+def by_name(name: str) -> Case:
+    """Builds one workload case from its name (as in all_cases())."""
+    if name == "softmax_1k":
+        return softmax_1k()
+    if name.startswith("short_rows_"):
+        _, _, op, cols = name.split("_")
+        return short_rows(int(cols), op)
+    if name.startswith("medium_norm_"):
+        return medium_norm(name[len("medium_norm_"):])
+    if name.startswith("long_rows_"):
+        return long_rows(op=name[len("long_rows_"):])
+    if name.startswith("ragged_"):
+        return ragged_ln(op=name[len("ragged_"):])
+    raise KeyError(name)
