@@ -1,9 +1,9 @@
 // classify.cuh -- device-side launch_by_rows for ragged rows (§2.1): reads the
-// int64 CSR offsets, gives every row its bucket, and writes the row indices of
-// each bucket, in increasing row order, to three lists by a block-wide prefix
-// scan.  It also resets the work counters the fused kernel pulls MEDIUM and
-// SMALL rows from.  No host round trip: the fused kernel that follows on the
-// same stream reads the counts from device memory.
+// int64 CSR offsets, gives every row its bucket, and appends each non-empty
+// row's (start, length) record, in increasing row order, to its bucket's list
+// by a block-wide prefix scan.  It also resets the work counters the fused
+// kernel pulls MEDIUM and SMALL rows from.  No host round trip: the fused
+// kernel that follows on the same stream reads the counts from device memory.
 #pragma once
 
 #include "common.cuh"
@@ -19,15 +19,16 @@ struct ClassifyParams {
   int64_t rows;
   int64_t max_len;
   int esize;
-  uint8_t *bucket;        // [rows]
-  int32_t *list[3];       // [rows] each: SMALL, MEDIUM, LARGE
-  int32_t *counts;        // [3]
-  unsigned int *counters; // [3]
+  uint8_t *bucket;          // [rows]
+  RowRec *list[3];       // [rows] each: SMALL, MEDIUM, LARGE
+  int32_t *counts;          // [3]
+  unsigned int *counters;   // [3]
   unsigned int *ws_status;
-  unsigned int *status;   // device status word
+  unsigned int *status;     // device status word
 };
 
-static __global__ void __launch_bounds__(kClassifyThreads) ragged_classify_kernel(const ClassifyParams p) {
+static __global__ void __launch_bounds__(kClassifyThreads)
+    ragged_classify_kernel(const ClassifyParams p) {
   __shared__ int warp_tot[kClassifyThreads / 32][3];
   __shared__ int base[3];
   const int tid = threadIdx.x;
@@ -36,23 +37,28 @@ static __global__ void __launch_bounds__(kClassifyThreads) ragged_classify_kerne
   if (tid < 3) base[tid] = 0;
   __syncthreads();
   int any_bad = 0;
-  for (int64_t blk = 0; blk < p.rows; blk += static_cast<int64_t>(kClassifyThreads) * kClassifyPerThread) {
+  for (int64_t blk = 0; blk < p.rows;
+       blk += static_cast<int64_t>(kClassifyThreads) * kClassifyPerThread) {
     int b[kClassifyPerThread];
+    int64_t st[kClassifyPerThread], ln[kClassifyPerThread];
     int cnt[3] = {0, 0, 0};
     const int64_t r0 = blk + static_cast<int64_t>(tid) * kClassifyPerThread;
 #pragma unroll
     for (int i = 0; i < kClassifyPerThread; ++i) {
       const int64_t r = r0 + i;
       b[i] = -1;  // not listed
+      st[i] = 0;
+      ln[i] = 0;
       if (r < p.rows) {
-        const int64_t len = p.offsets[r + 1] - p.offsets[r];
-        if (len < 0 || len > p.max_len) {
+        st[i] = p.offsets[r];
+        ln[i] = p.offsets[r + 1] - st[i];
+        if (ln[i] < 0 || ln[i] > p.max_len) {
           p.bucket[r] = kBucketRejected;
           any_bad = 1;
         } else {
-          const int k = bucket_of(len, p.esize);
+          const int k = bucket_of(ln[i], p.esize);
           p.bucket[r] = static_cast<uint8_t>(k);
-          if (len > 0) {
+          if (ln[i] > 0) {
             b[i] = k;
             ++cnt[k];
           }
@@ -94,7 +100,12 @@ static __global__ void __launch_bounds__(kClassifyThreads) ragged_classify_kerne
     for (int k = 0; k < 3; ++k) pos[k] = base[k] + warp_tot[warp][k] + inc[k] - cnt[k];
 #pragma unroll
     for (int i = 0; i < kClassifyPerThread; ++i) {
-      if (b[i] >= 0) p.list[b[i]][pos[b[i]]++] = static_cast<int32_t>(r0 + i);
+      if (b[i] >= 0) {
+        RowRec rec;
+        rec.start = st[i];
+        rec.n = ln[i];
+        p.list[b[i]][pos[b[i]]++] = rec;
+      }
     }
     __syncthreads();
     if (tid == kClassifyThreads - 1) {

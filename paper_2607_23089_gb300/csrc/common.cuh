@@ -48,6 +48,12 @@ __host__ __device__ __forceinline__ int bucket_of(int64_t len, int esize) {
   return bytes <= kSmallMaxBytes ? kSmall : (bytes <= kMediumMaxBytes ? kMedium : kLarge);
 }
 
+// One ragged row as the classify pass lists it.
+struct RowRec {
+  int64_t start;  // first element of the row in the packed buffer
+  int64_t n;      // its length
+};
+
 template <typename T>
 struct Elem;
 template <>
@@ -159,30 +165,103 @@ __device__ __forceinline__ uint4 shift_chunk<__nv_bfloat16>(const uint4 &A, cons
   }
 }
 
-// gamma/beta values for window chunk c of a row with head offset h: element e
-// of the chunk is column j = c*E + e - h.  `vec` says the parameter vector is
-// 16-byte aligned; columns outside [0, glen) read as `fill`.
-template <typename T>
-__device__ __forceinline__ void load_param_chunk(const T *__restrict__ g, int64_t glen,
-                                                 int64_t c, int h, bool vec, float fill,
-                                                 float (&out)[Elem<T>::kPerChunk]) {
-  constexpr int E = Elem<T>::kPerChunk;
-  const int64_t j0 = c * E - h;
-  if (vec && j0 >= 0 && j0 + E <= glen && h == 0) {
-    unpack(__ldg(reinterpret_cast<const uint4 *>(g + j0)), out);
-    return;
-  }
-  if (vec && h > 0 && c >= 1 && (c + 1) * E <= glen) {
-    const uint4 A = __ldg(reinterpret_cast<const uint4 *>(g + (c - 1) * E));
-    const uint4 B = __ldg(reinterpret_cast<const uint4 *>(g + c * E));
-    unpack(shift_chunk<T>(A, B, h), out);
-    return;
-  }
-#pragma unroll
-  for (int e = 0; e < E; ++e) {
-    const int64_t j = j0 + e;
-    out[e] = (j >= 0 && j < glen) ? load_elem(g + j) : fill;
-  }
+// ---------------------------------------------------------------------------
+// Packed fp32 pairs (Blackwell f32x2 arithmetic): a pair holds the even
+// element of a chunk in its low half and the odd element in its high half.
+// Every sum over a chunk run accumulates even and odd elements separately and
+// adds the two halves at the end, in that fixed order.
+// ---------------------------------------------------------------------------
+typedef unsigned long long f2;
+
+__device__ __forceinline__ f2 f2_make(float lo, float hi) {
+  f2 r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ float f2_lo(f2 v) {
+  float lo, hi;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+  return lo;
+}
+__device__ __forceinline__ float f2_hi(f2 v) {
+  float lo, hi;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+  return hi;
+}
+__device__ __forceinline__ float f2_total(f2 v) { return __fadd_rn(f2_lo(v), f2_hi(v)); }
+__device__ __forceinline__ f2 f2_add(f2 a, f2 b) {
+  f2 d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ f2 f2_sub(f2 a, f2 b) {
+  f2 d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ f2 f2_mul(f2 a, f2 b) {
+  f2 d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ f2 f2_fma(f2 a, f2 b, f2 c) {
+  f2 d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ f2 f2_bcast(float v) { return f2_make(v, v); }
+// Keeps the halves whose mask bit is set, the other halves become `fill`.
+__device__ __forceinline__ f2 f2_select(f2 v, bool keep_lo, bool keep_hi, float fill) {
+  return f2_make(keep_lo ? f2_lo(v) : fill, keep_hi ? f2_hi(v) : fill);
+}
+
+// 16-byte chunk <-> pairs.  fp32: 2 pairs, bf16: 4 pairs.
+__device__ __forceinline__ void chunk_to_pairs(const uint4 &v, f2 (&p)[2]) {
+  p[0] = (static_cast<f2>(v.y) << 32) | v.x;
+  p[1] = (static_cast<f2>(v.w) << 32) | v.z;
+}
+__device__ __forceinline__ f2 bf16x2_to_pair(uint32_t w) {
+  return f2_make(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
+}
+__device__ __forceinline__ void chunk_to_pairs(const uint4 &v, f2 (&p)[4]) {
+  p[0] = bf16x2_to_pair(v.x);
+  p[1] = bf16x2_to_pair(v.y);
+  p[2] = bf16x2_to_pair(v.z);
+  p[3] = bf16x2_to_pair(v.w);
+}
+__device__ __forceinline__ uint4 pairs_to_chunk(const f2 (&p)[2]) {
+  return make_uint4(static_cast<uint32_t>(p[0]), static_cast<uint32_t>(p[0] >> 32),
+                    static_cast<uint32_t>(p[1]), static_cast<uint32_t>(p[1] >> 32));
+}
+__device__ __forceinline__ uint32_t pair_to_bf16x2(f2 v) {
+  uint32_t r;  // cvt packs its first source into the upper half
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(f2_hi(v)), "f"(f2_lo(v)));
+  return r;
+}
+__device__ __forceinline__ uint4 pairs_to_chunk(const f2 (&p)[4]) {
+  return make_uint4(pair_to_bf16x2(p[0]), pair_to_bf16x2(p[1]), pair_to_bf16x2(p[2]),
+                    pair_to_bf16x2(p[3]));
+}
+// element e of a chunk's pair array
+template <int NP>
+__device__ __forceinline__ float pair_elem(const f2 (&p)[NP], int e) {
+  return (e & 1) ? f2_hi(p[e >> 1]) : f2_lo(p[e >> 1]);
+}
+
+// e^v as 2^(v * log2 e) on the MUFU unit; v is a difference x - m <= 0 here.
+constexpr float kLog2e = 1.4426950408889634f;
+__device__ __forceinline__ float ex2_approx(float v) {
+  float r;
+  asm("ex2.approx.f32 %0, %1;" : "=f"(r) : "f"(v));
+  return r;
+}
+// exp(x - m) for both halves of a pair
+__device__ __forceinline__ f2 f2_exp_shifted(f2 x, f2 m) {
+  const f2 u = f2_mul(f2_sub(x, m), f2_bcast(kLog2e));
+  return f2_make(ex2_approx(f2_lo(u)), ex2_approx(f2_hi(u)));
+}
+__device__ __forceinline__ float exp_shifted(float x, float m) {
+  return ex2_approx(__fmul_rn(__fsub_rn(x, m), kLog2e));
 }
 
 // ---------------------------------------------------------------------------
@@ -339,6 +418,59 @@ __device__ __forceinline__ float4 ld_dsmem_f4(uint32_t addr) {
                : "r"(addr)
                : "memory");
   return v;
+}
+
+// Named barrier over `nthreads` threads (a multiple of 32) of the CTA.
+__device__ __forceinline__ void named_sync(uint32_t id, uint32_t nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+// Named barrier that also ORs a predicate over the participating threads.
+__device__ __forceinline__ bool named_sync_or(uint32_t id, uint32_t nthreads, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.or.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(pred)), "r"(id), "r"(nthreads)
+      : "memory");
+  return r != 0;
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+// Arrive, with release at cluster scope, on the barrier at the same shared
+// memory offset in the CTA of the given cluster rank.
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t local_bar, uint32_t rank) {
+  const uint32_t remote = map_to_rank(local_bar, rank);
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait with acquire at cluster scope (for barriers peers arrive on).
+__device__ __forceinline__ bool mbar_wait_cluster_bounded(uint32_t bar, uint32_t parity,
+                                                          uint64_t limit_ns) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  for (;;) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    if (global_timer_ns() - t0 > limit_ns) return false;
+  }
+}
+__device__ __forceinline__ void fence_cluster() {
+  asm volatile("fence.acq_rel.cluster;" ::: "memory");
 }
 
 // Streaming 16-byte global load / store (evict-first in L1/L2).

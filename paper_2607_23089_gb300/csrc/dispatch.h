@@ -42,17 +42,19 @@ struct RaggedCall {
 
 // Ragged workspace layout (bytes): [0,4) status bits of the call, [64,76)
 // int32 counts per bucket, [128,140) uint32 work counters, [256, 256+rows)
-// uint8 bucket per row, then three int32 row lists of `rows` entries each
-// starting at ragged_lists_offset(rows).
+// uint8 bucket per row, then three lists (SMALL, MEDIUM, LARGE) of `rows`
+// records {int64 start, int64 length} each, starting at
+// ragged_lists_offset(rows).
 constexpr size_t kWsStatus = 0;
 constexpr size_t kWsCounts = 64;
 constexpr size_t kWsCounters = 128;
 constexpr size_t kWsBuckets = 256;
+constexpr size_t kWsRecordBytes = 16;
 inline size_t ragged_lists_offset(int64_t rows) {
   return (kWsBuckets + static_cast<size_t>(rows) + 255) & ~static_cast<size_t>(255);
 }
 inline size_t ragged_ws_bytes(int64_t rows) {
-  return ragged_lists_offset(rows) + 3 * 4 * static_cast<size_t>(rows) + 256;
+  return ragged_lists_offset(rows) + 3 * kWsRecordBytes * static_cast<size_t>(rows) + 256;
 }
 
 // Tile budget of one CTA portion: the longest row the resident split-row

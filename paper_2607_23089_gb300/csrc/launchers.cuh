@@ -23,14 +23,14 @@ inline bool congruent16(const void *a, const void *b) {
 }
 inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
-// Occupancy answers are cached per (kernel, shared memory, cluster size).
-inline int cached_occupancy(const void *kernel, size_t smem, int cluster,
+// Occupancy answers are cached per (kernel, block, shared memory, cluster size, device).
+inline int cached_occupancy(const void *kernel, int threads, size_t smem, int cluster,
                             const cudaLaunchConfig_t *cfg) {
   static std::mutex mu;
-  static std::map<std::tuple<const void *, size_t, int, int>, int> cache;
+  static std::map<std::tuple<const void *, int, size_t, int, int>, int> cache;
   int dev = 0;
   cudaGetDevice(&dev);
-  const auto key = std::make_tuple(kernel, smem, cluster, dev);
+  const auto key = std::make_tuple(kernel, threads, smem, cluster, dev);
   {
     std::lock_guard<std::mutex> lk(mu);
     auto it = cache.find(key);
@@ -41,7 +41,7 @@ inline int cached_occupancy(const void *kernel, size_t smem, int cluster,
   if (cluster > 1) {
     e = cudaOccupancyMaxActiveClusters(&n, kernel, cfg);
   } else {
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel, kCtaThreads, smem);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel, threads, smem);
   }
   if (e != cudaSuccess) {
     cudaGetLastError();
@@ -52,7 +52,9 @@ inline int cached_occupancy(const void *kernel, size_t smem, int cluster,
   return n;
 }
 
-// Kernel attributes are raised once per kernel and device.
+// Kernel attributes are raised once per kernel and device: the full opt-in
+// shared memory, the shared-memory carveout, and (cluster kernels) clusters
+// of up to 16 CTAs.
 inline cudaError_t prepare_kernel(const void *kernel, const DeviceInfo &d, bool cluster) {
   static std::mutex mu;
   static std::map<std::pair<const void *, int>, bool> done;
@@ -62,7 +64,10 @@ inline cudaError_t prepare_kernel(const void *kernel, const DeviceInfo &d, bool 
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        d.max_smem_optin);
   if (e != cudaSuccess) return e;
-  if (cluster) {  // clusters of up to 16 CTAs
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared);
+  if (e != cudaSuccess) return e;
+  if (cluster) {
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
   }
@@ -76,7 +81,8 @@ inline cudaError_t prepare_kernel(const void *kernel, const DeviceInfo &d, bool 
 template <int OP, typename T, int CPL, bool EXACT>
 cudaError_t launch_small_k(const SmallParams &p, const DeviceInfo &d, cudaStream_t stream) {
   auto kern = small_row_kernel<OP, T, CPL, EXACT>;
-  const int bps = cached_occupancy(reinterpret_cast<const void *>(kern), 0, 1, nullptr);
+  const int bps = cached_occupancy(reinterpret_cast<const void *>(kern), kCtaThreads, 0, 1,
+                                   nullptr);
   const int64_t rows_per_cta = static_cast<int64_t>(kCtaWarps) * (32 / p.G);
   const int64_t want = ceil_div(p.rows, rows_per_cta);
   const int64_t cap = static_cast<int64_t>(std::max(bps, 1)) * d.sm_count;
@@ -118,28 +124,32 @@ cudaError_t launch_small(const DenseCall &c, const DeviceInfo &d, bool exact, bo
 // ---------------------------------------------------------------------------
 // MEDIUM / LARGE / ragged: the tile kernel
 // ---------------------------------------------------------------------------
+// min_stage_area: bytes the stages must span together (ragged SMALL staging)
 template <int OP, typename T, bool EXACT, bool CLUSTER, bool RAGGED>
 cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int64_t items,
-                          const DeviceInfo &d, cudaStream_t stream) {
+                          const DeviceInfo &d, cudaStream_t stream, uint32_t min_stage_area = 0) {
   auto kern = tile_row_kernel<OP, T, EXACT, CLUSTER, RAGGED>;
   const void *kp = reinterpret_cast<const void *>(kern);
   p.stage_bytes = static_cast<uint32_t>(stage_tiles) * kTileBytes;
   p.max_tiles = stage_tiles;
+  p.gather_tiles = CLUSTER ? cs * stage_tiles : 0;
+  while (static_cast<uint64_t>(stages) * p.stage_bytes < min_stage_area) ++stages;
+  const auto total = [&](int s) {
+    return TileSmemLayout(p.stage_bytes, s, stage_tiles, p.gather_tiles).total;
+  };
   // as many of the wanted stages as fit in the CTA's shared memory
-  while (stages > 1 &&
-         TileSmemLayout(p.stage_bytes, stages, stage_tiles).total >
-             static_cast<uint32_t>(d.max_smem_optin))
-    --stages;
+  while (stages > 1 && total(stages) > static_cast<uint32_t>(d.max_smem_optin)) --stages;
+  if (static_cast<uint64_t>(stages) * p.stage_bytes < min_stage_area)
+    return cudaErrorInvalidConfiguration;
   p.stages = stages;
-  const TileSmemLayout L(p.stage_bytes, stages, stage_tiles);
-  const size_t smem = L.total;
+  const size_t smem = total(stages);
   if (smem > static_cast<size_t>(d.max_smem_optin)) return cudaErrorInvalidConfiguration;
   cudaError_t e = prepare_kernel(kp, d, CLUSTER);
   if (e != cudaSuccess) return e;
 
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
-  cfg.blockDim = dim3(kCtaThreads, 1, 1);
+  cfg.blockDim = dim3(kTileThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   int grid;
@@ -151,11 +161,11 @@ cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     cfg.gridDim = dim3(cs * std::max(1, d.sm_count / cs), 1, 1);
-    int ncl = cached_occupancy(kp, smem, cs, &cfg);
+    int ncl = cached_occupancy(kp, kTileThreads, smem, cs, &cfg);
     if (ncl < 1) ncl = 1;
     grid = static_cast<int>(cs * std::max<int64_t>(1, std::min<int64_t>(items, ncl)));
   } else {
-    const int bps = std::max(1, cached_occupancy(kp, smem, 1, nullptr));
+    const int bps = std::max(1, cached_occupancy(kp, kTileThreads, smem, 1, nullptr));
     grid = static_cast<int>(std::max<int64_t>(
         1, std::min<int64_t>(items, static_cast<int64_t>(bps) * d.sm_count)));
   }
@@ -167,8 +177,8 @@ cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int
 
 inline int pick_stages(int stage_tiles, int knob) {
   if (knob > 0) return std::min(knob, 16);
-  // about 48 KiB of stages per CTA, at least 2 so loads overlap compute
-  return std::max(2, std::min(8, 48 / std::max(1, stage_tiles)));
+  // about 32 KiB of stages per CTA, at least 2 so loads overlap compute
+  return std::max(2, std::min(8, 32 / std::max(1, stage_tiles)));
 }
 
 // Smallest cluster (power of two, >= 2) whose portions of a K-tile row hold
@@ -243,8 +253,7 @@ cudaError_t launch_ragged_t(const RaggedCall &c, const DeviceInfo &d) {
   constexpr int E = 16 / SZ;
   const Knobs kn = read_knobs();
   unsigned char *ws = static_cast<unsigned char *>(c.ws);
-  const size_t lists = ragged_lists_offset(c.rows);
-  int32_t *list0 = reinterpret_cast<int32_t *>(ws + lists);
+  const RowRec *list0 = reinterpret_cast<const RowRec *>(ws + ragged_lists_offset(c.rows));
   if (c.classify) {
     const cudaError_t e = launch_classify(c, d);
     if (e != cudaSuccess) return e;
@@ -262,10 +271,9 @@ cudaError_t launch_ragged_t(const RaggedCall &c, const DeviceInfo &d) {
   p.gvec = (!c.gamma || aligned16(c.gamma)) && (!c.beta || aligned16(c.beta));
   p.timeout_ns = kWaitLimitNs;
   p.status = d.status;
-  p.offsets = c.offsets;
-  p.list_small = list0;
-  p.list_medium = list0 + c.rows;
-  p.list_large = list0 + 2 * c.rows;
+  p.rec_small = list0;
+  p.rec_medium = list0 + c.rows;
+  p.rec_large = list0 + 2 * c.rows;
   p.counts = reinterpret_cast<const int32_t *>(ws + kWsCounts);
   p.counters = reinterpret_cast<unsigned int *>(ws + kWsCounters);
 
@@ -281,11 +289,12 @@ cudaError_t launch_ragged_t(const RaggedCall &c, const DeviceInfo &d) {
   }
   if (st > kMaxPortionTiles) return cudaErrorInvalidValue;
   const int S = pick_stages(static_cast<int>(st), kn.stages);
+  const uint32_t small_area = kConsumerWarps * kSmallSliceBytes;
   if (cs > 1)
     return launch_tile_k<OP, T, false, true, true>(p, cs, S, static_cast<int>(st), c.rows, d,
-                                                   c.stream);
+                                                   c.stream, small_area);
   return launch_tile_k<OP, T, false, false, true>(p, 1, S, static_cast<int>(st), c.rows, d,
-                                                  c.stream);
+                                                  c.stream, small_area);
 }
 
 template <int OP>

@@ -42,7 +42,7 @@ Knobs read_knobs() {
 
 cudaError_t launch_classify(const RaggedCall &c, const DeviceInfo &d) {
   unsigned char *ws = static_cast<unsigned char *>(c.ws);
-  int32_t *list0 = reinterpret_cast<int32_t *>(ws + ragged_lists_offset(c.rows));
+  RowRec *list0 = reinterpret_cast<RowRec *>(ws + ragged_lists_offset(c.rows));
   ClassifyParams cp;
   cp.offsets = c.offsets;
   cp.rows = c.rows;
