@@ -147,13 +147,27 @@ class L2Flusher:
 
 
 def time_calls(torch, fn, steps, warmup, flush=None):
-    """Per-call device time (ms) with CUDA events on the current stream; an
-    L2 flush, when given, runs before each call outside the timed span."""
+    """Device time per call (ms) with CUDA events on the current stream.
+
+    With an L2 flush, each call is timed alone and the flush (outside the
+    timed span) keeps the GPU busy while the host enqueues the call.  Without
+    one, `steps` calls run back to back between one pair of events, so the
+    host's launch overhead never shows up as idle GPU time; every entry of the
+    returned list is then that batch's mean."""
     for _ in range(warmup):
         if flush:
             flush()
         fn()
     torch.cuda.synchronize()
+    if flush is None:
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(steps):
+            fn()
+        b.record()
+        b.synchronize()
+        return [a.elapsed_time(b) / steps] * steps
     times = []
     for _ in range(steps):
         if flush:

@@ -166,62 +166,35 @@ __device__ __forceinline__ uint4 shift_chunk<__nv_bfloat16>(const uint4 &A, cons
 }
 
 // ---------------------------------------------------------------------------
-// Packed fp32 pairs (Blackwell f32x2 arithmetic): a pair holds the even
-// element of a chunk in its low half and the odd element in its high half.
-// Every sum over a chunk run accumulates even and odd elements separately and
+// Packed fp32 pairs (Blackwell f32x2 arithmetic, float2 builtins): a pair
+// holds the even element of a chunk in .x and the odd element in .y.  Every
+// sum over a run of chunks accumulates even and odd elements separately and
 // adds the two halves at the end, in that fixed order.
 // ---------------------------------------------------------------------------
-typedef unsigned long long f2;
+typedef float2 f2;
 
-__device__ __forceinline__ f2 f2_make(float lo, float hi) {
-  f2 r;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
-  return r;
-}
-__device__ __forceinline__ float f2_lo(f2 v) {
-  float lo, hi;
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
-  return lo;
-}
-__device__ __forceinline__ float f2_hi(f2 v) {
-  float lo, hi;
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
-  return hi;
-}
-__device__ __forceinline__ float f2_total(f2 v) { return __fadd_rn(f2_lo(v), f2_hi(v)); }
-__device__ __forceinline__ f2 f2_add(f2 a, f2 b) {
-  f2 d;
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-__device__ __forceinline__ f2 f2_sub(f2 a, f2 b) {
-  f2 d;
-  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-__device__ __forceinline__ f2 f2_mul(f2 a, f2 b) {
-  f2 d;
-  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-__device__ __forceinline__ f2 f2_fma(f2 a, f2 b, f2 c) {
-  f2 d;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
-  return d;
-}
-__device__ __forceinline__ f2 f2_bcast(float v) { return f2_make(v, v); }
-// Keeps the halves whose mask bit is set, the other halves become `fill`.
+__device__ __forceinline__ f2 f2_make(float lo, float hi) { return make_float2(lo, hi); }
+__device__ __forceinline__ float f2_lo(f2 v) { return v.x; }
+__device__ __forceinline__ float f2_hi(f2 v) { return v.y; }
+__device__ __forceinline__ float f2_total(f2 v) { return __fadd_rn(v.x, v.y); }
+__device__ __forceinline__ f2 f2_add(f2 a, f2 b) { return __fadd2_rn(a, b); }
+__device__ __forceinline__ f2 f2_mul(f2 a, f2 b) { return __fmul2_rn(a, b); }
+__device__ __forceinline__ f2 f2_fma(f2 a, f2 b, f2 c) { return __ffma2_rn(a, b, c); }
+__device__ __forceinline__ f2 f2_bcast(float v) { return make_float2(v, v); }
+// a - b as a + (-b); callers pass the negated operand once per row
+__device__ __forceinline__ f2 f2_neg(f2 v) { return make_float2(-v.x, -v.y); }
+// Keeps the halves whose flag is set, the other halves become `fill`.
 __device__ __forceinline__ f2 f2_select(f2 v, bool keep_lo, bool keep_hi, float fill) {
-  return f2_make(keep_lo ? f2_lo(v) : fill, keep_hi ? f2_hi(v) : fill);
+  return make_float2(keep_lo ? v.x : fill, keep_hi ? v.y : fill);
 }
 
 // 16-byte chunk <-> pairs.  fp32: 2 pairs, bf16: 4 pairs.
 __device__ __forceinline__ void chunk_to_pairs(const uint4 &v, f2 (&p)[2]) {
-  p[0] = (static_cast<f2>(v.y) << 32) | v.x;
-  p[1] = (static_cast<f2>(v.w) << 32) | v.z;
+  p[0] = make_float2(__uint_as_float(v.x), __uint_as_float(v.y));
+  p[1] = make_float2(__uint_as_float(v.z), __uint_as_float(v.w));
 }
 __device__ __forceinline__ f2 bf16x2_to_pair(uint32_t w) {
-  return f2_make(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
+  return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
 }
 __device__ __forceinline__ void chunk_to_pairs(const uint4 &v, f2 (&p)[4]) {
   p[0] = bf16x2_to_pair(v.x);
@@ -230,13 +203,12 @@ __device__ __forceinline__ void chunk_to_pairs(const uint4 &v, f2 (&p)[4]) {
   p[3] = bf16x2_to_pair(v.w);
 }
 __device__ __forceinline__ uint4 pairs_to_chunk(const f2 (&p)[2]) {
-  return make_uint4(static_cast<uint32_t>(p[0]), static_cast<uint32_t>(p[0] >> 32),
-                    static_cast<uint32_t>(p[1]), static_cast<uint32_t>(p[1] >> 32));
+  return make_uint4(__float_as_uint(p[0].x), __float_as_uint(p[0].y), __float_as_uint(p[1].x),
+                    __float_as_uint(p[1].y));
 }
 __device__ __forceinline__ uint32_t pair_to_bf16x2(f2 v) {
-  uint32_t r;  // cvt packs its first source into the upper half
-  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(f2_hi(v)), "f"(f2_lo(v)));
-  return r;
+  __nv_bfloat162 b = __float22bfloat162_rn(v);  // round to nearest even, .x in the low half
+  return *reinterpret_cast<uint32_t *>(&b);
 }
 __device__ __forceinline__ uint4 pairs_to_chunk(const f2 (&p)[4]) {
   return make_uint4(pair_to_bf16x2(p[0]), pair_to_bf16x2(p[1]), pair_to_bf16x2(p[2]),
@@ -245,7 +217,7 @@ __device__ __forceinline__ uint4 pairs_to_chunk(const f2 (&p)[4]) {
 // element e of a chunk's pair array
 template <int NP>
 __device__ __forceinline__ float pair_elem(const f2 (&p)[NP], int e) {
-  return (e & 1) ? f2_hi(p[e >> 1]) : f2_lo(p[e >> 1]);
+  return (e & 1) ? p[e >> 1].y : p[e >> 1].x;
 }
 
 // e^v as 2^(v * log2 e) on the MUFU unit; v is a difference x - m <= 0 here.
@@ -255,10 +227,10 @@ __device__ __forceinline__ float ex2_approx(float v) {
   asm("ex2.approx.f32 %0, %1;" : "=f"(r) : "f"(v));
   return r;
 }
-// exp(x - m) for both halves of a pair
-__device__ __forceinline__ f2 f2_exp_shifted(f2 x, f2 m) {
-  const f2 u = f2_mul(f2_sub(x, m), f2_bcast(kLog2e));
-  return f2_make(ex2_approx(f2_lo(u)), ex2_approx(f2_hi(u)));
+// exp(x - m) for both halves of a pair, given neg_m = (-m, -m)
+__device__ __forceinline__ f2 f2_exp_shifted(f2 x, f2 neg_m) {
+  const f2 u = __fmul2_rn(__fadd2_rn(x, neg_m), f2_bcast(kLog2e));
+  return make_float2(ex2_approx(u.x), ex2_approx(u.y));
 }
 __device__ __forceinline__ float exp_shifted(float x, float m) {
   return ex2_approx(__fmul_rn(__fsub_rn(x, m), kLog2e));
@@ -339,14 +311,18 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
       "mbarrier.arrive.shared::cta.b64 st, [%0];\n\t}" ::"r"(bar)
       : "memory");
 }
+// A waiting thread is suspended until the phase completes or this many
+// nanoseconds pass, whichever comes first, instead of re-polling.
+constexpr uint32_t kWaitSuspendNs = 1000000;
+
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(bar), "r"(parity)
+      : "r"(bar), "r"(parity), "r"(kWaitSuspendNs)
       : "memory");
   return ok != 0;
 }
@@ -408,15 +384,18 @@ __device__ __forceinline__ void cluster_sync() {
 }
 __device__ __forceinline__ uint32_t map_to_rank(uint32_t local_smem, uint32_t rank) {
   uint32_t r;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local_smem), "r"(rank));
+  asm("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local_smem), "r"(rank));
   return r;
 }
+// Load from a peer CTA's shared memory.  Volatile, so it stays after the
+// (volatile) barrier wait that publishes the data, but without a memory
+// clobber, so independent loads issue back to back before their results are
+// stored anywhere.
 __device__ __forceinline__ float4 ld_dsmem_f4(uint32_t addr) {
   float4 v;
   asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
                : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(addr)
-               : "memory");
+               : "r"(addr));
   return v;
 }
 
@@ -452,10 +431,10 @@ __device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t par
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(bar), "r"(parity)
+      : "r"(bar), "r"(parity), "r"(kWaitSuspendNs)
       : "memory");
   return ok != 0;
 }

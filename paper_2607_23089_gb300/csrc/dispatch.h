@@ -71,10 +71,12 @@ inline int64_t max_row_len_elems(int esize) {
 //                       the row (SMALL only for rows of <= 288 chunks)
 //   ROWOP_CLUSTER       cluster size for split rows (1, 2, 4, 8, 16)
 //   ROWOP_STAGES        stage-ring depth of the tile kernel
+//   ROWOP_CTAS_PER_SM   upper bound on resident tile-kernel CTAs per SM
 struct Knobs {
   int force_bucket = -1;
   int cluster = 0;
   int stages = 0;
+  int ctas_per_sm = 0;
 };
 Knobs read_knobs();
 

@@ -130,6 +130,7 @@ cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int
                           const DeviceInfo &d, cudaStream_t stream, uint32_t min_stage_area = 0) {
   auto kern = tile_row_kernel<OP, T, EXACT, CLUSTER, RAGGED>;
   const void *kp = reinterpret_cast<const void *>(kern);
+  const int max_ctas_per_sm = read_knobs().ctas_per_sm;
   p.stage_bytes = static_cast<uint32_t>(stage_tiles) * kTileBytes;
   p.max_tiles = stage_tiles;
   p.gather_tiles = CLUSTER ? cs * stage_tiles : 0;
@@ -162,10 +163,12 @@ cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int
     cfg.numAttrs = 1;
     cfg.gridDim = dim3(cs * std::max(1, d.sm_count / cs), 1, 1);
     int ncl = cached_occupancy(kp, kTileThreads, smem, cs, &cfg);
+    if (max_ctas_per_sm > 0) ncl = std::min(ncl, max_ctas_per_sm * d.sm_count / cs);
     if (ncl < 1) ncl = 1;
     grid = static_cast<int>(cs * std::max<int64_t>(1, std::min<int64_t>(items, ncl)));
   } else {
-    const int bps = std::max(1, cached_occupancy(kp, kTileThreads, smem, 1, nullptr));
+    int bps = std::max(1, cached_occupancy(kp, kTileThreads, smem, 1, nullptr));
+    if (max_ctas_per_sm > 0) bps = std::min(bps, max_ctas_per_sm);
     grid = static_cast<int>(std::max<int64_t>(
         1, std::min<int64_t>(items, static_cast<int64_t>(bps) * d.sm_count)));
   }
@@ -232,7 +235,8 @@ cudaError_t launch_dense_t(const DenseCall &c, const DeviceInfo &d) {
   const int cs = pick_cluster(K, 64, kn.cluster);
   const int st = static_cast<int>(ceil_div(K, cs));
   if (st > kMaxPortionTiles) return cudaErrorInvalidValue;
-  const int S = kn.stages > 0 ? std::min(kn.stages, 16) : (st >= 32 ? 1 : 2);
+  // two stages when they fit, so the next portion loads while this one is used
+  const int S = kn.stages > 0 ? std::min(kn.stages, 16) : 2;
   if (cs == 1) {
     if (exact) return launch_tile_k<OP, T, true, false, false>(p, 1, S, st, c.rows, d, c.stream);
     return launch_tile_k<OP, T, false, false, false>(p, 1, S, st, c.rows, d, c.stream);

@@ -46,7 +46,7 @@ __device__ __forceinline__ f2 chunk_sum_exp(const f2 (&p)[NP], f2 m2, f2 acc, in
   const bool full = (lo == 0 && hi == 2 * NP);
 #pragma unroll
   for (int i = 0; i < NP; ++i) {
-    f2 e = f2_exp_shifted(p[i], m2);
+    f2 e = f2_exp_shifted(p[i], f2_neg(m2));
     if (!full) e = f2_select(e, in_range(2 * i, lo, hi), in_range(2 * i + 1, lo, hi), 0.f);
     acc = f2_add(acc, e);
   }
@@ -73,7 +73,7 @@ __device__ __forceinline__ f2 chunk_sum_sqdev(const f2 (&p)[NP], f2 mean2, f2 ac
   const bool full = (lo == 0 && hi == 2 * NP);
 #pragma unroll
   for (int i = 0; i < NP; ++i) {
-    f2 d = f2_sub(p[i], mean2);
+    f2 d = f2_add(p[i], f2_neg(mean2));
     if (!full) d = f2_select(d, in_range(2 * i, lo, hi), in_range(2 * i + 1, lo, hi), 0.f);
     acc = f2_fma(d, d, acc);
   }
@@ -122,33 +122,42 @@ __device__ __forceinline__ void load_param_pairs(const T *__restrict__ g, int64_
 }
 
 // In place: x pairs -> y pairs.  (s0, s1) are (M, 1/S) for softmax,
-// (M, log S) for log-softmax, (mu, rstd) for LayerNorm, (-, rstd) for RMSNorm.
+// (M, log S) for log-softmax, (mu, rstd) for LayerNorm, (-, rstd) for RMSNorm;
+// g / b are the gamma / beta pairs (read only by the norms).
+template <int OP, int NP>
+__device__ __forceinline__ void normalize_pairs(f2 (&p)[NP], float s0, float s1,
+                                                const f2 (&g)[NP], const f2 (&b)[NP]) {
+  const f2 na = f2_bcast(-s0);
+  const f2 b2 = f2_bcast(s1);
+  if constexpr (OP == kSoftmax) {
+#pragma unroll
+    for (int i = 0; i < NP; ++i) p[i] = f2_mul(f2_exp_shifted(p[i], na), b2);
+  } else if constexpr (OP == kLogSoftmax) {
+    const f2 nb = f2_bcast(-s1);
+#pragma unroll
+    for (int i = 0; i < NP; ++i) p[i] = f2_add(f2_add(p[i], na), nb);
+  } else if constexpr (OP == kLayerNorm) {
+#pragma unroll
+    for (int i = 0; i < NP; ++i) p[i] = f2_fma(f2_mul(f2_add(p[i], na), b2), g[i], b[i]);
+  } else {
+#pragma unroll
+    for (int i = 0; i < NP; ++i) p[i] = f2_mul(f2_mul(p[i], b2), g[i]);
+  }
+}
+
+// chunk_normalize: normalize_pairs with gamma/beta of window chunk c read
+// through the general (bounds-checked, any alignment) loader.
 template <int OP, typename T>
 __device__ __forceinline__ void chunk_normalize(f2 (&p)[Elem<T>::kPerChunk / 2], float s0,
                                                 float s1, const T *gamma, int64_t glen_g,
                                                 const T *beta, int64_t glen_b, int64_t c, int h,
                                                 bool gvec) {
   constexpr int NP = Elem<T>::kPerChunk / 2;
-  const f2 a2 = f2_bcast(s0);
-  const f2 b2 = f2_bcast(s1);
-  if constexpr (OP == kSoftmax) {
-#pragma unroll
-    for (int i = 0; i < NP; ++i) p[i] = f2_mul(f2_exp_shifted(p[i], a2), b2);
-  } else if constexpr (OP == kLogSoftmax) {
-#pragma unroll
-    for (int i = 0; i < NP; ++i) p[i] = f2_sub(f2_sub(p[i], a2), b2);
-  } else if constexpr (OP == kLayerNorm) {
-    f2 g[NP], b[NP];
+  f2 g[NP], b[NP];
+  if constexpr (OP == kLayerNorm || OP == kRmsNorm)
     load_param_pairs<T>(gamma, glen_g, c, h, gvec, 1.f, g);
-    load_param_pairs<T>(beta, glen_b, c, h, gvec, 0.f, b);
-#pragma unroll
-    for (int i = 0; i < NP; ++i) p[i] = f2_fma(f2_mul(f2_sub(p[i], a2), b2), g[i], b[i]);
-  } else {
-    f2 g[NP];
-    load_param_pairs<T>(gamma, glen_g, c, h, gvec, 1.f, g);
-#pragma unroll
-    for (int i = 0; i < NP; ++i) p[i] = f2_mul(f2_mul(p[i], b2), g[i]);
-  }
+  if constexpr (OP == kLayerNorm) load_param_pairs<T>(beta, glen_b, c, h, gvec, 0.f, b);
+  normalize_pairs<OP, NP>(p, s0, s1, g, b);
 }
 
 // Writes the row's elements of chunk c: one 128-bit store when the chunk is

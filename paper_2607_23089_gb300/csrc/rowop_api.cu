@@ -37,6 +37,7 @@ Knobs read_knobs() {
   k.force_bucket = env_int("ROWOP_FORCE_BUCKET", -1);
   k.cluster = env_int("ROWOP_CLUSTER", 0);
   k.stages = env_int("ROWOP_STAGES", 0);
+  k.ctas_per_sm = env_int("ROWOP_CTAS_PER_SM", 0);
   return k;
 }
 

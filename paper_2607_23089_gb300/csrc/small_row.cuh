@@ -45,19 +45,22 @@ struct SmallRowArgs {
 // the lane's index in its group).  `get(k)` returns the 16 bytes of window
 // chunk sub + k*G.  All 32 lanes of the warp must call this together (the
 // butterflies use the full mask); groups never mix since every xor offset is
-// below G.  Inactive groups pass nc = 0.
-template <int OP, typename T, int CPL, bool EXACT, class Get>
+// below G.  Inactive groups pass nc = 0.  UNROLL = false keeps the chunk
+// loops rolled (for chunk sources that can be indexed at run time); the
+// operations and their order do not change.
+template <int OP, typename T, int CPL, bool EXACT, bool UNROLL, class Get>
 __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, int h, int64_t nc,
                                                int G, int sub, const SmallRowArgs &a) {
   constexpr int E = Elem<T>::kPerChunk;
   constexpr int NP = E / 2;
+  constexpr int kUnroll = UNROLL ? CPL : 1;
   const int64_t hn = h + n;
   float s0 = 0.f, s1 = 0.f;
 
   // ---- statistics ----
   if constexpr (OP == kSoftmax || OP == kLogSoftmax) {
     float m = -INFINITY;
-#pragma unroll
+#pragma unroll(kUnroll)
     for (int k = 0; k < CPL; ++k) {
       const int64_t c = sub + static_cast<int64_t>(k) * G;
       if (c < nc) {
@@ -71,7 +74,7 @@ __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, i
     m = group_max(m, G);
     const f2 m2 = f2_bcast(m);
     f2 acc = f2_bcast(0.f);
-#pragma unroll
+#pragma unroll(kUnroll)
     for (int k = 0; k < CPL; ++k) {
       const int64_t c = sub + static_cast<int64_t>(k) * G;
       if (c < nc) {
@@ -87,7 +90,7 @@ __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, i
     s1 = (OP == kSoftmax) ? __frcp_rn(s) : logf(s);
   } else if constexpr (OP == kLayerNorm) {
     f2 acc = f2_bcast(0.f);
-#pragma unroll
+#pragma unroll(kUnroll)
     for (int k = 0; k < CPL; ++k) {
       const int64_t c = sub + static_cast<int64_t>(k) * G;
       if (c < nc) {
@@ -101,7 +104,7 @@ __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, i
     const float mean = __fdiv_rn(group_sum(f2_total(acc), G), static_cast<float>(n));
     const f2 mean2 = f2_bcast(mean);
     acc = f2_bcast(0.f);
-#pragma unroll
+#pragma unroll(kUnroll)
     for (int k = 0; k < CPL; ++k) {
       const int64_t c = sub + static_cast<int64_t>(k) * G;
       if (c < nc) {
@@ -117,7 +120,7 @@ __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, i
     s1 = __frsqrt_rn(__fadd_rn(__fdiv_rn(q, static_cast<float>(n)), a.eps));
   } else {
     f2 acc = f2_bcast(0.f);
-#pragma unroll
+#pragma unroll(kUnroll)
     for (int k = 0; k < CPL; ++k) {
       const int64_t c = sub + static_cast<int64_t>(k) * G;
       if (c < nc) {
@@ -134,7 +137,7 @@ __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, i
 
   // ---- normalise and store ----
   char *owin = reinterpret_cast<char *>(out_row) - static_cast<int64_t>(h) * Elem<T>::kSize;
-#pragma unroll
+#pragma unroll(kUnroll)
   for (int k = 0; k < CPL; ++k) {
     const int64_t c = sub + static_cast<int64_t>(k) * G;
     if (c < nc) {
@@ -195,7 +198,7 @@ __global__ void __launch_bounds__(kCtaThreads) small_row_kernel(const SmallParam
                                        : load_chunk_elems<T>(in_row, c, h, p.cols);
       }
     }
-    small_row_core<OP, T, CPL, EXACT>([&](int k) { return raw[k]; }, out_row, p.cols, h, nc, G,
+    small_row_core<OP, T, CPL, EXACT, true>([&](int k) { return raw[k]; }, out_row, p.cols, h, nc, G,
                                       sub, p.a);
   }
 }

@@ -38,6 +38,7 @@ constexpr int kTileThreads = kConsumerThreads + 32;  // + the producer warp
 constexpr int kPieceTiles = 16;                      // tiles per piece barrier (16 KiB)
 constexpr uint32_t kBarConsumers = 1;                // named barrier of the consumer warps
 constexpr int kSmallSliceBytes = 4096 + 128;         // per-warp staging of a ragged SMALL row
+constexpr int kShortCombineTiles = 64;  // rows of up to this many tiles: every warp combines
 
 struct TileParams {
   const void *in;
@@ -74,7 +75,7 @@ struct ItemMeta {
 
 // Shared-memory layout of the tile kernel (host and device agree on it).
 struct TileSmemLayout {
-  uint32_t part_c, part_m, gather, meta, bar_meta, bar_piece, bar_empty, bar_ready,
+  uint32_t part_c, part_m, gather, meta, xw, bar_meta, bar_piece, bar_empty, bar_ready,
       bar_released, flags, total;
   int pieces;
   __host__ __device__ TileSmemLayout(uint32_t stage_bytes, int stages, int max_tiles,
@@ -89,6 +90,8 @@ struct TileSmemLayout {
     off += static_cast<uint32_t>(gather_tiles) * 16u;
     meta = off;
     off += stages * 32u;
+    xw = off;  // 2 x 8 per-warp values of the cooperative combine
+    off += 2u * kConsumerWarps * 4u;
     bar_meta = off;
     off += stages * 8u;
     bar_piece = off;
@@ -105,11 +108,13 @@ struct TileSmemLayout {
   }
 };
 
+// Row geometry in chunks and tiles.  Rows are at most rowop_max_row_len()
+// elements, so every per-row chunk and tile index fits in 32 bits.
 struct ItemGeo {
   int64_t start, n;
   int h;
-  int64_t nc, K, t0, t1;
-  int64_t cf, cl;  // chunks [cf, cl) are entirely the row's
+  int nc, K, t0, t1;
+  int cf, cl;  // chunks [cf, cl) are entirely the row's
 };
 
 template <typename T, bool EXACT>
@@ -122,10 +127,11 @@ __device__ __forceinline__ ItemGeo item_geo(const void *in, int64_t start, int64
   g.n = n;
   const uintptr_t a = reinterpret_cast<uintptr_t>(static_cast<const T *>(in) + start);
   g.h = EXACT ? 0 : static_cast<int>((a & 15) / SZ);
-  g.nc = (g.h + n + E - 1) / E;
+  const int hn = g.h + static_cast<int>(n);
+  g.nc = (hn + E - 1) / E;
   g.K = (g.nc + kTileChunks - 1) / kTileChunks;
   if (split) {
-    const int64_t tpc = (g.K + cs - 1) / cs;
+    const int tpc = (g.K + cs - 1) / cs;
     g.t0 = min(g.K, rank * tpc);
     g.t1 = min(g.K, g.t0 + tpc);
   } else {
@@ -133,128 +139,292 @@ __device__ __forceinline__ ItemGeo item_geo(const void *in, int64_t start, int64
     g.t1 = g.K;
   }
   g.cf = (g.h > 0) ? 1 : 0;
-  g.cl = (((g.h + n) % E) != 0) ? g.nc - 1 : g.nc;
+  g.cl = ((hn % E) != 0) ? g.nc - 1 : g.nc;
   return g;
 }
 
-__device__ __forceinline__ bool tile_is_full(int64_t t, const ItemGeo &g) {
+__device__ __forceinline__ bool tile_is_full(int t, const ItemGeo &g) {
   return t * kTileChunks >= g.cf && (t + 1) * kTileChunks <= g.cl;
 }
 
 // ---------------------------------------------------------------------------
-// pass 1: one warp reduces tile t (its 64 chunks at `tsm`) to a tile partial
-//   softmax / log-softmax (m_t, s_t = sum exp(x - m_t)), LayerNorm (sum,
-//   mean_t, sum (x - mean_t)^2, n_t), RMSNorm (sum x^2).
+// pass 1: tile partials.  One warp reduces tile t (its 64 chunks; lane l
+// holds chunks l and l+32) to a tile partial:
+//   softmax / log-softmax  (m_t, s_t = sum exp(x - m_t))
+//   LayerNorm              (sum_t, mean_t, sum (x - mean_t)^2, n_t)
+//   RMSNorm                (sum x^2)
+// A warp takes up to kPass1Batch of its tiles at once, so several independent
+// shuffle chains are in flight.
 // ---------------------------------------------------------------------------
-template <int OP, typename T, bool EXACT>
-__device__ __forceinline__ float4 tile_partial(const unsigned char *tsm, int64_t t,
-                                               const ItemGeo &g, int lane) {
+constexpr int kPass1Batch = 4;
+
+struct TileMask {
+  int lo0, hi0, lo1, hi1;  // valid element ranges of the lane's two chunks
+};
+
+template <typename T>
+__device__ __forceinline__ TileMask tile_mask(int t, const ItemGeo &g, int lane, bool full) {
   constexpr int E = Elem<T>::kPerChunk;
-  constexpr int NP = E / 2;
-  const bool full = tile_is_full(t, g);  // the row's last tile may hold < 64 chunks
+  TileMask m{0, E, 0, E};
+  if (!full) {
+    const int hn = g.h + static_cast<int>(g.n);
+    const int c0 = t * kTileChunks + lane;
+    const int c1 = c0 + 32;
+    if (c0 < g.nc) chunk_valid_range(c0, g.nc, g.h, hn, E, m.lo0, m.hi0); else m.lo0 = m.hi0 = 0;
+    if (c1 < g.nc) chunk_valid_range(c1, g.nc, g.h, hn, E, m.lo1, m.hi1); else m.lo1 = m.hi1 = 0;
+  }
+  return m;
+}
+
+// first lane-level statistic of a tile: max (softmax family), sum
+// (LayerNorm), sum of squares (RMSNorm)
+template <int OP, typename T>
+__device__ __forceinline__ float tile_lane_first(const unsigned char *tsm, const TileMask &m,
+                                                 int lane) {
+  constexpr int NP = Elem<T>::kPerChunk / 2;
   f2 p0[NP], p1[NP];
   chunk_to_pairs(*reinterpret_cast<const uint4 *>(tsm + lane * kChunkBytes), p0);
   chunk_to_pairs(*reinterpret_cast<const uint4 *>(tsm + (lane + 32) * kChunkBytes), p1);
-  int lo0 = 0, hi0 = E, lo1 = 0, hi1 = E;
-  const int64_t hn = g.h + g.n;
-  if (!full) {
-    const int64_t c0 = t * kTileChunks + lane;
-    const int64_t c1 = c0 + 32;
-    if (c0 < g.nc) chunk_valid_range(c0, g.nc, g.h, hn, E, lo0, hi0); else lo0 = hi0 = 0;
-    if (c1 < g.nc) chunk_valid_range(c1, g.nc, g.h, hn, E, lo1, hi1); else lo1 = hi1 = 0;
-  }
   if constexpr (OP == kSoftmax || OP == kLogSoftmax) {
-    float m = chunk_max<NP>(p0, -INFINITY, lo0, hi0);
-    m = warp_max(chunk_max<NP>(p1, m, lo1, hi1));
-    f2 acc = f2_bcast(0.f);
-    if (m != -INFINITY) {
-      const f2 m2 = f2_bcast(m);
-      acc = chunk_sum_exp<NP>(p0, m2, acc, lo0, hi0);
-      acc = chunk_sum_exp<NP>(p1, m2, acc, lo1, hi1);
-    }
-    return make_float4(m, warp_sum(f2_total(acc)), 0.f, 0.f);
+    return chunk_max<NP>(p1, chunk_max<NP>(p0, -INFINITY, m.lo0, m.hi0), m.lo1, m.hi1);
   } else if constexpr (OP == kLayerNorm) {
-    f2 acc = chunk_sum<NP>(p0, f2_bcast(0.f), lo0, hi0);
-    acc = chunk_sum<NP>(p1, acc, lo1, hi1);
-    const float sum = warp_sum(f2_total(acc));
-    float mean, ntf;
-    if (full) {
-      ntf = static_cast<float>(kTileChunks * E);
-      mean = __fmul_rn(sum, 1.f / static_cast<float>(kTileChunks * E));  // exact: power of 2
-    } else {
-      const int64_t w0 = t * kTileChunks * E;
-      const int64_t w1 = min(g.nc, (t + 1) * kTileChunks) * E;
-      const int64_t nt = max(static_cast<int64_t>(0),
-                             min(hn, w1) - max(static_cast<int64_t>(g.h), w0));
-      ntf = static_cast<float>(nt);
-      mean = nt > 0 ? __fdiv_rn(sum, ntf) : 0.f;
-    }
-    const f2 mean2 = f2_bcast(mean);
-    acc = chunk_sum_sqdev<NP>(p0, mean2, f2_bcast(0.f), lo0, hi0);
-    acc = chunk_sum_sqdev<NP>(p1, mean2, acc, lo1, hi1);
-    return make_float4(sum, mean, warp_sum(f2_total(acc)), ntf);
+    return f2_total(chunk_sum<NP>(p1, chunk_sum<NP>(p0, f2_bcast(0.f), m.lo0, m.hi0), m.lo1, m.hi1));
   } else {
-    f2 acc = chunk_sum_sq<NP>(p0, f2_bcast(0.f), lo0, hi0);
-    acc = chunk_sum_sq<NP>(p1, acc, lo1, hi1);
-    return make_float4(warp_sum(f2_total(acc)), 0.f, 0.f, 0.f);
+    return f2_total(
+        chunk_sum_sq<NP>(p1, chunk_sum_sq<NP>(p0, f2_bcast(0.f), m.lo0, m.hi0), m.lo1, m.hi1));
   }
 }
 
+// second lane-level statistic: sum exp(x - ref) (softmax family, ref = m_t)
+// or sum (x - ref)^2 (LayerNorm, ref = mean_t)
+template <int OP, typename T>
+__device__ __forceinline__ float tile_lane_second(const unsigned char *tsm, const TileMask &m,
+                                                  int lane, float ref) {
+  constexpr int NP = Elem<T>::kPerChunk / 2;
+  f2 p0[NP], p1[NP];
+  chunk_to_pairs(*reinterpret_cast<const uint4 *>(tsm + lane * kChunkBytes), p0);
+  chunk_to_pairs(*reinterpret_cast<const uint4 *>(tsm + (lane + 32) * kChunkBytes), p1);
+  const f2 r2 = f2_bcast(ref);
+  if constexpr (OP == kSoftmax || OP == kLogSoftmax) {
+    if (ref == -INFINITY) return 0.f;  // no element of the tile is above -inf
+    return f2_total(chunk_sum_exp<NP>(p1, r2, chunk_sum_exp<NP>(p0, r2, f2_bcast(0.f), m.lo0, m.hi0),
+                                      m.lo1, m.hi1));
+  } else {
+    return f2_total(chunk_sum_sqdev<NP>(p1, r2, chunk_sum_sqdev<NP>(p0, r2, f2_bcast(0.f), m.lo0, m.hi0),
+                                        m.lo1, m.hi1));
+  }
+}
+
+// B tiles of one warp, lt0, lt0 + 8, ..., lt0 + 8(B-1), all below the item's
+// tile count: lane-level sums of all of them first, then their butterflies
+// interleaved.  Waits on each stage piece before the first tile read from it
+// (`waited` is the last piece waited for); returns false when such a wait
+// ran out.
+template <int OP, typename T, int B>
+__device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const ItemGeo &g, int lt0,
+                                            int lane, float4 *part, uint32_t piece_bar0,
+                                            uint32_t par, uint64_t timeout_ns, int &waited) {
+  constexpr int E = Elem<T>::kPerChunk;
+  constexpr bool kMaxFirst = (OP == kSoftmax || OP == kLogSoftmax);
+  float a[B], b[B];
+#pragma unroll
+  for (int q = 0; q < B; ++q) {
+    const int lt = lt0 + q * kConsumerWarps;
+    const int pc = lt / kPieceTiles;
+    if (pc != waited) {
+      if (!mbar_wait_bounded(piece_bar0 + 8u * pc, par, timeout_ns)) return false;
+      waited = pc;
+    }
+    const int t = g.t0 + lt;
+    a[q] = tile_lane_first<OP, T>(stage + lt * kTileBytes,
+                                  tile_mask<T>(t, g, lane, tile_is_full(t, g)), lane);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+    for (int q = 0; q < B; ++q) {
+      const float y = __shfl_xor_sync(kFullMask, a[q], o);
+      a[q] = kMaxFirst ? fmaxf(a[q], y) : __fadd_rn(a[q], y);
+    }
+  }
+  if constexpr (OP == kRmsNorm) {
+    if (lane == 0) {
+#pragma unroll
+      for (int q = 0; q < B; ++q) part[lt0 + q * kConsumerWarps] = make_float4(a[q], 0.f, 0.f, 0.f);
+    }
+  } else {
+    float ref[B], ntf[B];
+#pragma unroll
+    for (int q = 0; q < B; ++q) {
+      const int lt = lt0 + q * kConsumerWarps;
+      const int t = g.t0 + lt;
+      const bool full = tile_is_full(t, g);
+      ref[q] = a[q];
+      ntf[q] = 0.f;
+      if constexpr (OP == kLayerNorm) {
+        if (full) {
+          ntf[q] = static_cast<float>(kTileChunks * E);
+          ref[q] = __fmul_rn(a[q], 1.f / static_cast<float>(kTileChunks * E));  // exact
+        } else {
+          const int hn = g.h + static_cast<int>(g.n);
+          const int w0 = t * kTileChunks * E;
+          const int w1 = min(g.nc, (t + 1) * kTileChunks) * E;
+          const int nt = max(0, min(hn, w1) - max(g.h, w0));
+          ntf[q] = static_cast<float>(nt);
+          ref[q] = nt > 0 ? __fdiv_rn(a[q], ntf[q]) : 0.f;
+        }
+      }
+      b[q] = tile_lane_second<OP, T>(stage + lt * kTileBytes, tile_mask<T>(t, g, lane, full), lane,
+                                     ref[q]);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+      for (int q = 0; q < B; ++q) b[q] = __fadd_rn(b[q], __shfl_xor_sync(kFullMask, b[q], o));
+    }
+    if (lane == 0) {
+#pragma unroll
+      for (int q = 0; q < B; ++q)
+        part[lt0 + q * kConsumerWarps] = (OP == kLayerNorm) ? make_float4(a[q], ref[q], b[q], ntf[q])
+                                                            : make_float4(a[q], b[q], 0.f, 0.f);
+    }
+  }
+  return true;
+}
+
+// Pass 1 of an item for one warp: part[lt] for its tiles lt = warp, warp + 8,
+// ..., taken kPass1Batch at a time while that many remain, then in a batch of
+// two and one.  Each tile's arithmetic (and its butterfly order) is the same
+// whatever batch it falls in.
+template <int OP, typename T>
+__device__ __forceinline__ bool pass1_warp(const unsigned char *stage, const ItemGeo &g, int warp,
+                                           int lane, float4 *part, uint32_t piece_bar0,
+                                           uint32_t par, uint64_t timeout_ns) {
+  const int ntl = g.t1 - g.t0;
+  int waited = -1;
+  int lt0 = warp;
+  while (lt0 < ntl) {
+    const int left = (ntl - lt0 + kConsumerWarps - 1) / kConsumerWarps;
+    bool ok;
+    if (left >= kPass1Batch) {
+      ok = pass1_batch<OP, T, kPass1Batch>(stage, g, lt0, lane, part, piece_bar0, par, timeout_ns, waited);
+      lt0 += kPass1Batch * kConsumerWarps;
+    } else if (left >= 2) {
+      ok = pass1_batch<OP, T, 2>(stage, g, lt0, lane, part, piece_bar0, par, timeout_ns, waited);
+      lt0 += 2 * kConsumerWarps;
+    } else {
+      ok = pass1_batch<OP, T, 1>(stage, g, lt0, lane, part, piece_bar0, par, timeout_ns, waited);
+      lt0 += kConsumerWarps;
+    }
+    if (!ok) return false;
+  }
+  return true;
+}
+
 // ---------------------------------------------------------------------------
-// combine: the row statistics from its K tile partials (part[t], t < K), in
-// the fixed order lane l: t = l, l+32, ..., then a 5-level butterfly.  Every
-// lane of the calling warp ends with the same (s0, s1).
+// combine: the row statistics from its K tile partials part[0..K), in a fixed
+// order that depends on K only.
+//   K <= 64: lane l of a warp takes t = l, l+32 in turn, then a 5-level
+//            butterfly; every warp computes it, so nothing is broadcast.
+//   K > 64:  thread v of the 256 consumer threads takes t = v, v+256, ... in
+//            turn, a butterfly per warp, then the 8 warp results in warp
+//            order; the warps cooperate through `xw` and named barriers.
+// (s0, s1): softmax (M, 1/S), log-softmax (M, log S), LayerNorm (mu, rstd),
+// RMSNorm (-, rstd).
 // ---------------------------------------------------------------------------
 template <int OP>
-__device__ __forceinline__ void combine_stats(const float4 *part, int64_t K, int64_t n,
-                                              float eps, int lane, float &s0, float &s1) {
-  if constexpr (OP == kSoftmax || OP == kLogSoftmax) {
-    float m = -INFINITY;
-    for (int64_t t = lane; t < K; t += 32) m = fmaxf(m, part[t].x);
-    const float M = warp_max(m);
-    float s = 0.f;
-    for (int64_t t = lane; t < K; t += 32) {
-      const float4 pt = part[t];
-      if (pt.x != -INFINITY) s = __fadd_rn(s, __fmul_rn(pt.y, exp_shifted(pt.x, M)));
-    }
-    const float S = warp_sum(s);
-    s0 = M;
-    s1 = (OP == kSoftmax) ? __frcp_rn(S) : logf(S);
+__device__ __forceinline__ void finish_stats(float first, float second, float inv_n, float eps,
+                                             float &s0, float &s1) {
+  if constexpr (OP == kSoftmax) {
+    s0 = first;
+    s1 = __frcp_rn(second);
+  } else if constexpr (OP == kLogSoftmax) {
+    s0 = first;
+    s1 = logf(second);
   } else if constexpr (OP == kLayerNorm) {
-    float s = 0.f;
-    for (int64_t t = lane; t < K; t += 32) s = __fadd_rn(s, part[t].x);
-    const float nf = static_cast<float>(n);
-    const float mean = __fdiv_rn(warp_sum(s), nf);
-    float v = 0.f;
-    for (int64_t t = lane; t < K; t += 32) {
-      const float4 pt = part[t];
-      const float d = __fsub_rn(pt.y, mean);
-      v = __fadd_rn(v, __fmaf_rn(__fmul_rn(pt.w, d), d, pt.z));
-    }
-    s0 = mean;
-    s1 = __frsqrt_rn(__fadd_rn(__fdiv_rn(warp_sum(v), nf), eps));
+    s0 = first;  // the mean
+    s1 = rsqrtf(__fadd_rn(__fmul_rn(second, inv_n), eps));
   } else {
-    float q = 0.f;
-    for (int64_t t = lane; t < K; t += 32) q = __fadd_rn(q, part[t].x);
     s0 = 0.f;
-    s1 = __frsqrt_rn(__fadd_rn(__fdiv_rn(warp_sum(q), static_cast<float>(n)), eps));
+    s1 = rsqrtf(__fadd_rn(__fmul_rn(first, inv_n), eps));
   }
+}
+
+// per-partial terms of the second sweep
+template <int OP>
+__device__ __forceinline__ float second_term(const float4 &pt, float first) {
+  if constexpr (OP == kSoftmax || OP == kLogSoftmax) {
+    return pt.x == -INFINITY ? 0.f : __fmul_rn(pt.y, exp_shifted(pt.x, first));
+  } else {
+    const float d = __fsub_rn(pt.y, first);
+    return __fmaf_rn(__fmul_rn(pt.w, d), d, pt.z);
+  }
+}
+
+template <int OP>
+__device__ __forceinline__ void combine_short(const float4 *part, int K, float inv_n, float eps,
+                                              int lane, float &s0, float &s1) {
+  constexpr bool kMax = (OP == kSoftmax || OP == kLogSoftmax);
+  const float4 z = make_float4(kMax ? -INFINITY : 0.f, 0.f, 0.f, 0.f);
+  const float4 p0 = lane < K ? part[lane] : z;
+  const float4 p1 = lane + 32 < K ? part[lane + 32] : z;
+  float first;
+  if constexpr (kMax) {
+    first = warp_max(fmaxf(p0.x, p1.x));
+  } else {
+    first = warp_sum(__fadd_rn(p0.x, p1.x));
+    if constexpr (OP == kLayerNorm) first = __fmul_rn(first, inv_n);
+  }
+  float second = 0.f;
+  if constexpr (OP != kRmsNorm) {
+    float v = lane < K ? second_term<OP>(p0, first) : 0.f;
+    if (lane + 32 < K) v = __fadd_rn(v, second_term<OP>(p1, first));
+    second = warp_sum(v);
+  }
+  finish_stats<OP>(first, second, inv_n, eps, s0, s1);
+}
+
+template <int OP>
+__device__ __forceinline__ void combine_long(const float4 *part, int K, float inv_n, float eps,
+                                             int tid, int lane, int warp, volatile float *xw,
+                                             float &s0, float &s1) {
+  constexpr bool kMax = (OP == kSoftmax || OP == kLogSoftmax);
+  float v = kMax ? -INFINITY : 0.f;
+  for (int t = tid; t < K; t += kConsumerThreads)
+    v = kMax ? fmaxf(v, part[t].x) : __fadd_rn(v, part[t].x);
+  v = kMax ? warp_max(v) : warp_sum(v);
+  if (lane == 0) xw[warp] = v;
+  named_sync(kBarConsumers, kConsumerThreads);
+  float first = xw[0];
+  for (int w = 1; w < kConsumerWarps; ++w) first = kMax ? fmaxf(first, xw[w]) : __fadd_rn(first, xw[w]);
+  if constexpr (OP == kLayerNorm) first = __fmul_rn(first, inv_n);
+  float second = 0.f;
+  if constexpr (OP != kRmsNorm) {
+    float u = 0.f;
+    for (int t = tid; t < K; t += kConsumerThreads) u = __fadd_rn(u, second_term<OP>(part[t], first));
+    u = warp_sum(u);
+    if (lane == 0) xw[kConsumerWarps + warp] = u;
+    named_sync(kBarConsumers, kConsumerThreads);
+    second = xw[kConsumerWarps];
+    for (int w = 1; w < kConsumerWarps; ++w) second = __fadd_rn(second, xw[kConsumerWarps + w]);
+  }
+  finish_stats<OP>(first, second, inv_n, eps, s0, s1);
 }
 
 // pass 2: normalise tile t from the stage and store it
 template <int OP, typename T, bool EXACT>
-__device__ __forceinline__ void tile_store(const unsigned char *tsm, int64_t t, const ItemGeo &g,
+__device__ __forceinline__ void tile_store(const unsigned char *tsm, int t, const ItemGeo &g,
                                            int lane, float s0, float s1, const TileParams &p,
                                            char *owin, T *out_row) {
   constexpr int E = Elem<T>::kPerChunk;
   constexpr int NP = E / 2;
   const bool full = tile_is_full(t, g);  // the row's last tile may hold < 64 chunks
-  const int64_t hn = g.h + g.n;
+  const int hn = g.h + static_cast<int>(g.n);
   const T *gamma = static_cast<const T *>(p.gamma);
   const T *beta = static_cast<const T *>(p.beta);
 #pragma unroll
   for (int u = 0; u < 2; ++u) {
-    const int64_t c = t * kTileChunks + lane + 32 * u;
+    const int c = t * kTileChunks + lane + 32 * u;
     if (!full && c >= g.nc) continue;
     f2 v[NP];
     chunk_to_pairs(*reinterpret_cast<const uint4 *>(tsm + (lane + 32 * u) * kChunkBytes), v);
@@ -266,16 +436,134 @@ __device__ __forceinline__ void tile_store(const unsigned char *tsm, int64_t t, 
   }
 }
 
+// gamma/beta chunk for window chunk c of a row with compile-time head offset
+// H; every column it covers is inside [0, glen) and the vector is 16-byte
+// aligned (the caller checked).
+template <typename T, int H>
+__device__ __forceinline__ uint4 param_chunk_fixed(const T *__restrict__ g, int c) {
+  constexpr int E = Elem<T>::kPerChunk;
+  const uint4 *v = reinterpret_cast<const uint4 *>(g);
+  if constexpr (H == 0) {
+    return __ldg(v + c);
+  } else {
+    const uint4 A = __ldg(v + (c - 1));
+    const uint4 B = __ldg(v + c);
+    if constexpr (E == 4) {
+      return shift_words<H>(A, B);
+    } else if constexpr ((H & 1) == 0) {
+      return shift_words<H / 2>(A, B);
+    } else {
+      return shift_half<(H + 1) / 2>(A, B);
+    }
+  }
+}
+
+// pass 2 fast path: tile t lies entirely in the row, the output takes
+// 128-bit stores, and (norms) gamma/beta cover the tile's columns with
+// aligned vector loads.  Same arithmetic as tile_store.
+template <int OP, typename T, int H>
+__device__ __forceinline__ void tile_store_fast(const unsigned char *tsm, int t, int lane,
+                                                float s0, float s1, const T *gamma,
+                                                const T *beta, char *owin) {
+  constexpr int NP = Elem<T>::kPerChunk / 2;
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    const int c = t * kTileChunks + lane + 32 * u;
+    f2 v[NP], g[NP], b[NP];
+    chunk_to_pairs(*reinterpret_cast<const uint4 *>(tsm + (lane + 32 * u) * kChunkBytes), v);
+    if constexpr (OP == kLayerNorm || OP == kRmsNorm)
+      chunk_to_pairs(param_chunk_fixed<T, H>(gamma, c), g);
+    if constexpr (OP == kLayerNorm) chunk_to_pairs(param_chunk_fixed<T, H>(beta, c), b);
+    normalize_pairs<OP, NP>(v, s0, s1, g, b);
+    stg_stream(owin + static_cast<int64_t>(c) * kChunkBytes, pairs_to_chunk(v));
+  }
+}
+
+// Whether tile t of an item takes the pass-2 fast path.
+template <int OP, typename T>
+__device__ __forceinline__ bool tile_fast(int t, const ItemGeo &g, const TileParams &p,
+                                          bool params_ok) {
+  constexpr int E = Elem<T>::kPerChunk;
+  constexpr bool kAffine = (OP == kLayerNorm || OP == kRmsNorm);
+  // the vector parameter loads reach column (t + 1) * 64 * E - 1 at most
+  return tile_is_full(t, g) && p.out_vec && params_ok &&
+         (!kAffine || static_cast<int64_t>(t + 1) * kTileChunks * E <= p.glen);
+}
+
+// pass 2 fast path over this warp's tiles of an item whose head offset is H
+template <int OP, typename T, int H>
+__device__ __forceinline__ void pass2_fast_tiles(const unsigned char *stage, const ItemGeo &g,
+                                                 int warp, int lane, float s0, float s1,
+                                                 const TileParams &p, char *owin,
+                                                 bool params_ok) {
+  const T *gamma = static_cast<const T *>(p.gamma);
+  const T *beta = static_cast<const T *>(p.beta);
+  const int ntl = g.t1 - g.t0;
+  for (int lt = warp; lt < ntl; lt += kConsumerWarps) {
+    const int t = g.t0 + lt;
+    if (tile_fast<OP, T>(t, g, p, params_ok))
+      tile_store_fast<OP, T, H>(stage + lt * kTileBytes, t, lane, s0, s1, gamma, beta, owin);
+  }
+}
+
+// pass 2 of an item: the fast tiles with the gamma/beta realignment compiled
+// for the item's head offset (one dispatch per item, not per chunk), then the
+// tiles the fast path does not take (the row's ends, unaligned output, rows
+// reaching the end of gamma/beta) through the general path.
+template <int OP, typename T, bool EXACT>
+__device__ __forceinline__ void pass2_item(const unsigned char *stage, const ItemGeo &g, int warp,
+                                           int lane, float s0, float s1, const TileParams &p,
+                                           char *owin, T *out_row) {
+  constexpr int E = Elem<T>::kPerChunk;
+  constexpr bool kAffine = (OP == kLayerNorm || OP == kRmsNorm);
+  const bool params_ok =
+      !kAffine || (p.gvec && p.gamma && (OP == kRmsNorm || p.beta != nullptr));
+  if constexpr (EXACT || !kAffine) {
+    pass2_fast_tiles<OP, T, 0>(stage, g, warp, lane, s0, s1, p, owin, params_ok);
+  } else {
+    switch (g.h) {
+      case 0: pass2_fast_tiles<OP, T, 0>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
+      case 1: pass2_fast_tiles<OP, T, 1>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
+      case 2: pass2_fast_tiles<OP, T, 2>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
+      case 3: pass2_fast_tiles<OP, T, 3>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
+      default:
+        if constexpr (E == 8) {
+          switch (g.h) {
+            case 4: pass2_fast_tiles<OP, T, 4>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
+            case 5: pass2_fast_tiles<OP, T, 5>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
+            case 6: pass2_fast_tiles<OP, T, 6>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
+            default: pass2_fast_tiles<OP, T, 7>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
+          }
+        }
+        break;
+    }
+  }
+  const int ntl = g.t1 - g.t0;
+  for (int lt = warp; lt < ntl; lt += kConsumerWarps) {
+    const int t = g.t0 + lt;
+    if (!tile_fast<OP, T>(t, g, p, params_ok))
+      tile_store<OP, T, EXACT>(stage + lt * kTileBytes, t, g, lane, s0, s1, p, owin, out_row);
+  }
+}
+
 // ---------------------------------------------------------------------------
 // producer: edge chunks loaded now, written into the stage one item later
 // ---------------------------------------------------------------------------
+// The head chunk (window chunk 0) and the tail chunk (the last) of an item,
+// in fixed fields so nothing is indexed at run time.
 struct PendingEdges {
-  int count;  // chunks pending; -1 = nothing pending
-  int nbars;
-  uint32_t dst[2];
-  uint4 val[2];
-  uint32_t bar[2];
+  bool active;        // an item's edges still have to be written
+  bool head, tail;    // which edge chunks it has
+  bool tail_own_bar;  // the tail chunk lies in another piece than the head
+  uint32_t head_dst, tail_dst, head_bar, tail_bar;
+  uint4 head_val, tail_val;
 };
+
+__device__ __forceinline__ void st_shared_u4(uint32_t dst, const uint4 &v) {
+  asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(v.x), "r"(v.y),
+               "r"(v.z), "r"(v.w)
+               : "memory");
+}
 
 __device__ __forceinline__ uint32_t ld_u16_issue(const void *p) {
   unsigned short v;
@@ -307,14 +595,12 @@ __device__ __forceinline__ uint4 issue_edge_chunk(const T *in_row, int64_t c, in
 }
 
 __device__ __forceinline__ void complete_pending(PendingEdges &pe) {
-  if (pe.count < 0) return;
-  for (int i = 0; i < pe.count; ++i) {
-    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(pe.dst[i]), "r"(pe.val[i].x),
-                 "r"(pe.val[i].y), "r"(pe.val[i].z), "r"(pe.val[i].w)
-                 : "memory");
-  }
-  for (int i = 0; i < pe.nbars; ++i) mbar_arrive(pe.bar[i]);
-  pe.count = -1;
+  if (!pe.active) return;
+  if (pe.head) st_shared_u4(pe.head_dst, pe.head_val);
+  if (pe.tail) st_shared_u4(pe.tail_dst, pe.tail_val);
+  if (pe.head) mbar_arrive(pe.head_bar);
+  if (pe.tail && (pe.tail_own_bar || !pe.head)) mbar_arrive(pe.tail_bar);
+  pe.active = false;
 }
 
 template <typename T, bool EXACT, bool CLUSTER, bool RAGGED>
@@ -330,25 +616,15 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
   int64_t k_large = 0, k_dense = 0;
   bool medium_phase = false;
   PendingEdges pend;
-  pend.count = -1;
+  pend.active = false;
   uint32_t fill_mask = 0, fill_parity = 0;
 
-  for (int64_t it = 0;; ++it) {
-    const int s = static_cast<int>(it % S);
-    if (it >= S) {
-      if (!mbar_wait_bounded(sbase + L.bar_empty + 8u * s,
-                             static_cast<uint32_t>(((it / S) - 1) & 1), p.timeout_ns)) {
-        atomicOr(p.status, kStatusTimeout);
-        flags[0] = 1;
-        break;
-      }
-      fill_mask &= ~(1u << s);
-    }
-    if (flags[0]) break;
-    complete_pending(pend);
-
-    int kind = kItemEnd;
-    int64_t start = 0, n = 0;
+  // The next item of this CTA: its record is fetched one step ahead, so the
+  // load (and the work-counter round trip) overlaps the wait for a free stage.
+  auto fetch = [&](int &kind, int64_t &start, int64_t &n) {
+    kind = kItemEnd;
+    start = 0;
+    n = 0;
     if (RAGGED) {
       if (!medium_phase) {
         const int64_t li = cid + k_large * ncl;
@@ -380,6 +656,28 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
         n = p.cols;
       }
     }
+  };
+  int next_kind;
+  int64_t next_start, next_n;
+  fetch(next_kind, next_start, next_n);
+
+  for (int64_t it = 0;; ++it) {
+    const int s = static_cast<int>(it % S);
+    const int kind = next_kind;
+    const int64_t start = next_start, n = next_n;
+    if (kind != kItemEnd) fetch(next_kind, next_start, next_n);
+    if (it >= S) {
+      if (!mbar_wait_bounded(sbase + L.bar_empty + 8u * s,
+                             static_cast<uint32_t>(((it / S) - 1) & 1), p.timeout_ns)) {
+        atomicOr(p.status, kStatusTimeout);
+        flags[0] = 1;
+        break;
+      }
+      fill_mask &= ~(1u << s);
+    }
+    if (flags[0]) break;
+    complete_pending(pend);
+
     meta[s].start = start;
     meta[s].n = n;
     meta[s].kind = kind;
@@ -402,8 +700,8 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
       const uint32_t bar = sbase + L.bar_piece + 8u * (s * L.pieces + pc);
       const int64_t q0 = c0 + static_cast<int64_t>(pc) * kPieceTiles * kTileChunks;
       const int64_t q1 = min(c1, q0 + kPieceTiles * kTileChunks);
-      const int64_t b0 = max(q0, g.cf);
-      const int64_t b1 = min(q1, g.cl);
+      const int64_t b0 = max(q0, static_cast<int64_t>(g.cf));
+      const int64_t b1 = min(q1, static_cast<int64_t>(g.cl));
       const uint32_t bytes = (q0 < c1 && b1 > b0) ? static_cast<uint32_t>((b1 - b0) * kChunkBytes)
                                                   : 0u;
       const bool edge = (head && pc == head_pc) || (tail && pc == tail_pc);
@@ -427,21 +725,16 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
     }
     if (head || tail) {
       PendingEdges pe;
-      pe.count = 0;
-      pe.nbars = 0;
-      if (head) {
-        pe.dst[pe.count] = stage;
-        pe.val[pe.count] = issue_edge_chunk<T>(in_row, 0, g.h, g.n);
-        ++pe.count;
-        pe.bar[pe.nbars++] = sbase + L.bar_piece + 8u * (s * L.pieces + head_pc);
-      }
-      if (tail) {
-        pe.dst[pe.count] = stage + static_cast<uint32_t>((g.nc - 1 - c0) * kChunkBytes);
-        pe.val[pe.count] = issue_edge_chunk<T>(in_row, g.nc - 1, g.h, g.n);
-        ++pe.count;
-        if (!(head && tail_pc == head_pc))
-          pe.bar[pe.nbars++] = sbase + L.bar_piece + 8u * (s * L.pieces + tail_pc);
-      }
+      pe.active = true;
+      pe.head = head;
+      pe.tail = tail;
+      pe.tail_own_bar = tail && !(head && tail_pc == head_pc);
+      pe.head_dst = stage;
+      pe.head_bar = sbase + L.bar_piece + 8u * (s * L.pieces + head_pc);
+      pe.tail_dst = stage + static_cast<uint32_t>((g.nc - 1 - c0) * kChunkBytes);
+      pe.tail_bar = sbase + L.bar_piece + 8u * (s * L.pieces + (tail ? tail_pc : 0));
+      pe.head_val = head ? issue_edge_chunk<T>(in_row, 0, g.h, g.n) : make_uint4(0, 0, 0, 0);
+      pe.tail_val = tail ? issue_edge_chunk<T>(in_row, g.nc - 1, g.h, g.n) : make_uint4(0, 0, 0, 0);
       pend = pe;
       if (S == 1) complete_pending(pend);
     }
@@ -500,12 +793,15 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
   }
 
   // ------------------------------ consumers ------------------------------
-  int64_t uses[2] = {0, 0};  // cluster items that used part_c[b]
+  // cluster items that used part_c[0] / part_c[1] (kept as scalars: a
+  // runtime-indexed array would live in local memory)
+  uint32_t uses0 = 0, uses1 = 0;
   bool ended = false;
   for (int64_t it = 0;; ++it) {
     const int s = static_cast<int>(it % S);
     const uint32_t par = static_cast<uint32_t>((it / S) & 1);
     const int b = static_cast<int>(it & 1);
+    const uint32_t uses_b = b ? uses1 : uses0;
     bool bad = !mbar_wait_bounded(sbase + L.bar_meta + 8u * s, par, p.timeout_ns);
     int kind = kItemEnd;
     ItemGeo g;
@@ -516,33 +812,20 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
       if (kind != kItemEnd) {
         const bool split = CLUSTER && kind == kItemLarge;
         g = item_geo<T, EXACT>(p.in, meta[s].start, meta[s].n, split, rank, cs);
-        if (split && uses[b] > 0)
-          bad = !mbar_wait_cluster_bounded(sbase + L.bar_released + 8u * b,
-                                           static_cast<uint32_t>((uses[b] - 1) & 1), p.timeout_ns);
+        if (split && uses_b > 0)
+          bad = !mbar_wait_cluster_bounded(sbase + L.bar_released + 8u * b, (uses_b - 1) & 1,
+                                           p.timeout_ns);
       }
     }
     const bool split = CLUSTER && kind == kItemLarge;
     const unsigned char *stage = smem + static_cast<size_t>(s) * p.stage_bytes;
-    const int64_t ntl = g.t1 - g.t0;
+    const int ntl = g.t1 - g.t0;
     float4 *part = (split ? part_c : part_m) + static_cast<size_t>(b) * p.max_tiles;
 
     // ---- pass 1 ----
-    if (!bad && kind != kItemEnd) {
-      int waited = -1;
-      for (int64_t lt = warp; lt < ntl; lt += kConsumerWarps) {
-        const int pc = static_cast<int>(lt / kPieceTiles);
-        if (pc != waited) {
-          if (!mbar_wait_bounded(sbase + L.bar_piece + 8u * (s * L.pieces + pc), par,
-                                 p.timeout_ns)) {
-            bad = true;
-            break;
-          }
-          waited = pc;
-        }
-        const float4 pt = tile_partial<OP, T, EXACT>(stage + lt * kTileBytes, g.t0 + lt, g, lane);
-        if (lane == 0) part[lt] = pt;
-      }
-    }
+    if (!bad && kind != kItemEnd)
+      bad = !pass1_warp<OP, T>(stage, g, warp, lane, part,
+                               sbase + L.bar_piece + 8u * (s * L.pieces), par, p.timeout_ns);
     if (named_sync_or(kBarConsumers, kConsumerThreads, bad)) {
       if (tid == 0) {
         atomicOr(p.status, kStatusTimeout);
@@ -559,17 +842,31 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
     const float4 *src = part;
     if (split) {
       const uint32_t ready = sbase + L.bar_ready + 8u * b;
-      if (tid == 0)
-        for (int r = 0; r < cs; ++r) mbar_arrive_remote(ready, static_cast<uint32_t>(r));
-      bool ok = mbar_wait_cluster_bounded(ready, static_cast<uint32_t>(uses[b] & 1), p.timeout_ns);
+      // thread r signals rank r; the named barrier above already ordered
+      // every warp's partial writes before these releases
+      if (tid < cs) mbar_arrive_remote(ready, static_cast<uint32_t>(tid));
+      bool ok = mbar_wait_cluster_bounded(ready, uses_b & 1, p.timeout_ns);
       if (ok) {
-        const int64_t tpc = (g.K + cs - 1) / cs;
+        const int tpc = (g.K + cs - 1) / cs;
         const uint32_t mine = smem_addr(part_c + static_cast<size_t>(b) * p.max_tiles);
-        for (int64_t t = tid; t < g.K; t += kConsumerThreads) {
-          const int64_t r = t / tpc;
-          gather[t] = ld_dsmem_f4(map_to_rank(mine + static_cast<uint32_t>((t - r * tpc) * 16),
-                                              static_cast<uint32_t>(r)));
+        auto peer_addr = [&](int t) {
+          const int r = t / tpc;
+          return map_to_rank(mine + static_cast<uint32_t>((t - r * tpc) * 16),
+                             static_cast<uint32_t>(r));
+        };
+        // four loads in flight per thread before their results are stored
+        int t = tid;
+        for (; t + 3 * kConsumerThreads < g.K; t += 4 * kConsumerThreads) {
+          const float4 v0 = ld_dsmem_f4(peer_addr(t));
+          const float4 v1 = ld_dsmem_f4(peer_addr(t + kConsumerThreads));
+          const float4 v2 = ld_dsmem_f4(peer_addr(t + 2 * kConsumerThreads));
+          const float4 v3 = ld_dsmem_f4(peer_addr(t + 3 * kConsumerThreads));
+          gather[t] = v0;
+          gather[t + kConsumerThreads] = v1;
+          gather[t + 2 * kConsumerThreads] = v2;
+          gather[t + 3 * kConsumerThreads] = v3;
         }
+        for (; t < g.K; t += kConsumerThreads) gather[t] = ld_dsmem_f4(peer_addr(t));
       }
       if (named_sync_or(kBarConsumers, kConsumerThreads, !ok)) {
         if (tid == 0) {
@@ -578,21 +875,27 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
         }
         break;
       }
-      if (tid == 0)
-        for (int r = 0; r < cs; ++r)
-          mbar_arrive_remote(sbase + L.bar_released + 8u * b, static_cast<uint32_t>(r));
-      ++uses[b];
+      if (tid < cs) mbar_arrive_remote(sbase + L.bar_released + 8u * b, static_cast<uint32_t>(tid));
+      if (b) {
+        ++uses1;
+      } else {
+        ++uses0;
+      }
       src = gather;
     }
     float s0, s1;
-    combine_stats<OP>(src, g.K, g.n, p.eps, lane, s0, s1);
+    const float inv_n = __frcp_rn(static_cast<float>(g.n));
+    if (g.K <= kShortCombineTiles) {
+      combine_short<OP>(src, g.K, inv_n, p.eps, lane, s0, s1);
+    } else {
+      combine_long<OP>(src, g.K, inv_n, p.eps, tid, lane, warp,
+                       reinterpret_cast<volatile float *>(smem + L.xw), s0, s1);
+    }
 
     // ---- pass 2 ----
     T *out_row = static_cast<T *>(p.out) + g.start;
     char *owin = reinterpret_cast<char *>(out_row) - g.h * SZ;
-    for (int64_t lt = warp; lt < ntl; lt += kConsumerWarps)
-      tile_store<OP, T, EXACT>(stage + lt * kTileBytes, g.t0 + lt, g, lane, s0, s1, p, owin,
-                               out_row);
+    pass2_item<OP, T, EXACT>(stage, g, warp, lane, s0, s1, p, owin, out_row);
     __syncwarp();
     if (lane == 0) mbar_arrive(sbase + L.bar_empty + 8u * s);
   }
@@ -636,24 +939,17 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
         return *reinterpret_cast<const uint4 *>(slice + (sub + static_cast<int64_t>(k) * G) *
                                                             kChunkBytes);
       };
-      const int cpl = small_cpl_class((rec.n + E - 1) / E + 1, G);
-      if (cpl == 4) {
-        small_row_core<OP, T, 4, false>(get, out + rec.start, rec.n, h, ncg, G, sub, sa);
-      } else if (cpl == 8) {
-        small_row_core<OP, T, 8, false>(get, out + rec.start, rec.n, h, ncg, G, sub, sa);
-      } else {
-        small_row_core<OP, T, 9, false>(get, out + rec.start, rec.n, h, ncg, G, sub, sa);
-      }
+      small_row_core<OP, T, 9, false, false>(get, out + rec.start, rec.n, h, ncg, G, sub, sa);
       __syncwarp();
     }
   }
 
   // ---- no CTA leaves while a peer may still read its partials ----
   if (CLUSTER) {
-    for (int bb = 0; bb < 2; ++bb)
-      if (uses[bb] > 0)
-        (void)mbar_wait_cluster_bounded(sbase + L.bar_released + 8u * bb,
-                                        static_cast<uint32_t>((uses[bb] - 1) & 1), p.timeout_ns);
+    if (uses0 > 0)
+      (void)mbar_wait_cluster_bounded(sbase + L.bar_released, (uses0 - 1) & 1, p.timeout_ns);
+    if (uses1 > 0)
+      (void)mbar_wait_cluster_bounded(sbase + L.bar_released + 8u, (uses1 - 1) & 1, p.timeout_ns);
   }
 
   // ---- ragged: the last CTA to finish resets the work counters, so a plan
