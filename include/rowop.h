@@ -187,6 +187,32 @@ ROWOP_API int rowop_rmsnorm_ragged_planned(const void *in, void *out,
                                            float eps, void *ws, size_t ws_bytes,
                                            cudaStream_t stream);
 
+/* ---- ragged LayerNorm without a caller workspace ---------------------------
+ * The paper has no counterpart: this is a library convenience for callers
+ * that must not allocate (or cannot pass) device memory for the workspace.
+ * rowop_layernorm_ragged with the same arguments minus ws / ws_bytes: the
+ * workspace is a fixed array in the library's device memory, sized for
+ * ROWOP_STATIC_MAX_ROWS rows (about 3.2 MB), one per device.  Nothing is
+ * allocated or freed by the call.  Results equal those of
+ * rowop_layernorm_ragged bit for bit.
+ *   rows > ROWOP_STATIC_MAX_ROWS  -> ROWOP_ERR_WORKSPACE, nothing launched.
+ * The first call on a device looks the array's address up (a CUDA runtime
+ * query, made with that device current); make it before capturing the stream
+ * into a graph.  Every call starts with the classify pass, which rewrites the
+ * per-call state the fused kernel needs zeroed (bucket counts, work counters,
+ * status) before that kernel reads it, so nothing carries over from a
+ * previous call.  All calls on one device share the one array: calls that
+ * may run at the same time (on different streams, or from different host
+ * threads without ordering) race on it and give undefined results.  The
+ * bucket bytes described for ws above are not exposed. */
+#define ROWOP_STATIC_MAX_ROWS 65536
+
+ROWOP_API int rowop_layernorm_ragged_static(const void *in, void *out,
+                                            const void *gamma, const void *beta,
+                                            const int64_t *offsets, int64_t rows,
+                                            int64_t max_len, rowop_dtype_t dtype,
+                                            float eps, cudaStream_t stream);
+
 /* ---- dispatch rule, limits, status ---------------------------------------- */
 
 /* launch_by_rows (§2.1): the bucket for a row of len elements (len >= 0):

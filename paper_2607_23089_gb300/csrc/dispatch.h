@@ -50,10 +50,10 @@ constexpr size_t kWsCounts = 64;
 constexpr size_t kWsCounters = 128;
 constexpr size_t kWsBuckets = 256;
 constexpr size_t kWsRecordBytes = 16;
-inline size_t ragged_lists_offset(int64_t rows) {
+constexpr size_t ragged_lists_offset(int64_t rows) {
   return (kWsBuckets + static_cast<size_t>(rows) + 255) & ~static_cast<size_t>(255);
 }
-inline size_t ragged_ws_bytes(int64_t rows) {
+constexpr size_t ragged_ws_bytes(int64_t rows) {
   return ragged_lists_offset(rows) + 3 * kWsRecordBytes * static_cast<size_t>(rows) + 256;
 }
 

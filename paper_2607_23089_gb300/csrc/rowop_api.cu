@@ -90,6 +90,34 @@ static int device_info(DeviceInfo *out) {
   return ROWOP_OK;
 }
 
+// Library-owned ragged workspace of rowop_layernorm_ragged_static: one array
+// per device (a __device__ variable has one instance in every device's
+// context), sized for ROWOP_STATIC_MAX_ROWS rows.
+constexpr size_t kStaticWsBytes = ragged_ws_bytes(ROWOP_STATIC_MAX_ROWS);
+static __device__ __align__(256) unsigned char g_static_ws[kStaticWsBytes];
+
+// Address of the current device's g_static_ws, looked up once per device.
+static int static_workspace(void **ws) {
+  static std::mutex mu;
+  static void *addr[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    cudaGetLastError();
+    return ROWOP_ERR_CUDA;
+  }
+  std::lock_guard<std::mutex> lk(mu);
+  if (!addr[dev]) {
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_ws) != cudaSuccess || p == nullptr) {
+      cudaGetLastError();
+      return ROWOP_ERR_CUDA;
+    }
+    addr[dev] = p;
+  }
+  *ws = addr[dev];
+  return ROWOP_OK;
+}
+
 static int esize_of(int dtype) { return dtype == ROWOP_F32 ? 4 : (dtype == ROWOP_BF16 ? 2 : 0); }
 
 static bool elem_aligned(const void *p, int esize) {
@@ -307,6 +335,21 @@ int rowop_rmsnorm_ragged_planned(const void *in, void *out, const void *gamma,
                                  cudaStream_t stream) {
   return run_ragged(kRmsNorm, in, out, gamma, nullptr, offsets, rows, max_len, dtype, eps, ws,
                     ws_bytes, stream, false);
+}
+
+int rowop_layernorm_ragged_static(const void *in, void *out, const void *gamma,
+                                  const void *beta, const int64_t *offsets, int64_t rows,
+                                  int64_t max_len, rowop_dtype_t dtype, float eps,
+                                  cudaStream_t stream) {
+  if (rows > ROWOP_STATIC_MAX_ROWS) return ROWOP_ERR_WORKSPACE;
+  if (rows <= 0)  // nothing to stage: same checks and result as the caller-workspace call
+    return run_ragged(kLayerNorm, in, out, gamma, beta, offsets, rows, max_len, dtype, eps,
+                      nullptr, 0, stream, true);
+  void *ws = nullptr;
+  const int st = static_workspace(&ws);
+  if (st != ROWOP_OK) return st;
+  return run_ragged(kLayerNorm, in, out, gamma, beta, offsets, rows, max_len, dtype, eps, ws,
+                    kStaticWsBytes, stream, true);
 }
 
 int rowop_select_bucket(int64_t len, rowop_dtype_t dtype) {

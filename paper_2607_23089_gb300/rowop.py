@@ -57,6 +57,7 @@ SIGNATURES = {
     "rowop_layernorm_ragged_planned": ([_P, _P, _P, _P, _P, _I64, _I64, _I, _F, _P, _SZ,
                                         _P], _I),
     "rowop_rmsnorm_ragged_planned": ([_P, _P, _P, _P, _I64, _I64, _I, _F, _P, _SZ, _P], _I),
+    "rowop_layernorm_ragged_static": ([_P, _P, _P, _P, _P, _I64, _I64, _I, _F, _P], _I),
     "rowop_select_bucket": ([_I64, _I], _I),
     "rowop_max_row_len": ([_I], _I64),
     "rowop_status_string": ([_I], ctypes.c_char_p),
