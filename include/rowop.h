@@ -188,11 +188,16 @@ ROWOP_API int rowop_rmsnorm_ragged_planned(const void *in, void *out,
                                            cudaStream_t stream);
 
 /* ---- ragged LayerNorm without a caller workspace ---------------------------
- * The paper has no counterpart: this is a library convenience for callers
- * that must not allocate (or cannot pass) device memory for the workspace.
+ * The paper has no counterpart: this is a library convenience.  Some callers
+ * cannot provide the workspace: a kernel plugin inside another runtime (an
+ * inference engine, a framework's custom-op slot) is handed only its input
+ * and output buffers and has no allocator of its own to ask; and code on a
+ * latency-critical path often may not call cudaMalloc / cudaFree, which can
+ * synchronise the device and stall every stream.  For them this is
  * rowop_layernorm_ragged with the same arguments minus ws / ws_bytes: the
  * workspace is a fixed array in the library's device memory, sized for
- * ROWOP_STATIC_MAX_ROWS rows (about 3.2 MB), one per device.  Nothing is
+ * ROWOP_STATIC_MAX_ROWS rows (about 3.2 MB), one per device, held by every
+ * GPU that loads the library until the process exits.  Nothing is
  * allocated or freed by the call.  Results equal those of
  * rowop_layernorm_ragged bit for bit.
  *   rows > ROWOP_STATIC_MAX_ROWS  -> ROWOP_ERR_WORKSPACE, nothing launched.

@@ -1,6 +1,7 @@
 """rowop_layernorm_ragged_static, the ragged LayerNorm entry point that takes
 its workspace from a fixed array inside the library instead of caller
-memory.  Called through the C ABI and compared, bit for bit, with
+memory, for callers that cannot allocate one (a plugin that is handed only
+its input and output buffers, a path that may not call cudaMalloc).  Called through the C ABI and compared, bit for bit, with
 rowop_layernorm_ragged on a caller-owned workspace, on calls made one after
 another (so any state left over from the previous call would show), at the
 largest row count it accepts, and one row beyond it (rejected).  Collected
