@@ -72,11 +72,13 @@ inline int64_t max_row_len_elems(int esize) {
 //   ROWOP_CLUSTER       cluster size for split rows (1, 2, 4, 8, 16)
 //   ROWOP_STAGES        stage-ring depth of the tile kernel
 //   ROWOP_CTAS_PER_SM   upper bound on resident tile-kernel CTAs per SM
+//   ROWOP_GROUP_WARPS   consumer warps per item group of the tile kernel (1, 2, 4, 8)
 struct Knobs {
   int force_bucket = -1;
   int cluster = 0;
   int stages = 0;
   int ctas_per_sm = 0;
+  int group_warps = 0;
 };
 Knobs read_knobs();
 

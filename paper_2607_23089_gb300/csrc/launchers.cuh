@@ -124,26 +124,40 @@ cudaError_t launch_small(const DenseCall &c, const DeviceInfo &d, bool exact, bo
 // ---------------------------------------------------------------------------
 // MEDIUM / LARGE / ragged: the tile kernel
 // ---------------------------------------------------------------------------
-// min_stage_area: bytes the stages must span together (ragged SMALL staging)
+// group_warps: consumer warps per item group (W); the stage ring holds at
+// least one item per group.  min_stage_area: bytes the stages must span
+// together (ragged SMALL staging).
 template <int OP, typename T, bool EXACT, bool CLUSTER, bool RAGGED>
-cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int64_t items,
-                          const DeviceInfo &d, cudaStream_t stream, uint32_t min_stage_area = 0) {
+cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int group_warps,
+                          int64_t items, const DeviceInfo &d, cudaStream_t stream,
+                          uint32_t min_stage_area = 0) {
   auto kern = tile_row_kernel<OP, T, EXACT, CLUSTER, RAGGED>;
   const void *kp = reinterpret_cast<const void *>(kern);
   const int max_ctas_per_sm = read_knobs().ctas_per_sm;
   p.stage_bytes = static_cast<uint32_t>(stage_tiles) * kTileBytes;
   p.max_tiles = stage_tiles;
-  p.gather_tiles = CLUSTER ? cs * stage_tiles : 0;
   while (static_cast<uint64_t>(stages) * p.stage_bytes < min_stage_area) ++stages;
-  const auto total = [&](int s) {
-    return TileSmemLayout(p.stage_bytes, s, stage_tiles, p.gather_tiles).total;
+  const auto total = [&](int s, int w) {
+    return TileSmemLayout(p.stage_bytes, s, stage_tiles, kConsumerWarps / w, CLUSTER,
+                          !CLUSTER || RAGGED).total;
   };
-  // as many of the wanted stages as fit in the CTA's shared memory
-  while (stages > 1 && total(stages) > static_cast<uint32_t>(d.max_smem_optin)) --stages;
+  // as many of the wanted stages as fit in the CTA's shared memory, at least
+  // one per group: fewer, larger groups when even that does not fit
+  const uint32_t optin = static_cast<uint32_t>(d.max_smem_optin);
+  int W = group_warps;
+  stages = std::max(stages, kConsumerWarps / W);
+  for (;;) {
+    const int G = kConsumerWarps / W;
+    while (stages > G && total(stages, W) > optin) --stages;
+    if (total(stages, W) <= optin) break;
+    if (W == kConsumerWarps) return cudaErrorInvalidConfiguration;
+    W *= 2;
+  }
   if (static_cast<uint64_t>(stages) * p.stage_bytes < min_stage_area)
     return cudaErrorInvalidConfiguration;
   p.stages = stages;
-  const size_t smem = total(stages);
+  p.group_warps = W;
+  const size_t smem = total(stages, W);
   if (smem > static_cast<size_t>(d.max_smem_optin)) return cudaErrorInvalidConfiguration;
   cudaError_t e = prepare_kernel(kp, d, CLUSTER);
   if (e != cudaSuccess) return e;
@@ -178,10 +192,31 @@ cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int
   return cudaGetLastError();
 }
 
-inline int pick_stages(int stage_tiles, int knob) {
-  if (knob > 0) return std::min(knob, 16);
-  // about 32 KiB of stages per CTA, at least 2 so loads overlap compute
-  return std::max(2, std::min(8, 32 / std::max(1, stage_tiles)));
+// Consumer warps per item group.  Dense rows of a few tiles: several groups,
+// so one group's waits overlap the others' work while each warp still has a
+// few tiles per item.  Ragged launches keep one group of 8: their items are
+// of mixed size and two fixed-size stages per CTA is all that lets three
+// CTAs share an SM (measured fastest on the ragged workload).
+inline int pick_group_warps(int64_t stage_tiles, bool ragged, int knob) {
+  if (knob == 1 || knob == 2 || knob == 4 || knob == 8) return knob;
+  if (ragged) return 8;
+  if (stage_tiles <= 16) return 2;
+  if (stage_tiles <= 64) return 4;
+  return 8;
+}
+
+// Shared memory one CTA may spend on stages so that three CTAs fit an SM.
+constexpr int64_t kStageBudgetBytes = 72 * 1024;
+
+// Stages: at least one per group and up to one and a half per group within
+// the three-CTA budget; stages too large for that budget get two per group
+// (launch_tile_k then keeps as many as fit the CTA's shared memory).
+inline int pick_stages(int64_t stage_tiles, int group_warps, int knob) {
+  if (knob > 0) return std::min(knob, 32);
+  const int G = kConsumerWarps / group_warps;
+  const int64_t fit = kStageBudgetBytes / (stage_tiles * kTileBytes);
+  if (fit >= G) return static_cast<int>(std::max<int64_t>(2, std::min<int64_t>(G + G / 2, fit)));
+  return std::max(2, 2 * G);
 }
 
 // Smallest cluster (power of two, >= 2) whose portions of a K-tile row hold
@@ -226,23 +261,19 @@ cudaError_t launch_dense_t(const DenseCall &c, const DeviceInfo &d) {
   p.gvec = gvec;
   p.timeout_ns = kWaitLimitNs;
   p.status = d.status;
-  if (bucket == kMedium) {
-    const int st = static_cast<int>(K);
-    const int S = pick_stages(st, kn.stages);
-    if (exact) return launch_tile_k<OP, T, true, false, false>(p, 1, S, st, c.rows, d, c.stream);
-    return launch_tile_k<OP, T, false, false, false>(p, 1, S, st, c.rows, d, c.stream);
-  }
-  const int cs = pick_cluster(K, 64, kn.cluster);
+  // portions of up to 128 tiles: a 1 MiB fp32 row goes to clusters of 8
+  // (19 clusters fill the 152 SMs; 16-CTA clusters would leave 8 idle)
+  const int cs = bucket == kMedium ? 1 : pick_cluster(K, 128, kn.cluster);
   const int st = static_cast<int>(ceil_div(K, cs));
   if (st > kMaxPortionTiles) return cudaErrorInvalidValue;
-  // two stages when they fit, so the next portion loads while this one is used
-  const int S = kn.stages > 0 ? std::min(kn.stages, 16) : 2;
+  const int W = pick_group_warps(st, false, kn.group_warps);
+  const int S = pick_stages(st, W, kn.stages);
   if (cs == 1) {
-    if (exact) return launch_tile_k<OP, T, true, false, false>(p, 1, S, st, c.rows, d, c.stream);
-    return launch_tile_k<OP, T, false, false, false>(p, 1, S, st, c.rows, d, c.stream);
+    if (exact) return launch_tile_k<OP, T, true, false, false>(p, 1, S, st, W, c.rows, d, c.stream);
+    return launch_tile_k<OP, T, false, false, false>(p, 1, S, st, W, c.rows, d, c.stream);
   }
-  if (exact) return launch_tile_k<OP, T, true, true, false>(p, cs, S, st, c.rows, d, c.stream);
-  return launch_tile_k<OP, T, false, true, false>(p, cs, S, st, c.rows, d, c.stream);
+  if (exact) return launch_tile_k<OP, T, true, true, false>(p, cs, S, st, W, c.rows, d, c.stream);
+  return launch_tile_k<OP, T, false, true, false>(p, cs, S, st, W, c.rows, d, c.stream);
 }
 
 template <int OP>
@@ -292,12 +323,13 @@ cudaError_t launch_ragged_t(const RaggedCall &c, const DeviceInfo &d) {
     st = std::max<int64_t>(st, ceil_div(kmax, cs));
   }
   if (st > kMaxPortionTiles) return cudaErrorInvalidValue;
-  const int S = pick_stages(static_cast<int>(st), kn.stages);
+  const int W = pick_group_warps(st, true, kn.group_warps);
+  const int S = pick_stages(st, W, kn.stages);
   const uint32_t small_area = kConsumerWarps * kSmallSliceBytes;
   if (cs > 1)
-    return launch_tile_k<OP, T, false, true, true>(p, cs, S, static_cast<int>(st), c.rows, d,
+    return launch_tile_k<OP, T, false, true, true>(p, cs, S, static_cast<int>(st), W, c.rows, d,
                                                    c.stream, small_area);
-  return launch_tile_k<OP, T, false, false, true>(p, 1, S, static_cast<int>(st), c.rows, d,
+  return launch_tile_k<OP, T, false, false, true>(p, 1, S, static_cast<int>(st), W, c.rows, d,
                                                   c.stream, small_area);
 }
 

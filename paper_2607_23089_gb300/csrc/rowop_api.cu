@@ -38,6 +38,7 @@ Knobs read_knobs() {
   k.cluster = env_int("ROWOP_CLUSTER", 0);
   k.stages = env_int("ROWOP_STAGES", 0);
   k.ctas_per_sm = env_int("ROWOP_CTAS_PER_SM", 0);
+  k.group_warps = env_int("ROWOP_GROUP_WARPS", 0);
   return k;
 }
 

@@ -10,15 +10,21 @@
 //     while later ones land -- and reads the at most two 16-byte chunks the
 //     row only partly covers element by element (never outside the row),
 //     writing them into the stage one item later so their latency overlaps;
-//   * consumers reduce one 1 KiB tile per warp to a tile partial, meet at one
-//     named barrier per item, combine the K tile partials of the row in a
-//     fixed order (every warp redundantly, so no broadcast is needed),
-//     normalise their tiles from the stage, store with 128-bit streaming
-//     stores and release the stage to the producer.
+//   * the 8 consumer warps form 8/W groups of W warps (W = 1, 2, 4 or 8,
+//     chosen per launch from the item size); item `it` goes to group
+//     it mod (8/W), so groups work on different items at the same time and
+//     one group's waits (its loads, the cluster exchange) overlap the others'
+//     work.  In a group, each warp reduces its 1 KiB tiles to tile partials,
+//     the warps meet at one named barrier per item, combine the K tile
+//     partials of the row in a fixed order (every warp redundantly, so no
+//     broadcast is needed), normalise their tiles from the stage, store with
+//     128-bit streaming stores and release the stage to the producer.  Which
+//     warp handles which tile never changes the arithmetic, so the result
+//     does not depend on W.
 // Dense MEDIUM rows: one CTA per row.  LARGE rows: the cs CTAs of a cluster
 // split the row's tiles into contiguous portions resident in shared memory;
 // after pass 1 every CTA signals the others with remote mbarrier arrives,
-// gathers all K partials through distributed shared memory and combines them
+// reads all K partials through distributed shared memory and combines them
 // exactly like the MEDIUM path -- the row is read from HBM once and the result
 // does not depend on cs.  Ragged: the LARGE rows (cluster-split, round-robin
 // over clusters), then the MEDIUM rows (pulled from a device counter), then
@@ -36,7 +42,8 @@ constexpr int kConsumerWarps = 8;
 constexpr int kConsumerThreads = kConsumerWarps * 32;
 constexpr int kTileThreads = kConsumerThreads + 32;  // + the producer warp
 constexpr int kPieceTiles = 16;                      // tiles per piece barrier (16 KiB)
-constexpr uint32_t kBarConsumers = 1;                // named barrier of the consumer warps
+constexpr uint32_t kBarConsumers = 1;                // named barrier of all consumer warps
+constexpr uint32_t kBarGroup0 = 2;                   // named barrier of consumer group g: 2 + g
 constexpr int kSmallSliceBytes = 4096 + 128;         // per-warp staging of a ragged SMALL row
 constexpr int kShortCombineTiles = 64;  // rows of up to this many tiles: every warp combines
 
@@ -53,7 +60,7 @@ struct TileParams {
   uint32_t stage_bytes;  // = max_tiles * kTileBytes
   int stages;
   int max_tiles;     // tiles one stage holds
-  int gather_tiles;  // partials the gather buffer holds (cluster launches)
+  int group_warps;   // W: consumer warps that share one item (1, 2, 4 or 8)
   int out_vec;
   int gvec;
   uint64_t timeout_ns;
@@ -74,24 +81,30 @@ struct ItemMeta {
 };
 
 // Shared-memory layout of the tile kernel (host and device agree on it).
+// Per consumer group: tile partials of split items (part_c) and of items a
+// CTA handles alone (part_m), both double-buffered by the parity of the
+// group's item count; the two halves of the cooperative combine's scratch
+// (xw); the partials of a short split row gathered from the peers (gather);
+// the cluster barriers ready / released, one per buffer.
 struct TileSmemLayout {
   uint32_t part_c, part_m, gather, meta, xw, bar_meta, bar_piece, bar_empty, bar_ready,
       bar_released, flags, total;
   int pieces;
-  __host__ __device__ TileSmemLayout(uint32_t stage_bytes, int stages, int max_tiles,
-                                     int gather_tiles) {
+  __host__ __device__ TileSmemLayout(uint32_t stage_bytes, int stages, int max_tiles, int groups,
+                                     bool split_items, bool local_items) {
     pieces = (max_tiles + kPieceTiles - 1) / kPieceTiles;
+    const uint32_t part_bytes = static_cast<uint32_t>(groups) * 2u * max_tiles * 16u;
     uint32_t off = stage_bytes * stages;
     part_c = off;
-    off += 2u * max_tiles * 16u;
+    off += split_items ? part_bytes : 0u;
     part_m = off;
-    off += 2u * max_tiles * 16u;
+    off += local_items ? part_bytes : 0u;
     gather = off;
-    off += static_cast<uint32_t>(gather_tiles) * 16u;
+    off += split_items ? static_cast<uint32_t>(groups) * kShortCombineTiles * 16u : 0u;
     meta = off;
     off += stages * 32u;
-    xw = off;  // 2 x 8 per-warp values of the cooperative combine
-    off += 2u * kConsumerWarps * 4u;
+    xw = off;
+    off += static_cast<uint32_t>(groups) * 2u * kConsumerWarps * 4u;
     bar_meta = off;
     off += stages * 8u;
     bar_piece = off;
@@ -99,9 +112,9 @@ struct TileSmemLayout {
     bar_empty = off;
     off += stages * 8u;
     bar_ready = off;
-    off += 16u;
+    off += static_cast<uint32_t>(groups) * 16u;
     bar_released = off;
-    off += 16u;
+    off += static_cast<uint32_t>(groups) * 16u;
     flags = off;
     off += 16u;
     total = off;
@@ -215,29 +228,31 @@ __device__ __forceinline__ float tile_lane_second(const unsigned char *tsm, cons
   }
 }
 
-// B tiles of one warp, lt0, lt0 + 8, ..., lt0 + 8(B-1), all below the item's
-// tile count: lane-level sums of all of them first, then their butterflies
-// interleaved.  Waits on each stage piece before the first tile read from it
-// (`waited` is the last piece waited for); returns false when such a wait
-// ran out.
-template <int OP, typename T, int B>
+// B tiles of one warp, lt0, lt0 + W, ..., lt0 + W(B-1), all below the item's
+// tile count (W = warps of the group): lane-level sums of all of them first,
+// then their butterflies interleaved.  FULL: the caller checked that every
+// one of them lies entirely in the row, so no element masks are evaluated
+// (same arithmetic: the masks of a full tile keep every element).  Waits on
+// each stage piece before the first tile read from it (`waited` is the last
+// piece waited for); returns false when such a wait ran out.
+template <int OP, typename T, int B, bool FULL>
 __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const ItemGeo &g, int lt0,
-                                            int lane, float4 *part, uint32_t piece_bar0,
+                                            int W, int lane, float4 *part, uint32_t piece_bar0,
                                             uint32_t par, uint64_t timeout_ns, int &waited) {
   constexpr int E = Elem<T>::kPerChunk;
   constexpr bool kMaxFirst = (OP == kSoftmax || OP == kLogSoftmax);
   float a[B], b[B];
 #pragma unroll
   for (int q = 0; q < B; ++q) {
-    const int lt = lt0 + q * kConsumerWarps;
+    const int lt = lt0 + q * W;
     const int pc = lt / kPieceTiles;
     if (pc != waited) {
       if (!mbar_wait_bounded(piece_bar0 + 8u * pc, par, timeout_ns)) return false;
       waited = pc;
     }
     const int t = g.t0 + lt;
-    a[q] = tile_lane_first<OP, T>(stage + lt * kTileBytes,
-                                  tile_mask<T>(t, g, lane, tile_is_full(t, g)), lane);
+    const TileMask m = FULL ? TileMask{0, E, 0, E} : tile_mask<T>(t, g, lane, tile_is_full(t, g));
+    a[q] = tile_lane_first<OP, T>(stage + lt * kTileBytes, m, lane);
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -250,15 +265,15 @@ __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const It
   if constexpr (OP == kRmsNorm) {
     if (lane == 0) {
 #pragma unroll
-      for (int q = 0; q < B; ++q) part[lt0 + q * kConsumerWarps] = make_float4(a[q], 0.f, 0.f, 0.f);
+      for (int q = 0; q < B; ++q) part[lt0 + q * W] = make_float4(a[q], 0.f, 0.f, 0.f);
     }
   } else {
     float ref[B], ntf[B];
 #pragma unroll
     for (int q = 0; q < B; ++q) {
-      const int lt = lt0 + q * kConsumerWarps;
+      const int lt = lt0 + q * W;
       const int t = g.t0 + lt;
-      const bool full = tile_is_full(t, g);
+      const bool full = FULL || tile_is_full(t, g);
       ref[q] = a[q];
       ntf[q] = 0.f;
       if constexpr (OP == kLayerNorm) {
@@ -274,8 +289,8 @@ __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const It
           ref[q] = nt > 0 ? __fdiv_rn(a[q], ntf[q]) : 0.f;
         }
       }
-      b[q] = tile_lane_second<OP, T>(stage + lt * kTileBytes, tile_mask<T>(t, g, lane, full), lane,
-                                     ref[q]);
+      const TileMask m = FULL ? TileMask{0, E, 0, E} : tile_mask<T>(t, g, lane, full);
+      b[q] = tile_lane_second<OP, T>(stage + lt * kTileBytes, m, lane, ref[q]);
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -285,38 +300,51 @@ __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const It
     if (lane == 0) {
 #pragma unroll
       for (int q = 0; q < B; ++q)
-        part[lt0 + q * kConsumerWarps] = (OP == kLayerNorm) ? make_float4(a[q], ref[q], b[q], ntf[q])
+        part[lt0 + q * W] = (OP == kLayerNorm) ? make_float4(a[q], ref[q], b[q], ntf[q])
                                                             : make_float4(a[q], b[q], 0.f, 0.f);
     }
   }
   return true;
 }
 
-// Pass 1 of an item for one warp: part[lt] for its tiles lt = warp, warp + 8,
-// ..., taken kPass1Batch at a time while that many remain, then in a batch of
-// two and one.  Each tile's arithmetic (and its butterfly order) is the same
+// Pass 1 of an item for warp `wig` of a group of W warps: part[lt] for its
+// tiles lt = wig, wig + W, ..., taken kPass1Batch at a time while that many
+// remain, then in a batch of two and one.  Each tile's arithmetic (and its butterfly order) is the same
 // whatever batch it falls in.
 template <int OP, typename T>
-__device__ __forceinline__ bool pass1_warp(const unsigned char *stage, const ItemGeo &g, int warp,
-                                           int lane, float4 *part, uint32_t piece_bar0,
+__device__ __forceinline__ bool pass1_warp(const unsigned char *stage, const ItemGeo &g, int wig,
+                                           int W, int lane, float4 *part, uint32_t piece_bar0,
                                            uint32_t par, uint64_t timeout_ns) {
   const int ntl = g.t1 - g.t0;
+  // tiles [full0, full1) of the row lie entirely in it (all but its ends)
+  const int full0 = g.cf > 0 ? 1 : 0;
+  const int full1 = g.cl / kTileChunks;
   int waited = -1;
-  int lt0 = warp;
+  int lt0 = wig;
   while (lt0 < ntl) {
-    const int left = (ntl - lt0 + kConsumerWarps - 1) / kConsumerWarps;
+    const int left = (ntl - lt0 + W - 1) / W;
+    const int bsz = left >= kPass1Batch ? kPass1Batch : (left >= 2 ? 2 : 1);
+    const int ta = g.t0 + lt0, tb = ta + (bsz - 1) * W;
+    const bool full = ta >= full0 && tb < full1;
     bool ok;
-    if (left >= kPass1Batch) {
-      ok = pass1_batch<OP, T, kPass1Batch>(stage, g, lt0, lane, part, piece_bar0, par, timeout_ns, waited);
-      lt0 += kPass1Batch * kConsumerWarps;
-    } else if (left >= 2) {
-      ok = pass1_batch<OP, T, 2>(stage, g, lt0, lane, part, piece_bar0, par, timeout_ns, waited);
-      lt0 += 2 * kConsumerWarps;
+    if (bsz == kPass1Batch) {
+      ok = full ? pass1_batch<OP, T, kPass1Batch, true>(stage, g, lt0, W, lane, part, piece_bar0,
+                                                         par, timeout_ns, waited)
+                : pass1_batch<OP, T, kPass1Batch, false>(stage, g, lt0, W, lane, part,
+                                                          piece_bar0, par, timeout_ns, waited);
+    } else if (bsz == 2) {
+      ok = full ? pass1_batch<OP, T, 2, true>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                                              timeout_ns, waited)
+                : pass1_batch<OP, T, 2, false>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                                               timeout_ns, waited);
     } else {
-      ok = pass1_batch<OP, T, 1>(stage, g, lt0, lane, part, piece_bar0, par, timeout_ns, waited);
-      lt0 += kConsumerWarps;
+      ok = full ? pass1_batch<OP, T, 1, true>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                                              timeout_ns, waited)
+                : pass1_batch<OP, T, 1, false>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                                               timeout_ns, waited);
     }
     if (!ok) return false;
+    lt0 += bsz * W;
   }
   return true;
 }
@@ -361,13 +389,15 @@ __device__ __forceinline__ float second_term(const float4 &pt, float first) {
   }
 }
 
-template <int OP>
-__device__ __forceinline__ void combine_short(const float4 *part, int K, float inv_n, float eps,
-                                              int lane, float &s0, float &s1) {
+// `get(t)` returns tile partial t (from this CTA's shared memory, or from a
+// peer's through distributed shared memory).
+template <int OP, class Get>
+__device__ __forceinline__ void combine_short(Get get, int K, float inv_n, float eps, int lane,
+                                              float &s0, float &s1) {
   constexpr bool kMax = (OP == kSoftmax || OP == kLogSoftmax);
   const float4 z = make_float4(kMax ? -INFINITY : 0.f, 0.f, 0.f, 0.f);
-  const float4 p0 = lane < K ? part[lane] : z;
-  const float4 p1 = lane + 32 < K ? part[lane + 32] : z;
+  const float4 p0 = lane < K ? get(lane) : z;
+  const float4 p1 = lane + 32 < K ? get(lane + 32) : z;
   float first;
   if constexpr (kMax) {
     first = warp_max(fmaxf(p0.x, p1.x));
@@ -384,27 +414,38 @@ __device__ __forceinline__ void combine_short(const float4 *part, int K, float i
   finish_stats<OP>(first, second, inv_n, eps, s0, s1);
 }
 
-template <int OP>
-__device__ __forceinline__ void combine_long(const float4 *part, int K, float inv_n, float eps,
-                                             int tid, int lane, int warp, volatile float *xw,
+// The 256 virtual lanes of the long combine are spread over the group's W
+// warps: warp `wig` plays virtual warps wig, wig + W, ...; the group meets at
+// its named barrier `bar` and shares the 8 virtual-warp results through xw.
+template <int OP, class Get>
+__device__ __forceinline__ void combine_long(Get get, int K, float inv_n, float eps, int lane,
+                                             int wig, int W, uint32_t bar, volatile float *xw,
                                              float &s0, float &s1) {
   constexpr bool kMax = (OP == kSoftmax || OP == kLogSoftmax);
-  float v = kMax ? -INFINITY : 0.f;
-  for (int t = tid; t < K; t += kConsumerThreads)
-    v = kMax ? fmaxf(v, part[t].x) : __fadd_rn(v, part[t].x);
-  v = kMax ? warp_max(v) : warp_sum(v);
-  if (lane == 0) xw[warp] = v;
-  named_sync(kBarConsumers, kConsumerThreads);
+  const uint32_t nthreads = static_cast<uint32_t>(W) * 32u;
+  for (int vw = wig; vw < kConsumerWarps; vw += W) {
+    float v = kMax ? -INFINITY : 0.f;
+    for (int t = vw * 32 + lane; t < K; t += kConsumerThreads) {
+      const float x = get(t).x;
+      v = kMax ? fmaxf(v, x) : __fadd_rn(v, x);
+    }
+    v = kMax ? warp_max(v) : warp_sum(v);
+    if (lane == 0) xw[vw] = v;
+  }
+  named_sync(bar, nthreads);
   float first = xw[0];
   for (int w = 1; w < kConsumerWarps; ++w) first = kMax ? fmaxf(first, xw[w]) : __fadd_rn(first, xw[w]);
   if constexpr (OP == kLayerNorm) first = __fmul_rn(first, inv_n);
   float second = 0.f;
   if constexpr (OP != kRmsNorm) {
-    float u = 0.f;
-    for (int t = tid; t < K; t += kConsumerThreads) u = __fadd_rn(u, second_term<OP>(part[t], first));
-    u = warp_sum(u);
-    if (lane == 0) xw[kConsumerWarps + warp] = u;
-    named_sync(kBarConsumers, kConsumerThreads);
+    for (int vw = wig; vw < kConsumerWarps; vw += W) {
+      float u = 0.f;
+      for (int t = vw * 32 + lane; t < K; t += kConsumerThreads)
+        u = __fadd_rn(u, second_term<OP>(get(t), first));
+      u = warp_sum(u);
+      if (lane == 0) xw[kConsumerWarps + vw] = u;
+    }
+    named_sync(bar, nthreads);
     second = xw[kConsumerWarps];
     for (int w = 1; w < kConsumerWarps; ++w) second = __fadd_rn(second, xw[kConsumerWarps + w]);
   }
@@ -490,16 +531,17 @@ __device__ __forceinline__ bool tile_fast(int t, const ItemGeo &g, const TilePar
          (!kAffine || static_cast<int64_t>(t + 1) * kTileChunks * E <= p.glen);
 }
 
-// pass 2 fast path over this warp's tiles of an item whose head offset is H
+// pass 2 fast path over this warp's tiles (wig, wig + W, ...) of an item
+// whose head offset is H
 template <int OP, typename T, int H>
 __device__ __forceinline__ void pass2_fast_tiles(const unsigned char *stage, const ItemGeo &g,
-                                                 int warp, int lane, float s0, float s1,
+                                                 int wig, int W, int lane, float s0, float s1,
                                                  const TileParams &p, char *owin,
                                                  bool params_ok) {
   const T *gamma = static_cast<const T *>(p.gamma);
   const T *beta = static_cast<const T *>(p.beta);
   const int ntl = g.t1 - g.t0;
-  for (int lt = warp; lt < ntl; lt += kConsumerWarps) {
+  for (int lt = wig; lt < ntl; lt += W) {
     const int t = g.t0 + lt;
     if (tile_fast<OP, T>(t, g, p, params_ok))
       tile_store_fast<OP, T, H>(stage + lt * kTileBytes, t, lane, s0, s1, gamma, beta, owin);
@@ -511,35 +553,35 @@ __device__ __forceinline__ void pass2_fast_tiles(const unsigned char *stage, con
 // tiles the fast path does not take (the row's ends, unaligned output, rows
 // reaching the end of gamma/beta) through the general path.
 template <int OP, typename T, bool EXACT>
-__device__ __forceinline__ void pass2_item(const unsigned char *stage, const ItemGeo &g, int warp,
-                                           int lane, float s0, float s1, const TileParams &p,
-                                           char *owin, T *out_row) {
+__device__ __forceinline__ void pass2_item(const unsigned char *stage, const ItemGeo &g, int wig,
+                                           int W, int lane, float s0, float s1,
+                                           const TileParams &p, char *owin, T *out_row) {
   constexpr int E = Elem<T>::kPerChunk;
   constexpr bool kAffine = (OP == kLayerNorm || OP == kRmsNorm);
   const bool params_ok =
       !kAffine || (p.gvec && p.gamma && (OP == kRmsNorm || p.beta != nullptr));
   if constexpr (EXACT || !kAffine) {
-    pass2_fast_tiles<OP, T, 0>(stage, g, warp, lane, s0, s1, p, owin, params_ok);
+    pass2_fast_tiles<OP, T, 0>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok);
   } else {
     switch (g.h) {
-      case 0: pass2_fast_tiles<OP, T, 0>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
-      case 1: pass2_fast_tiles<OP, T, 1>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
-      case 2: pass2_fast_tiles<OP, T, 2>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
-      case 3: pass2_fast_tiles<OP, T, 3>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
+      case 0: pass2_fast_tiles<OP, T, 0>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
+      case 1: pass2_fast_tiles<OP, T, 1>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
+      case 2: pass2_fast_tiles<OP, T, 2>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
+      case 3: pass2_fast_tiles<OP, T, 3>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
       default:
         if constexpr (E == 8) {
           switch (g.h) {
-            case 4: pass2_fast_tiles<OP, T, 4>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
-            case 5: pass2_fast_tiles<OP, T, 5>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
-            case 6: pass2_fast_tiles<OP, T, 6>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
-            default: pass2_fast_tiles<OP, T, 7>(stage, g, warp, lane, s0, s1, p, owin, params_ok); break;
+            case 4: pass2_fast_tiles<OP, T, 4>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
+            case 5: pass2_fast_tiles<OP, T, 5>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
+            case 6: pass2_fast_tiles<OP, T, 6>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
+            default: pass2_fast_tiles<OP, T, 7>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
           }
         }
         break;
     }
   }
   const int ntl = g.t1 - g.t0;
-  for (int lt = warp; lt < ntl; lt += kConsumerWarps) {
+  for (int lt = wig; lt < ntl; lt += W) {
     const int t = g.t0 + lt;
     if (!tile_fast<OP, T>(t, g, p, params_ok))
       tile_store<OP, T, EXACT>(stage + lt * kTileBytes, t, g, lane, s0, s1, p, owin, out_row);
@@ -609,6 +651,8 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
                                               int64_t ncl) {
   constexpr int SZ = Elem<T>::kSize;
   const int S = p.stages;
+  const int G = kConsumerWarps / p.group_warps;  // every group gets an end-of-work item
+  int ends = 0;
   const uint32_t sbase = smem_addr(smem);
   ItemMeta *meta = reinterpret_cast<ItemMeta *>(smem + L.meta);
   volatile int *flags = reinterpret_cast<volatile int *>(smem + L.flags);
@@ -682,7 +726,10 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
     meta[s].n = n;
     meta[s].kind = kind;
     mbar_arrive(sbase + L.bar_meta + 8u * s);
-    if (kind == kItemEnd) break;
+    if (kind == kItemEnd) {
+      if (++ends == G) break;
+      continue;
+    }
 
     const bool split = CLUSTER && kind == kItemLarge;
     const ItemGeo g = item_geo<T, EXACT>(p.in, start, n, split, rank, cs);
@@ -755,7 +802,9 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
   constexpr int E = Elem<T>::kPerChunk;
   constexpr int SZ = Elem<T>::kSize;
   extern __shared__ __align__(1024) unsigned char smem[];
-  const TileSmemLayout L(p.stage_bytes, p.stages, p.max_tiles, p.gather_tiles);
+  const int W = p.group_warps;
+  const int G = kConsumerWarps / W;
+  const TileSmemLayout L(p.stage_bytes, p.stages, p.max_tiles, G, CLUSTER, !CLUSTER || RAGGED);
   const int S = p.stages;
   const int tid = threadIdx.x;
   const int lane = tid & 31;
@@ -765,21 +814,18 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
   const int64_t cid = CLUSTER ? cluster_id_x() : blockIdx.x;
   const int64_t ncl = CLUSTER ? cluster_count_x() : gridDim.x;
   const uint32_t sbase = smem_addr(smem);
-  float4 *part_c = reinterpret_cast<float4 *>(smem + L.part_c);
-  float4 *part_m = reinterpret_cast<float4 *>(smem + L.part_m);
-  float4 *gather = reinterpret_cast<float4 *>(smem + L.gather);
   const ItemMeta *meta = reinterpret_cast<const ItemMeta *>(smem + L.meta);
   volatile int *flags = reinterpret_cast<volatile int *>(smem + L.flags);
 
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(sbase + L.bar_meta + 8u * s, 1);
-      mbar_init(sbase + L.bar_empty + 8u * s, kConsumerWarps);
+      mbar_init(sbase + L.bar_empty + 8u * s, W);
       for (int pc = 0; pc < L.pieces; ++pc) mbar_init(sbase + L.bar_piece + 8u * (s * L.pieces + pc), 1);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(sbase + L.bar_ready + 8u * b, cs);
-      mbar_init(sbase + L.bar_released + 8u * b, cs);
+    for (int i = 0; i < 2 * G; ++i) {
+      mbar_init(sbase + L.bar_ready + 8u * i, cs);           // one arrive per CTA
+      mbar_init(sbase + L.bar_released + 8u * i, cs * W);    // one per warp of the group
     }
     flags[0] = 0;
     fence_mbar_init();
@@ -793,14 +839,26 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
   }
 
   // ------------------------------ consumers ------------------------------
-  // cluster items that used part_c[0] / part_c[1] (kept as scalars: a
-  // runtime-indexed array would live in local memory)
+  const int grp = warp / W;       // this warp's group
+  const int wig = warp - grp * W; // its index in the group
+  const int gtid = tid - grp * W * 32;
+  const uint32_t gthreads = static_cast<uint32_t>(W) * 32u;
+  const uint32_t gbar = kBarGroup0 + static_cast<uint32_t>(grp);
+  float4 *part_c = reinterpret_cast<float4 *>(smem + L.part_c) + static_cast<size_t>(grp) * 2 * p.max_tiles;
+  float4 *part_m = reinterpret_cast<float4 *>(smem + L.part_m) + static_cast<size_t>(grp) * 2 * p.max_tiles;
+  volatile float *xw = reinterpret_cast<volatile float *>(smem + L.xw) + grp * 2 * kConsumerWarps;
+  float4 *gather = reinterpret_cast<float4 *>(smem + L.gather) + grp * kShortCombineTiles;
+  const uint32_t bar_ready = sbase + L.bar_ready + 16u * grp;        // + 8 b
+  const uint32_t bar_released = sbase + L.bar_released + 16u * grp;  // + 8 b
+  // split items of this group that used part_c[0] / part_c[1] (kept as
+  // scalars: a runtime-indexed array would live in local memory)
   uint32_t uses0 = 0, uses1 = 0;
   bool ended = false;
-  for (int64_t it = 0;; ++it) {
+  for (int64_t j = 0;; ++j) {
+    const int64_t it = grp + j * G;  // the group's j-th item
     const int s = static_cast<int>(it % S);
     const uint32_t par = static_cast<uint32_t>((it / S) & 1);
-    const int b = static_cast<int>(it & 1);
+    const int b = static_cast<int>(j & 1);
     const uint32_t uses_b = b ? uses1 : uses0;
     bool bad = !mbar_wait_bounded(sbase + L.bar_meta + 8u * s, par, p.timeout_ns);
     int kind = kItemEnd;
@@ -813,21 +871,19 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
         const bool split = CLUSTER && kind == kItemLarge;
         g = item_geo<T, EXACT>(p.in, meta[s].start, meta[s].n, split, rank, cs);
         if (split && uses_b > 0)
-          bad = !mbar_wait_cluster_bounded(sbase + L.bar_released + 8u * b, (uses_b - 1) & 1,
-                                           p.timeout_ns);
+          bad = !mbar_wait_cluster_bounded(bar_released + 8u * b, (uses_b - 1) & 1, p.timeout_ns);
       }
     }
     const bool split = CLUSTER && kind == kItemLarge;
     const unsigned char *stage = smem + static_cast<size_t>(s) * p.stage_bytes;
-    const int ntl = g.t1 - g.t0;
     float4 *part = (split ? part_c : part_m) + static_cast<size_t>(b) * p.max_tiles;
 
     // ---- pass 1 ----
     if (!bad && kind != kItemEnd)
-      bad = !pass1_warp<OP, T>(stage, g, warp, lane, part,
+      bad = !pass1_warp<OP, T>(stage, g, wig, W, lane, part,
                                sbase + L.bar_piece + 8u * (s * L.pieces), par, p.timeout_ns);
-    if (named_sync_or(kBarConsumers, kConsumerThreads, bad)) {
-      if (tid == 0) {
+    if (named_sync_or(gbar, gthreads, bad)) {
+      if (gtid == 0) {
         atomicOr(p.status, kStatusTimeout);
         flags[0] = 1;
       }
@@ -839,70 +895,68 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
     }
 
     // ---- combine ----
-    const float4 *src = part;
+    float s0, s1;
+    const float inv_n = __frcp_rn(static_cast<float>(g.n));
     if (split) {
-      const uint32_t ready = sbase + L.bar_ready + 8u * b;
+      const uint32_t ready = bar_ready + 8u * b;
       // thread r signals rank r; the named barrier above already ordered
       // every warp's partial writes before these releases
-      if (tid < cs) mbar_arrive_remote(ready, static_cast<uint32_t>(tid));
-      bool ok = mbar_wait_cluster_bounded(ready, uses_b & 1, p.timeout_ns);
-      if (ok) {
-        const int tpc = (g.K + cs - 1) / cs;
-        const uint32_t mine = smem_addr(part_c + static_cast<size_t>(b) * p.max_tiles);
-        auto peer_addr = [&](int t) {
-          const int r = t / tpc;
-          return map_to_rank(mine + static_cast<uint32_t>((t - r * tpc) * 16),
-                             static_cast<uint32_t>(r));
-        };
-        // four loads in flight per thread before their results are stored
-        int t = tid;
-        for (; t + 3 * kConsumerThreads < g.K; t += 4 * kConsumerThreads) {
-          const float4 v0 = ld_dsmem_f4(peer_addr(t));
-          const float4 v1 = ld_dsmem_f4(peer_addr(t + kConsumerThreads));
-          const float4 v2 = ld_dsmem_f4(peer_addr(t + 2 * kConsumerThreads));
-          const float4 v3 = ld_dsmem_f4(peer_addr(t + 3 * kConsumerThreads));
-          gather[t] = v0;
-          gather[t + kConsumerThreads] = v1;
-          gather[t + 2 * kConsumerThreads] = v2;
-          gather[t + 3 * kConsumerThreads] = v3;
-        }
-        for (; t < g.K; t += kConsumerThreads) gather[t] = ld_dsmem_f4(peer_addr(t));
-      }
-      if (named_sync_or(kBarConsumers, kConsumerThreads, !ok)) {
-        if (tid == 0) {
+      if (gtid < cs) mbar_arrive_remote(ready, static_cast<uint32_t>(gtid));
+      const bool ok = mbar_wait_cluster_bounded(ready, uses_b & 1, p.timeout_ns);
+      if (named_sync_or(gbar, gthreads, !ok)) {
+        if (gtid == 0) {
           atomicOr(p.status, kStatusTimeout);
           flags[0] = 1;
         }
         break;
       }
-      if (tid < cs) mbar_arrive_remote(sbase + L.bar_released + 8u * b, static_cast<uint32_t>(tid));
+      // partial t lives in rank t / tpc at the same offset of its part_c
+      const int tpc = (g.K + cs - 1) / cs;
+      const uint32_t mine = smem_addr(part);
+      auto peer = [&](int t) {
+        const int r = t / tpc;
+        return ld_dsmem_f4(map_to_rank(mine + static_cast<uint32_t>((t - r * tpc) * 16),
+                                       static_cast<uint32_t>(r)));
+      };
+      if (g.K <= kShortCombineTiles) {
+        // every warp combines all K partials: copy them here once, then
+        // combine from local shared memory
+        for (int t = gtid; t < g.K; t += static_cast<int>(gthreads)) gather[t] = peer(t);
+        named_sync(gbar, gthreads);
+        __syncwarp();
+        if (lane < cs) mbar_arrive_remote(bar_released + 8u * b, static_cast<uint32_t>(lane));
+        combine_short<OP>([&](int t) { return gather[t]; }, g.K, inv_n, p.eps, lane, s0, s1);
+      } else {
+        combine_long<OP>(peer, g.K, inv_n, p.eps, lane, wig, W, gbar, xw, s0, s1);
+        // this warp has read every peer partial it needs: let the peers reuse them
+        __syncwarp();
+        if (lane < cs) mbar_arrive_remote(bar_released + 8u * b, static_cast<uint32_t>(lane));
+      }
       if (b) {
         ++uses1;
       } else {
         ++uses0;
       }
-      src = gather;
-    }
-    float s0, s1;
-    const float inv_n = __frcp_rn(static_cast<float>(g.n));
-    if (g.K <= kShortCombineTiles) {
-      combine_short<OP>(src, g.K, inv_n, p.eps, lane, s0, s1);
     } else {
-      combine_long<OP>(src, g.K, inv_n, p.eps, tid, lane, warp,
-                       reinterpret_cast<volatile float *>(smem + L.xw), s0, s1);
+      auto local = [&](int t) { return part[t]; };
+      if (g.K <= kShortCombineTiles) {
+        combine_short<OP>(local, g.K, inv_n, p.eps, lane, s0, s1);
+      } else {
+        combine_long<OP>(local, g.K, inv_n, p.eps, lane, wig, W, gbar, xw, s0, s1);
+      }
     }
 
     // ---- pass 2 ----
     T *out_row = static_cast<T *>(p.out) + g.start;
     char *owin = reinterpret_cast<char *>(out_row) - g.h * SZ;
-    pass2_item<OP, T, EXACT>(stage, g, warp, lane, s0, s1, p, owin, out_row);
+    pass2_item<OP, T, EXACT>(stage, g, wig, W, lane, s0, s1, p, owin, out_row);
     __syncwarp();
     if (lane == 0) mbar_arrive(sbase + L.bar_empty + 8u * s);
   }
 
   // ---- ragged: the SMALL rows, one per warp, staged in a slice of the stages ----
-  if (RAGGED && ended) {
-    named_sync(kBarConsumers, kConsumerThreads);  // no warp reads the stages any more
+  // (every group has left its loop: no warp reads the stages any more)
+  if (RAGGED && !named_sync_or(kBarConsumers, kConsumerThreads, !ended)) {
     SmallRowArgs sa;
     sa.gamma = p.gamma;
     sa.beta = p.beta;
@@ -946,10 +1000,8 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
 
   // ---- no CTA leaves while a peer may still read its partials ----
   if (CLUSTER) {
-    if (uses0 > 0)
-      (void)mbar_wait_cluster_bounded(sbase + L.bar_released, (uses0 - 1) & 1, p.timeout_ns);
-    if (uses1 > 0)
-      (void)mbar_wait_cluster_bounded(sbase + L.bar_released + 8u, (uses1 - 1) & 1, p.timeout_ns);
+    if (uses0 > 0) (void)mbar_wait_cluster_bounded(bar_released, (uses0 - 1) & 1, p.timeout_ns);
+    if (uses1 > 0) (void)mbar_wait_cluster_bounded(bar_released + 8u, (uses1 - 1) & 1, p.timeout_ns);
   }
 
   // ---- ragged: the last CTA to finish resets the work counters, so a plan

@@ -125,14 +125,20 @@ def test_dense_deterministic(rw, op):
         assert torch.equal(a.view(torch.int32), b.view(torch.int32))
 
 
-def _forced(rw, op, dtype, rows, cols, bucket, cluster=None, ld=None, x_off=0):
-    old = {k: os.environ.get(k) for k in ("ROWOP_FORCE_BUCKET", "ROWOP_CLUSTER")}
+KNOBS = ("ROWOP_FORCE_BUCKET", "ROWOP_CLUSTER", "ROWOP_GROUP_WARPS", "ROWOP_STAGES")
+
+
+def _forced(rw, op, dtype, rows, cols, bucket, cluster=None, ld=None, x_off=0,
+            group_warps=None, stages=None):
+    old = {k: os.environ.get(k) for k in KNOBS}
     try:
         os.environ["ROWOP_FORCE_BUCKET"] = str(bucket)
-        if cluster:
-            os.environ["ROWOP_CLUSTER"] = str(cluster)
-        else:
-            os.environ.pop("ROWOP_CLUSTER", None)
+        for k, v in (("ROWOP_CLUSTER", cluster), ("ROWOP_GROUP_WARPS", group_warps),
+                     ("ROWOP_STAGES", stages)):
+            if v:
+                os.environ[k] = str(v)
+            else:
+                os.environ.pop(k, None)
         return run_case(rw, op, dtype, rows, cols, ld=ld, x_off=x_off, y_off=x_off,
                         seed=cols).clone()
     finally:
@@ -162,3 +168,26 @@ def test_forced_designs_agree(rw, op, dtype, cols, ld, x_off):
         assert torch.equal(_bits(medium), _bits(large)), f"cluster {cs}"
     if cols * ESIZE[dtype] <= 4096 + 512:
         _forced(rw, op, dtype, rows, cols, 0, ld=ld, x_off=x_off)
+
+
+@pytest.mark.parametrize("dtype", DTYPES, ids=["f32", "bf16"])
+@pytest.mark.parametrize("op", ALL_OPS)
+@pytest.mark.parametrize("cols,ld,x_off", [(3000, None, 0), (6000, 6003, 1),
+                                          (40001, 40005, 3)])
+def test_group_sizes_agree(rw, op, dtype, cols, ld, x_off):
+    """The tile kernel's consumer warps work in groups of W (1, 2, 4 or 8
+    warps per item, several items at once).  Which warp reduces which tile
+    does not change the arithmetic: every W, with few or many stages, gives
+    the same bits, in the one-CTA design and in the cluster split.  37 rows
+    give every group several items and a partial last round."""
+    rows = 37
+    ref = _forced(rw, op, dtype, rows, cols, 1, ld=ld, x_off=x_off, group_warps=8)
+    for w in (1, 2, 4):
+        for stages in (None, 8 // w):
+            got = _forced(rw, op, dtype, rows, cols, 1, ld=ld, x_off=x_off, group_warps=w,
+                          stages=stages)
+            assert torch.equal(_bits(ref), _bits(got)), f"MEDIUM W={w} stages={stages}"
+    for cs, w in ((2, 1), (4, 2), (8, 4)):
+        got = _forced(rw, op, dtype, rows, cols, 2, cluster=cs, ld=ld, x_off=x_off,
+                      group_warps=w)
+        assert torch.equal(_bits(ref), _bits(got)), f"cluster {cs} W={w}"

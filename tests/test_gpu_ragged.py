@@ -204,3 +204,24 @@ def test_ragged_all_empty_and_tiny(rw):
             continue
         ref = oracle_ragged("logsoftmax", r["x"][:covered].double().numpy(), r["off"])
         assert_close(to_f64(r["y"][:covered]), ref, torch.float32, "tiny")
+
+
+@pytest.mark.parametrize("dtype", DTYPES, ids=["f32", "bf16"])
+@pytest.mark.parametrize("op", ("softmax", "layernorm"))
+def test_ragged_group_sizes_agree(rw, op, dtype, monkeypatch):
+    """The fused ragged kernel gives the same bits whatever the consumer
+    group size (W warps per item) and cluster size it runs with."""
+    max_len = 70000 if dtype == torch.float32 else 40000
+    lens = mixed_lengths(dtype, 300, seed=41, max_len=max_len)
+    ref = run_ragged(rw, op, dtype, lens, max_len, seed=43, base_off=1)["y"].clone()
+    bits = (lambda t: t.view(torch.int32)) if dtype == torch.float32 else \
+        (lambda t: t.view(torch.int16))
+    for w, cs in ((1, None), (2, 4), (4, None), (8, 2)):
+        monkeypatch.setenv("ROWOP_GROUP_WARPS", str(w))
+        if cs:
+            monkeypatch.setenv("ROWOP_CLUSTER", str(cs))
+        else:
+            monkeypatch.delenv("ROWOP_CLUSTER", raising=False)
+        got = run_ragged(rw, op, dtype, lens, max_len, seed=43, base_off=1)["y"]
+        assert rw.check_status() == 0
+        assert torch.equal(bits(ref), bits(got)), f"W={w} cluster={cs}"
