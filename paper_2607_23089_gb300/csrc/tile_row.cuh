@@ -452,31 +452,6 @@ __device__ __forceinline__ void combine_long(Get get, int K, float inv_n, float 
   finish_stats<OP>(first, second, inv_n, eps, s0, s1);
 }
 
-// pass 2: normalise tile t from the stage and store it
-template <int OP, typename T, bool EXACT>
-__device__ __forceinline__ void tile_store(const unsigned char *tsm, int t, const ItemGeo &g,
-                                           int lane, float s0, float s1, const TileParams &p,
-                                           char *owin, T *out_row) {
-  constexpr int E = Elem<T>::kPerChunk;
-  constexpr int NP = E / 2;
-  const bool full = tile_is_full(t, g);  // the row's last tile may hold < 64 chunks
-  const int hn = g.h + static_cast<int>(g.n);
-  const T *gamma = static_cast<const T *>(p.gamma);
-  const T *beta = static_cast<const T *>(p.beta);
-#pragma unroll
-  for (int u = 0; u < 2; ++u) {
-    const int c = t * kTileChunks + lane + 32 * u;
-    if (!full && c >= g.nc) continue;
-    f2 v[NP];
-    chunk_to_pairs(*reinterpret_cast<const uint4 *>(tsm + (lane + 32 * u) * kChunkBytes), v);
-    int lo = 0, hi = E;
-    if (!full) chunk_valid_range(c, g.nc, g.h, hn, E, lo, hi);
-    chunk_normalize<OP, T>(v, s0, s1, gamma, gamma ? p.glen : 0, beta, beta ? p.glen : 0, c,
-                           g.h, p.gvec != 0);
-    store_chunk<T>(v, owin, out_row, c, g.h, lo, hi, p.out_vec != 0);
-  }
-}
-
 // gamma/beta chunk for window chunk c of a row with compile-time head offset
 // H; every column it covers is inside [0, glen) and the vector is 16-byte
 // aligned (the caller checked).
@@ -499,59 +474,117 @@ __device__ __forceinline__ uint4 param_chunk_fixed(const T *__restrict__ g, int 
   }
 }
 
-// pass 2 fast path: tile t lies entirely in the row, the output takes
-// 128-bit stores, and (norms) gamma/beta cover the tile's columns with
-// aligned vector loads.  Same arithmetic as tile_store.
+// pass 2 fast path for one chunk: entirely the row's, output 16-byte
+// congruent to the input, gamma/beta aligned and covering its columns.  Same
+// arithmetic as chunk_store_edge.
 template <int OP, typename T, int H>
-__device__ __forceinline__ void tile_store_fast(const unsigned char *tsm, int t, int lane,
-                                                float s0, float s1, const T *gamma,
-                                                const T *beta, char *owin) {
+__device__ __forceinline__ void chunk_store_fast(const unsigned char *csm, int c, float s0,
+                                                 float s1, const T *gamma, const T *beta,
+                                                 char *owin) {
   constexpr int NP = Elem<T>::kPerChunk / 2;
-#pragma unroll
-  for (int u = 0; u < 2; ++u) {
-    const int c = t * kTileChunks + lane + 32 * u;
-    f2 v[NP], g[NP], b[NP];
-    chunk_to_pairs(*reinterpret_cast<const uint4 *>(tsm + (lane + 32 * u) * kChunkBytes), v);
-    if constexpr (OP == kLayerNorm || OP == kRmsNorm)
-      chunk_to_pairs(param_chunk_fixed<T, H>(gamma, c), g);
-    if constexpr (OP == kLayerNorm) chunk_to_pairs(param_chunk_fixed<T, H>(beta, c), b);
-    normalize_pairs<OP, NP>(v, s0, s1, g, b);
-    stg_stream(owin + static_cast<int64_t>(c) * kChunkBytes, pairs_to_chunk(v));
-  }
+  f2 v[NP], g[NP], b[NP];
+  chunk_to_pairs(*reinterpret_cast<const uint4 *>(csm), v);
+  if constexpr (OP == kLayerNorm || OP == kRmsNorm)
+    chunk_to_pairs(param_chunk_fixed<T, H>(gamma, c), g);
+  if constexpr (OP == kLayerNorm) chunk_to_pairs(param_chunk_fixed<T, H>(beta, c), b);
+  normalize_pairs<OP, NP>(v, s0, s1, g, b);
+  stg_stream(owin + static_cast<int64_t>(c) * kChunkBytes, pairs_to_chunk(v));
 }
 
-// Whether tile t of an item takes the pass-2 fast path.
-template <int OP, typename T>
-__device__ __forceinline__ bool tile_fast(int t, const ItemGeo &g, const TileParams &p,
-                                          bool params_ok) {
-  constexpr int E = Elem<T>::kPerChunk;
-  constexpr bool kAffine = (OP == kLayerNorm || OP == kRmsNorm);
-  // the vector parameter loads reach column (t + 1) * 64 * E - 1 at most
-  return tile_is_full(t, g) && p.out_vec && params_ok &&
-         (!kAffine || static_cast<int64_t>(t + 1) * kTileChunks * E <= p.glen);
-}
-
-// pass 2 fast path over this warp's tiles (wig, wig + W, ...) of an item
-// whose head offset is H
+// pass 2, one chunk the fast path does not take: a row end the row only
+// partly covers, output not 16-byte congruent to the input, or gamma/beta
+// unaligned, absent or ending inside the chunk's window.  Elements outside
+// the row are masked and stored element by element.  Parameters come as
+// aligned vectors realigned for the compile-time head offset H (columns
+// before 0 read as zero and are masked) whenever they are aligned and reach
+// past the chunk, else element by element.
 template <int OP, typename T, int H>
-__device__ __forceinline__ void pass2_fast_tiles(const unsigned char *stage, const ItemGeo &g,
-                                                 int wig, int W, int lane, float s0, float s1,
-                                                 const TileParams &p, char *owin,
-                                                 bool params_ok) {
+__device__ __forceinline__ void chunk_store_edge(const unsigned char *csm, int c, const ItemGeo &g,
+                                                 float s0, float s1, const TileParams &p,
+                                                 char *owin, T *out_row) {
+  constexpr int E = Elem<T>::kPerChunk;
+  constexpr int NP = E / 2;
+  constexpr bool kAffine = (OP == kLayerNorm || OP == kRmsNorm);
+  const int hn = g.h + static_cast<int>(g.n);
+  const T *gamma = static_cast<const T *>(p.gamma);
+  const T *beta = static_cast<const T *>(p.beta);
+  f2 v[NP], gp[NP], bp[NP];
+  chunk_to_pairs(*reinterpret_cast<const uint4 *>(csm), v);
+  int lo, hi;
+  chunk_valid_range(c, g.nc, g.h, hn, E, lo, hi);
+  if constexpr (kAffine) {
+    const bool vec = p.gvec && gamma && (OP == kRmsNorm || beta) && g.h == H &&
+                     static_cast<int64_t>(c + 1) * E <= p.glen;
+    if (vec) {
+      auto realigned = [&](const T *a) {
+        const uint4 *w = reinterpret_cast<const uint4 *>(a);
+        if constexpr (H == 0) {
+          return __ldg(w + c);
+        } else {
+          const uint4 A = c > 0 ? __ldg(w + (c - 1)) : make_uint4(0u, 0u, 0u, 0u);
+          const uint4 B = __ldg(w + c);
+          if constexpr (E == 4) {
+            return shift_words<H>(A, B);
+          } else if constexpr ((H & 1) == 0) {
+            return shift_words<H / 2>(A, B);
+          } else {
+            return shift_half<(H + 1) / 2>(A, B);
+          }
+        }
+      };
+      chunk_to_pairs(realigned(gamma), gp);
+      if constexpr (OP == kLayerNorm) chunk_to_pairs(realigned(beta), bp);
+    } else {
+      load_param_pairs<T>(gamma, gamma ? p.glen : 0, c, g.h, p.gvec != 0, 1.f, gp);
+      if constexpr (OP == kLayerNorm)
+        load_param_pairs<T>(beta, beta ? p.glen : 0, c, g.h, p.gvec != 0, 0.f, bp);
+    }
+  }
+  normalize_pairs<OP, NP>(v, s0, s1, gp, bp);
+  store_chunk<T>(v, owin, out_row, c, g.h, lo, hi, p.out_vec != 0);
+}
+
+// pass 2 over this warp's tiles (wig, wig + W, ...) of an item whose head
+// offset is H.  Chunks [g.cf, cfast) take the fast path, the row's other
+// chunks the general one: tiles made only of fast chunks (all but the row's
+// ends, as a rule) run first with both chunks of a lane issued together, then
+// the remaining tiles chunk by chunk.
+template <int OP, typename T, int H>
+__device__ __forceinline__ void pass2_tiles(const unsigned char *stage, const ItemGeo &g, int wig,
+                                            int W, int lane, float s0, float s1,
+                                            const TileParams &p, char *owin, T *out_row,
+                                            int cfast) {
   const T *gamma = static_cast<const T *>(p.gamma);
   const T *beta = static_cast<const T *>(p.beta);
   const int ntl = g.t1 - g.t0;
+  // tiles [fa, fb) of the row hold only fast chunks
+  const int fa = (g.cf + kTileChunks - 1) / kTileChunks;
+  const int fb = cfast / kTileChunks;
   for (int lt = wig; lt < ntl; lt += W) {
     const int t = g.t0 + lt;
-    if (tile_fast<OP, T>(t, g, p, params_ok))
-      tile_store_fast<OP, T, H>(stage + lt * kTileBytes, t, lane, s0, s1, gamma, beta, owin);
+    if (t < fa || t >= fb) continue;
+#pragma unroll
+    for (int u = 0; u < 2; ++u)
+      chunk_store_fast<OP, T, H>(stage + lt * kTileBytes + (lane + 32 * u) * kChunkBytes,
+                                 t * kTileChunks + lane + 32 * u, s0, s1, gamma, beta, owin);
+  }
+  for (int lt = wig; lt < ntl; lt += W) {
+    const int t = g.t0 + lt;
+    if (t >= fa && t < fb) continue;
+    for (int u = 0; u < 2; ++u) {
+      const int c = t * kTileChunks + lane + 32 * u;
+      const unsigned char *csm = stage + lt * kTileBytes + (lane + 32 * u) * kChunkBytes;
+      if (c >= g.cf && c < cfast) {
+        chunk_store_fast<OP, T, H>(csm, c, s0, s1, gamma, beta, owin);
+      } else if (c < g.nc) {
+        chunk_store_edge<OP, T, H>(csm, c, g, s0, s1, p, owin, out_row);
+      }
+    }
   }
 }
 
-// pass 2 of an item: the fast tiles with the gamma/beta realignment compiled
-// for the item's head offset (one dispatch per item, not per chunk), then the
-// tiles the fast path does not take (the row's ends, unaligned output, rows
-// reaching the end of gamma/beta) through the general path.
+// pass 2 of an item, with the gamma/beta realignment compiled for the item's
+// head offset (one dispatch per item, not per chunk).
 template <int OP, typename T, bool EXACT>
 __device__ __forceinline__ void pass2_item(const unsigned char *stage, const ItemGeo &g, int wig,
                                            int W, int lane, float s0, float s1,
@@ -560,31 +593,31 @@ __device__ __forceinline__ void pass2_item(const unsigned char *stage, const Ite
   constexpr bool kAffine = (OP == kLayerNorm || OP == kRmsNorm);
   const bool params_ok =
       !kAffine || (p.gvec && p.gamma && (OP == kRmsNorm || p.beta != nullptr));
+  // fast chunks end where the row's full chunks end, or where the vector
+  // parameter loads would reach past gamma/beta (they read up to column
+  // (c + 1) * E - 1 for chunk c)
+  int cfast = g.cf;
+  if (p.out_vec && params_ok)
+    cfast = kAffine ? static_cast<int>(min(static_cast<int64_t>(g.cl), p.glen / E)) : g.cl;
   if constexpr (EXACT || !kAffine) {
-    pass2_fast_tiles<OP, T, 0>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok);
+    pass2_tiles<OP, T, 0>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast);
   } else {
     switch (g.h) {
-      case 0: pass2_fast_tiles<OP, T, 0>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
-      case 1: pass2_fast_tiles<OP, T, 1>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
-      case 2: pass2_fast_tiles<OP, T, 2>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
-      case 3: pass2_fast_tiles<OP, T, 3>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
+      case 0: pass2_tiles<OP, T, 0>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+      case 1: pass2_tiles<OP, T, 1>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+      case 2: pass2_tiles<OP, T, 2>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+      case 3: pass2_tiles<OP, T, 3>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
       default:
         if constexpr (E == 8) {
           switch (g.h) {
-            case 4: pass2_fast_tiles<OP, T, 4>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
-            case 5: pass2_fast_tiles<OP, T, 5>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
-            case 6: pass2_fast_tiles<OP, T, 6>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
-            default: pass2_fast_tiles<OP, T, 7>(stage, g, wig, W, lane, s0, s1, p, owin, params_ok); break;
+            case 4: pass2_tiles<OP, T, 4>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+            case 5: pass2_tiles<OP, T, 5>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+            case 6: pass2_tiles<OP, T, 6>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+            default: pass2_tiles<OP, T, 7>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
           }
         }
         break;
     }
-  }
-  const int ntl = g.t1 - g.t0;
-  for (int lt = wig; lt < ntl; lt += W) {
-    const int t = g.t0 + lt;
-    if (!tile_fast<OP, T>(t, g, p, params_ok))
-      tile_store<OP, T, EXACT>(stage + lt * kTileBytes, t, g, lane, s0, s1, p, owin, out_row);
   }
 }
 
