@@ -208,15 +208,17 @@ inline int pick_group_warps(int64_t stage_tiles, bool ragged, int knob) {
 // Shared memory one CTA may spend on stages so that three CTAs fit an SM.
 constexpr int64_t kStageBudgetBytes = 72 * 1024;
 
-// Stages: at least one per group and up to one and a half per group within
-// the three-CTA budget; stages too large for that budget get two per group
-// (launch_tile_k then keeps as many as fit the CTA's shared memory).
+// Stages: one per group and up to one and a half per group within the
+// three-CTA budget (a ragged launch, one group, gets a single stage: three
+// CTAs with one large stage each beat fewer CTAs with two, as measured);
+// stages too large for that budget get two per group (launch_tile_k then
+// keeps as many as fit the CTA's shared memory).
 inline int pick_stages(int64_t stage_tiles, int group_warps, int knob) {
   if (knob > 0) return std::min(knob, 32);
   const int G = kConsumerWarps / group_warps;
   const int64_t fit = kStageBudgetBytes / (stage_tiles * kTileBytes);
-  if (fit >= G) return static_cast<int>(std::max<int64_t>(2, std::min<int64_t>(G + G / 2, fit)));
-  return std::max(2, 2 * G);
+  if (fit >= G) return static_cast<int>(std::min<int64_t>(G + G / 2, fit));
+  return 2 * G;
 }
 
 // Smallest cluster (power of two, >= 2) whose portions of a K-tile row hold
@@ -319,7 +321,13 @@ cudaError_t launch_ragged_t(const RaggedCall &c, const DeviceInfo &d) {
   int cs = 1;
   int64_t st = std::max<int64_t>(1, kmed);
   if (has_large) {
-    cs = pick_cluster(kmax, std::max<int64_t>(kmed, 64), kn.cluster);
+    // rows that fit one CTA's stage budget run whole on one CTA: the
+    // cluster exchange costs more than it saves on them (measured); longer
+    // ones are split over the smallest cluster that brings the portions
+    // within that budget
+    const int64_t budget = kStageBudgetBytes / kTileBytes;
+    cs = (kn.cluster == 0 && kmax <= budget) ? 1
+                                              : pick_cluster(kmax, std::max(kmed, budget), kn.cluster);
     st = std::max<int64_t>(st, ceil_div(kmax, cs));
   }
   if (st > kMaxPortionTiles) return cudaErrorInvalidValue;
