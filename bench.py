@@ -433,7 +433,7 @@ def run_rowop(args, rank, world, local):
         "e2e": {"value": round(world * nbytes / (e2e_ms * 1e-3) / 1e9, 1), "unit": "GB/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": round(e2e_ms, 4)},
-        "roofline": {"bound": "hbm", "kernel": "tile_row_kernel<LayerNorm,bf16,ragged,cluster>",
+        "roofline": {"bound": "hbm", "kernel": "tile_row_kernel<LayerNorm,bf16,ragged> (fused launch)",
                      "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "peak_source": peak_src,
                      "traffic": profile_traffic(),

@@ -1,9 +1,11 @@
 // classify.cuh -- device-side launch_by_rows for ragged rows (§2.1): reads the
 // int64 CSR offsets, gives every row its bucket, and appends each non-empty
 // row's (start, length) record, in increasing row order, to its bucket's list
-// by a block-wide prefix scan.  It also resets the work counters the fused
-// kernel pulls MEDIUM and SMALL rows from.  No host round trip: the fused
-// kernel that follows on the same stream reads the counts from device memory.
+// by a block-wide prefix scan.  Every block handles its own contiguous range
+// of rows and writes into its own segment of each list, plus its per-bucket
+// counts, so blocks never wait on one another; the fused kernel that follows
+// on the same stream turns the block counts into list positions.  No host
+// round trip.
 #pragma once
 
 #include "common.cuh"
@@ -17,13 +19,13 @@ constexpr uint8_t kBucketRejected = 255;
 struct ClassifyParams {
   const int64_t *offsets;
   int64_t rows;
+  int64_t rows_per_block;
   int64_t max_len;
   int esize;
   uint8_t *bucket;          // [rows]
-  RowRec *list[3];       // [rows] each: SMALL, MEDIUM, LARGE
-  int32_t *counts;          // [3]
-  unsigned int *counters;   // [3]
-  unsigned int *ws_status;
+  RowRec *list[3];          // [rows] each: SMALL, MEDIUM, LARGE
+  int32_t *block_counts;    // [blocks][3]
+  unsigned int *ws_status;  // zeroed before the launch
   unsigned int *status;     // device status word
 };
 
@@ -34,10 +36,12 @@ static __global__ void __launch_bounds__(kClassifyThreads)
   const int tid = threadIdx.x;
   const int lane = tid & 31;
   const int warp = tid >> 5;
+  const int64_t row0 = static_cast<int64_t>(blockIdx.x) * p.rows_per_block;
+  const int64_t row1 = min(p.rows, row0 + p.rows_per_block);
   if (tid < 3) base[tid] = 0;
   __syncthreads();
   int any_bad = 0;
-  for (int64_t blk = 0; blk < p.rows;
+  for (int64_t blk = row0; blk < row1;
        blk += static_cast<int64_t>(kClassifyThreads) * kClassifyPerThread) {
     int b[kClassifyPerThread];
     int64_t st[kClassifyPerThread], ln[kClassifyPerThread];
@@ -49,7 +53,7 @@ static __global__ void __launch_bounds__(kClassifyThreads)
       b[i] = -1;  // not listed
       st[i] = 0;
       ln[i] = 0;
-      if (r < p.rows) {
+      if (r < row1) {
         st[i] = p.offsets[r];
         ln[i] = p.offsets[r + 1] - st[i];
         if (ln[i] < 0 || ln[i] > p.max_len) {
@@ -104,7 +108,7 @@ static __global__ void __launch_bounds__(kClassifyThreads)
         RowRec rec;
         rec.start = st[i];
         rec.n = ln[i];
-        p.list[b[i]][pos[b[i]]++] = rec;
+        p.list[b[i]][row0 + pos[b[i]]++] = rec;
       }
     }
     __syncthreads();
@@ -116,14 +120,13 @@ static __global__ void __launch_bounds__(kClassifyThreads)
   }
   any_bad = __syncthreads_or(any_bad);
   if (tid == 0) {
-    p.counts[0] = base[0];
-    p.counts[1] = base[1];
-    p.counts[2] = base[2];
-    p.counters[0] = 0u;
-    p.counters[1] = 0u;
-    p.counters[2] = 0u;
-    *p.ws_status = any_bad ? kStatusBadOffsets : 0u;
-    if (any_bad) atomicOr(p.status, kStatusBadOffsets);
+    p.block_counts[3 * blockIdx.x + 0] = base[0];
+    p.block_counts[3 * blockIdx.x + 1] = base[1];
+    p.block_counts[3 * blockIdx.x + 2] = base[2];
+    if (any_bad) {
+      atomicOr(p.ws_status, kStatusBadOffsets);
+      atomicOr(p.status, kStatusBadOffsets);
+    }
   }
 }
 

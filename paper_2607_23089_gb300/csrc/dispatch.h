@@ -40,18 +40,36 @@ struct RaggedCall {
   bool classify;  // run the classify pass first (false: reuse a plan in ws)
 };
 
-// Ragged workspace layout (bytes): [0,4) status bits of the call, [64,76)
-// int32 counts per bucket, [128,140) uint32 work counters, [256, 256+rows)
-// uint8 bucket per row, then three lists (SMALL, MEDIUM, LARGE) of `rows`
-// records {int64 start, int64 length} each, starting at
-// ragged_lists_offset(rows).
+// Ragged workspace layout (bytes): [0,4) status bits of the call, [128,140)
+// uint32 work counters, [256, 256+rows) uint8 bucket per row, then the int32
+// per-bucket row counts of every classify block ([blocks][3], at
+// ragged_counts_offset(rows)), then three lists (SMALL, MEDIUM, LARGE) of
+// `rows` records {int64 start, int64 length} each, starting at
+// ragged_lists_offset(rows).  Classify block b handles rows
+// [b*rpb, (b+1)*rpb) (rpb = ragged_rows_per_block(rows)) and writes its
+// records, in row order, from entry b*rpb of each list on.
 constexpr size_t kWsStatus = 0;
-constexpr size_t kWsCounts = 64;
 constexpr size_t kWsCounters = 128;
+constexpr size_t kWsHeader = 256;  // [0, 256) is zeroed before the classify launch
 constexpr size_t kWsBuckets = 256;
 constexpr size_t kWsRecordBytes = 16;
-constexpr size_t ragged_lists_offset(int64_t rows) {
+constexpr int64_t kClassifyRowsPerBlock = 1024;
+constexpr int64_t kClassifyMaxBlocks = 256;
+constexpr int64_t ragged_blocks(int64_t rows) {
+  return rows <= 0 ? 1
+                   : ((rows + kClassifyRowsPerBlock - 1) / kClassifyRowsPerBlock < kClassifyMaxBlocks
+                          ? (rows + kClassifyRowsPerBlock - 1) / kClassifyRowsPerBlock
+                          : kClassifyMaxBlocks);
+}
+constexpr int64_t ragged_rows_per_block(int64_t rows) {
+  return rows <= 0 ? 1 : (rows + ragged_blocks(rows) - 1) / ragged_blocks(rows);
+}
+constexpr size_t ragged_counts_offset(int64_t rows) {
   return (kWsBuckets + static_cast<size_t>(rows) + 255) & ~static_cast<size_t>(255);
+}
+constexpr size_t ragged_lists_offset(int64_t rows) {
+  return (ragged_counts_offset(rows) + 12 * static_cast<size_t>(ragged_blocks(rows)) + 255) &
+         ~static_cast<size_t>(255);
 }
 constexpr size_t ragged_ws_bytes(int64_t rows) {
   return ragged_lists_offset(rows) + 3 * kWsRecordBytes * static_cast<size_t>(rows) + 256;

@@ -139,7 +139,7 @@ cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int
   while (static_cast<uint64_t>(stages) * p.stage_bytes < min_stage_area) ++stages;
   const auto total = [&](int s, int w) {
     return TileSmemLayout(p.stage_bytes, s, stage_tiles, kConsumerWarps / w, CLUSTER,
-                          !CLUSTER || RAGGED).total;
+                          !CLUSTER || RAGGED, RAGGED ? p.blocks : 0).total;
   };
   // as many of the wanted stages as fit in the CTA's shared memory, at least
   // one per group: fewer, larger groups when even that does not fit
@@ -311,7 +311,9 @@ cudaError_t launch_ragged_t(const RaggedCall &c, const DeviceInfo &d) {
   p.rec_small = list0;
   p.rec_medium = list0 + c.rows;
   p.rec_large = list0 + 2 * c.rows;
-  p.counts = reinterpret_cast<const int32_t *>(ws + kWsCounts);
+  p.block_counts = reinterpret_cast<const int32_t *>(ws + ragged_counts_offset(c.rows));
+  p.blocks = static_cast<int>(ragged_blocks(c.rows));
+  p.rows_per_block = ragged_rows_per_block(c.rows);
   p.counters = reinterpret_cast<unsigned int *>(ws + kWsCounters);
 
   const int64_t kmax = ceil_div(ceil_div(c.max_len + E - 1, E), kTileChunks);

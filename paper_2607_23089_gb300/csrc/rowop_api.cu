@@ -48,17 +48,21 @@ cudaError_t launch_classify(const RaggedCall &c, const DeviceInfo &d) {
   ClassifyParams cp;
   cp.offsets = c.offsets;
   cp.rows = c.rows;
+  cp.rows_per_block = ragged_rows_per_block(c.rows);
   cp.max_len = c.max_len;
   cp.esize = c.dtype == 0 ? 4 : 2;
   cp.bucket = ws + kWsBuckets;
   cp.list[0] = list0;
   cp.list[1] = list0 + c.rows;
   cp.list[2] = list0 + 2 * c.rows;
-  cp.counts = reinterpret_cast<int32_t *>(ws + kWsCounts);
-  cp.counters = reinterpret_cast<unsigned int *>(ws + kWsCounters);
+  cp.block_counts = reinterpret_cast<int32_t *>(ws + ragged_counts_offset(c.rows));
   cp.ws_status = reinterpret_cast<unsigned int *>(ws + kWsStatus);
   cp.status = d.status;
-  ragged_classify_kernel<<<1, kClassifyThreads, 0, c.stream>>>(cp);
+  // status bits and work counters start at zero
+  cudaError_t e = cudaMemsetAsync(ws, 0, kWsHeader, c.stream);
+  if (e != cudaSuccess) return e;
+  const int blocks = static_cast<int>(ragged_blocks(c.rows));
+  ragged_classify_kernel<<<blocks, kClassifyThreads, 0, c.stream>>>(cp);
   return cudaGetLastError();
 }
 

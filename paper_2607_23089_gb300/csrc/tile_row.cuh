@@ -69,8 +69,10 @@ struct TileParams {
   const RowRec *rec_small;
   const RowRec *rec_medium;
   const RowRec *rec_large;
-  const int32_t *counts;   // [3]: SMALL, MEDIUM, LARGE
-  unsigned int *counters;  // [3]: next MEDIUM, next SMALL, CTAs finished
+  const int32_t *block_counts;  // [blocks][3] rows per bucket of each classify block
+  int blocks;                   // classify blocks (0: dense launch)
+  int64_t rows_per_block;       // classify block b lists from entry b * rows_per_block on
+  unsigned int *counters;       // [3]: next MEDIUM, next SMALL, CTAs finished
 };
 
 struct ItemMeta {
@@ -87,11 +89,11 @@ struct ItemMeta {
 // (xw); the partials of a short split row gathered from the peers (gather);
 // the cluster barriers ready / released, one per buffer.
 struct TileSmemLayout {
-  uint32_t part_c, part_m, gather, meta, xw, bar_meta, bar_piece, bar_empty, bar_ready,
+  uint32_t part_c, part_m, gather, meta, xw, pref, bar_meta, bar_piece, bar_empty, bar_ready,
       bar_released, flags, total;
   int pieces;
   __host__ __device__ TileSmemLayout(uint32_t stage_bytes, int stages, int max_tiles, int groups,
-                                     bool split_items, bool local_items) {
+                                     bool split_items, bool local_items, int blocks) {
     pieces = (max_tiles + kPieceTiles - 1) / kPieceTiles;
     const uint32_t part_bytes = static_cast<uint32_t>(groups) * 2u * max_tiles * 16u;
     uint32_t off = stage_bytes * stages;
@@ -105,6 +107,8 @@ struct TileSmemLayout {
     off += stages * 32u;
     xw = off;
     off += static_cast<uint32_t>(groups) * 2u * kConsumerWarps * 4u;
+    pref = off;  // ragged: [3][blocks + 1] list position where each classify block starts
+    off += (3u * (blocks + 1) * 4u + 15u) & ~15u;
     bar_meta = off;
     off += stages * 8u;
     bar_piece = off;
@@ -678,6 +682,23 @@ __device__ __forceinline__ void complete_pending(PendingEdges &pe) {
   pe.active = false;
 }
 
+// Record `idx` of a bucket's list: the classify block b with
+// pref[b] <= idx < pref[b + 1] wrote it at entry b * rows_per_block +
+// (idx - pref[b]) of the list (pref: that bucket's [blocks + 1] starts).
+__device__ __forceinline__ RowRec ragged_record(const TileParams &p, const int *pref,
+                                                const RowRec *list, int64_t idx) {
+  int lo = 0, hi = p.blocks;  // pref[lo] <= idx < pref[hi]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (pref[mid] <= idx) {
+      lo = mid;
+    } else {
+      hi = mid;
+    }
+  }
+  return list[static_cast<int64_t>(lo) * p.rows_per_block + (idx - pref[lo])];
+}
+
 template <typename T, bool EXACT, bool CLUSTER, bool RAGGED>
 __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSmemLayout &L,
                                               unsigned char *smem, int cs, int rank, int64_t cid,
@@ -690,6 +711,8 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
   ItemMeta *meta = reinterpret_cast<ItemMeta *>(smem + L.meta);
   volatile int *flags = reinterpret_cast<volatile int *>(smem + L.flags);
   const uint64_t pol = l2_evict_first_policy();
+  const int *pref = reinterpret_cast<const int *>(smem + L.pref);
+  const int nb1 = p.blocks + 1;
   int64_t k_large = 0, k_dense = 0;
   bool medium_phase = false;
   PendingEdges pend;
@@ -705,8 +728,8 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
     if (RAGGED) {
       if (!medium_phase) {
         const int64_t li = cid + k_large * ncl;
-        if (li < p.counts[2]) {
-          const RowRec r = p.rec_large[li];
+        if (li < pref[2 * nb1 + p.blocks]) {
+          const RowRec r = ragged_record(p, pref + 2 * nb1, p.rec_large, li);
           ++k_large;
           kind = kItemLarge;
           start = r.start;
@@ -717,8 +740,8 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
       }
       if (medium_phase) {
         const unsigned int m = atomicAdd(&p.counters[0], 1u);
-        if (m < static_cast<unsigned int>(p.counts[1])) {
-          const RowRec r = p.rec_medium[m];
+        if (m < static_cast<unsigned int>(pref[nb1 + p.blocks])) {
+          const RowRec r = ragged_record(p, pref + nb1, p.rec_medium, m);
           kind = kItemMedium;
           start = r.start;
           n = r.n;
@@ -837,7 +860,8 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
   extern __shared__ __align__(1024) unsigned char smem[];
   const int W = p.group_warps;
   const int G = kConsumerWarps / W;
-  const TileSmemLayout L(p.stage_bytes, p.stages, p.max_tiles, G, CLUSTER, !CLUSTER || RAGGED);
+  const TileSmemLayout L(p.stage_bytes, p.stages, p.max_tiles, G, CLUSTER, !CLUSTER || RAGGED,
+                         RAGGED ? p.blocks : 0);
   const int S = p.stages;
   const int tid = threadIdx.x;
   const int lane = tid & 31;
@@ -862,6 +886,24 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
     }
     flags[0] = 0;
     fence_mbar_init();
+  }
+  if (RAGGED && warp < 3) {
+    // warp k: exclusive scan of bucket k's row counts over the classify blocks
+    int *pref = reinterpret_cast<int *>(smem + L.pref) + warp * (p.blocks + 1);
+    int carry = 0;
+    for (int b0 = 0; b0 < p.blocks; b0 += 32) {
+      const int b = b0 + lane;
+      const int v = b < p.blocks ? p.block_counts[3 * b + warp] : 0;
+      int x = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(kFullMask, x, o);
+        if (lane >= o) x += y;
+      }
+      if (b < p.blocks) pref[b] = carry + x - v;
+      carry += __shfl_sync(kFullMask, x, 31);
+    }
+    if (lane == 0) pref[p.blocks] = carry;
   }
   __syncthreads();
   if (CLUSTER) cluster_sync();  // every peer's barriers exist before any remote arrive
@@ -1004,8 +1046,9 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
       unsigned int idx = 0;
       if (lane == 0) idx = atomicAdd(&p.counters[1], 1u);
       idx = __shfl_sync(kFullMask, idx, 0);
-      if (idx >= static_cast<unsigned int>(p.counts[0])) break;
-      const RowRec rec = p.rec_small[idx];
+      const int *pref = reinterpret_cast<const int *>(smem + L.pref);  // SMALL: bucket 0
+      if (idx >= static_cast<unsigned int>(pref[p.blocks])) break;
+      const RowRec rec = ragged_record(p, pref, p.rec_small, idx);
       const T *in_row = in + rec.start;
       const uintptr_t ia = reinterpret_cast<uintptr_t>(in_row);
       const int h = static_cast<int>((ia & 15) / SZ);

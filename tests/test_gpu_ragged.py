@@ -225,3 +225,52 @@ def test_ragged_group_sizes_agree(rw, op, dtype, monkeypatch):
         got = run_ragged(rw, op, dtype, lens, max_len, seed=43, base_off=1)["y"]
         assert rw.check_status() == 0
         assert torch.equal(bits(ref), bits(got)), f"W={w} cluster={cs}"
+
+
+@pytest.mark.parametrize("rows", [1025, 5000, 300000])
+def test_ragged_many_classify_blocks(rw, rows):
+    """Enough rows for several classify blocks (1024 rows each, at most 256
+    blocks): every block lists its own rows and the fused kernel maps list
+    positions across blocks.  Rows of every bucket sit in different blocks,
+    some rejected; values, dispatch bytes and the status all check out."""
+    dtype = torch.bfloat16
+    op = "layernorm"
+    g = np.random.default_rng(rows)
+    max_len = 20000
+    lens = g.integers(0, 40, size=rows)
+    lens[::997] = 3000      # MEDIUM
+    lens[5::1999] = 19000   # LARGE
+    lens[7::2503] = 0
+    r = run_ragged(rw, op, dtype, lens, max_len, seed=rows % 97)
+    assert rw.check_status() == 0
+    ref = oracle_ragged(op, r["x"].double().numpy(), r["off"], r["gam"].double().numpy(),
+                        r["bet"].double().numpy(), r["eps"])
+    assert_close(to_f64(r["y"]), ref, dtype, f"ragged {rows} rows")
+    buckets = r["ws"][256:256 + rows].cpu().numpy()
+    want = np.array([orc.bucket(int(n), ESIZE[dtype]) for n in lens], dtype=np.uint8)
+    assert (buckets == want).all()
+
+
+def test_ragged_bad_rows_in_several_blocks(rw):
+    """Rejected rows in different classify blocks all raise the status bit of
+    the call and are skipped; the others are normalised."""
+    dtype = torch.float32
+    rows = 3000
+    g = np.random.default_rng(3)
+    lens = g.integers(1, 300, size=rows)
+    bad = [10, 1500, 2990]
+    lens[bad] = 500  # longer than max_len
+    r = run_ragged(rw, "softmax", dtype, lens, 400, seed=5)
+    assert rw.check_status() == rw.ROWOP_ERR_BAD_OFFSETS
+    buckets = r["ws"][256:256 + rows].cpu().numpy()
+    assert all(buckets[i] == 255 for i in bad)
+    assert r["ws"][:4].view(torch.int32).item() == 2
+    off = r["off"]
+    for i in bad:
+        assert is_canary(r["y"][int(off[i]):int(off[i + 1])]).all()
+    good = np.ones(rows, dtype=bool)
+    good[bad] = False
+    for i in np.flatnonzero(good)[::97]:
+        seg = r["y"][int(off[i]):int(off[i + 1])]
+        ref = orc.softmax(r["x"][int(off[i]):int(off[i + 1])].double().numpy()[None])[0]
+        assert_close(to_f64(seg), ref, dtype, f"row {i}")
