@@ -192,16 +192,14 @@ cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int
   return cudaGetLastError();
 }
 
-// Consumer warps per item group.  Dense rows of a few tiles: several groups,
-// so one group's waits overlap the others' work while each warp still has a
-// few tiles per item.  Ragged launches keep one group of 8: their items are
-// of mixed size and two fixed-size stages per CTA is all that lets three
-// CTAs share an SM (measured fastest on the ragged workload).
+// Consumer warps per item group.  Items of a few tiles (dense rows of up to
+// 16 KiB): groups of 2 warps, so several items are in work per CTA and one
+// group's waits overlap the others' work.  Larger items: one group of all 8
+// warps and a single stage, which keeps three CTAs on every SM -- measured
+// faster than fewer CTAs that stage ahead (workloads 4 and 5).
 inline int pick_group_warps(int64_t stage_tiles, bool ragged, int knob) {
   if (knob == 1 || knob == 2 || knob == 4 || knob == 8) return knob;
-  if (ragged) return 8;
-  if (stage_tiles <= 16) return 2;
-  if (stage_tiles <= 64) return 4;
+  if (!ragged && stage_tiles <= 16) return 2;
   return 8;
 }
 
@@ -263,9 +261,10 @@ cudaError_t launch_dense_t(const DenseCall &c, const DeviceInfo &d) {
   p.gvec = gvec;
   p.timeout_ns = kWaitLimitNs;
   p.status = d.status;
-  // portions of up to 128 tiles: a 1 MiB fp32 row goes to clusters of 8
-  // (19 clusters fill the 152 SMs; 16-CTA clusters would leave 8 idle)
-  const int cs = bucket == kMedium ? 1 : pick_cluster(K, 128, kn.cluster);
+  // portions within the three-CTA stage budget: a 1 MiB fp32 row goes to
+  // clusters of 16 with 64 KiB per CTA, three CTAs per SM (0.17 ms on
+  // workload 4 against 0.23 ms for clusters of 8 with 128 KiB, one per SM)
+  const int cs = bucket == kMedium ? 1 : pick_cluster(K, kStageBudgetBytes / kTileBytes, kn.cluster);
   const int st = static_cast<int>(ceil_div(K, cs));
   if (st > kMaxPortionTiles) return cudaErrorInvalidValue;
   const int W = pick_group_warps(st, false, kn.group_warps);
