@@ -105,8 +105,11 @@ __device__ __forceinline__ void load_param_pairs(const T *__restrict__ g, int64_
     chunk_to_pairs(__ldg(reinterpret_cast<const uint4 *>(g + j0)), out);
     return;
   }
-  if (vec && h > 0 && c >= 1 && (c + 1) * E <= glen) {
-    const uint4 A = __ldg(reinterpret_cast<const uint4 *>(g + (c - 1) * E));
+  if (vec && h > 0 && (c + 1) * E <= glen) {
+    // columns before 0 (chunk 0 of the row) read as zero: they lie outside
+    // the row and are never used
+    const uint4 A = c >= 1 ? __ldg(reinterpret_cast<const uint4 *>(g + (c - 1) * E))
+                           : make_uint4(0u, 0u, 0u, 0u);
     const uint4 B = __ldg(reinterpret_cast<const uint4 *>(g + c * E));
     chunk_to_pairs(shift_chunk<T>(A, B, h), out);
     return;

@@ -170,10 +170,9 @@ __device__ __forceinline__ bool tile_is_full(int t, const ItemGeo &g) {
 //   softmax / log-softmax  (m_t, s_t = sum exp(x - m_t))
 //   LayerNorm              (sum_t, mean_t, sum (x - mean_t)^2, n_t)
 //   RMSNorm                (sum x^2)
-// A warp takes up to kPass1Batch of its tiles at once, so several independent
-// shuffle chains are in flight.
+// A warp takes up to PB (4 or 2) of its tiles at once, so several
+// independent shuffle chains are in flight.
 // ---------------------------------------------------------------------------
-constexpr int kPass1Batch = 4;
 
 struct TileMask {
   int lo0, hi0, lo1, hi1;  // valid element ranges of the lane's two chunks
@@ -312,10 +311,10 @@ __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const It
 }
 
 // Pass 1 of an item for warp `wig` of a group of W warps: part[lt] for its
-// tiles lt = wig, wig + W, ..., taken kPass1Batch at a time while that many
-// remain, then in a batch of two and one.  Each tile's arithmetic (and its butterfly order) is the same
-// whatever batch it falls in.
-template <int OP, typename T>
+// tiles lt = wig, wig + W, ..., taken PB at a time while that many remain,
+// then in a batch of two and one.  Each tile's arithmetic (and its butterfly
+// order) is the same whatever batch it falls in.
+template <int OP, typename T, int PB>
 __device__ __forceinline__ bool pass1_warp(const unsigned char *stage, const ItemGeo &g, int wig,
                                            int W, int lane, float4 *part, uint32_t piece_bar0,
                                            uint32_t par, uint64_t timeout_ns) {
@@ -327,15 +326,15 @@ __device__ __forceinline__ bool pass1_warp(const unsigned char *stage, const Ite
   int lt0 = wig;
   while (lt0 < ntl) {
     const int left = (ntl - lt0 + W - 1) / W;
-    const int bsz = left >= kPass1Batch ? kPass1Batch : (left >= 2 ? 2 : 1);
+    const int bsz = left >= PB ? PB : (left >= 2 ? 2 : 1);
     const int ta = g.t0 + lt0, tb = ta + (bsz - 1) * W;
     const bool full = ta >= full0 && tb < full1;
     bool ok;
-    if (bsz == kPass1Batch) {
-      ok = full ? pass1_batch<OP, T, kPass1Batch, true>(stage, g, lt0, W, lane, part, piece_bar0,
-                                                         par, timeout_ns, waited)
-                : pass1_batch<OP, T, kPass1Batch, false>(stage, g, lt0, W, lane, part,
-                                                          piece_bar0, par, timeout_ns, waited);
+    if (PB > 2 && bsz == PB) {
+      ok = full ? pass1_batch<OP, T, PB, true>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                                               timeout_ns, waited)
+                : pass1_batch<OP, T, PB, false>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                                                timeout_ns, waited);
     } else if (bsz == 2) {
       ok = full ? pass1_batch<OP, T, 2, true>(stage, g, lt0, W, lane, part, piece_bar0, par,
                                               timeout_ns, waited)
@@ -858,6 +857,12 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
   constexpr int E = Elem<T>::kPerChunk;
   constexpr int SZ = Elem<T>::kSize;
   extern __shared__ __align__(1024) unsigned char smem[];
+  // pass-1 batch: four tiles for dense one-CTA rows (groups of two warps, few
+  // tiles each), two with the cluster exchange, one in the ragged kernel,
+  // whose 72 registers also carry the edge paths and the SMALL phase: larger
+  // batches spill there (ragged bf16 LayerNorm 0.58 / 0.40 / 0.32 ms with
+  // batches of 4 / 2 / 1)
+  constexpr int kPass1Batch = RAGGED ? 1 : (CLUSTER ? 2 : 4);
   const int W = p.group_warps;
   const int G = kConsumerWarps / W;
   const TileSmemLayout L(p.stage_bytes, p.stages, p.max_tiles, G, CLUSTER, !CLUSTER || RAGGED,
@@ -955,7 +960,7 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
 
     // ---- pass 1 ----
     if (!bad && kind != kItemEnd)
-      bad = !pass1_warp<OP, T>(stage, g, wig, W, lane, part,
+      bad = !pass1_warp<OP, T, kPass1Batch>(stage, g, wig, W, lane, part,
                                sbase + L.bar_piece + 8u * (s * L.pieces), par, p.timeout_ns);
     if (named_sync_or(gbar, gthreads, bad)) {
       if (gtid == 0) {
