@@ -32,6 +32,7 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "rowop_oracle.c")
+_SRCS = [_SRC, os.path.join(_HERE, "pad_moe_oracle.c")]
 _BUILD_DIR = os.path.join(_HERE, "_build")
 _LIB_PATH = os.path.join(_BUILD_DIR, "liboracle.so")
 _lock = threading.Lock()
@@ -41,16 +42,16 @@ SMALL, MEDIUM, LARGE = 0, 1, 2
 
 
 def build(force: bool = False) -> str:
-    """Compile ``rowop_oracle.c`` with gcc (-O2, no fast-math) into a shared
-    library next to it.  OpenMP is used when the compiler offers it; without
-    it the row loop simply runs on one thread."""
+    """Compile ``rowop_oracle.c`` and ``pad_moe_oracle.c`` with gcc (-O2, no
+    fast-math) into a shared library next to them.  OpenMP is used when the
+    compiler offers it; without it the row loop simply runs on one thread."""
     os.makedirs(_BUILD_DIR, exist_ok=True)
     if (not force and os.path.exists(_LIB_PATH)
-            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+            and all(os.path.getmtime(_LIB_PATH) >= os.path.getmtime(s) for s in _SRCS)):
         return _LIB_PATH
     tmp = _LIB_PATH + f".tmp{os.getpid()}"
     base = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fno-fast-math",
-            "-ffp-contract=off", _SRC, "-o", tmp, "-lm"]
+            "-ffp-contract=off", *_SRCS, "-o", tmp, "-lm"]
     try:
         subprocess.run(base[:1] + ["-fopenmp"] + base[1:], check=True,
                        capture_output=True)
@@ -78,10 +79,13 @@ def _load():
         lib.oracle_rmsnorm_ragged.argtypes = [d, d, d, d, i64, dbl, ci]
         lib.oracle_bucket.argtypes = [i64, i64]
         lib.oracle_bucket.restype = ci
+        lib.oracle_pad_scale.argtypes = [d, d, i64, i64, i64, dbl]
+        lib.oracle_moe_group_top2.argtypes = [d, d, i64, i64, i64]
         for name in ("oracle_softmax", "oracle_logsoftmax", "oracle_layernorm",
                      "oracle_rmsnorm", "oracle_softmax_ragged",
                      "oracle_logsoftmax_ragged", "oracle_layernorm_ragged",
-                     "oracle_rmsnorm_ragged"):
+                     "oracle_rmsnorm_ragged", "oracle_pad_scale",
+                     "oracle_moe_group_top2"):
             getattr(lib, name).restype = None
         _lib = lib
         return lib
@@ -212,3 +216,35 @@ def bucket(length: int, esize: int) -> int:
 __all__ = ["build", "softmax", "logsoftmax", "layernorm", "rmsnorm",
            "softmax_ragged", "logsoftmax_ragged", "layernorm_ragged",
            "rmsnorm_ragged", "bucket", "SMALL", "MEDIUM", "LARGE"]
+
+
+# ---------------------------------------------------------------------------
+# Hyena FFT-size padding and the MoE group score (pad_moe_oracle.c)
+# ---------------------------------------------------------------------------
+def pad_scale(x, fft_size: int, scale: float):
+    """``y[r, c] = scale * x[r, c]`` for ``c < seqlen``, then zeros up to
+    ``fft_size`` (§6).  ``scale`` is taken as the float32 value the GPU
+    multiplies by, widened to double; the product of two float32 values is
+    exact in double."""
+    x = _f64(x)
+    if x.ndim != 2:
+        raise ValueError("pad_scale wants a 2-D rows x seqlen array")
+    rows, seqlen = x.shape
+    if fft_size < seqlen:
+        raise ValueError("fft_size < seqlen")
+    y = np.empty((rows, fft_size), dtype=np.float64)
+    _load().oracle_pad_scale(_ptr(x), _ptr(y), rows, seqlen, fft_size,
+                             float(np.float32(scale)))
+    return y
+
+
+def moe_group_top2(scores, group: int = 32):
+    """``out[t, g] = max_{i != j} (v_i + v_j)`` over each group of ``group``
+    consecutive scores of token ``t`` (§2.1), by brute force over the pairs."""
+    v = _f64(scores)
+    if v.ndim != 2 or v.shape[1] % group:
+        raise ValueError("moe_group_top2 wants tokens x experts, experts a multiple of group")
+    tokens, experts = v.shape
+    out = np.empty((tokens, experts // group), dtype=np.float64)
+    _load().oracle_moe_group_top2(_ptr(v), _ptr(out), tokens, experts, group)
+    return out

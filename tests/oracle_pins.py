@@ -253,6 +253,57 @@ def pin_bucket_rule(orc):
         assert orc.bucket(1 << 20, esize) == 2
 
 
+def pin_pad_scale(orc):
+    """Hyena FFT-size padding (§6): a hand-worked case, the zero tail, the
+    identity at scale 1, linearity in the scale and row independence."""
+    x = np.array([[1.0, 2.0, 3.0], [4.0, 5.0, 6.0]])
+    want = np.array([[0.5, 1.0, 1.5, 0.0, 0.0], [2.0, 2.5, 3.0, 0.0, 0.0]])
+    _close(orc.pad_scale(x, 5, 0.5), want, rtol=0, atol=0)
+    g = np.random.default_rng(11)
+    x = g.standard_normal((7, 13)).astype(np.float32).astype(np.float64)
+    y = orc.pad_scale(x, 32, 0.25)
+    assert y.shape == (7, 32)
+    assert (y[:, 13:] == 0).all()
+    _close(orc.pad_scale(x, 13, 1.0), x, rtol=0, atol=0)
+    _close(orc.pad_scale(x, 20, 0.75), orc.pad_scale(x, 20, 0.5) + orc.pad_scale(x, 20, 0.25))
+    perm = g.permutation(7)
+    _close(orc.pad_scale(x[perm], 20, 0.5), orc.pad_scale(x, 20, 0.5)[perm], rtol=0, atol=0)
+    # every live element is the scaled input element at the same position
+    for r, c in ((0, 0), (3, 7), (6, 12)):
+        assert y[r, c] == 0.25 * x[r, c]
+
+
+def pin_moe_group_top2(orc):
+    """MoE group score (§2.1): hand cases with ties and masked experts, the
+    paper's statement that the largest off-diagonal pair sum is the sum of
+    the two largest values (checked by sorting), invariance under permuting a
+    group, and a shift by c moving the score by 2c."""
+    inf = np.inf
+    cases = [([5.0, 5.0, 1.0, 2.0], 10.0), ([1.0, 2.0, 3.0, 4.0], 7.0),
+             ([-inf, 3.0, -inf, -inf], -inf), ([3.0, -1.0, -2.0, -5.0], 2.0),
+             ([-inf, -inf, -inf, -inf], -inf), ([0.5, 0.5, 0.5, 0.5], 1.0)]
+    for v, want in cases:
+        got = orc.moe_group_top2(np.array([v]), group=4)
+        assert got.shape == (1, 1)
+        assert got[0, 0] == want, (v, got, want)
+    g = np.random.default_rng(12)
+    # coarse values so that ties, including tied maxima, are frequent
+    v = np.round(g.standard_normal((50, 256)) * 4) / 4
+    v[3, 40:72] = 1.0
+    v[7, :32] = -inf
+    v[7, 5] = 2.0
+    got = orc.moe_group_top2(v)
+    assert got.shape == (50, 8)
+    top2 = np.sort(v.reshape(50, 8, 32), axis=2)[:, :, -2:].sum(axis=2)
+    _close(got, top2, rtol=0, atol=0)
+    assert got[3, 1] == 2.0 or got[3, 1] >= 2.0
+    assert got[7, 0] == -inf
+    perm = g.permutation(32)
+    w = v.reshape(50, 8, 32)[:, :, perm].reshape(50, 256)
+    _close(orc.moe_group_top2(w), got, rtol=0, atol=0)
+    _close(orc.moe_group_top2(v + 1.5), got + 3.0, rtol=0, atol=0)
+
+
 ALL_PINS = [pin_hand_cases, pin_softmax_invariants, pin_layernorm_invariants,
             pin_rmsnorm_invariants, pin_brute_force, pin_torch_float64,
-            pin_ragged, pin_bucket_rule]
+            pin_ragged, pin_bucket_rule, pin_pad_scale, pin_moe_group_top2]

@@ -12,6 +12,7 @@ from tests.oracle_pins import ALL_PINS
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 SRC = os.path.join(ROOT, "oracle", "rowop_oracle.c")
+SRC_PM = os.path.join(ROOT, "oracle", "pad_moe_oracle.c")
 WRAPPER = os.path.join(ROOT, "oracle", "rowop_oracle.py")
 
 # (function whose body is edited, text, replacement, what the mistake is)
@@ -44,7 +45,20 @@ MUTANTS = [
      "SMALL threshold off by one"),
     ("oracle_bucket", "bytes <= 32768", "bytes <= 65536",
      "MEDIUM threshold"),
+    ("oracle_pad_scale", "c < seqlen ?", "c <= seqlen - 2 ?", "last live column zeroed"),
+    ("oracle_pad_scale", "scale * x[r * seqlen + c]", "x[r * seqlen + c]", "scale dropped"),
+    ("oracle_pad_scale", "x[r * seqlen + c]", "x[r * seqlen + (seqlen - 1 - c)]",
+     "row read backwards"),
+    ("oracle_moe_group_top2", "if (i != j && ", "if (", "pair of a score with itself"),
+    ("oracle_moe_group_top2", "g * group", "g", "groups overlap"),
+    ("oracle_moe_group_top2", "j < group;", "j < group - 1 && i < group - 1;",
+     "last member skipped"),
+    ("oracle_moe_group_top2", "w[i] + w[j] > best", "w[i] + w[j] >= best + 1.0",
+     "comparison off"),
 ]
+
+# functions defined in pad_moe_oracle.c rather than rowop_oracle.c
+PM_FUNCS = {"oracle_pad_scale", "oracle_moe_group_top2"}
 
 
 def _mutate(src: str, func: str, old: str, new: str) -> str:
@@ -57,14 +71,16 @@ def _mutate(src: str, func: str, old: str, new: str) -> str:
     return src[:start] + body.replace(old, new, 1) + src[end:]
 
 
-def _load_mutant(tmp_path, text):
+def _load_mutant(tmp_path, text, text_pm):
     d = tmp_path / "mut"
     d.mkdir()
     (d / "rowop_oracle.c").write_text(text)
+    (d / "pad_moe_oracle.c").write_text(text_pm)
     spec = importlib.util.spec_from_file_location("oracle_mutant", WRAPPER)
     mod = importlib.util.module_from_spec(spec)
     spec.loader.exec_module(mod)
     mod._SRC = str(d / "rowop_oracle.c")
+    mod._SRCS = [str(d / "rowop_oracle.c"), str(d / "pad_moe_oracle.c")]
     mod._BUILD_DIR = str(d / "_build")
     mod._LIB_PATH = str(d / "_build" / "liboracle.so")
     mod._lib = None
@@ -76,7 +92,13 @@ def _load_mutant(tmp_path, text):
 def test_pins_catch_mutant(tmp_path, func, old, new, what):
     with open(SRC) as f:
         src = f.read()
-    mod = _load_mutant(tmp_path, _mutate(src, func, old, new))
+    with open(SRC_PM) as f:
+        src_pm = f.read()
+    if func in PM_FUNCS:
+        src_pm = _mutate(src_pm, func, old, new)
+    else:
+        src = _mutate(src, func, old, new)
+    mod = _load_mutant(tmp_path, src, src_pm)
     caught = []
     for pin in ALL_PINS:
         try:
