@@ -197,6 +197,10 @@ def per_config(torch, rw, wl, device, peak, steps):
             ws = rw.ragged_workspace(case.rows, device)
             fn = lambda: rw.run(case.op, x, offsets=off, max_len=case.max_len,  # noqa: E731
                                 gamma=g, beta=b, eps=case.eps, out=y, ws=ws)
+        elif case.op in ("pad_scale", "moe_group_top2"):
+            kw = dict(fft_size=case.meta.get("fft_size"), scale=case.meta.get("scale"))
+            y = rw.run(case.op, x, **kw)
+            fn = lambda: rw.run(case.op, x, out=y, **kw)  # noqa: E731
         else:
             y = torch.empty_like(x)
             fn = lambda: rw.run(case.op, x, gamma=g, beta=b, eps=case.eps, out=y)  # noqa: E731
@@ -470,6 +474,9 @@ def run_only(args, local):
     g = case.gamma.to(device) if case.gamma is not None else None
     b = case.beta.to(device) if case.beta is not None else None
     kw = dict(gamma=g, beta=b, eps=case.eps, out=y)
+    if case.op in ("pad_scale", "moe_group_top2"):
+        kw = dict(fft_size=case.meta.get("fft_size"), scale=case.meta.get("scale"))
+        kw["out"] = rw.run(case.op, x, **kw)
     if case.ragged:
         kw.update(offsets=case.offsets.to(device), max_len=case.max_len,
                   ws=rw.ragged_workspace(case.rows, device))

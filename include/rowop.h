@@ -218,6 +218,32 @@ ROWOP_API int rowop_layernorm_ragged_static(const void *in, void *out,
                                             int64_t max_len, rowop_dtype_t dtype,
                                             float eps, cudaStream_t stream);
 
+/* ---- Hyena FFT-size padding (§6, "Representative cross-layer trace") -------
+ * out[r][c] = scale * in[r][c] for 0 <= c < seqlen and 0 for
+ * seqlen <= c < fft_size, for every row r < rows: the zero-padded, scaled
+ * input of an FFT convolution.
+ * in    : rows x seqlen elements of dtype, row stride ld_in >= seqlen (may be
+ *         NULL when seqlen == 0)
+ * out   : rows x fft_size elements of dtype, row stride ld_out >= fft_size;
+ *         written in full for every row (columns past fft_size untouched)
+ * fft_size >= seqlen >= 0; scale finite.  bf16: the product is formed in
+ * fp32 and rounded to nearest even.  in and out must not overlap.          */
+ROWOP_API int rowop_pad_scale(const void *in, void *out, int64_t rows, int64_t seqlen,
+                              int64_t fft_size, int64_t ld_in, int64_t ld_out,
+                              float scale, rowop_dtype_t dtype, cudaStream_t stream);
+
+/* ---- MoE group score (§2.1, "A Running Example") --------------------------
+ * For every token t and every group g of 32 consecutive experts:
+ *   out[t][g] = max over i != j of (s[t][32g+i] + s[t][32g+j]),
+ * the sum of the group's two largest scores, a tied maximum counting twice.
+ * Computed by value only (no index is ever produced), in fp32.
+ * scores : tokens x experts of dtype, row stride ld >= experts; experts a
+ *          positive multiple of 32; scores finite or -inf
+ * out    : tokens x (experts / 32) float32, contiguous                     */
+ROWOP_API int rowop_moe_group_top2(const void *scores, float *out, int64_t tokens,
+                                   int64_t experts, int64_t ld, rowop_dtype_t dtype,
+                                   cudaStream_t stream);
+
 /* ---- dispatch rule, limits, status ---------------------------------------- */
 
 /* launch_by_rows (§2.1): the bucket for a row of len elements (len >= 0):

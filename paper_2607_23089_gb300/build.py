@@ -25,7 +25,7 @@ NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
                      "-Xcompiler", "-fvisibility=hidden", "-I", CSRC,
                      "-I", INCLUDE]
 UNITS = ["rowop_api.cu", "ops_softmax.cu", "ops_logsoftmax.cu",
-         "ops_layernorm.cu", "ops_rmsnorm.cu"]
+         "ops_layernorm.cu", "ops_rmsnorm.cu", "pad_moe.cu"]
 
 
 def nvcc() -> str:

@@ -222,9 +222,12 @@ __device__ __forceinline__ float pair_elem(const f2 (&p)[NP], int e) {
 
 // e^v as 2^(v * log2 e) on the MUFU unit; v is a difference x - m <= 0 here.
 constexpr float kLog2e = 1.4426950408889634f;
+// 2^v, the hardware approximation, with subnormal results flushed to zero:
+// they arise only for exp(x - m) < 2^-126, terms that cannot move a row sum
+// of at least 1 and outputs far below every absolute tolerance.
 __device__ __forceinline__ float ex2_approx(float v) {
   float r;
-  asm("ex2.approx.f32 %0, %1;" : "=f"(r) : "f"(v));
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(v));
   return r;
 }
 // exp(x - m) for both halves of a pair, given neg_m = (-m, -m)

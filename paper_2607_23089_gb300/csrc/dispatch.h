@@ -40,6 +40,28 @@ struct RaggedCall {
   bool classify;  // run the classify pass first (false: reuse a plan in ws)
 };
 
+// Hyena FFT-size padding: out[r][c] = scale * in[r][c] (c < seqlen), else 0.
+struct PadCall {
+  int dtype;
+  const void *in;
+  void *out;
+  int64_t rows, seqlen, fft, ld_in, ld_out;
+  float scale;
+  cudaStream_t stream;
+};
+
+// MoE group score over groups of 32 consecutive experts (fp32 output).
+struct MoeCall {
+  int dtype;
+  const void *scores;
+  float *out;
+  int64_t tokens, experts, ld;
+  cudaStream_t stream;
+};
+
+cudaError_t launch_pad_scale(const PadCall &c, const DeviceInfo &d);
+cudaError_t launch_moe_group_top2(const MoeCall &c, const DeviceInfo &d);
+
 // Ragged workspace layout (bytes): [0,4) status bits of the call, [128,140)
 // uint32 work counters, [256, 256+rows) uint8 bucket per row, then the int32
 // per-bucket row counts of every classify block ([blocks][3], at

@@ -357,6 +357,60 @@ int rowop_layernorm_ragged_static(const void *in, void *out, const void *gamma,
                     kStaticWsBytes, stream, true);
 }
 
+int rowop_pad_scale(const void *in, void *out, int64_t rows, int64_t seqlen, int64_t fft_size,
+                    int64_t ld_in, int64_t ld_out, float scale, rowop_dtype_t dtype,
+                    cudaStream_t stream) {
+  const int es = esize_of(dtype);
+  if (es == 0) return ROWOP_ERR_UNSUPPORTED_DTYPE;
+  if (rows < 0 || seqlen < 0 || fft_size < seqlen || !std::isfinite(scale))
+    return ROWOP_ERR_INVALID_ARG;
+  if (rows == 0 || fft_size == 0) return ROWOP_OK;
+  if (!out || ld_out < fft_size || (seqlen > 0 && (!in || ld_in < seqlen)))
+    return ROWOP_ERR_INVALID_ARG;
+  if (!elem_aligned(out, es) || (in && !elem_aligned(in, es))) return ROWOP_ERR_INVALID_ARG;
+  if (ld_out > INT64_MAX / es / rows || (seqlen > 0 && ld_in > INT64_MAX / es / rows))
+    return ROWOP_ERR_INVALID_ARG;
+  DeviceInfo d;
+  const int st = device_info(&d);
+  if (st != ROWOP_OK) return st;
+  PadCall c;
+  c.dtype = dtype;
+  c.in = in;
+  c.out = out;
+  c.rows = rows;
+  c.seqlen = seqlen;
+  c.fft = fft_size;
+  c.ld_in = seqlen > 0 ? ld_in : 0;
+  c.ld_out = ld_out;
+  c.scale = scale;
+  c.stream = stream;
+  return from_cuda(launch_pad_scale(c, d));
+}
+
+int rowop_moe_group_top2(const void *scores, float *out, int64_t tokens, int64_t experts,
+                         int64_t ld, rowop_dtype_t dtype, cudaStream_t stream) {
+  const int es = esize_of(dtype);
+  if (es == 0) return ROWOP_ERR_UNSUPPORTED_DTYPE;
+  if (tokens < 0 || experts <= 0 || experts % 32 != 0 || ld < experts)
+    return ROWOP_ERR_INVALID_ARG;
+  if (tokens == 0) return ROWOP_OK;
+  if (!scores || !out || !elem_aligned(scores, es) || !elem_aligned(out, 4))
+    return ROWOP_ERR_INVALID_ARG;
+  if (ld > INT64_MAX / es / tokens) return ROWOP_ERR_INVALID_ARG;
+  DeviceInfo d;
+  const int st = device_info(&d);
+  if (st != ROWOP_OK) return st;
+  MoeCall c;
+  c.dtype = dtype;
+  c.scores = scores;
+  c.out = out;
+  c.tokens = tokens;
+  c.experts = experts;
+  c.ld = ld;
+  c.stream = stream;
+  return from_cuda(launch_moe_group_top2(c, d));
+}
+
 int rowop_select_bucket(int64_t len, rowop_dtype_t dtype) {
   const int es = esize_of(dtype);
   if (es == 0 || len < 0) return -1;

@@ -58,6 +58,8 @@ SIGNATURES = {
                                         _P], _I),
     "rowop_rmsnorm_ragged_planned": ([_P, _P, _P, _P, _I64, _I64, _I, _F, _P, _SZ, _P], _I),
     "rowop_layernorm_ragged_static": ([_P, _P, _P, _P, _P, _I64, _I64, _I, _F, _P], _I),
+    "rowop_pad_scale": ([_P, _P, _I64, _I64, _I64, _I64, _I64, _F, _I, _P], _I),
+    "rowop_moe_group_top2": ([_P, _P, _I64, _I64, _I64, _I, _P], _I),
     "rowop_select_bucket": ([_I64, _I], _I),
     "rowop_max_row_len": ([_I], _I64),
     "rowop_status_string": ([_I], ctypes.c_char_p),
@@ -267,10 +269,42 @@ def select_bucket(length: int, dtype) -> int:
     return rowop_select_bucket(int(length), code)  # noqa: F821
 
 
+def pad_scale(x, fft_size: int, scale: float, out=None, stream=None):
+    """Hyena FFT-size padding of a rows x seqlen tensor to rows x fft_size
+    (``rowop_pad_scale``)."""
+    torch = _torch()
+    _check_cuda(x)
+    rows, seqlen = x.shape
+    if out is None:
+        out = torch.empty((rows, fft_size), dtype=x.dtype, device=x.device)
+    _ok(rowop_pad_scale(x.data_ptr(), out.data_ptr(), rows, seqlen, int(fft_size),  # noqa: F821
+                        x.stride(0), out.stride(0), float(scale), dtype_code(x.dtype),
+                        _stream(stream)), "rowop_pad_scale")
+    return out
+
+
+def moe_group_top2(scores, out=None, stream=None):
+    """Per-group sum of the two largest of every 32 consecutive expert scores,
+    float32 (``rowop_moe_group_top2``)."""
+    torch = _torch()
+    _check_cuda(scores)
+    tokens, experts = scores.shape
+    if out is None:
+        out = torch.empty((tokens, experts // 32), dtype=torch.float32, device=scores.device)
+    _ok(rowop_moe_group_top2(scores.data_ptr(), out.data_ptr(), tokens, experts,  # noqa: F821
+                             scores.stride(0), dtype_code(scores.dtype), _stream(stream)),
+        "rowop_moe_group_top2")
+    return out
+
+
 def run(op: str, x, *, offsets=None, max_len=None, gamma=None, beta=None,
-        eps=None, out=None, ws=None, stream=None):
+        eps=None, out=None, ws=None, stream=None, fft_size=None, scale=None):
     """One call of ``op`` on dense or ragged input (ragged when offsets is
     given); returns the output tensor."""
+    if op == "pad_scale":
+        return pad_scale(x, fft_size, scale, out, stream)
+    if op == "moe_group_top2":
+        return moe_group_top2(x, out, stream)
     if offsets is None:
         if op == "softmax":
             return softmax(x, out, stream)

@@ -63,6 +63,10 @@ class Case:
         """Bytes the operator must move: read x once, write y once, read
         gamma/beta once, read the offsets once."""
         es = ESIZE[self.dtype]
+        if self.op == "pad_scale":  # read rows x seqlen, write rows x fft_size
+            return self.x.numel() * es + self.x.shape[0] * self.meta["fft_size"] * es
+        if self.op == "moe_group_top2":  # read the scores, write one float per group
+            return self.x.numel() * es + self.x.shape[0] * (self.x.shape[1] // 32) * 4
         b = 2 * self.elements * es
         ncol = self.max_len if self.ragged else self.x.shape[1]
         if self.gamma is not None:
@@ -150,6 +154,30 @@ def ragged_ln(rows: int = 16384, max_len: int = 32768, op: str = "layernorm",
                 eps=eps, max_len=max_len)
 
 
+def hyena_pad(rows: int = 16384, seqlen: int = 4096, fft_size: int = 8192,
+              seed: int = 5) -> Case:
+    """Hyena FFT-size padding (§6): fp32 rows x seqlen, x = N(0,1), padded
+    with zeros to fft_size = 2*seqlen and scaled by 1/fft_size (the usual
+    normalisation of an FFT convolution).  Not one of the five workloads
+    above; the shapes are those of a long-convolution layer (rows = batch x
+    channels)."""
+    g = _gen(seed)
+    x = torch.randn(rows, seqlen, generator=g)
+    return Case("hyena_pad_scale", "pad_scale", x, torch.float32,
+                meta={"fft_size": fft_size, "scale": 1.0 / fft_size})
+
+
+def moe_group(tokens: int = 131072, experts: int = 256, seed: int = 6,
+              dtype=torch.float32) -> Case:
+    """MoE group score (§2.1): tokens x 256 expert scores in 8 groups of 32,
+    s = sigmoid(N(0,1)) rounded to multiples of 1/256 so that ties, tied
+    maxima included, are common.  Not one of the five workloads above."""
+    g = _gen(seed)
+    s = torch.sigmoid(torch.randn(tokens, experts, generator=g))
+    s = torch.round(s * 256) / 256
+    return Case("moe_group_top2", "moe_group_top2", s.to(dtype), dtype)
+
+
 def all_cases(scale_down: int = 1):
     """The five workloads as a flat list of cases.  ``scale_down`` > 1 divides
     every row count (not the row lengths) for quicker runs."""
@@ -162,6 +190,8 @@ def all_cases(scale_down: int = 1):
         out.append(medium_norm(op, rows=max(1, 8192 // s)))
     out.append(long_rows(rows=max(1, 256 // s)))
     out.append(ragged_ln(rows=max(1, 16384 // s)))
+    out.append(hyena_pad(rows=max(1, 16384 // s)))
+    out.append(moe_group(tokens=max(1, 131072 // s)))
     return out
 
 
@@ -178,4 +208,8 @@ def by_name(name: str) -> Case:
         return long_rows(op=name[len("long_rows_"):])
     if name.startswith("ragged_"):
         return ragged_ln(op=name[len("ragged_"):])
+    if name == "hyena_pad_scale":
+        return hyena_pad()
+    if name == "moe_group_top2":
+        return moe_group()
     raise KeyError(name)

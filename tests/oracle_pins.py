@@ -33,7 +33,8 @@ def _close(a, b, rtol=1e-13, atol=1e-14):
     assert a.shape == b.shape, (a.shape, b.shape)
     ok = np.isclose(a, b, rtol=rtol, atol=atol, equal_nan=True)
     if not ok.all():
-        d = np.where(ok, 0.0, np.abs(np.nan_to_num(a - b, nan=np.inf)))
+        with np.errstate(invalid="ignore"):
+            d = np.where(ok, 0.0, np.abs(np.nan_to_num(a - b, nan=np.inf)))
         raise AssertionError(f"max |diff| {d.max()}\n{a}\n{b}")
 
 

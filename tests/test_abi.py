@@ -125,3 +125,21 @@ def test_binding_refuses_cpu_tensors(lib):
     import torch
     with pytest.raises(ValueError):
         lib.softmax(torch.zeros(4, 8))
+
+
+def test_pad_and_moe_validation(lib):
+    """Bad shapes are refused before anything touches the device."""
+    F32 = lib.ROWOP_F32
+    assert lib.rowop_pad_scale(None, None, 0, 4, 8, 4, 8, 1.0, F32, None) == lib.ROWOP_OK
+    assert lib.rowop_pad_scale(None, None, 4, 9, 8, 9, 8, 1.0, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert lib.rowop_pad_scale(None, None, 4, 4, 8, 4, 8, 1.0, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert lib.rowop_pad_scale(16, 16, 4, 4, 8, 3, 8, 1.0, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert lib.rowop_pad_scale(16, 16, 4, 4, 8, 4, 8, float("nan"), F32, None) == \
+        lib.ROWOP_ERR_INVALID_ARG
+    assert lib.rowop_pad_scale(16, 16, 4, 4, 8, 4, 8, 1.0, 7, None) == \
+        lib.ROWOP_ERR_UNSUPPORTED_DTYPE
+    assert lib.rowop_moe_group_top2(16, 16, 0, 64, 64, F32, None) == lib.ROWOP_OK
+    assert lib.rowop_moe_group_top2(16, 16, 4, 48, 48, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert lib.rowop_moe_group_top2(16, 16, 4, 64, 32, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert lib.rowop_moe_group_top2(None, 16, 4, 64, 64, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert lib.rowop_moe_group_top2(16, 18, 4, 64, 64, F32, None) == lib.ROWOP_ERR_INVALID_ARG
