@@ -18,8 +18,8 @@
  * ---------------------------------------
  * - All pointers are DEVICE pointers owned by the caller; the library never
  *   allocates device memory on a call and keeps no pointer after it returns.
- * - Element type is rowop_dtype_t: float32, or bfloat16 with float32
- *   arithmetic inside and round-to-nearest-even on output.  gamma and beta
+ * - Element type is rowop_dtype_t: float32, or bfloat16 / float16 with
+ *   float32 arithmetic inside and round-to-nearest-even on output.  gamma and beta
  *   have the element type of the data.  gamma == NULL means all ones and
  *   beta == NULL all zeros.
  * - Dense layout: row r starts at element r*ld of `in` and of `out`; ld is in
@@ -67,13 +67,14 @@ extern "C" {
 
 typedef enum rowop_dtype {
     ROWOP_F32 = 0,  /* float32 in, float32 out                         */
-    ROWOP_BF16 = 1  /* bfloat16 in/out, float32 arithmetic, RNE output */
+    ROWOP_BF16 = 1, /* bfloat16 in/out, float32 arithmetic, RNE output */
+    ROWOP_F16 = 2   /* float16 in/out, float32 arithmetic, RNE output  */
 } rowop_dtype_t;
 
 typedef enum rowop_status {
     ROWOP_OK = 0,
     ROWOP_ERR_INVALID_ARG = 1,        /* NULL / misaligned pointer, bad size, ld < cols, eps < 0 */
-    ROWOP_ERR_UNSUPPORTED_DTYPE = 2,  /* dtype is not ROWOP_F32 or ROWOP_BF16 */
+    ROWOP_ERR_UNSUPPORTED_DTYPE = 2,  /* dtype is not ROWOP_F32, ROWOP_BF16 or ROWOP_F16 */
     ROWOP_ERR_WORKSPACE = 3,          /* ragged workspace NULL, misaligned or too small */
     ROWOP_ERR_CUDA = 4,               /* a CUDA runtime call or launch failed */
     ROWOP_ERR_TIMEOUT = 5,            /* a bounded device wait ran out (see rowop_check_status) */

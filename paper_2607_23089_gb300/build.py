@@ -24,8 +24,14 @@ ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
                      "-Xcompiler", "-fvisibility=hidden", "-I", CSRC,
                      "-I", INCLUDE]
-UNITS = ["rowop_api.cu", "ops_softmax.cu", "ops_logsoftmax.cu",
-         "ops_layernorm.cu", "ops_rmsnorm.cu", "pad_moe.cu"]
+# (source, object name, extra flags): ops_instance.cu once per operator and
+# element type
+_OPS = [("kSoftmax", "softmax"), ("kLogSoftmax", "logsoftmax"), ("kLayerNorm", "layernorm"),
+        ("kRmsNorm", "rmsnorm")]
+_TYPES = [("float", "f32"), ("__nv_bfloat16", "bf16"), ("__half", "f16")]
+UNITS = [("rowop_api.cu", "rowop_api.o", []), ("pad_moe.cu", "pad_moe.o", [])] + [
+    ("ops_instance.cu", f"ops_{on}_{tn}.o", [f"-DROWOP_INST_OP={o}", f"-DROWOP_INST_T={t}"])
+    for o, on in _OPS for t, tn in _TYPES]
 
 
 def nvcc() -> str:
@@ -62,14 +68,15 @@ def build(force: bool = False, extra_flags=(), verbose: bool = False) -> str:
     cc = nvcc()
 
     def compile_one(unit):
-        src = os.path.join(CSRC, unit)
-        obj = os.path.join(BUILD, unit.replace(".cu", ".o"))
-        cmd = [cc] + NVCC_FLAGS + list(extra_flags) + ["-c", src, "-o", obj]
+        name, objname, defs = unit
+        src = os.path.join(CSRC, name)
+        obj = os.path.join(BUILD, objname)
+        cmd = [cc] + NVCC_FLAGS + defs + list(extra_flags) + ["-c", src, "-o", obj]
         if verbose:
             print(" ".join(cmd))
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
-            raise RuntimeError(f"nvcc failed on {unit}:\n{r.stderr}")
+            raise RuntimeError(f"nvcc failed on {objname}:\n{r.stderr}")
         return obj, r.stderr
 
     with cf.ThreadPoolExecutor(max_workers=min(len(UNITS), os.cpu_count() or 4)) as ex:

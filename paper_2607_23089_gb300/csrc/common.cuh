@@ -21,6 +21,7 @@
 #pragma once
 
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -66,41 +67,82 @@ struct Elem<__nv_bfloat16> {
   static constexpr int kPerChunk = 8;
   static constexpr int kSize = 2;
 };
+template <>
+struct Elem<__half> {
+  static constexpr int kPerChunk = 8;
+  static constexpr int kSize = 2;
+};
 
 // ---------------------------------------------------------------------------
 // fp32 <-> element conversion, whole 16-byte chunks
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ void unpack(const uint4 &v, float (&f)[4]) {
-  f[0] = __uint_as_float(v.x);
-  f[1] = __uint_as_float(v.y);
-  f[2] = __uint_as_float(v.z);
-  f[3] = __uint_as_float(v.w);
-}
 __device__ __forceinline__ void unpack_bf16x2(uint32_t w, float &lo, float &hi) {
   lo = __uint_as_float(w << 16);
   hi = __uint_as_float(w & 0xffff0000u);
-}
-__device__ __forceinline__ void unpack(const uint4 &v, float (&f)[8]) {
-  unpack_bf16x2(v.x, f[0], f[1]);
-  unpack_bf16x2(v.y, f[2], f[3]);
-  unpack_bf16x2(v.z, f[4], f[5]);
-  unpack_bf16x2(v.w, f[6], f[7]);
-}
-__device__ __forceinline__ uint4 pack(const float (&f)[4]) {
-  return make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]),
-                    __float_as_uint(f[2]), __float_as_uint(f[3]));
 }
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 b = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t *>(&b);
 }
-__device__ __forceinline__ uint4 pack(const float (&f)[8]) {
+__device__ __forceinline__ float2 half2_bits_to_float2(uint32_t w) {
+  __half2 h = *reinterpret_cast<const __half2 *>(&w);
+  return __half22float2(h);
+}
+__device__ __forceinline__ uint32_t float2_to_half2_bits(float2 v) {
+  __half2 h = __float22half2_rn(v);  // round to nearest even, .x in the low half
+  return *reinterpret_cast<uint32_t *>(&h);
+}
+
+// A 16-byte chunk of T <-> its E values in fp32.
+template <typename T>
+__device__ __forceinline__ void unpack(const uint4 &v, float (&f)[Elem<T>::kPerChunk]);
+template <typename T>
+__device__ __forceinline__ uint4 pack(const float (&f)[Elem<T>::kPerChunk]);
+template <>
+__device__ __forceinline__ void unpack<float>(const uint4 &v, float (&f)[4]) {
+  f[0] = __uint_as_float(v.x);
+  f[1] = __uint_as_float(v.y);
+  f[2] = __uint_as_float(v.z);
+  f[3] = __uint_as_float(v.w);
+}
+template <>
+__device__ __forceinline__ void unpack<__nv_bfloat16>(const uint4 &v, float (&f)[8]) {
+  unpack_bf16x2(v.x, f[0], f[1]);
+  unpack_bf16x2(v.y, f[2], f[3]);
+  unpack_bf16x2(v.z, f[4], f[5]);
+  unpack_bf16x2(v.w, f[6], f[7]);
+}
+template <>
+__device__ __forceinline__ void unpack<__half>(const uint4 &v, float (&f)[8]) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 t = half2_bits_to_float2(w[i]);
+    f[2 * i] = t.x;
+    f[2 * i + 1] = t.y;
+  }
+}
+template <>
+__device__ __forceinline__ uint4 pack<float>(const float (&f)[4]) {
+  return make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]),
+                    __float_as_uint(f[2]), __float_as_uint(f[3]));
+}
+template <>
+__device__ __forceinline__ uint4 pack<__nv_bfloat16>(const float (&f)[8]) {
   return make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]),
                     pack_bf16x2(f[4], f[5]), pack_bf16x2(f[6], f[7]));
+}
+template <>
+__device__ __forceinline__ uint4 pack<__half>(const float (&f)[8]) {
+  return make_uint4(float2_to_half2_bits(make_float2(f[0], f[1])),
+                    float2_to_half2_bits(make_float2(f[2], f[3])),
+                    float2_to_half2_bits(make_float2(f[4], f[5])),
+                    float2_to_half2_bits(make_float2(f[6], f[7])));
 }
 
 __device__ __forceinline__ float to_f32(float v) { return v; }
 __device__ __forceinline__ float to_f32(__nv_bfloat16 v) { return __bfloat162float(v); }
+__device__ __forceinline__ float to_f32(__half v) { return __half2float(v); }
 template <typename T>
 __device__ __forceinline__ T from_f32(float v);
 template <>
@@ -108,6 +150,10 @@ __device__ __forceinline__ float from_f32<float>(float v) { return v; }
 template <>
 __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) {
   return __float2bfloat16_rn(v);
+}
+template <>
+__device__ __forceinline__ __half from_f32<__half>(float v) {
+  return __float2half_rn(v);
 }
 
 // One element of type T read as its raw bits into an fp32 value.
@@ -152,6 +198,13 @@ __device__ __forceinline__ uint4 shift_chunk<float>(const uint4 &A, const uint4 
 }
 template <>
 __device__ __forceinline__ uint4 shift_chunk<__nv_bfloat16>(const uint4 &A, const uint4 &B,
+                                                            int h);
+template <>
+__device__ __forceinline__ uint4 shift_chunk<__half>(const uint4 &A, const uint4 &B, int h) {
+  return shift_chunk<__nv_bfloat16>(A, B, h);  // both are 2-byte elements
+}
+template <>
+__device__ __forceinline__ uint4 shift_chunk<__nv_bfloat16>(const uint4 &A, const uint4 &B,
                                                             int h) {
   switch (h) {
     case 1: return shift_half<1>(A, B);
@@ -188,31 +241,51 @@ __device__ __forceinline__ f2 f2_select(f2 v, bool keep_lo, bool keep_hi, float 
   return make_float2(keep_lo ? v.x : fill, keep_hi ? v.y : fill);
 }
 
-// 16-byte chunk <-> pairs.  fp32: 2 pairs, bf16: 4 pairs.
-__device__ __forceinline__ void chunk_to_pairs(const uint4 &v, f2 (&p)[2]) {
-  p[0] = make_float2(__uint_as_float(v.x), __uint_as_float(v.y));
-  p[1] = make_float2(__uint_as_float(v.z), __uint_as_float(v.w));
-}
+// 16-byte chunk of T <-> pairs.  fp32: 2 pairs, bf16 / fp16: 4 pairs.
 __device__ __forceinline__ f2 bf16x2_to_pair(uint32_t w) {
   return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
-}
-__device__ __forceinline__ void chunk_to_pairs(const uint4 &v, f2 (&p)[4]) {
-  p[0] = bf16x2_to_pair(v.x);
-  p[1] = bf16x2_to_pair(v.y);
-  p[2] = bf16x2_to_pair(v.z);
-  p[3] = bf16x2_to_pair(v.w);
-}
-__device__ __forceinline__ uint4 pairs_to_chunk(const f2 (&p)[2]) {
-  return make_uint4(__float_as_uint(p[0].x), __float_as_uint(p[0].y), __float_as_uint(p[1].x),
-                    __float_as_uint(p[1].y));
 }
 __device__ __forceinline__ uint32_t pair_to_bf16x2(f2 v) {
   __nv_bfloat162 b = __float22bfloat162_rn(v);  // round to nearest even, .x in the low half
   return *reinterpret_cast<uint32_t *>(&b);
 }
-__device__ __forceinline__ uint4 pairs_to_chunk(const f2 (&p)[4]) {
+template <typename T>
+__device__ __forceinline__ void chunk_to_pairs(const uint4 &v, f2 (&p)[Elem<T>::kPerChunk / 2]);
+template <typename T>
+__device__ __forceinline__ uint4 pairs_to_chunk(const f2 (&p)[Elem<T>::kPerChunk / 2]);
+template <>
+__device__ __forceinline__ void chunk_to_pairs<float>(const uint4 &v, f2 (&p)[2]) {
+  p[0] = make_float2(__uint_as_float(v.x), __uint_as_float(v.y));
+  p[1] = make_float2(__uint_as_float(v.z), __uint_as_float(v.w));
+}
+template <>
+__device__ __forceinline__ void chunk_to_pairs<__nv_bfloat16>(const uint4 &v, f2 (&p)[4]) {
+  p[0] = bf16x2_to_pair(v.x);
+  p[1] = bf16x2_to_pair(v.y);
+  p[2] = bf16x2_to_pair(v.z);
+  p[3] = bf16x2_to_pair(v.w);
+}
+template <>
+__device__ __forceinline__ void chunk_to_pairs<__half>(const uint4 &v, f2 (&p)[4]) {
+  p[0] = half2_bits_to_float2(v.x);
+  p[1] = half2_bits_to_float2(v.y);
+  p[2] = half2_bits_to_float2(v.z);
+  p[3] = half2_bits_to_float2(v.w);
+}
+template <>
+__device__ __forceinline__ uint4 pairs_to_chunk<float>(const f2 (&p)[2]) {
+  return make_uint4(__float_as_uint(p[0].x), __float_as_uint(p[0].y), __float_as_uint(p[1].x),
+                    __float_as_uint(p[1].y));
+}
+template <>
+__device__ __forceinline__ uint4 pairs_to_chunk<__nv_bfloat16>(const f2 (&p)[4]) {
   return make_uint4(pair_to_bf16x2(p[0]), pair_to_bf16x2(p[1]), pair_to_bf16x2(p[2]),
                     pair_to_bf16x2(p[3]));
+}
+template <>
+__device__ __forceinline__ uint4 pairs_to_chunk<__half>(const f2 (&p)[4]) {
+  return make_uint4(float2_to_half2_bits(p[0]), float2_to_half2_bits(p[1]),
+                    float2_to_half2_bits(p[2]), float2_to_half2_bits(p[3]));
 }
 // element e of a chunk's pair array
 template <int NP>

@@ -125,9 +125,6 @@ Knobs read_knobs();
 // Ragged classify pass into the workspace (defined in rowop_api.cu).
 cudaError_t launch_classify(const RaggedCall &c, const DeviceInfo &d);
 
-template <int OP>
-cudaError_t launch_dense(const DenseCall &c, const DeviceInfo &d);
-template <int OP>
-cudaError_t launch_ragged(const RaggedCall &c, const DeviceInfo &d);
+
 
 }  // namespace rowop

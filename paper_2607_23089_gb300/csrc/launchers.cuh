@@ -277,11 +277,6 @@ cudaError_t launch_dense_t(const DenseCall &c, const DeviceInfo &d) {
   return launch_tile_k<OP, T, false, true, false>(p, cs, S, st, W, c.rows, d, c.stream);
 }
 
-template <int OP>
-cudaError_t launch_dense(const DenseCall &c, const DeviceInfo &d) {
-  if (c.dtype == 0) return launch_dense_t<OP, float>(c, d);
-  return launch_dense_t<OP, __nv_bfloat16>(c, d);
-}
 
 template <int OP, typename T>
 cudaError_t launch_ragged_t(const RaggedCall &c, const DeviceInfo &d) {
@@ -342,10 +337,5 @@ cudaError_t launch_ragged_t(const RaggedCall &c, const DeviceInfo &d) {
                                                   c.stream, small_area);
 }
 
-template <int OP>
-cudaError_t launch_ragged(const RaggedCall &c, const DeviceInfo &d) {
-  if (c.dtype == 0) return launch_ragged_t<OP, float>(c, d);
-  return launch_ragged_t<OP, __nv_bfloat16>(c, d);
-}
 
 }  // namespace rowop

@@ -36,7 +36,7 @@ __device__ __forceinline__ uint4 pad_chunk(const T *in_row, int64_t c, int64_t s
   constexpr int E = Elem<T>::kPerChunk;
   float v[E];
   if (full_live) {
-    unpack(raw, v);
+    unpack<T>(raw, v);
 #pragma unroll
     for (int e = 0; e < E; ++e) v[e] = __fmul_rn(v[e], scale);
   } else {
@@ -46,7 +46,7 @@ __device__ __forceinline__ uint4 pad_chunk(const T *in_row, int64_t c, int64_t s
       v[e] = j < seqlen ? __fmul_rn(load_elem(in_row + j), scale) : 0.f;
     }
   }
-  return pack(v);
+  return pack<T>(v);
 }
 
 // VEC: in/out rows 16-byte aligned and fft a whole number of chunks.  Work
@@ -127,6 +127,7 @@ cudaError_t launch_pad_scale_t(const PadCall &c, const DeviceInfo &d) {
 
 cudaError_t launch_pad_scale(const PadCall &c, const DeviceInfo &d) {
   if (c.dtype == 0) return launch_pad_scale_t<float>(c, d);
+  if (c.dtype == 2) return launch_pad_scale_t<__half>(c, d);
   return launch_pad_scale_t<__nv_bfloat16>(c, d);
 }
 
@@ -184,7 +185,7 @@ __global__ void __launch_bounds__(kMoeThreads) moe_group_top2_kernel(const MoePa
         float t1 = -INFINITY, t2 = -INFINITY;
         if (c < nchunks) {
           float v[E];
-          unpack(ldg_stream(row + c * E), v);
+          unpack<T>(ldg_stream(row + c * E), v);
 #pragma unroll
           for (int e = 0; e < E; ++e) top2_add(t1, t2, v[e]);
         }
@@ -227,6 +228,7 @@ cudaError_t launch_moe_t(const MoeCall &c, const DeviceInfo &d) {
 
 cudaError_t launch_moe_group_top2(const MoeCall &c, const DeviceInfo &d) {
   if (c.dtype == 0) return launch_moe_t<float>(c, d);
+  if (c.dtype == 2) return launch_moe_t<__half>(c, d);
   return launch_moe_t<__nv_bfloat16>(c, d);
 }
 

@@ -102,7 +102,7 @@ __device__ __forceinline__ void load_param_pairs(const T *__restrict__ g, int64_
   constexpr int E = Elem<T>::kPerChunk;
   const int64_t j0 = c * E - h;
   if (vec && h == 0 && j0 + E <= glen) {
-    chunk_to_pairs(__ldg(reinterpret_cast<const uint4 *>(g + j0)), out);
+    chunk_to_pairs<T>(__ldg(reinterpret_cast<const uint4 *>(g + j0)), out);
     return;
   }
   if (vec && h > 0 && (c + 1) * E <= glen) {
@@ -111,7 +111,7 @@ __device__ __forceinline__ void load_param_pairs(const T *__restrict__ g, int64_
     const uint4 A = c >= 1 ? __ldg(reinterpret_cast<const uint4 *>(g + (c - 1) * E))
                            : make_uint4(0u, 0u, 0u, 0u);
     const uint4 B = __ldg(reinterpret_cast<const uint4 *>(g + c * E));
-    chunk_to_pairs(shift_chunk<T>(A, B, h), out);
+    chunk_to_pairs<T>(shift_chunk<T>(A, B, h), out);
     return;
   }
   float v[E];
@@ -172,7 +172,7 @@ __device__ __forceinline__ void store_chunk(const f2 (&p)[Elem<T>::kPerChunk / 2
                                             bool out_vec) {
   constexpr int E = Elem<T>::kPerChunk;
   if (lo == 0 && hi == E && out_vec) {
-    stg_stream(owin + c * kChunkBytes, pairs_to_chunk(p));
+    stg_stream(owin + c * kChunkBytes, pairs_to_chunk<T>(p));
   } else {
 #pragma unroll
     for (int e = 0; e < E; ++e)

@@ -13,14 +13,25 @@
 
 namespace rowop {
 
-extern template cudaError_t launch_dense<kSoftmax>(const DenseCall &, const DeviceInfo &);
-extern template cudaError_t launch_dense<kLogSoftmax>(const DenseCall &, const DeviceInfo &);
-extern template cudaError_t launch_dense<kLayerNorm>(const DenseCall &, const DeviceInfo &);
-extern template cudaError_t launch_dense<kRmsNorm>(const DenseCall &, const DeviceInfo &);
-extern template cudaError_t launch_ragged<kSoftmax>(const RaggedCall &, const DeviceInfo &);
-extern template cudaError_t launch_ragged<kLogSoftmax>(const RaggedCall &, const DeviceInfo &);
-extern template cudaError_t launch_ragged<kLayerNorm>(const RaggedCall &, const DeviceInfo &);
-extern template cudaError_t launch_ragged<kRmsNorm>(const RaggedCall &, const DeviceInfo &);
+// The per-type launch paths, instantiated one (operator, type) pair per
+// object file from ops_instance.cu.
+template <int OP, typename T>
+cudaError_t launch_dense_t(const DenseCall &c, const DeviceInfo &d);
+template <int OP, typename T>
+cudaError_t launch_ragged_t(const RaggedCall &c, const DeviceInfo &d);
+
+template <int OP>
+static cudaError_t launch_dense(const DenseCall &c, const DeviceInfo &d) {
+  if (c.dtype == ROWOP_F32) return launch_dense_t<OP, float>(c, d);
+  if (c.dtype == ROWOP_F16) return launch_dense_t<OP, __half>(c, d);
+  return launch_dense_t<OP, __nv_bfloat16>(c, d);
+}
+template <int OP>
+static cudaError_t launch_ragged(const RaggedCall &c, const DeviceInfo &d) {
+  if (c.dtype == ROWOP_F32) return launch_ragged_t<OP, float>(c, d);
+  if (c.dtype == ROWOP_F16) return launch_ragged_t<OP, __half>(c, d);
+  return launch_ragged_t<OP, __nv_bfloat16>(c, d);
+}
 
 // Device-side status bits (kStatusTimeout, kStatusBadOffsets), one word per
 // device; kernels receive its address.
@@ -123,7 +134,9 @@ static int static_workspace(void **ws) {
   return ROWOP_OK;
 }
 
-static int esize_of(int dtype) { return dtype == ROWOP_F32 ? 4 : (dtype == ROWOP_BF16 ? 2 : 0); }
+static int esize_of(int dtype) {
+  return dtype == ROWOP_F32 ? 4 : ((dtype == ROWOP_BF16 || dtype == ROWOP_F16) ? 2 : 0);
+}
 
 static bool elem_aligned(const void *p, int esize) {
   return (reinterpret_cast<uintptr_t>(p) % static_cast<uintptr_t>(esize)) == 0;

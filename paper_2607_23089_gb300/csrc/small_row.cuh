@@ -65,7 +65,7 @@ __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, i
       const int64_t c = sub + static_cast<int64_t>(k) * G;
       if (c < nc) {
         f2 p[NP];
-        chunk_to_pairs(get(k), p);
+        chunk_to_pairs<T>(get(k), p);
         int lo = 0, hi = E;
         if (!EXACT) chunk_valid_range(c, nc, h, hn, E, lo, hi);
         m = chunk_max<NP>(p, m, lo, hi);
@@ -79,7 +79,7 @@ __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, i
       const int64_t c = sub + static_cast<int64_t>(k) * G;
       if (c < nc) {
         f2 p[NP];
-        chunk_to_pairs(get(k), p);
+        chunk_to_pairs<T>(get(k), p);
         int lo = 0, hi = E;
         if (!EXACT) chunk_valid_range(c, nc, h, hn, E, lo, hi);
         acc = chunk_sum_exp<NP>(p, m2, acc, lo, hi);
@@ -95,7 +95,7 @@ __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, i
       const int64_t c = sub + static_cast<int64_t>(k) * G;
       if (c < nc) {
         f2 p[NP];
-        chunk_to_pairs(get(k), p);
+        chunk_to_pairs<T>(get(k), p);
         int lo = 0, hi = E;
         if (!EXACT) chunk_valid_range(c, nc, h, hn, E, lo, hi);
         acc = chunk_sum<NP>(p, acc, lo, hi);
@@ -109,7 +109,7 @@ __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, i
       const int64_t c = sub + static_cast<int64_t>(k) * G;
       if (c < nc) {
         f2 p[NP];
-        chunk_to_pairs(get(k), p);
+        chunk_to_pairs<T>(get(k), p);
         int lo = 0, hi = E;
         if (!EXACT) chunk_valid_range(c, nc, h, hn, E, lo, hi);
         acc = chunk_sum_sqdev<NP>(p, mean2, acc, lo, hi);
@@ -125,7 +125,7 @@ __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, i
       const int64_t c = sub + static_cast<int64_t>(k) * G;
       if (c < nc) {
         f2 p[NP];
-        chunk_to_pairs(get(k), p);
+        chunk_to_pairs<T>(get(k), p);
         int lo = 0, hi = E;
         if (!EXACT) chunk_valid_range(c, nc, h, hn, E, lo, hi);
         acc = chunk_sum_sq<NP>(p, acc, lo, hi);
@@ -142,7 +142,7 @@ __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, i
     const int64_t c = sub + static_cast<int64_t>(k) * G;
     if (c < nc) {
       f2 p[NP];
-      chunk_to_pairs(get(k), p);
+      chunk_to_pairs<T>(get(k), p);
       int lo = 0, hi = E;
       if (!EXACT) chunk_valid_range(c, nc, h, hn, E, lo, hi);
       chunk_normalize<OP, T>(p, s0, s1, static_cast<const T *>(a.gamma),

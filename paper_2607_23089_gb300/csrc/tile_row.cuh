@@ -199,8 +199,8 @@ __device__ __forceinline__ float tile_lane_first(const unsigned char *tsm, const
                                                  int lane) {
   constexpr int NP = Elem<T>::kPerChunk / 2;
   f2 p0[NP], p1[NP];
-  chunk_to_pairs(*reinterpret_cast<const uint4 *>(tsm + lane * kChunkBytes), p0);
-  chunk_to_pairs(*reinterpret_cast<const uint4 *>(tsm + (lane + 32) * kChunkBytes), p1);
+  chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(tsm + lane * kChunkBytes), p0);
+  chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(tsm + (lane + 32) * kChunkBytes), p1);
   if constexpr (OP == kSoftmax || OP == kLogSoftmax) {
     return chunk_max<NP>(p1, chunk_max<NP>(p0, -INFINITY, m.lo0, m.hi0), m.lo1, m.hi1);
   } else if constexpr (OP == kLayerNorm) {
@@ -218,8 +218,8 @@ __device__ __forceinline__ float tile_lane_second(const unsigned char *tsm, cons
                                                   int lane, float ref) {
   constexpr int NP = Elem<T>::kPerChunk / 2;
   f2 p0[NP], p1[NP];
-  chunk_to_pairs(*reinterpret_cast<const uint4 *>(tsm + lane * kChunkBytes), p0);
-  chunk_to_pairs(*reinterpret_cast<const uint4 *>(tsm + (lane + 32) * kChunkBytes), p1);
+  chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(tsm + lane * kChunkBytes), p0);
+  chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(tsm + (lane + 32) * kChunkBytes), p1);
   const f2 r2 = f2_bcast(ref);
   if constexpr (OP == kSoftmax || OP == kLogSoftmax) {
     if (ref == -INFINITY) return 0.f;  // no element of the tile is above -inf
@@ -486,12 +486,12 @@ __device__ __forceinline__ void chunk_store_fast(const unsigned char *csm, int c
                                                  char *owin) {
   constexpr int NP = Elem<T>::kPerChunk / 2;
   f2 v[NP], g[NP], b[NP];
-  chunk_to_pairs(*reinterpret_cast<const uint4 *>(csm), v);
+  chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(csm), v);
   if constexpr (OP == kLayerNorm || OP == kRmsNorm)
-    chunk_to_pairs(param_chunk_fixed<T, H>(gamma, c), g);
-  if constexpr (OP == kLayerNorm) chunk_to_pairs(param_chunk_fixed<T, H>(beta, c), b);
+    chunk_to_pairs<T>(param_chunk_fixed<T, H>(gamma, c), g);
+  if constexpr (OP == kLayerNorm) chunk_to_pairs<T>(param_chunk_fixed<T, H>(beta, c), b);
   normalize_pairs<OP, NP>(v, s0, s1, g, b);
-  stg_stream(owin + static_cast<int64_t>(c) * kChunkBytes, pairs_to_chunk(v));
+  stg_stream(owin + static_cast<int64_t>(c) * kChunkBytes, pairs_to_chunk<T>(v));
 }
 
 // pass 2, one chunk the fast path does not take: a row end the row only
@@ -512,7 +512,7 @@ __device__ __forceinline__ void chunk_store_edge(const unsigned char *csm, int c
   const T *gamma = static_cast<const T *>(p.gamma);
   const T *beta = static_cast<const T *>(p.beta);
   f2 v[NP], gp[NP], bp[NP];
-  chunk_to_pairs(*reinterpret_cast<const uint4 *>(csm), v);
+  chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(csm), v);
   int lo, hi;
   chunk_valid_range(c, g.nc, g.h, hn, E, lo, hi);
   if constexpr (kAffine) {
@@ -535,8 +535,8 @@ __device__ __forceinline__ void chunk_store_edge(const unsigned char *csm, int c
           }
         }
       };
-      chunk_to_pairs(realigned(gamma), gp);
-      if constexpr (OP == kLayerNorm) chunk_to_pairs(realigned(beta), bp);
+      chunk_to_pairs<T>(realigned(gamma), gp);
+      if constexpr (OP == kLayerNorm) chunk_to_pairs<T>(realigned(beta), bp);
     } else {
       load_param_pairs<T>(gamma, gamma ? p.glen : 0, c, g.h, p.gvec != 0, 1.f, gp);
       if constexpr (OP == kLayerNorm)

@@ -22,7 +22,7 @@ import threading
 HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "_build", "librowop.so")
 
-ROWOP_F32, ROWOP_BF16 = 0, 1
+ROWOP_F32, ROWOP_BF16, ROWOP_F16 = 0, 1, 2
 SMALL, MEDIUM, LARGE = 0, 1, 2
 STATUS = {
     0: "ROWOP_OK", 1: "ROWOP_ERR_INVALID_ARG", 2: "ROWOP_ERR_UNSUPPORTED_DTYPE",
@@ -121,7 +121,9 @@ def dtype_code(dtype) -> int:
         return ROWOP_F32
     if dtype == torch.bfloat16:
         return ROWOP_BF16
-    raise TypeError(f"librowop supports float32 and bfloat16, not {dtype}")
+    if dtype == torch.float16:
+        return ROWOP_F16
+    raise TypeError(f"librowop supports float32, bfloat16 and float16, not {dtype}")
 
 
 def _stream(stream):

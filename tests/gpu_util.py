@@ -13,12 +13,14 @@ import torch
 
 from oracle import rowop_oracle as orc
 
-TOL = {torch.float32: (1e-5, 1e-6), torch.bfloat16: (1e-2, 1e-6)}
-CANARY = {torch.float32: 0x7FC0DEAD, torch.bfloat16: 0x7FC1}
-ESIZE = {torch.float32: 4, torch.bfloat16: 2}
+TOL = {torch.float32: (1e-5, 1e-6), torch.bfloat16: (1e-2, 1e-6),
+       torch.float16: (1e-3, 1e-6)}
+CANARY = {torch.float32: 0x7FC0DEAD, torch.bfloat16: 0x7FC1, torch.float16: 0x7FC1}
+ESIZE = {torch.float32: 4, torch.bfloat16: 2, torch.float16: 2}
 NORM_OPS = ("layernorm", "rmsnorm")
 ALL_OPS = ("softmax", "logsoftmax", "layernorm", "rmsnorm")
-DTYPES = (torch.float32, torch.bfloat16)
+DTYPES = (torch.float32, torch.bfloat16, torch.float16)
+DTYPE_IDS = ["f32", "bf16", "f16"]
 
 
 def assert_close(got, ref, dtype, what=""):
@@ -45,7 +47,7 @@ def canary_tensor(n, dtype, device="cuda"):
         raw = torch.full((n,), CANARY[dtype], dtype=torch.int32, device=device)
         return raw.view(torch.float32)
     raw = torch.full((n,), CANARY[dtype], dtype=torch.int16, device=device)
-    return raw.view(torch.bfloat16)
+    return raw.view(dtype)
 
 
 def is_canary(t):

@@ -12,7 +12,7 @@ import numpy as np
 import pytest
 import torch
 
-from tests.gpu_util import (ALL_OPS, DTYPES, ESIZE, assert_close, canary_tensor,
+from tests.gpu_util import (DTYPE_IDS, ALL_OPS, DTYPES, ESIZE, assert_close, canary_tensor,
                             eps_for, gen, gen_affine, is_canary, oracle_dense, to_f64)
 
 pytestmark = pytest.mark.gpu
@@ -85,7 +85,7 @@ COLS = [1, 2, 3, 5, 8, 31, 64, 100, 128, 257, 512, 1000, 1023, 1024, 1025, 2047,
         65539, 262144]
 
 
-@pytest.mark.parametrize("dtype", DTYPES, ids=["f32", "bf16"])
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
 @pytest.mark.parametrize("op", ALL_OPS)
 @pytest.mark.parametrize("cols", COLS)
 def test_dense_parity(rw, op, dtype, cols):
@@ -93,7 +93,7 @@ def test_dense_parity(rw, op, dtype, cols):
     run_case(rw, op, dtype, rows, cols, seed=cols)
 
 
-@pytest.mark.parametrize("dtype", DTYPES, ids=["f32", "bf16"])
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
 @pytest.mark.parametrize("op", ALL_OPS)
 @pytest.mark.parametrize("cols,extra,x_off,y_off", [
     (7, 1, 0, 0), (1000, 1, 1, 1), (1000, 3, 2, 0), (5000, 1, 0, 0),
@@ -104,7 +104,7 @@ def test_dense_misaligned(rw, op, dtype, cols, extra, x_off, y_off):
              seed=cols + extra)
 
 
-@pytest.mark.parametrize("dtype", DTYPES, ids=["f32", "bf16"])
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
 @pytest.mark.parametrize("op", ALL_OPS)
 @pytest.mark.parametrize("cols", [100, 6000, 50000])
 def test_dense_inplace(rw, op, dtype, cols):
@@ -153,7 +153,7 @@ def _bits(t):
     return t.view(torch.int32) if t.dtype == torch.float32 else t.view(torch.int16)
 
 
-@pytest.mark.parametrize("dtype", DTYPES, ids=["f32", "bf16"])
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
 @pytest.mark.parametrize("op", ALL_OPS)
 @pytest.mark.parametrize("cols,ld,x_off", [(900, None, 0), (6000, None, 0),
                                           (6000, 6003, 1), (40000, None, 0),
@@ -170,7 +170,7 @@ def test_forced_designs_agree(rw, op, dtype, cols, ld, x_off):
         _forced(rw, op, dtype, rows, cols, 0, ld=ld, x_off=x_off)
 
 
-@pytest.mark.parametrize("dtype", DTYPES, ids=["f32", "bf16"])
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
 @pytest.mark.parametrize("op", ALL_OPS)
 @pytest.mark.parametrize("cols,ld,x_off", [(3000, None, 0), (6000, 6003, 1),
                                           (40001, 40005, 3)])

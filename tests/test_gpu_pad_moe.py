@@ -4,8 +4,8 @@ the C ABI, against the double-precision oracle.
 fp32 padding is compared bit for bit: the product of two float32 values is
 exact in double, so the oracle's value rounded to float32 is the correctly
 rounded product the GPU forms.  bf16 padding rounds that fp32 product once
-more and is held to the bf16 tolerance.  The group score is compared bit for
-bit in both dtypes: the sum of the two largest scores is exact in double and
+more and is held to its tolerance (so is fp16).  The group score is compared bit for
+bit in every dtype: the sum of the two largest scores is exact in double and
 the GPU rounds it to float32 once.
 """
 import numpy as np
@@ -13,7 +13,7 @@ import pytest
 import torch
 
 from oracle import rowop_oracle as orc
-from tests.gpu_util import ESIZE, assert_close, canary_tensor, is_canary, to_f64
+from tests.gpu_util import DTYPE_IDS, DTYPES, ESIZE, assert_close, canary_tensor, is_canary, to_f64
 
 pytestmark = pytest.mark.gpu
 
@@ -70,7 +70,7 @@ PAD_CASES = [
 ]
 
 
-@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16], ids=["f32", "bf16"])
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
 @pytest.mark.parametrize("case", PAD_CASES, ids=lambda c: f"{c[0]}x{c[1]}->{c[2]}")
 def test_pad_scale_parity(rw, dtype, case):
     rows, seqlen, fft, scale, ld_in, ld_out, off_in, off_out = case
@@ -82,7 +82,7 @@ def test_pad_scale_parity(rw, dtype, case):
         want = torch.from_numpy(ref.astype(np.float32))
         assert torch.equal(_bits(y.cpu()), _bits(want))
     else:
-        assert_close(to_f64(y), ref, dtype, "pad_scale bf16")
+        assert_close(to_f64(y), ref, dtype, f"pad_scale {dtype}")
 
 
 def test_pad_scale_workload_sampled(rw):
@@ -125,7 +125,7 @@ MOE_CASES = [(1000, 256, None, 0, False), (333, 32, None, 0, False),
              (97, 256, None, 1, True), (50000, 64, None, 0, False)]
 
 
-@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16], ids=["f32", "bf16"])
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
 @pytest.mark.parametrize("case", MOE_CASES, ids=lambda c: f"{c[0]}x{c[1]}-ld{c[2]}-off{c[3]}")
 def test_moe_group_top2_parity(rw, dtype, case):
     tokens, experts, ld, off, masked = case

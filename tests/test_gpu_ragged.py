@@ -12,7 +12,7 @@ import pytest
 import torch
 
 from oracle import rowop_oracle as orc
-from tests.gpu_util import (ALL_OPS, DTYPES, ESIZE, assert_close, canary_tensor,
+from tests.gpu_util import (DTYPE_IDS, ALL_OPS, DTYPES, ESIZE, assert_close, canary_tensor,
                             eps_for, gen_affine, is_canary, oracle_ragged, to_f64)
 
 pytestmark = pytest.mark.gpu
@@ -91,7 +91,7 @@ def run_ragged(rw, op, dtype, lens, max_len, seed, base_off=0, inplace=False,
                 G=G, base_off=base_off, total=total)
 
 
-@pytest.mark.parametrize("dtype", DTYPES, ids=["f32", "bf16"])
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
 @pytest.mark.parametrize("op", ALL_OPS)
 @pytest.mark.parametrize("base_off", [0, 3])
 def test_ragged_parity(rw, op, dtype, base_off):
@@ -113,7 +113,7 @@ def test_ragged_parity(rw, op, dtype, base_off):
     assert r["ws"][:4].view(torch.int32).item() == 0
 
 
-@pytest.mark.parametrize("dtype", DTYPES, ids=["f32", "bf16"])
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
 @pytest.mark.parametrize("op", ALL_OPS)
 def test_ragged_row_equals_dense_row(rw, op, dtype):
     """A ragged row and a dense call on the same row at the same 16-byte
@@ -206,7 +206,7 @@ def test_ragged_all_empty_and_tiny(rw):
         assert_close(to_f64(r["y"][:covered]), ref, torch.float32, "tiny")
 
 
-@pytest.mark.parametrize("dtype", DTYPES, ids=["f32", "bf16"])
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
 @pytest.mark.parametrize("op", ("softmax", "layernorm"))
 def test_ragged_group_sizes_agree(rw, op, dtype, monkeypatch):
     """The fused ragged kernel gives the same bits whatever the consumer
