@@ -248,3 +248,29 @@ def moe_group_top2(scores, group: int = 32):
     out = np.empty((tokens, experts // group), dtype=np.float64)
     _load().oracle_moe_group_top2(_ptr(v), _ptr(out), tokens, experts, group)
     return out
+
+
+# ---------------------------------------------------------------------------
+# Fused residual add + norm
+# ---------------------------------------------------------------------------
+def residual_sum(x, r, dtype):
+    """The residual stream after the add, ``s = x + r``, as stored: the sum
+    (exact in double for float32 / bfloat16 / float16 inputs but in
+    pathological exponent gaps) rounded to nearest even in the I/O type
+    ``dtype`` (a torch dtype), returned as float64."""
+    import torch
+    s = _f64(x) + _f64(r)
+    return torch.from_numpy(s).to(dtype).double().numpy()
+
+
+def add_layernorm(x, r, dtype, gamma=None, beta=None, eps=1e-5, nthreads=1):
+    """``s = x + r`` stored in ``dtype``, then ``y = LayerNorm(s)``: the norm
+    reads the sum as stored.  Returns ``(s, y)``."""
+    s = residual_sum(x, r, dtype)
+    return s, layernorm(s, gamma, beta, eps, nthreads)
+
+
+def add_rmsnorm(x, r, dtype, gamma=None, eps=1e-6, nthreads=1):
+    """``s = x + r`` stored in ``dtype``, then ``y = RMSNorm(s)``."""
+    s = residual_sum(x, r, dtype)
+    return s, rmsnorm(s, gamma, eps, nthreads)

@@ -305,6 +305,36 @@ def pin_moe_group_top2(orc):
     _close(orc.moe_group_top2(v + 1.5), got + 3.0, rtol=0, atol=0)
 
 
+def pin_residual_norm(orc):
+    """Fused residual add + norm: the stored sum of small integers is exact,
+    a zero residual gives the plain norm of x, x and r commute, the sum is
+    rounded to the I/O type before the norm reads it (a bf16 hand case), and
+    the norms of the sum keep their invariants (mean 0 / unit RMS)."""
+    import torch
+    x = np.array([[1.0, 2.0, 3.0, 4.0], [-8.0, 0.0, 8.0, 16.0]])
+    r = np.array([[10.0, 20.0, 30.0, 40.0], [1.0, 1.0, 1.0, 1.0]])
+    s, y = orc.add_layernorm(x, r, torch.float32, eps=0.0)
+    _close(s, [[11.0, 22.0, 33.0, 44.0], [-7.0, 1.0, 9.0, 17.0]], rtol=0, atol=0)
+    # row 0 of s is 11 * (1, 2, 3, 4): mean 27.5, biased var 151.25
+    _close(y[0], (np.array([11.0, 22.0, 33.0, 44.0]) - 27.5) / math.sqrt(151.25))
+    # 256 + 1 is not a bf16 value: the sum rounds to 256 (ties to even) first
+    s, _ = orc.add_rmsnorm(np.array([[256.0, 3.0]]), np.array([[1.0, 0.0]]), torch.bfloat16)
+    _close(s, [[256.0, 3.0]], rtol=0, atol=0)
+    g = np.random.default_rng(13)
+    xv = g.standard_normal((6, 50)).astype(np.float32).astype(np.float64)
+    rv = g.standard_normal((6, 50)).astype(np.float32).astype(np.float64)
+    zero = np.zeros_like(xv)
+    _close(orc.add_layernorm(xv, zero, torch.float32)[1], orc.layernorm(xv))
+    _close(orc.add_rmsnorm(xv, zero, torch.float32)[1], orc.rmsnorm(xv))
+    _close(orc.add_layernorm(xv, rv, torch.float32)[1], orc.add_layernorm(rv, xv, torch.float32)[1])
+    s, y = orc.add_layernorm(xv, rv, torch.bfloat16, eps=0.0)
+    assert (torch.from_numpy(s).to(torch.bfloat16).double().numpy() == s).all()
+    _close(y.mean(axis=1), np.zeros(6), atol=1e-13)
+    s, y = orc.add_rmsnorm(xv, rv, torch.float16, eps=0.0)
+    _close(np.sqrt((y * y).mean(axis=1)), np.ones(6))
+
+
 ALL_PINS = [pin_hand_cases, pin_softmax_invariants, pin_layernorm_invariants,
             pin_rmsnorm_invariants, pin_brute_force, pin_torch_float64,
-            pin_ragged, pin_bucket_rule, pin_pad_scale, pin_moe_group_top2]
+            pin_ragged, pin_bucket_rule, pin_pad_scale, pin_moe_group_top2,
+            pin_residual_norm]
