@@ -197,6 +197,12 @@ def per_config(torch, rw, wl, device, peak, steps):
             ws = rw.ragged_workspace(case.rows, device)
             fn = lambda: rw.run(case.op, x, offsets=off, max_len=case.max_len,  # noqa: E731
                                 gamma=g, beta=b, eps=case.eps, out=y, ws=ws)
+        elif case.resid is not None:
+            rr = case.resid.to(device)
+            y = torch.empty_like(x)
+            sm = torch.empty_like(x)
+            fn = lambda: rw.run(case.op, x, gamma=g, beta=b, eps=case.eps, out=y,  # noqa: E731
+                                resid=rr, sum_out=sm)
         elif case.op in ("pad_scale", "moe_group_top2"):
             kw = dict(fft_size=case.meta.get("fft_size"), scale=case.meta.get("scale"))
             y = rw.run(case.op, x, **kw)
@@ -477,6 +483,8 @@ def run_only(args, local):
     if case.op in ("pad_scale", "moe_group_top2"):
         kw = dict(fft_size=case.meta.get("fft_size"), scale=case.meta.get("scale"))
         kw["out"] = rw.run(case.op, x, **kw)
+    if case.resid is not None:
+        kw.update(resid=case.resid.to(device), sum_out=torch.empty_like(x))
     if case.ragged:
         kw.update(offsets=case.offsets.to(device), max_len=case.max_len,
                   ws=rw.ragged_workspace(case.rows, device))

@@ -114,6 +114,22 @@ ROWOP_API int rowop_rmsnorm(const void *in, void *out, const void *gamma, int64_
                   int64_t cols, int64_t ld, rowop_dtype_t dtype, float eps,
                   cudaStream_t stream);
 
+/* ---- fused residual add + norm (dense) ------------------------------------
+ * sum_out = x + r (rounded to dtype: the updated residual stream), then
+ * y = LayerNorm(sum_out) or RMSNorm(sum_out) of the sum as stored -- the two
+ * steps of a pre-norm transformer block in one pass over HBM (read x and r,
+ * write sum_out and y).  x, r, sum_out and y share the rows x cols layout and
+ * ld; gamma/beta as above.  sum_out may be x or r itself (the residual stream
+ * updated in place); y must not overlap x, r or sum_out.                    */
+ROWOP_API int rowop_add_layernorm(const void *x, const void *r, void *sum_out, void *y,
+                                  const void *gamma, const void *beta, int64_t rows,
+                                  int64_t cols, int64_t ld, rowop_dtype_t dtype, float eps,
+                                  cudaStream_t stream);
+
+ROWOP_API int rowop_add_rmsnorm(const void *x, const void *r, void *sum_out, void *y,
+                                const void *gamma, int64_t rows, int64_t cols, int64_t ld,
+                                rowop_dtype_t dtype, float eps, cudaStream_t stream);
+
 /* ---- ragged rows (int64 CSR offsets into one packed buffer) ---------------
  * offsets : device int64[rows + 1], non-decreasing
  * max_len : an upper bound on every row's length (>= 0); sizes the on-chip

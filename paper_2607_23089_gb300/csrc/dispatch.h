@@ -24,6 +24,10 @@ struct DenseCall {
   int64_t rows, cols, ld;
   float eps;
   cudaStream_t stream;
+  // fused residual add (norms only): sum_out = in + resid, then the norm of
+  // sum_out; both NULL for the plain operator
+  const void *resid = nullptr;
+  void *sum_out = nullptr;
 };
 
 struct RaggedCall {

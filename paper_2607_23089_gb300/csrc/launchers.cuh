@@ -78,9 +78,9 @@ inline cudaError_t prepare_kernel(const void *kernel, const DeviceInfo &d, bool 
 // ---------------------------------------------------------------------------
 // SMALL: register-resident rows, G lanes per row
 // ---------------------------------------------------------------------------
-template <int OP, typename T, int CPL, bool EXACT>
+template <int OP, typename T, int CPL, bool EXACT, bool RESID>
 cudaError_t launch_small_k(const SmallParams &p, const DeviceInfo &d, cudaStream_t stream) {
-  auto kern = small_row_kernel<OP, T, CPL, EXACT>;
+  auto kern = small_row_kernel<OP, T, CPL, EXACT, RESID>;
   const int bps = cached_occupancy(reinterpret_cast<const void *>(kern), kCtaThreads, 0, 1,
                                    nullptr);
   const int64_t rows_per_cta = static_cast<int64_t>(kCtaWarps) * (32 / p.G);
@@ -91,7 +91,7 @@ cudaError_t launch_small_k(const SmallParams &p, const DeviceInfo &d, cudaStream
   return cudaGetLastError();
 }
 
-template <int OP, typename T>
+template <int OP, typename T, bool RESID>
 cudaError_t launch_small(const DenseCall &c, const DeviceInfo &d, bool exact, bool out_vec,
                          bool gvec) {
   constexpr int SZ = sizeof(T);
@@ -109,16 +109,19 @@ cudaError_t launch_small(const DenseCall &c, const DeviceInfo &d, bool exact, bo
   p.a.eps = c.eps;
   p.a.gvec = gvec;
   p.a.out_vec = out_vec;
+  p.resid = c.resid;
+  p.sum_out = c.sum_out;
+  p.rvec = RESID && congruent16(c.in, c.resid) && congruent16(c.in, c.sum_out);
   const int64_t max_chunks = ceil_div(c.cols, E) + (exact ? 0 : 1);
   const int cpl = small_cpl_class(max_chunks, p.G);
   if (exact) {
-    if (cpl == 4) return launch_small_k<OP, T, 4, true>(p, d, c.stream);
-    if (cpl == 8) return launch_small_k<OP, T, 8, true>(p, d, c.stream);
-    return launch_small_k<OP, T, 9, true>(p, d, c.stream);
+    if (cpl == 4) return launch_small_k<OP, T, 4, true, RESID>(p, d, c.stream);
+    if (cpl == 8) return launch_small_k<OP, T, 8, true, RESID>(p, d, c.stream);
+    return launch_small_k<OP, T, 9, true, RESID>(p, d, c.stream);
   }
-  if (cpl == 4) return launch_small_k<OP, T, 4, false>(p, d, c.stream);
-  if (cpl == 8) return launch_small_k<OP, T, 8, false>(p, d, c.stream);
-  return launch_small_k<OP, T, 9, false>(p, d, c.stream);
+  if (cpl == 4) return launch_small_k<OP, T, 4, false, RESID>(p, d, c.stream);
+  if (cpl == 8) return launch_small_k<OP, T, 8, false, RESID>(p, d, c.stream);
+  return launch_small_k<OP, T, 9, false, RESID>(p, d, c.stream);
 }
 
 // ---------------------------------------------------------------------------
@@ -127,11 +130,11 @@ cudaError_t launch_small(const DenseCall &c, const DeviceInfo &d, bool exact, bo
 // group_warps: consumer warps per item group (W); the stage ring holds at
 // least one item per group.  min_stage_area: bytes the stages must span
 // together (ragged SMALL staging).
-template <int OP, typename T, bool EXACT, bool CLUSTER, bool RAGGED>
+template <int OP, typename T, bool EXACT, bool CLUSTER, bool RAGGED, bool RESID = false>
 cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int group_warps,
                           int64_t items, const DeviceInfo &d, cudaStream_t stream,
                           uint32_t min_stage_area = 0) {
-  auto kern = tile_row_kernel<OP, T, EXACT, CLUSTER, RAGGED>;
+  auto kern = tile_row_kernel<OP, T, EXACT, CLUSTER, RAGGED, RESID>;
   const void *kp = reinterpret_cast<const void *>(kern);
   const int max_ctas_per_sm = read_knobs().ctas_per_sm;
   p.stage_bytes = static_cast<uint32_t>(stage_tiles) * kTileBytes;
@@ -228,8 +231,8 @@ inline int pick_cluster(int64_t K, int64_t cap, int knob) {
   return cs;
 }
 
-template <int OP, typename T>
-cudaError_t launch_dense_t(const DenseCall &c, const DeviceInfo &d) {
+template <int OP, typename T, bool RESID>
+cudaError_t launch_dense_impl(const DenseCall &c, const DeviceInfo &d) {
   constexpr int SZ = sizeof(T);
   constexpr int E = 16 / SZ;
   const Knobs kn = read_knobs();
@@ -245,7 +248,7 @@ cudaError_t launch_dense_t(const DenseCall &c, const DeviceInfo &d) {
   if (kn.force_bucket == kLarge) bucket = kLarge;
   if (bucket == kMedium && K > kMaxPortionTiles) bucket = kLarge;
 
-  if (bucket == kSmall) return launch_small<OP, T>(c, d, exact, out_vec, gvec);
+  if (bucket == kSmall) return launch_small<OP, T, RESID>(c, d, exact, out_vec, gvec);
 
   TileParams p = {};
   p.in = c.in;
@@ -261,6 +264,9 @@ cudaError_t launch_dense_t(const DenseCall &c, const DeviceInfo &d) {
   p.gvec = gvec;
   p.timeout_ns = kWaitLimitNs;
   p.status = d.status;
+  p.resid = c.resid;
+  p.sum_out = c.sum_out;
+  p.rvec = RESID && congruent16(c.in, c.resid) && congruent16(c.in, c.sum_out);
   // portions within the three-CTA stage budget: a 1 MiB fp32 row goes to
   // clusters of 16 with 64 KiB per CTA, three CTAs per SM (0.17 ms on
   // workload 4 against 0.23 ms for clusters of 8 with 128 KiB, one per SM)
@@ -270,11 +276,23 @@ cudaError_t launch_dense_t(const DenseCall &c, const DeviceInfo &d) {
   const int W = pick_group_warps(st, false, kn.group_warps);
   const int S = pick_stages(st, W, kn.stages);
   if (cs == 1) {
-    if (exact) return launch_tile_k<OP, T, true, false, false>(p, 1, S, st, W, c.rows, d, c.stream);
-    return launch_tile_k<OP, T, false, false, false>(p, 1, S, st, W, c.rows, d, c.stream);
+    if (exact)
+      return launch_tile_k<OP, T, true, false, false, RESID>(p, 1, S, st, W, c.rows, d, c.stream);
+    return launch_tile_k<OP, T, false, false, false, RESID>(p, 1, S, st, W, c.rows, d, c.stream);
   }
-  if (exact) return launch_tile_k<OP, T, true, true, false>(p, cs, S, st, W, c.rows, d, c.stream);
-  return launch_tile_k<OP, T, false, true, false>(p, cs, S, st, W, c.rows, d, c.stream);
+  if (exact)
+    return launch_tile_k<OP, T, true, true, false, RESID>(p, cs, S, st, W, c.rows, d, c.stream);
+  return launch_tile_k<OP, T, false, true, false, RESID>(p, cs, S, st, W, c.rows, d, c.stream);
+}
+
+// The dense launch path of one operator and type; the norms also serve the
+// fused residual add when the call carries a residual.
+template <int OP, typename T>
+cudaError_t launch_dense_t(const DenseCall &c, const DeviceInfo &d) {
+  if constexpr (OP == kLayerNorm || OP == kRmsNorm) {
+    if (c.resid) return launch_dense_impl<OP, T, true>(c, d);
+  }
+  return launch_dense_impl<OP, T, false>(c, d);
 }
 
 

@@ -170,10 +170,15 @@ static int check_dense(const void *in, const void *out, const void *gamma, const
 
 static int run_dense(int op, const void *in, void *out, const void *gamma, const void *beta,
                      int64_t rows, int64_t cols, int64_t ld, rowop_dtype_t dtype, float eps,
-                     cudaStream_t stream) {
+                     cudaStream_t stream, const void *resid = nullptr, void *sum_out = nullptr) {
   const bool norm = (op == kLayerNorm || op == kRmsNorm);
   const int chk = check_dense(in, out, gamma, beta, rows, cols, ld, dtype, eps, norm);
   if (chk < 0) return -chk;
+  if (resid || sum_out) {
+    const int es = esize_of(dtype);
+    if (!norm || !resid || !sum_out || !elem_aligned(resid, es) || !elem_aligned(sum_out, es))
+      return ROWOP_ERR_INVALID_ARG;
+  }
   if (chk == 1) return ROWOP_OK;
   DeviceInfo d;
   const int st = device_info(&d);
@@ -189,6 +194,8 @@ static int run_dense(int op, const void *in, void *out, const void *gamma, const
   c.ld = ld;
   c.eps = eps;
   c.stream = stream;
+  c.resid = resid;
+  c.sum_out = sum_out;
   switch (op) {
     case kSoftmax: return from_cuda(launch_dense<kSoftmax>(c, d));
     case kLogSoftmax: return from_cuda(launch_dense<kLogSoftmax>(c, d));
@@ -284,6 +291,22 @@ int rowop_layernorm(const void *in, void *out, const void *gamma, const void *be
 int rowop_rmsnorm(const void *in, void *out, const void *gamma, int64_t rows, int64_t cols,
                   int64_t ld, rowop_dtype_t dtype, float eps, cudaStream_t stream) {
   return run_dense(kRmsNorm, in, out, gamma, nullptr, rows, cols, ld, dtype, eps, stream);
+}
+
+int rowop_add_layernorm(const void *x, const void *r, void *sum_out, void *y,
+                        const void *gamma, const void *beta, int64_t rows, int64_t cols,
+                        int64_t ld, rowop_dtype_t dtype, float eps, cudaStream_t stream) {
+  if (!r || !sum_out) return rows == 0 ? ROWOP_OK : ROWOP_ERR_INVALID_ARG;
+  return run_dense(kLayerNorm, x, y, gamma, beta, rows, cols, ld, dtype, eps, stream, r,
+                   sum_out);
+}
+
+int rowop_add_rmsnorm(const void *x, const void *r, void *sum_out, void *y, const void *gamma,
+                      int64_t rows, int64_t cols, int64_t ld, rowop_dtype_t dtype, float eps,
+                      cudaStream_t stream) {
+  if (!r || !sum_out) return rows == 0 ? ROWOP_OK : ROWOP_ERR_INVALID_ARG;
+  return run_dense(kRmsNorm, x, y, gamma, nullptr, rows, cols, ld, dtype, eps, stream, r,
+                   sum_out);
 }
 
 size_t rowop_ragged_workspace_size(int64_t rows) {

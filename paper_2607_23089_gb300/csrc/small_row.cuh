@@ -161,11 +161,42 @@ struct SmallParams {
   int64_t ld;
   int G;
   SmallRowArgs a;
+  // fused residual add: sum_out = in + resid (same layout), normalised after
+  const void *resid;
+  void *sum_out;
+  int rvec;  // resid and sum_out 16-byte congruent to in
 };
+
+// Residual add for one window chunk c of a row: chunk x (the row's elements,
+// zeros elsewhere) plus the same chunk of the residual, rounded to T, stored
+// to sum_out and returned -- the norm reads the sum as stored.
+template <typename T>
+__device__ __forceinline__ uint4 residual_chunk(const uint4 &x, const T *r_row, T *s_row,
+                                                const char *rwin, char *swin, int64_t c, int h,
+                                                int lo, int hi, int64_t n, bool rvec) {
+  constexpr int E = Elem<T>::kPerChunk;
+  constexpr int NP = E / 2;
+  const bool full = lo == 0 && hi == E;
+  const uint4 rr = (full && rvec) ? ldg_stream(rwin + c * kChunkBytes)
+                                  : load_chunk_elems<T>(r_row, c, h, n);
+  f2 a[NP], b[NP];
+  chunk_to_pairs<T>(x, a);
+  chunk_to_pairs<T>(rr, b);
+#pragma unroll
+  for (int i = 0; i < NP; ++i) a[i] = f2_add(a[i], b[i]);
+  const uint4 sv = pairs_to_chunk<T>(a);
+  if (full && rvec) {
+    stg_stream(swin + c * kChunkBytes, sv);
+  } else {
+    chunk_to_pairs<T>(sv, a);  // the stored (rounded) values, element by element
+    store_chunk<T>(a, swin, s_row, c, h, lo, hi, false);
+  }
+  return sv;
+}
 
 // Dense SMALL kernel: persistent grid; each warp takes BLOCK_ROWS = 32/G
 // consecutive rows per step, every lane loads its chunks into registers first.
-template <int OP, typename T, int CPL, bool EXACT>
+template <int OP, typename T, int CPL, bool EXACT, bool RESID = false>
 __global__ void __launch_bounds__(kCtaThreads) small_row_kernel(const SmallParams p) {
   constexpr int E = Elem<T>::kPerChunk;
   constexpr int SZ = Elem<T>::kSize;
@@ -196,6 +227,22 @@ __global__ void __launch_bounds__(kCtaThreads) small_row_kernel(const SmallParam
         if (!EXACT) chunk_valid_range(c, nc, h, h + p.cols, E, lo, hi);
         raw[k] = (lo == 0 && hi == E) ? ldg_stream(win + c * kChunkBytes)
                                        : load_chunk_elems<T>(in_row, c, h, p.cols);
+      }
+    }
+    if constexpr (RESID) {
+      const T *r_row = static_cast<const T *>(p.resid) + (active ? r : 0) * p.ld;
+      T *s_row = static_cast<T *>(p.sum_out) + (active ? r : 0) * p.ld;
+      const char *rwin = reinterpret_cast<const char *>(r_row) - h * SZ;
+      char *swin = reinterpret_cast<char *>(s_row) - h * SZ;
+#pragma unroll
+      for (int k = 0; k < CPL; ++k) {
+        const int64_t c = sub + static_cast<int64_t>(k) * G;
+        if (c < nc) {
+          int lo = 0, hi = E;
+          if (!EXACT) chunk_valid_range(c, nc, h, h + p.cols, E, lo, hi);
+          raw[k] = residual_chunk<T>(raw[k], r_row, s_row, rwin, swin, c, h, lo, hi, p.cols,
+                                     p.rvec != 0);
+        }
       }
     }
     small_row_core<OP, T, CPL, EXACT, true>([&](int k) { return raw[k]; }, out_row, p.cols, h, nc, G,

@@ -73,6 +73,10 @@ struct TileParams {
   int blocks;                   // classify blocks (0: dense launch)
   int64_t rows_per_block;       // classify block b lists from entry b * rows_per_block on
   unsigned int *counters;       // [3]: next MEDIUM, next SMALL, CTAs finished
+  // fused residual add (dense norms): sum_out = in + resid, same layout
+  const void *resid;
+  void *sum_out;
+  int rvec;  // resid and sum_out 16-byte congruent to in
 };
 
 struct ItemMeta {
@@ -238,10 +242,35 @@ __device__ __forceinline__ float tile_lane_second(const unsigned char *tsm, cons
 // (same arithmetic: the masks of a full tile keep every element).  Waits on
 // each stage piece before the first tile read from it (`waited` is the last
 // piece waited for); returns false when such a wait ran out.
-template <int OP, typename T, int B, bool FULL>
+// Fused residual add for this lane's two chunks of tile t, in the stage:
+// each becomes the stored sum x + r (written to sum_out too), so the
+// statistics and pass 2 read the sum as stored.
+template <typename T>
+__device__ __forceinline__ void residual_tile(unsigned char *tsm, int t, const ItemGeo &g,
+                                              int lane, const TileParams &p) {
+  constexpr int E = Elem<T>::kPerChunk;
+  constexpr int SZ = Elem<T>::kSize;
+  const T *r_row = static_cast<const T *>(p.resid) + g.start;
+  T *s_row = static_cast<T *>(p.sum_out) + g.start;
+  const char *rwin = reinterpret_cast<const char *>(r_row) - g.h * SZ;
+  char *swin = reinterpret_cast<char *>(s_row) - g.h * SZ;
+  const int hn = g.h + static_cast<int>(g.n);
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    const int c = t * kTileChunks + lane + 32 * u;
+    if (c >= g.nc) continue;
+    uint4 *slot = reinterpret_cast<uint4 *>(tsm + (lane + 32 * u) * kChunkBytes);
+    int lo, hi;
+    chunk_valid_range(c, g.nc, g.h, hn, E, lo, hi);
+    *slot = residual_chunk<T>(*slot, r_row, s_row, rwin, swin, c, g.h, lo, hi, g.n, p.rvec != 0);
+  }
+}
+
+template <int OP, typename T, int B, bool FULL, bool RESID>
 __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const ItemGeo &g, int lt0,
                                             int W, int lane, float4 *part, uint32_t piece_bar0,
-                                            uint32_t par, uint64_t timeout_ns, int &waited) {
+                                            uint32_t par, uint64_t timeout_ns, int &waited,
+                                            const TileParams &p) {
   constexpr int E = Elem<T>::kPerChunk;
   constexpr bool kMaxFirst = (OP == kSoftmax || OP == kLogSoftmax);
   float a[B], b[B];
@@ -254,6 +283,8 @@ __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const It
       waited = pc;
     }
     const int t = g.t0 + lt;
+    if constexpr (RESID)
+      residual_tile<T>(const_cast<unsigned char *>(stage) + lt * kTileBytes, t, g, lane, p);
     const TileMask m = FULL ? TileMask{0, E, 0, E} : tile_mask<T>(t, g, lane, tile_is_full(t, g));
     a[q] = tile_lane_first<OP, T>(stage + lt * kTileBytes, m, lane);
   }
@@ -314,10 +345,10 @@ __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const It
 // tiles lt = wig, wig + W, ..., taken PB at a time while that many remain,
 // then in a batch of two and one.  Each tile's arithmetic (and its butterfly
 // order) is the same whatever batch it falls in.
-template <int OP, typename T, int PB>
+template <int OP, typename T, int PB, bool RESID>
 __device__ __forceinline__ bool pass1_warp(const unsigned char *stage, const ItemGeo &g, int wig,
                                            int W, int lane, float4 *part, uint32_t piece_bar0,
-                                           uint32_t par, uint64_t timeout_ns) {
+                                           uint32_t par, uint64_t timeout_ns, const TileParams &p) {
   const int ntl = g.t1 - g.t0;
   // tiles [full0, full1) of the row lie entirely in it (all but its ends)
   const int full0 = g.cf > 0 ? 1 : 0;
@@ -331,20 +362,20 @@ __device__ __forceinline__ bool pass1_warp(const unsigned char *stage, const Ite
     const bool full = ta >= full0 && tb < full1;
     bool ok;
     if (PB > 2 && bsz == PB) {
-      ok = full ? pass1_batch<OP, T, PB, true>(stage, g, lt0, W, lane, part, piece_bar0, par,
-                                               timeout_ns, waited)
-                : pass1_batch<OP, T, PB, false>(stage, g, lt0, W, lane, part, piece_bar0, par,
-                                                timeout_ns, waited);
+      ok = full ? pass1_batch<OP, T, PB, true, RESID>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                                               timeout_ns, waited, p)
+                : pass1_batch<OP, T, PB, false, RESID>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                                                timeout_ns, waited, p);
     } else if (bsz == 2) {
-      ok = full ? pass1_batch<OP, T, 2, true>(stage, g, lt0, W, lane, part, piece_bar0, par,
-                                              timeout_ns, waited)
-                : pass1_batch<OP, T, 2, false>(stage, g, lt0, W, lane, part, piece_bar0, par,
-                                               timeout_ns, waited);
+      ok = full ? pass1_batch<OP, T, 2, true, RESID>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                                              timeout_ns, waited, p)
+                : pass1_batch<OP, T, 2, false, RESID>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                                               timeout_ns, waited, p);
     } else {
-      ok = full ? pass1_batch<OP, T, 1, true>(stage, g, lt0, W, lane, part, piece_bar0, par,
-                                              timeout_ns, waited)
-                : pass1_batch<OP, T, 1, false>(stage, g, lt0, W, lane, part, piece_bar0, par,
-                                               timeout_ns, waited);
+      ok = full ? pass1_batch<OP, T, 1, true, RESID>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                                              timeout_ns, waited, p)
+                : pass1_batch<OP, T, 1, false, RESID>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                                               timeout_ns, waited, p);
     }
     if (!ok) return false;
     lt0 += bsz * W;
@@ -852,7 +883,7 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
   }
 }
 
-template <int OP, typename T, bool EXACT, bool CLUSTER, bool RAGGED>
+template <int OP, typename T, bool EXACT, bool CLUSTER, bool RAGGED, bool RESID = false>
 __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TileParams p) {
   constexpr int E = Elem<T>::kPerChunk;
   constexpr int SZ = Elem<T>::kSize;
@@ -960,8 +991,9 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
 
     // ---- pass 1 ----
     if (!bad && kind != kItemEnd)
-      bad = !pass1_warp<OP, T, kPass1Batch>(stage, g, wig, W, lane, part,
-                               sbase + L.bar_piece + 8u * (s * L.pieces), par, p.timeout_ns);
+      bad = !pass1_warp<OP, T, kPass1Batch, RESID>(stage, g, wig, W, lane, part,
+                                                  sbase + L.bar_piece + 8u * (s * L.pieces), par,
+                                                  p.timeout_ns, p);
     if (named_sync_or(gbar, gthreads, bad)) {
       if (gtid == 0) {
         atomicOr(p.status, kStatusTimeout);
@@ -1030,6 +1062,9 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
     T *out_row = static_cast<T *>(p.out) + g.start;
     char *owin = reinterpret_cast<char *>(out_row) - g.h * SZ;
     pass2_item<OP, T, EXACT>(stage, g, wig, W, lane, s0, s1, p, owin, out_row);
+    // the stage was written through the generic proxy (the residual sums):
+    // order that before the producer's next bulk copies into it
+    if constexpr (RESID) fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0) mbar_arrive(sbase + L.bar_empty + 8u * s);
   }

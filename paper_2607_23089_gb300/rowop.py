@@ -58,6 +58,8 @@ SIGNATURES = {
                                         _P], _I),
     "rowop_rmsnorm_ragged_planned": ([_P, _P, _P, _P, _I64, _I64, _I, _F, _P, _SZ, _P], _I),
     "rowop_layernorm_ragged_static": ([_P, _P, _P, _P, _P, _I64, _I64, _I, _F, _P], _I),
+    "rowop_add_layernorm": ([_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _F, _P], _I),
+    "rowop_add_rmsnorm": ([_P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _F, _P], _I),
     "rowop_pad_scale": ([_P, _P, _I64, _I64, _I64, _I64, _I64, _F, _I, _P], _I),
     "rowop_moe_group_top2": ([_P, _P, _I64, _I64, _I64, _I, _P], _I),
     "rowop_select_bucket": ([_I64, _I], _I),
@@ -271,6 +273,36 @@ def select_bucket(length: int, dtype) -> int:
     return rowop_select_bucket(int(length), code)  # noqa: F821
 
 
+def add_layernorm(x, r, gamma=None, beta=None, eps=1e-5, sum_out=None, out=None, stream=None):
+    """Fused residual add + LayerNorm (``rowop_add_layernorm``): returns
+    ``(x + r, LayerNorm(x + r))``."""
+    torch = _torch()
+    _check_cuda(x, r, gamma, beta)
+    rows, cols = x.shape
+    sum_out = torch.empty_like(x) if sum_out is None else sum_out
+    out = torch.empty_like(x) if out is None else out
+    _ok(rowop_add_layernorm(x.data_ptr(), r.data_ptr(), sum_out.data_ptr(),  # noqa: F821
+                            out.data_ptr(), _ptr(gamma), _ptr(beta), rows, cols, x.stride(0),
+                            dtype_code(x.dtype), float(eps), _stream(stream)),
+        "rowop_add_layernorm")
+    return sum_out, out
+
+
+def add_rmsnorm(x, r, gamma=None, eps=1e-6, sum_out=None, out=None, stream=None):
+    """Fused residual add + RMSNorm (``rowop_add_rmsnorm``): returns
+    ``(x + r, RMSNorm(x + r))``."""
+    torch = _torch()
+    _check_cuda(x, r, gamma)
+    rows, cols = x.shape
+    sum_out = torch.empty_like(x) if sum_out is None else sum_out
+    out = torch.empty_like(x) if out is None else out
+    _ok(rowop_add_rmsnorm(x.data_ptr(), r.data_ptr(), sum_out.data_ptr(),  # noqa: F821
+                          out.data_ptr(), _ptr(gamma), rows, cols, x.stride(0),
+                          dtype_code(x.dtype), float(eps), _stream(stream)),
+        "rowop_add_rmsnorm")
+    return sum_out, out
+
+
 def pad_scale(x, fft_size: int, scale: float, out=None, stream=None):
     """Hyena FFT-size padding of a rows x seqlen tensor to rows x fft_size
     (``rowop_pad_scale``)."""
@@ -300,11 +332,17 @@ def moe_group_top2(scores, out=None, stream=None):
 
 
 def run(op: str, x, *, offsets=None, max_len=None, gamma=None, beta=None,
-        eps=None, out=None, ws=None, stream=None, fft_size=None, scale=None):
+        eps=None, out=None, ws=None, stream=None, fft_size=None, scale=None, resid=None,
+        sum_out=None):
     """One call of ``op`` on dense or ragged input (ragged when offsets is
     given); returns the output tensor."""
     if op == "pad_scale":
         return pad_scale(x, fft_size, scale, out, stream)
+    if op == "add_layernorm":
+        return add_layernorm(x, resid, gamma, beta, 1e-5 if eps is None else eps, sum_out, out,
+                             stream)[1]
+    if op == "add_rmsnorm":
+        return add_rmsnorm(x, resid, gamma, 1e-6 if eps is None else eps, sum_out, out, stream)[1]
     if op == "moe_group_top2":
         return moe_group_top2(x, out, stream)
     if offsets is None:

@@ -46,6 +46,7 @@ class Case:
     eps: float = 0.0
     max_len: int = 0
     meta: dict = field(default_factory=dict)
+    resid: Optional[torch.Tensor] = None     # fused residual add: the residual r
 
     @property
     def ragged(self) -> bool:
@@ -68,6 +69,8 @@ class Case:
         if self.op == "moe_group_top2":  # read the scores, write one float per group
             return self.x.numel() * es + self.x.shape[0] * (self.x.shape[1] // 32) * 4
         b = 2 * self.elements * es
+        if self.resid is not None:  # also read r and write the sum
+            b += 2 * self.elements * es
         ncol = self.max_len if self.ragged else self.x.shape[1]
         if self.gamma is not None:
             b += ncol * es
@@ -154,6 +157,23 @@ def ragged_ln(rows: int = 16384, max_len: int = 32768, op: str = "layernorm",
                 eps=eps, max_len=max_len)
 
 
+def medium_add_norm(op: str, rows: int = 8192, cols: int = 4096, seed: int = 7) -> Case:
+    """Fused residual add + norm on the workload-3 shape: bf16 x as in
+    workload 3, residual r = N(0,1), gamma/beta as there.  Not one of the five
+    workloads."""
+    g = _gen(seed)
+    x = torch.randn(rows, cols, generator=g)
+    scale = 0.1 + 9.9 * torch.rand(rows, 1, generator=g)
+    x = (x * scale).to(torch.bfloat16)
+    r = torch.randn(rows, cols, generator=g).to(torch.bfloat16)
+    gamma, beta = _affine(g, cols, torch.bfloat16)
+    if op == "rmsnorm":
+        return Case("medium_add_rmsnorm", "add_rmsnorm", x, torch.bfloat16, gamma=gamma,
+                    eps=1e-6, resid=r)
+    return Case("medium_add_layernorm", "add_layernorm", x, torch.bfloat16, gamma=gamma,
+                beta=beta, eps=1e-5, resid=r)
+
+
 def hyena_pad(rows: int = 16384, seqlen: int = 4096, fft_size: int = 8192,
               seed: int = 5) -> Case:
     """Hyena FFT-size padding (§6): fp32 rows x seqlen, x = N(0,1), padded
@@ -190,6 +210,8 @@ def all_cases(scale_down: int = 1):
         out.append(medium_norm(op, rows=max(1, 8192 // s)))
     out.append(long_rows(rows=max(1, 256 // s)))
     out.append(ragged_ln(rows=max(1, 16384 // s)))
+    for op in ("rmsnorm", "layernorm"):
+        out.append(medium_add_norm(op, rows=max(1, 8192 // s)))
     out.append(hyena_pad(rows=max(1, 16384 // s)))
     out.append(moe_group(tokens=max(1, 131072 // s)))
     return out
@@ -208,6 +230,8 @@ def by_name(name: str) -> Case:
         return long_rows(op=name[len("long_rows_"):])
     if name.startswith("ragged_"):
         return ragged_ln(op=name[len("ragged_"):])
+    if name.startswith("medium_add_"):
+        return medium_add_norm(name[len("medium_add_"):])
     if name == "hyena_pad_scale":
         return hyena_pad()
     if name == "moe_group_top2":
