@@ -456,12 +456,21 @@ __device__ __forceinline__ void combine_long(Get get, int K, float inv_n, float 
                                              int wig, int W, uint32_t bar, volatile float *xw,
                                              float &s0, float &s1) {
   constexpr bool kMax = (OP == kSoftmax || OP == kLogSoftmax);
+  constexpr int kAhead = 4;  // partials a lane fetches before folding them (in order)
   const uint32_t nthreads = static_cast<uint32_t>(W) * 32u;
+  const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
   for (int vw = wig; vw < kConsumerWarps; vw += W) {
     float v = kMax ? -INFINITY : 0.f;
-    for (int t = vw * 32 + lane; t < K; t += kConsumerThreads) {
-      const float x = get(t).x;
-      v = kMax ? fmaxf(v, x) : __fadd_rn(v, x);
+    for (int t0 = vw * 32 + lane; t0 < K; t0 += kAhead * kConsumerThreads) {
+      float4 q[kAhead];
+#pragma unroll
+      for (int i = 0; i < kAhead; ++i) {
+        const int t = t0 + i * kConsumerThreads;
+        q[i] = t < K ? get(t) : z;
+      }
+#pragma unroll
+      for (int i = 0; i < kAhead; ++i)
+        if (t0 + i * kConsumerThreads < K) v = kMax ? fmaxf(v, q[i].x) : __fadd_rn(v, q[i].x);
     }
     v = kMax ? warp_max(v) : warp_sum(v);
     if (lane == 0) xw[vw] = v;
@@ -474,8 +483,17 @@ __device__ __forceinline__ void combine_long(Get get, int K, float inv_n, float 
   if constexpr (OP != kRmsNorm) {
     for (int vw = wig; vw < kConsumerWarps; vw += W) {
       float u = 0.f;
-      for (int t = vw * 32 + lane; t < K; t += kConsumerThreads)
-        u = __fadd_rn(u, second_term<OP>(get(t), first));
+      for (int t0 = vw * 32 + lane; t0 < K; t0 += kAhead * kConsumerThreads) {
+        float4 q[kAhead];
+#pragma unroll
+        for (int i = 0; i < kAhead; ++i) {
+          const int t = t0 + i * kConsumerThreads;
+          q[i] = t < K ? get(t) : z;
+        }
+#pragma unroll
+        for (int i = 0; i < kAhead; ++i)
+          if (t0 + i * kConsumerThreads < K) u = __fadd_rn(u, second_term<OP>(q[i], first));
+      }
       u = warp_sum(u);
       if (lane == 0) xw[kConsumerWarps + vw] = u;
     }
