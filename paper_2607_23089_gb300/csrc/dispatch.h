@@ -110,19 +110,24 @@ inline int64_t max_row_len_elems(int esize) {
   return static_cast<int64_t>(kMaxPortionTiles) * kMaxCluster * 64 * e - (e - 1);
 }
 
-// Test-and-tuning knobs read from the environment (never change results):
+// Test-and-tuning knobs read from the environment (none changes results but
+// ROWOP_SOFTMAX_ONLINE, which selects another way to round):
 //   ROWOP_FORCE_BUCKET  0/1/2 -> dense rows use that design when it can hold
 //                       the row (SMALL only for rows of <= 288 chunks)
 //   ROWOP_CLUSTER       cluster size for split rows (1, 2, 4, 8, 16)
 //   ROWOP_STAGES        stage-ring depth of the tile kernel
 //   ROWOP_CTAS_PER_SM   upper bound on resident tile-kernel CTAs per SM
 //   ROWOP_GROUP_WARPS   consumer warps per item group of the tile kernel (1, 2, 4, 8)
+//   ROWOP_SOFTMAX_ONLINE 1 -> dense SMALL softmax / log-softmax use the online
+//                       one-pass statistics instead of the two-pass ones (a
+//                       comparison variant: its results differ by rounding)
 struct Knobs {
   int force_bucket = -1;
   int cluster = 0;
   int stages = 0;
   int ctas_per_sm = 0;
   int group_warps = 0;
+  int softmax_online = 0;
 };
 Knobs read_knobs();
 

@@ -81,6 +81,9 @@ inline cudaError_t prepare_kernel(const void *kernel, const DeviceInfo &d, bool 
 template <int OP, typename T, int CPL, bool EXACT, bool RESID>
 cudaError_t launch_small_k(const SmallParams &p, const DeviceInfo &d, cudaStream_t stream) {
   auto kern = small_row_kernel<OP, T, CPL, EXACT, RESID>;
+  if constexpr (OP == kSoftmax || OP == kLogSoftmax) {
+    if (read_knobs().softmax_online) kern = small_row_kernel<OP, T, CPL, EXACT, RESID, true>;
+  }
   const int bps = cached_occupancy(reinterpret_cast<const void *>(kern), kCtaThreads, 0, 1,
                                    nullptr);
   const int64_t rows_per_cta = static_cast<int64_t>(kCtaWarps) * (32 / p.G);

@@ -50,6 +50,7 @@ Knobs read_knobs() {
   k.stages = env_int("ROWOP_STAGES", 0);
   k.ctas_per_sm = env_int("ROWOP_CTAS_PER_SM", 0);
   k.group_warps = env_int("ROWOP_GROUP_WARPS", 0);
+  k.softmax_online = env_int("ROWOP_SOFTMAX_ONLINE", 0);
   return k;
 }
 

@@ -48,7 +48,22 @@ struct SmallRowArgs {
 // below G.  Inactive groups pass nc = 0.  UNROLL = false keeps the chunk
 // loops rolled (for chunk sources that can be indexed at run time); the
 // operations and their order do not change.
-template <int OP, typename T, int CPL, bool EXACT, bool UNROLL, class Get>
+// Online (one-pass) softmax statistics of a lane's chunks: a running maximum
+// m and sum s of exp(x - m), rescaled when a chunk raises the maximum.
+// Groups then merge their (m, s) pairs: M = max, S = s e^(m-M) + s' e^(m'-M).
+__device__ __forceinline__ void online_merge(float &m, float &s, float m2, float s2) {
+  if (m2 == -INFINITY) return;
+  if (m == -INFINITY) {
+    m = m2;
+    s = s2;
+    return;
+  }
+  const float M = fmaxf(m, m2);
+  s = __fadd_rn(__fmul_rn(s, exp_shifted(m, M)), __fmul_rn(s2, exp_shifted(m2, M)));
+  m = M;
+}
+
+template <int OP, typename T, int CPL, bool EXACT, bool UNROLL, bool ONLINE = false, class Get>
 __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, int h, int64_t nc,
                                                int G, int sub, const SmallRowArgs &a) {
   constexpr int E = Elem<T>::kPerChunk;
@@ -58,7 +73,33 @@ __device__ __forceinline__ void small_row_core(Get get, T *out_row, int64_t n, i
   float s0 = 0.f, s1 = 0.f;
 
   // ---- statistics ----
-  if constexpr (OP == kSoftmax || OP == kLogSoftmax) {
+  if constexpr ((OP == kSoftmax || OP == kLogSoftmax) && ONLINE) {
+    float m = -INFINITY, sl = 0.f;
+#pragma unroll(kUnroll)
+    for (int k = 0; k < CPL; ++k) {
+      const int64_t c = sub + static_cast<int64_t>(k) * G;
+      if (c < nc) {
+        f2 p[NP];
+        chunk_to_pairs<T>(get(k), p);
+        int lo = 0, hi = E;
+        if (!EXACT) chunk_valid_range(c, nc, h, hn, E, lo, hi);
+        const float cm = chunk_max<NP>(p, -INFINITY, lo, hi);
+        if (cm > m) {  // the chunk raises the maximum: rescale what was summed
+          sl = m == -INFINITY ? 0.f : __fmul_rn(sl, exp_shifted(m, cm));
+          m = cm;
+        }
+        if (m != -INFINITY)
+          sl = __fadd_rn(sl, f2_total(chunk_sum_exp<NP>(p, f2_bcast(m), f2_bcast(0.f), lo, hi)));
+      }
+    }
+    for (int o = 1; o < G; o <<= 1) {
+      const float m2 = __shfl_xor_sync(kFullMask, m, o);
+      const float s2 = __shfl_xor_sync(kFullMask, sl, o);
+      online_merge(m, sl, m2, s2);
+    }
+    s0 = m;
+    s1 = (OP == kSoftmax) ? __frcp_rn(sl) : logf(sl);
+  } else if constexpr (OP == kSoftmax || OP == kLogSoftmax) {
     float m = -INFINITY;
 #pragma unroll(kUnroll)
     for (int k = 0; k < CPL; ++k) {
@@ -196,7 +237,7 @@ __device__ __forceinline__ uint4 residual_chunk(const uint4 &x, const T *r_row, 
 
 // Dense SMALL kernel: persistent grid; each warp takes BLOCK_ROWS = 32/G
 // consecutive rows per step, every lane loads its chunks into registers first.
-template <int OP, typename T, int CPL, bool EXACT, bool RESID = false>
+template <int OP, typename T, int CPL, bool EXACT, bool RESID = false, bool ONLINE = false>
 __global__ void __launch_bounds__(kCtaThreads) small_row_kernel(const SmallParams p) {
   constexpr int E = Elem<T>::kPerChunk;
   constexpr int SZ = Elem<T>::kSize;
@@ -245,8 +286,8 @@ __global__ void __launch_bounds__(kCtaThreads) small_row_kernel(const SmallParam
         }
       }
     }
-    small_row_core<OP, T, CPL, EXACT, true>([&](int k) { return raw[k]; }, out_row, p.cols, h, nc, G,
-                                      sub, p.a);
+    small_row_core<OP, T, CPL, EXACT, true, ONLINE>([&](int k) { return raw[k]; }, out_row, p.cols,
+                                                    h, nc, G, sub, p.a);
   }
 }
 

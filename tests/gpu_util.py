@@ -30,8 +30,12 @@ def assert_close(got, ref, dtype, what=""):
     rtol, atol = TOL[dtype]
     nan_g, nan_r = np.isnan(got), np.isnan(ref)
     assert (nan_g == nan_r).all(), f"{what}: NaN pattern differs"
-    err = np.abs(np.where(nan_r, 0.0, got - ref))
-    lim = atol + rtol * np.abs(np.where(nan_r, 0.0, ref))
+    inf_g, inf_r = np.isinf(got), np.isinf(ref)
+    assert (inf_g == inf_r).all(), f"{what}: infinity pattern differs"
+    assert (got[inf_r] == ref[inf_r]).all(), f"{what}: infinity of the wrong sign"
+    special = nan_r | inf_r
+    err = np.abs(np.where(special, 0.0, got - np.where(special, 0.0, ref)))
+    lim = atol + rtol * np.abs(np.where(special, 0.0, ref))
     bad = err > lim
     if bad.any():
         i = np.unravel_index(np.argmax(err - lim), err.shape)

@@ -191,3 +191,22 @@ def test_group_sizes_agree(rw, op, dtype, cols, ld, x_off):
         got = _forced(rw, op, dtype, rows, cols, 2, cluster=cs, ld=ld, x_off=x_off,
                       group_warps=w)
         assert torch.equal(_bits(ref), _bits(got)), f"cluster {cs} W={w}"
+
+
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
+@pytest.mark.parametrize("op", ["softmax", "logsoftmax"])
+@pytest.mark.parametrize("cols", [1, 5, 64, 255, 1000, 2047])
+def test_online_softmax_variant(rw, op, dtype, cols, monkeypatch):
+    """The one-pass (online) softmax statistics of the SMALL design, selected
+    by ROWOP_SOFTMAX_ONLINE, meet the same tolerance against the oracle,
+    also on rows whose maximum arrives late and rows with -inf entries."""
+    monkeypatch.setenv("ROWOP_SOFTMAX_ONLINE", "1")
+    run_case(rw, op, dtype, 37, cols, seed=cols + 3)
+    rows = 6
+    x = torch.linspace(-20, 20, cols).repeat(rows, 1)  # increasing: the maximum is last
+    x[1] = x[1].flip(0)
+    x[2, ::3] = -float("inf")
+    x = x.to(dtype)
+    y = rw.run(op, x.cuda()).cpu()
+    ref = oracle_dense(op, x.double().numpy())
+    assert_close(to_f64(y), ref, dtype, f"online {op}")
