@@ -32,7 +32,7 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "rowop_oracle.c")
-_SRCS = [_SRC, os.path.join(_HERE, "pad_moe_oracle.c")]
+_SRCS = [_SRC, os.path.join(_HERE, "pad_moe_oracle.c"), os.path.join(_HERE, "backward_oracle.c")]
 _BUILD_DIR = os.path.join(_HERE, "_build")
 _LIB_PATH = os.path.join(_BUILD_DIR, "liboracle.so")
 _lock = threading.Lock()
@@ -42,8 +42,8 @@ SMALL, MEDIUM, LARGE = 0, 1, 2
 
 
 def build(force: bool = False) -> str:
-    """Compile ``rowop_oracle.c`` and ``pad_moe_oracle.c`` with gcc (-O2, no
-    fast-math) into a shared library next to them.  OpenMP is used when the
+    """Compile ``rowop_oracle.c``, ``pad_moe_oracle.c`` and
+    ``backward_oracle.c`` with gcc (-O2, no fast-math) into a shared library next to them.  OpenMP is used when the
     compiler offers it; without it the row loop simply runs on one thread."""
     os.makedirs(_BUILD_DIR, exist_ok=True)
     if (not force and os.path.exists(_LIB_PATH)
@@ -81,6 +81,14 @@ def _load():
         lib.oracle_bucket.restype = ci
         lib.oracle_pad_scale.argtypes = [d, d, i64, i64, i64, dbl]
         lib.oracle_moe_group_top2.argtypes = [d, d, i64, i64, i64]
+        lib.oracle_softmax_backward.argtypes = [d, d, d, i64, i64, ci]
+        lib.oracle_logsoftmax_backward.argtypes = [d, d, d, i64, i64, ci]
+        lib.oracle_layernorm_backward.argtypes = [d, d, d, d, d, d, i64, i64, dbl, ci]
+        lib.oracle_layernorm_backward.restype = ci
+        lib.oracle_rmsnorm_backward.argtypes = [d, d, d, d, d, i64, i64, dbl, ci]
+        lib.oracle_rmsnorm_backward.restype = ci
+        lib.oracle_softmax_backward.restype = None
+        lib.oracle_logsoftmax_backward.restype = None
         for name in ("oracle_softmax", "oracle_logsoftmax", "oracle_layernorm",
                      "oracle_rmsnorm", "oracle_softmax_ragged",
                      "oracle_logsoftmax_ragged", "oracle_layernorm_ragged",
@@ -274,3 +282,64 @@ def add_rmsnorm(x, r, dtype, gamma=None, eps=1e-6, nthreads=1):
     """``s = x + r`` stored in ``dtype``, then ``y = RMSNorm(s)``."""
     s = residual_sum(x, r, dtype)
     return s, rmsnorm(s, gamma, eps, nthreads)
+
+
+# ---------------------------------------------------------------------------
+# Backward passes (backward_oracle.c): analytic derivatives of the forward
+# definitions above for an upstream gradient dy
+# ---------------------------------------------------------------------------
+def _pair(a, b, what):
+    a = _f64(a)
+    b = _f64(b)
+    if a.ndim != 2 or a.shape != b.shape:
+        raise ValueError(f"{what} wants two 2-D arrays of the same shape")
+    return a, b
+
+
+def softmax_backward(y, dy, nthreads=1):
+    """``dx = y * (dy - sum(dy * y))`` per row, ``y`` the softmax output."""
+    y, dy = _pair(y, dy, "softmax_backward")
+    dx = np.empty_like(y)
+    _load().oracle_softmax_backward(_ptr(y), _ptr(dy), _ptr(dx), y.shape[0], y.shape[1],
+                                    _threads(nthreads))
+    return dx
+
+
+def logsoftmax_backward(y, dy, nthreads=1):
+    """``dx = dy - exp(y) * sum(dy)`` per row, ``y`` the log-softmax output."""
+    y, dy = _pair(y, dy, "logsoftmax_backward")
+    dx = np.empty_like(y)
+    _load().oracle_logsoftmax_backward(_ptr(y), _ptr(dy), _ptr(dx), y.shape[0], y.shape[1],
+                                       _threads(nthreads))
+    return dx
+
+
+def layernorm_backward(x, dy, gamma=None, eps=1e-5, nthreads=1):
+    """LayerNorm backward from the input ``x`` (statistics recomputed as the
+    forward forms them).  Returns ``(dx, dgamma, dbeta)``; ``dgamma`` and
+    ``dbeta`` are column sums over all rows."""
+    x, dy = _pair(x, dy, "layernorm_backward")
+    rows, cols = x.shape
+    g = _vec(gamma, cols, 1.0)
+    dx = np.empty_like(x)
+    dg = np.empty(cols, dtype=np.float64)
+    db = np.empty(cols, dtype=np.float64)
+    rc = _load().oracle_layernorm_backward(_ptr(x), _ptr(dy), _ptr(g), _ptr(dx), _ptr(dg),
+                                           _ptr(db), rows, cols, _as_eps(eps), _threads(nthreads))
+    if rc != 0:
+        raise MemoryError("oracle_layernorm_backward could not allocate its row statistics")
+    return dx, dg, db
+
+
+def rmsnorm_backward(x, dy, gamma=None, eps=1e-6, nthreads=1):
+    """RMSNorm backward from the input ``x``.  Returns ``(dx, dgamma)``."""
+    x, dy = _pair(x, dy, "rmsnorm_backward")
+    rows, cols = x.shape
+    g = _vec(gamma, cols, 1.0)
+    dx = np.empty_like(x)
+    dg = np.empty(cols, dtype=np.float64)
+    rc = _load().oracle_rmsnorm_backward(_ptr(x), _ptr(dy), _ptr(g), _ptr(dx), _ptr(dg),
+                                         rows, cols, _as_eps(eps), _threads(nthreads))
+    if rc != 0:
+        raise MemoryError("oracle_rmsnorm_backward could not allocate its row statistics")
+    return dx, dg

@@ -334,7 +334,141 @@ def pin_residual_norm(orc):
     _close(np.sqrt((y * y).mean(axis=1)), np.ones(6))
 
 
+# --------------------------------------------------------------------------
+# backward passes
+# --------------------------------------------------------------------------
+def _fd_grad(f, a, h=1e-5):
+    """Central differences of the scalar function f at every entry of a."""
+    a = np.array(a, dtype=np.float64)
+    g = np.empty_like(a)
+    flat = a.reshape(-1)
+    gf = g.reshape(-1)
+    for k in range(flat.size):
+        old = flat[k]
+        flat[k] = old + h
+        fp = f(a)
+        flat[k] = old - h
+        fm = f(a)
+        flat[k] = old
+        gf[k] = (fp - fm) / (2 * h)
+    return g
+
+
+def pin_backward_finite_difference(orc):
+    """Every backward pass against central differences of the (separately
+    pinned) forward oracle: dx for all four operators, and dgamma / dbeta of
+    the norms, of the loss sum(dy * f(x, gamma, beta))."""
+    rng = np.random.default_rng(31)
+    rows, n = 3, 9
+    x = rng.normal(0.3, 2.0, (rows, n))
+    dy = rng.normal(0.0, 1.0, (rows, n))
+    g = rng.normal(1.0, 0.3, n)
+    b = rng.normal(0.0, 0.3, n)
+    tol = dict(rtol=1e-6, atol=1e-8)
+    y = orc.softmax(x)
+    _close(orc.softmax_backward(y, dy), _fd_grad(lambda a: np.sum(dy * orc.softmax(a)), x), **tol)
+    y = orc.logsoftmax(x)
+    _close(orc.logsoftmax_backward(y, dy),
+           _fd_grad(lambda a: np.sum(dy * orc.logsoftmax(a)), x), **tol)
+    eps = float(np.float32(1e-5))
+    dx, dg, db = orc.layernorm_backward(x, dy, g, eps=eps)
+    _close(dx, _fd_grad(lambda a: np.sum(dy * orc.layernorm(a, g, b, eps=eps)), x), **tol)
+    _close(dg, _fd_grad(lambda a: np.sum(dy * orc.layernorm(x, a, b, eps=eps)), g), **tol)
+    _close(db, _fd_grad(lambda a: np.sum(dy * orc.layernorm(x, g, a, eps=eps)), b), **tol)
+    eps = float(np.float32(1e-6))
+    dx, dg = orc.rmsnorm_backward(x, dy, g, eps=eps)
+    _close(dx, _fd_grad(lambda a: np.sum(dy * orc.rmsnorm(a, g, eps=eps)), x), **tol)
+    _close(dg, _fd_grad(lambda a: np.sum(dy * orc.rmsnorm(x, a, eps=eps)), g), **tol)
+
+
+def pin_backward_invariants(orc):
+    """Properties any correct backward pass has: softmax-family gradients sum
+    to zero over a row; a constant upstream gradient gives no softmax
+    gradient; the log-softmax gradient of one log-probability is e_k - p;
+    the two-element softmax closed form; LayerNorm gradients are orthogonal
+    to 1 and to xhat (eps = 0), vanish for two-element rows (eps = 0) and are
+    unchanged by a shift of x; RMSNorm gradients are orthogonal to x and
+    scale as 1/c when x does (eps = 0); dbeta is the column sum of dy."""
+    rng = np.random.default_rng(32)
+    x = rng.normal(0.0, 2.0, (5, 17))
+    dy = rng.normal(0.0, 1.0, (5, 17))
+    g = rng.normal(1.0, 0.3, 17)
+    p = orc.softmax(x)
+    _close(orc.softmax_backward(p, dy).sum(axis=1), np.zeros(5), atol=1e-14)
+    _close(orc.softmax_backward(p, np.full_like(x, 0.7)), np.zeros_like(x), atol=1e-15)
+    lp = orc.logsoftmax(x)
+    _close(orc.logsoftmax_backward(lp, dy).sum(axis=1), np.zeros(5), atol=1e-13)
+    onehot = np.zeros_like(x)
+    onehot[np.arange(5), [0, 3, 16, 8, 8]] = 1.0
+    _close(orc.logsoftmax_backward(lp, onehot), onehot - p, rtol=1e-13, atol=1e-15)
+    # two elements: y1 = 1 / (1 + exp(x2 - x1)); dx1 = y1 y2 (dy1 - dy2) = -dx2
+    x2 = np.array([[0.5, -1.25]])
+    d2 = np.array([[2.0, -0.5]])
+    s1 = 1.0 / (1.0 + math.exp(-1.75))
+    want = s1 * (1.0 - s1) * 2.5
+    _close(orc.softmax_backward(orc.softmax(x2), d2), [[want, -want]], rtol=1e-14)
+    # LayerNorm, eps = 0
+    dx, dg, db = orc.layernorm_backward(x, dy, g, eps=0.0)
+    mu = x.mean(axis=1, keepdims=True)
+    xhat = (x - mu) / np.sqrt(((x - mu) ** 2).mean(axis=1, keepdims=True))
+    _close(dx.sum(axis=1), np.zeros(5), atol=1e-13)
+    _close((dx * xhat).sum(axis=1), np.zeros(5), atol=1e-13)
+    _close(db, dy.sum(axis=0), rtol=1e-15, atol=1e-15)
+    _close(orc.layernorm_backward(x + 3.5, dy, g, eps=1e-3)[0],
+           orc.layernorm_backward(x, dy, g, eps=1e-3)[0], rtol=1e-9, atol=1e-12)
+    _close(orc.layernorm_backward(2.0 * x, dy, g, eps=0.0)[0], dx / 2.0, rtol=1e-12, atol=1e-14)
+    _close(orc.layernorm_backward(x[:, :2], dy[:, :2], g[:2], eps=0.0)[0], np.zeros((5, 2)),
+           atol=1e-14)
+    # RMSNorm, eps = 0
+    dx, dg = orc.rmsnorm_backward(x, dy, g, eps=0.0)
+    _close((dx * x).sum(axis=1), np.zeros(5), atol=1e-13)
+    _close(orc.rmsnorm_backward(4.0 * x, dy, g, eps=0.0)[0], dx / 4.0, rtol=1e-12, atol=1e-14)
+    _close(orc.rmsnorm_backward(4.0 * x, dy, g, eps=0.0)[1], dg, rtol=1e-12, atol=1e-14)
+    # one-element rows: LayerNorm's output is beta whatever x is
+    _close(orc.layernorm_backward(x[:, :1], dy[:, :1], g[:1], eps=1e-5)[0], np.zeros((5, 1)),
+           atol=0)
+
+
+def pin_backward_torch(orc):
+    """Against PyTorch autograd in float64 (a library, used only here),
+    including dgamma / dbeta summed over many rows."""
+    import torch
+    import torch.nn.functional as F
+    rng = np.random.default_rng(33)
+    x = rng.normal(0.5, 3.0, (40, 130))
+    dy = rng.normal(0.0, 1.0, (40, 130))
+    gam = rng.normal(1.0, 0.2, 130)
+    bet = rng.normal(0.0, 0.2, 130)
+    td = torch.from_numpy(dy)
+
+    def grads(fn, *args):
+        ts = [torch.from_numpy(a.copy()).requires_grad_(True) for a in args]
+        (fn(*ts) * td).sum().backward()
+        return [t.grad.numpy() for t in ts]
+
+    t = torch.from_numpy(x)
+    y = torch.softmax(t, dim=1).numpy()
+    _close(orc.softmax_backward(y, dy), grads(lambda a: torch.softmax(a, dim=1), x)[0],
+           rtol=1e-11, atol=1e-14)
+    y = torch.log_softmax(t, dim=1).numpy()
+    _close(orc.logsoftmax_backward(y, dy), grads(lambda a: torch.log_softmax(a, dim=1), x)[0],
+           rtol=1e-11, atol=1e-13)
+    eps = float(np.float32(1e-5))
+    dx, dg, db = orc.layernorm_backward(x, dy, gam, eps=eps)
+    want = grads(lambda a, g_, b_: F.layer_norm(a, (130,), g_, b_, eps=eps), x, gam, bet)
+    _close(dx, want[0], rtol=1e-10, atol=1e-12)
+    _close(dg, want[1], rtol=1e-10, atol=1e-11)
+    _close(db, want[2], rtol=1e-10, atol=1e-11)
+    if hasattr(F, "rms_norm"):
+        eps = float(np.float32(1e-6))
+        dx, dg = orc.rmsnorm_backward(x, dy, gam, eps=eps)
+        want = grads(lambda a, g_: F.rms_norm(a, (130,), g_, eps=eps), x, gam)
+        _close(dx, want[0], rtol=1e-10, atol=1e-12)
+        _close(dg, want[1], rtol=1e-10, atol=1e-11)
+
+
 ALL_PINS = [pin_hand_cases, pin_softmax_invariants, pin_layernorm_invariants,
             pin_rmsnorm_invariants, pin_brute_force, pin_torch_float64,
             pin_ragged, pin_bucket_rule, pin_pad_scale, pin_moe_group_top2,
-            pin_residual_norm]
+            pin_residual_norm, pin_backward_finite_difference, pin_backward_invariants,
+            pin_backward_torch]

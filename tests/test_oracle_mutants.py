@@ -13,6 +13,7 @@ from tests.oracle_pins import ALL_PINS
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 SRC = os.path.join(ROOT, "oracle", "rowop_oracle.c")
 SRC_PM = os.path.join(ROOT, "oracle", "pad_moe_oracle.c")
+SRC_BW = os.path.join(ROOT, "oracle", "backward_oracle.c")
 WRAPPER = os.path.join(ROOT, "oracle", "rowop_oracle.py")
 
 # (function whose body is edited, text, replacement, what the mistake is)
@@ -55,10 +56,32 @@ MUTANTS = [
      "last member skipped"),
     ("oracle_moe_group_top2", "w[i] + w[j] > best", "w[i] + w[j] >= best + 1.0",
      "comparison off"),
+    ("softmax_bwd_row", "(dy[j] - s)", "(dy[j] + s)", "softmax backward sign"),
+    ("softmax_bwd_row", "s += dy[j] * y[j];", "s += dy[j];", "softmax backward dot without y"),
+    ("logsoftmax_bwd_row", "exp(y[j]) * s", "y[j] * s", "log-softmax backward without exp"),
+    ("layernorm_bwd_row", "- a - xhat * b", "- xhat * b", "LayerNorm backward mean term dropped"),
+    ("layernorm_bwd_row", "rstd * (dy[j]", "(dy[j]", "LayerNorm backward rstd factor dropped"),
+    ("layernorm_bwd_row", "sgx += g * ((x[j] - mu) * rstd);", "sgx += g * (x[j] - mu);",
+     "LayerNorm backward xhat without rstd"),
+    ("layernorm_bwd_row", "dy[j] * gamma[j] - a", "dy[j] - a", "LayerNorm backward gamma dropped"),
+    ("layernorm_stats", "sq / (double)n + eps", "sq / (double)(n - 1) + eps",
+     "LayerNorm backward unbiased variance"),
+    ("oracle_layernorm_backward", "sg += dy[r * cols + j] * xhat;", "sg += dy[r * cols + j];",
+     "dgamma without xhat"),
+    ("oracle_layernorm_backward", "for (int64_t r = 0; r < rows; ++r) {\n            const",
+     "for (int64_t r = 1; r < rows; ++r) {\n            const", "column sums skip row 0"),
+    ("rmsnorm_bwd_row", "- (x[j] * rstd) * b", "- x[j] * b", "RMSNorm backward xhat without rstd"),
+    ("rmsnorm_rstd", "sq / (double)n + eps", "sq + eps", "RMSNorm backward sum of squares"),
+    ("oracle_rmsnorm_backward", "(x[r * cols + j] * rs[r])", "x[r * cols + j]",
+     "RMSNorm dgamma uses x"),
 ]
 
 # functions defined in pad_moe_oracle.c rather than rowop_oracle.c
 PM_FUNCS = {"oracle_pad_scale", "oracle_moe_group_top2"}
+# functions defined in backward_oracle.c
+BW_FUNCS = {"softmax_bwd_row", "logsoftmax_bwd_row", "layernorm_bwd_row", "layernorm_stats",
+            "oracle_layernorm_backward", "rmsnorm_bwd_row", "rmsnorm_rstd",
+            "oracle_rmsnorm_backward"}
 
 
 def _mutate(src: str, func: str, old: str, new: str) -> str:
@@ -71,16 +94,18 @@ def _mutate(src: str, func: str, old: str, new: str) -> str:
     return src[:start] + body.replace(old, new, 1) + src[end:]
 
 
-def _load_mutant(tmp_path, text, text_pm):
+def _load_mutant(tmp_path, text, text_pm, text_bw):
     d = tmp_path / "mut"
     d.mkdir()
     (d / "rowop_oracle.c").write_text(text)
     (d / "pad_moe_oracle.c").write_text(text_pm)
+    (d / "backward_oracle.c").write_text(text_bw)
     spec = importlib.util.spec_from_file_location("oracle_mutant", WRAPPER)
     mod = importlib.util.module_from_spec(spec)
     spec.loader.exec_module(mod)
     mod._SRC = str(d / "rowop_oracle.c")
-    mod._SRCS = [str(d / "rowop_oracle.c"), str(d / "pad_moe_oracle.c")]
+    mod._SRCS = [str(d / "rowop_oracle.c"), str(d / "pad_moe_oracle.c"),
+                 str(d / "backward_oracle.c")]
     mod._BUILD_DIR = str(d / "_build")
     mod._LIB_PATH = str(d / "_build" / "liboracle.so")
     mod._lib = None
@@ -94,11 +119,15 @@ def test_pins_catch_mutant(tmp_path, func, old, new, what):
         src = f.read()
     with open(SRC_PM) as f:
         src_pm = f.read()
+    with open(SRC_BW) as f:
+        src_bw = f.read()
     if func in PM_FUNCS:
         src_pm = _mutate(src_pm, func, old, new)
+    elif func in BW_FUNCS:
+        src_bw = _mutate(src_bw, func, old, new)
     else:
         src = _mutate(src, func, old, new)
-    mod = _load_mutant(tmp_path, src, src_pm)
+    mod = _load_mutant(tmp_path, src, src_pm, src_bw)
     caught = []
     for pin in ALL_PINS:
         try:
