@@ -207,6 +207,8 @@ def per_config(torch, rw, wl, device, peak, steps):
             kw = dict(fft_size=case.meta.get("fft_size"), scale=case.meta.get("scale"))
             y = rw.run(case.op, x, **kw)
             fn = lambda: rw.run(case.op, x, out=y, **kw)  # noqa: E731
+        elif case.dy is not None:
+            fn, y = backward_call(torch, rw, case, x, device)
         else:
             y = torch.empty_like(x)
             fn = lambda: rw.run(case.op, x, gamma=g, beta=b, eps=case.eps, out=y)  # noqa: E731
@@ -221,7 +223,7 @@ def per_config(torch, rw, wl, device, peak, steps):
         gbs = nbytes / (med * 1e-3) / 1e9
         out.append({
             "name": case.name, "op": case.op,
-            "dtype": "bf16" if case.dtype == torch.bfloat16 else "f32",
+            "dtype": {torch.bfloat16: "bf16", torch.float16: "f16"}.get(case.dtype, "f32"),
             "shape": ([case.rows, "ragged", case.max_len] if case.ragged
                       else list(case.x.shape)),
             "bytes": nbytes, "ms_median": round(med, 5), "ms_best": round(best, 5),
@@ -234,6 +236,31 @@ def per_config(torch, rw, wl, device, peak, steps):
         })
         del x, y, g, b
     return out
+
+
+def backward_call(torch, rw, case, x, device):
+    """A backward-pass case on device buffers: returns (fn, dx).  The softmax
+    family's forward output y is formed once, by the library's forward, from
+    the case's forward input; dgamma / dbeta and the workspace are allocated
+    once, outside the timed calls."""
+    dy = case.dy.to(device)
+    a = x
+    if case.op in ("softmax_backward", "logsoftmax_backward"):
+        a = rw.run(case.op[:-len("_backward")], x)
+    dx = torch.empty_like(a)
+    g = case.gamma.to(device) if case.gamma is not None else None
+    cols = a.shape[1]
+    kw = dict(dy=dy, gamma=g, eps=case.eps, out=dx)
+    if case.op == "layernorm_backward":
+        kw.update(dgamma=torch.empty(cols, dtype=a.dtype, device=device),
+                  dbeta=torch.empty(cols, dtype=a.dtype, device=device),
+                  ws=torch.empty(rw.rowop_layernorm_backward_workspace_size(cols),
+                                 dtype=torch.uint8, device=device))
+    elif case.op == "rmsnorm_backward":
+        kw.update(dgamma=torch.empty(cols, dtype=a.dtype, device=device),
+                  ws=torch.empty(rw.rowop_rmsnorm_backward_workspace_size(cols),
+                                 dtype=torch.uint8, device=device))
+    return (lambda: rw.run(case.op, a, **kw)), dx
 
 
 def profile_traffic():
@@ -488,7 +515,10 @@ def run_only(args, local):
     if case.ragged:
         kw.update(offsets=case.offsets.to(device), max_len=case.max_len,
                   ws=rw.ragged_workspace(case.rows, device))
-    ts = time_calls(torch, lambda: rw.run(case.op, x, **kw), args.steps, args.warmup)
+    fn = lambda: rw.run(case.op, x, **kw)  # noqa: E731
+    if case.dy is not None:
+        fn, _ = backward_call(torch, rw, case, x, device)
+    ts = time_calls(torch, fn, args.steps, args.warmup)
     st = rw.check_status()
     if st != 0:
         raise RuntimeError(rw.STATUS.get(st, st))

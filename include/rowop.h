@@ -130,6 +130,69 @@ ROWOP_API int rowop_add_rmsnorm(const void *x, const void *r, void *sum_out, voi
                                 const void *gamma, int64_t rows, int64_t cols, int64_t ld,
                                 rowop_dtype_t dtype, float eps, cudaStream_t stream);
 
+/* ---- backward passes (dense) ----------------------------------------------
+ * The paper states only the forward operators of this family (§2.1); the
+ * backward passes are their derivatives (chain rule) for an upstream
+ * gradient dy of the output:
+ *
+ *   softmax      dx_j = y_j (dy_j - s),        s = sum_j dy_j y_j
+ *   log-softmax  dx_j = dy_j - exp(y_j) s,     s = sum_j dy_j
+ *   LayerNorm    xhat_j = (x_j - mu) rstd, rstd = 1/sqrt(var + eps), g_j = dy_j gamma_j,
+ *                dx_j = rstd (g_j - mean(g) - xhat_j mean(g xhat)),
+ *                dgamma_j = sum over rows of dy_j xhat_j,  dbeta_j = sum over rows of dy_j
+ *   RMSNorm      xhat_j = x_j rstd, rstd = 1/sqrt(mean(x^2) + eps), g_j = dy_j gamma_j,
+ *                dx_j = rstd (g_j - xhat_j mean(g xhat)),
+ *                dgamma_j = sum over rows of dy_j xhat_j
+ *
+ * The softmax family takes the forward OUTPUT y; the norms take the forward
+ * INPUT x and recompute mu / rstd exactly as the forward defines them (no
+ * saved statistics are needed).  y or x, dy and dx share the rows x cols
+ * layout and ld (ld >= cols); dx may be dy itself, or x / y itself (exact
+ * in-place); partial overlap is undefined.  gamma: cols elements or NULL
+ * (ones).  dgamma / dbeta: cols elements of dtype, or NULL when not wanted;
+ * they are sums over ALL rows, and rows == 0 sets them to zero.  Rows that
+ * are 16-byte congruent across y/x, dy and dx (and ld*esize a multiple of 16)
+ * take 16-byte loads and stores, other rows element accesses.
+ *
+ * Norm workspace: when dgamma or dbeta is requested, `ws` (device, 16-byte
+ * aligned, ws_bytes >= rowop_{layernorm,rmsnorm}_backward_workspace_size(cols)
+ * on the current device) receives one float32 partial row per CTA; the
+ * partials are then added in index order, so the result is reproducible bit
+ * for bit on one device (the number of partials follows its SM count).  ws
+ * may be NULL when neither is requested.  The workspace must not be shared
+ * by calls that can run concurrently.
+ *
+ * Rows up to ROWOP_BWD_MAX_COLS_SOFTMAX (softmax family) or
+ * ROWOP_BWD_MAX_COLS_NORM (norms) elements; longer rows return
+ * ROWOP_ERR_TOO_LONG.  Errors: ROWOP_ERR_INVALID_ARG (NULL or misaligned
+ * pointer, cols <= 0 with work to do, ld < cols, eps < 0),
+ * ROWOP_ERR_WORKSPACE, ROWOP_ERR_UNSUPPORTED_DTYPE, ROWOP_ERR_CUDA.        */
+#define ROWOP_BWD_MAX_COLS_SOFTMAX 262144
+#define ROWOP_BWD_MAX_COLS_NORM 262144
+
+ROWOP_API int rowop_softmax_backward(const void *y, const void *dy, void *dx, int64_t rows,
+                                     int64_t cols, int64_t ld, rowop_dtype_t dtype,
+                                     cudaStream_t stream);
+
+ROWOP_API int rowop_logsoftmax_backward(const void *y, const void *dy, void *dx, int64_t rows,
+                                        int64_t cols, int64_t ld, rowop_dtype_t dtype,
+                                        cudaStream_t stream);
+
+ROWOP_API int rowop_layernorm_backward(const void *x, const void *dy, const void *gamma,
+                                       void *dx, void *dgamma, void *dbeta, int64_t rows,
+                                       int64_t cols, int64_t ld, rowop_dtype_t dtype, float eps,
+                                       void *ws, size_t ws_bytes, cudaStream_t stream);
+
+ROWOP_API int rowop_rmsnorm_backward(const void *x, const void *dy, const void *gamma,
+                                     void *dx, void *dgamma, int64_t rows, int64_t cols,
+                                     int64_t ld, rowop_dtype_t dtype, float eps, void *ws,
+                                     size_t ws_bytes, cudaStream_t stream);
+
+/* Workspace bytes for dgamma (and dbeta) of rows of `cols` elements on the
+ * current device; 0 if cols <= 0 or the device cannot be queried. */
+ROWOP_API size_t rowop_layernorm_backward_workspace_size(int64_t cols);
+ROWOP_API size_t rowop_rmsnorm_backward_workspace_size(int64_t cols);
+
 /* ---- ragged rows (int64 CSR offsets into one packed buffer) ---------------
  * offsets : device int64[rows + 1], non-decreasing
  * max_len : an upper bound on every row's length (>= 0); sizes the on-chip

@@ -24,13 +24,14 @@ ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
                      "-Xcompiler", "-fvisibility=hidden", "-I", CSRC,
                      "-I", INCLUDE]
-# (source, object name, extra flags): ops_instance.cu once per operator and
-# element type
+# (source, object name, extra flags): ops_instance.cu (forward) and
+# bwd_instance.cu (backward) once per operator and element type
 _OPS = [("kSoftmax", "softmax"), ("kLogSoftmax", "logsoftmax"), ("kLayerNorm", "layernorm"),
         ("kRmsNorm", "rmsnorm")]
 _TYPES = [("float", "f32"), ("__nv_bfloat16", "bf16"), ("__half", "f16")]
 UNITS = [("rowop_api.cu", "rowop_api.o", []), ("pad_moe.cu", "pad_moe.o", [])] + [
-    ("ops_instance.cu", f"ops_{on}_{tn}.o", [f"-DROWOP_INST_OP={o}", f"-DROWOP_INST_T={t}"])
+    (src, f"{pre}_{on}_{tn}.o", [f"-DROWOP_INST_OP={o}", f"-DROWOP_INST_T={t}"])
+    for src, pre in (("ops_instance.cu", "ops"), ("bwd_instance.cu", "bwd"))
     for o, on in _OPS for t, tn in _TYPES]
 
 

@@ -1,0 +1,183 @@
+// bwd_launch.cuh -- host side of the backward passes: the team shape for the
+// row length, the grid, and the dgamma / dbeta finalize launch.  Included by
+// one translation unit per (operator, type) pair (bwd_instance.cu).
+#pragma once
+
+#include "bwd_row.cuh"
+#include "launch_util.cuh"
+
+namespace rowop {
+
+struct BwdShape {
+  int tpr;  // threads of one CTA per row
+  int nt;   // threads per CTA
+  int cs;   // CTAs per row (cluster size)
+};
+
+// Team shape for rows of `units` chunk slots (16-byte window chunks, or
+// groups of E elements) held CPT per thread: lane groups of a power of two up
+// to a warp, whole warps up to 512 threads in one CTA, else a cluster of a
+// power of two CTAs (up to 16).  CTAs of lane groups or small teams hold
+// several teams: `small_cta` threads (256 for the softmax family; 128 for the
+// norms, whose per-thread shared memory grows with the CTA).  `force_cs`
+// (2..16) splits every row.
+inline bool bwd_shape(int64_t units, int cpt, int force_cs, int small_cta, BwdShape &s) {
+  const int64_t need = std::max<int64_t>(1, ceil_div(units, cpt));
+  const auto warps32 = [](int64_t n) { return static_cast<int>(ceil_div(n, 32) * 32); };
+  if (force_cs == 2 || force_cs == 4 || force_cs == 8 || force_cs == 16) {
+    const int64_t per = ceil_div(need, force_cs);
+    if (per <= kBwdMaxThreads) {
+      s = {warps32(per), warps32(per), force_cs};
+      return true;
+    }
+  }
+  if (need <= 32) {
+    int t = 1;
+    while (t < need) t <<= 1;
+    s = {t, small_cta, 1};
+  } else if (need <= small_cta) {
+    const int t = warps32(need);
+    s = {t, t * (small_cta / t), 1};
+  } else if (need <= kBwdMaxThreads) {
+    const int t = warps32(need);
+    s = {t, t, 1};
+  } else {
+    int cs = 2;
+    while (cs < kMaxCluster && ceil_div(need, cs) > kBwdMaxThreads) cs <<= 1;
+    if (ceil_div(need, cs) > kBwdMaxThreads) return false;
+    const int t = warps32(ceil_div(need, cs));
+    s = {t, t, cs};
+  }
+  return true;
+}
+
+template <typename T>
+cudaError_t launch_bwd_finalize(const float *part, int64_t nparts, int64_t cols, int nacc,
+                                void *dgamma, void *dbeta, cudaStream_t stream) {
+  const dim3 grid(static_cast<unsigned>(ceil_div(cols, 32)), static_cast<unsigned>(nacc), 1);
+  bwd_param_finalize_kernel<T><<<grid, 256, 0, stream>>>(part, nparts, cols, nacc,
+                                                         static_cast<T *>(dgamma),
+                                                         static_cast<T *>(dbeta));
+  return cudaGetLastError();
+}
+
+template <int OP, typename T, int CPT, bool VEC, bool CLUSTER>
+cudaError_t launch_bwd_k(const BwdParams &p, const BwdShape &s, const BwdCall &c,
+                         const DeviceInfo &d) {
+  auto kern = bwd_row_kernel<OP, T, CPT, VEC, CLUSTER>;
+  const void *kp = reinterpret_cast<const void *>(kern);
+  constexpr bool kNorm = (OP == kLayerNorm || OP == kRmsNorm);
+  const int teams_cta = s.nt / s.tpr;
+  // CTAs that hold several teams sum their dgamma / dbeta in shared memory
+  const bool multi = !CLUSTER && (s.tpr < 32 || teams_cta > 1);
+  constexpr int S = CPT * Elem<T>::kPerChunk;
+  const size_t na = static_cast<size_t>(p.nacc);
+  const size_t smem = (kNorm ? static_cast<size_t>(CPT) * s.nt * 16 : 0) +
+                      ((kNorm && p.part) ? na * S * s.nt * sizeof(float) : 0) +
+                      ((kNorm && p.part && multi) ? na * static_cast<size_t>(c.cols) * sizeof(float)
+                                                  : 0);
+  if (smem > static_cast<size_t>(d.max_smem_optin)) return cudaErrorInvalidConfiguration;
+  {
+    static std::mutex mu;
+    static std::map<std::pair<const void *, int>, bool> done;
+    std::lock_guard<std::mutex> lk(mu);
+    const auto key = std::make_pair(kp, d.device);
+    if (!done.count(key)) {
+      cudaFuncAttributes fa;
+      cudaError_t e = cudaFuncGetAttributes(&fa, kp);
+      if (e != cudaSuccess) return e;
+      e = cudaFuncSetAttribute(kp, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               d.max_smem_optin - static_cast<int>(fa.sharedSizeBytes));
+      if (e != cudaSuccess) return e;
+      if (CLUSTER) {
+        e = cudaFuncSetAttribute(kp, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (e != cudaSuccess) return e;
+      }
+      done[key] = true;
+    }
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  cfg.blockDim = dim3(s.nt, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = c.stream;
+  const int64_t part_cap = static_cast<int64_t>(kBwdMaxPartsPerSm) * d.sm_count;
+  int64_t grid, nparts;
+  if (CLUSTER) {
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = s.cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cfg.gridDim = dim3(s.cs * std::max(1, d.sm_count / s.cs), 1, 1);
+    int64_t ncl = std::max(1, cached_occupancy(kp, s.nt, smem, s.cs, &cfg));
+    ncl = std::min<int64_t>(ncl, std::max<int64_t>(1, part_cap / s.cs));
+    nparts = std::max<int64_t>(1, std::min<int64_t>(c.rows, ncl));
+    grid = nparts * s.cs;
+  } else {
+    const int bps = std::max(1, cached_occupancy(kp, s.nt, smem, 1, nullptr));
+    grid = std::max<int64_t>(1, std::min<int64_t>({ceil_div(c.rows, teams_cta),
+                                                   static_cast<int64_t>(bps) * d.sm_count,
+                                                   part_cap}));
+    nparts = grid;
+  }
+  cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
+  cudaError_t e = cudaLaunchKernelEx(&cfg, kern, p);
+  if (e != cudaSuccess) return e;
+  e = cudaGetLastError();
+  if (e != cudaSuccess || !p.part) return e;
+  return launch_bwd_finalize<T>(p.part, nparts, c.cols, p.nacc, c.dgamma, c.dbeta, c.stream);
+}
+
+template <int OP, typename T>
+cudaError_t launch_bwd_t(const BwdCall &c, const DeviceInfo &d) {
+  constexpr int SZ = sizeof(T);
+  constexpr int E = 16 / SZ;
+  constexpr bool kNorm = (OP == kLayerNorm || OP == kRmsNorm);
+  constexpr int CPT = kBwdSlots / E;
+  const int small_cta = kNorm ? 128 : 256;
+  const int nacc = OP == kLayerNorm ? 2 : 1;
+  const bool want_params = kNorm && (c.dgamma || c.dbeta);
+  if (c.rows == 0) {  // the parameter gradients of no rows are zero
+    if (!want_params) return cudaSuccess;
+    return launch_bwd_finalize<T>(nullptr, 0, c.cols, nacc, c.dgamma, c.dbeta, c.stream);
+  }
+  bool vec = ((c.ld * SZ) % 16 == 0) && congruent16(c.a, c.dy) && congruent16(c.a, c.dx);
+  int h = vec ? static_cast<int>((reinterpret_cast<uintptr_t>(c.a) & 15u) / SZ) : 0;
+  int64_t units = vec ? ceil_div(h + c.cols, E) : ceil_div(c.cols, E);
+  const int force_cs = read_knobs().bwd_cluster;
+  BwdShape s;
+  if (!bwd_shape(units, CPT, force_cs, small_cta, s)) {
+    // a row of the longest length that starts mid-chunk needs one window
+    // chunk more than the largest cluster holds: take the element path
+    vec = false;
+    h = 0;
+    units = ceil_div(c.cols, E);
+    if (!bwd_shape(units, CPT, force_cs, small_cta, s)) return cudaErrorInvalidValue;
+  }
+  BwdParams p = {};
+  p.a = c.a;
+  p.dy = c.dy;
+  p.dx = c.dx;
+  p.gamma = c.gamma;
+  p.part = want_params ? static_cast<float *>(c.ws) : nullptr;
+  p.rows = c.rows;
+  p.cols = c.cols;
+  p.ld = c.ld;
+  p.eps = c.eps;
+  p.tpr = s.tpr;
+  p.h = h;
+  p.nc = static_cast<int>(units);
+  p.nacc = nacc;
+  p.timeout_ns = kWaitLimitNs;
+  p.status = d.status;
+  if (s.cs > 1) {
+    if (vec) return launch_bwd_k<OP, T, CPT, true, true>(p, s, c, d);
+    return launch_bwd_k<OP, T, CPT, false, true>(p, s, c, d);
+  }
+  if (vec) return launch_bwd_k<OP, T, CPT, true, false>(p, s, c, d);
+  return launch_bwd_k<OP, T, CPT, false, false>(p, s, c, d);
+}
+
+}  // namespace rowop

@@ -63,6 +63,36 @@ struct MoeCall {
   cudaStream_t stream;
 };
 
+// Backward pass of one operator over dense rows: `a` is the forward output y
+// (softmax family) or the forward input x (norms); dgamma / dbeta (norms,
+// either may be NULL) are column sums over all rows, formed from per-CTA
+// partials in `ws`.
+struct BwdCall {
+  int dtype;
+  const void *a;
+  const void *dy;
+  void *dx;
+  const void *gamma;
+  void *dgamma;
+  void *dbeta;
+  int64_t rows, cols, ld;
+  float eps;
+  void *ws;
+  cudaStream_t stream;
+};
+
+// Partial rows of dgamma / dbeta: the backward launch never runs more than
+// this many CTAs per SM (one partial row each).
+constexpr int kBwdMaxPartsPerSm = 8;
+// bytes of the partials workspace: nacc = 2 (LayerNorm) or 1 (RMSNorm)
+inline size_t bwd_ws_bytes(int nacc, int64_t cols, int sm_count) {
+  return static_cast<size_t>(kBwdMaxPartsPerSm) * static_cast<size_t>(sm_count) *
+         static_cast<size_t>(nacc) * static_cast<size_t>(cols) * sizeof(float);
+}
+// Longest backward row: 16 CTAs of 512 threads holding 32 elements each.
+constexpr int64_t kBwdMaxColsSoftmax = 16 * 512 * 32;
+constexpr int64_t kBwdMaxColsNorm = 16 * 512 * 32;
+
 cudaError_t launch_pad_scale(const PadCall &c, const DeviceInfo &d);
 cudaError_t launch_moe_group_top2(const MoeCall &c, const DeviceInfo &d);
 
@@ -111,7 +141,8 @@ inline int64_t max_row_len_elems(int esize) {
 }
 
 // Test-and-tuning knobs read from the environment (none changes results but
-// ROWOP_SOFTMAX_ONLINE, which selects another way to round):
+// ROWOP_SOFTMAX_ONLINE and ROWOP_BWD_CLUSTER, which select another way to
+// round):
 //   ROWOP_FORCE_BUCKET  0/1/2 -> dense rows use that design when it can hold
 //                       the row (SMALL only for rows of <= 288 chunks)
 //   ROWOP_CLUSTER       cluster size for split rows (1, 2, 4, 8, 16)
@@ -121,6 +152,8 @@ inline int64_t max_row_len_elems(int esize) {
 //   ROWOP_SOFTMAX_ONLINE 1 -> dense SMALL softmax / log-softmax use the online
 //                       one-pass statistics instead of the two-pass ones (a
 //                       comparison variant: its results differ by rounding)
+//   ROWOP_BWD_CLUSTER   backward passes: split every row over a cluster of
+//                       this many CTAs (2, 4, 8, 16); changes rounding order
 struct Knobs {
   int force_bucket = -1;
   int cluster = 0;
@@ -128,6 +161,7 @@ struct Knobs {
   int ctas_per_sm = 0;
   int group_warps = 0;
   int softmax_online = 0;
+  int bwd_cluster = 0;
 };
 Knobs read_knobs();
 

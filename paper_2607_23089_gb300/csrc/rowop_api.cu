@@ -20,6 +20,18 @@ cudaError_t launch_dense_t(const DenseCall &c, const DeviceInfo &d);
 template <int OP, typename T>
 cudaError_t launch_ragged_t(const RaggedCall &c, const DeviceInfo &d);
 
+// The backward passes, instantiated one (operator, type) pair per object file
+// from bwd_instance.cu.
+template <int OP, typename T>
+cudaError_t launch_bwd_t(const BwdCall &c, const DeviceInfo &d);
+
+template <int OP>
+static cudaError_t launch_bwd(const BwdCall &c, const DeviceInfo &d) {
+  if (c.dtype == ROWOP_F32) return launch_bwd_t<OP, float>(c, d);
+  if (c.dtype == ROWOP_F16) return launch_bwd_t<OP, __half>(c, d);
+  return launch_bwd_t<OP, __nv_bfloat16>(c, d);
+}
+
 template <int OP>
 static cudaError_t launch_dense(const DenseCall &c, const DeviceInfo &d) {
   if (c.dtype == ROWOP_F32) return launch_dense_t<OP, float>(c, d);
@@ -51,6 +63,7 @@ Knobs read_knobs() {
   k.ctas_per_sm = env_int("ROWOP_CTAS_PER_SM", 0);
   k.group_warps = env_int("ROWOP_GROUP_WARPS", 0);
   k.softmax_online = env_int("ROWOP_SOFTMAX_ONLINE", 0);
+  k.bwd_cluster = env_int("ROWOP_BWD_CLUSTER", 0);
   return k;
 }
 
@@ -250,6 +263,65 @@ static int run_ragged(int op, const void *in, void *out, const void *gamma, cons
   }
 }
 
+// Backward passes.  a = y (softmax family) or x (norms).
+static int run_bwd(int op, const void *a, const void *dy, void *dx, const void *gamma,
+                   void *dgamma, void *dbeta, int64_t rows, int64_t cols, int64_t ld,
+                   rowop_dtype_t dtype, float eps, void *ws, size_t ws_bytes,
+                   cudaStream_t stream) {
+  const int es = esize_of(dtype);
+  const bool norm = (op == kLayerNorm || op == kRmsNorm);
+  if (es == 0) return ROWOP_ERR_UNSUPPORTED_DTYPE;
+  if (rows < 0) return ROWOP_ERR_INVALID_ARG;
+  if (norm && !eps_ok(eps)) return ROWOP_ERR_INVALID_ARG;
+  const bool want = norm && (dgamma || dbeta);
+  if (rows == 0 && !want) return ROWOP_OK;
+  if (cols <= 0) return ROWOP_ERR_INVALID_ARG;
+  if ((gamma && !elem_aligned(gamma, es)) || (dgamma && !elem_aligned(dgamma, es)) ||
+      (dbeta && !elem_aligned(dbeta, es)))
+    return ROWOP_ERR_INVALID_ARG;
+  if (rows > 0) {
+    if (ld < cols || !a || !dy || !dx) return ROWOP_ERR_INVALID_ARG;
+    if (!elem_aligned(a, es) || !elem_aligned(dy, es) || !elem_aligned(dx, es))
+      return ROWOP_ERR_INVALID_ARG;
+    if (ld > INT64_MAX / es / rows) return ROWOP_ERR_INVALID_ARG;
+  }
+  if (cols > (norm ? kBwdMaxColsNorm : kBwdMaxColsSoftmax)) return ROWOP_ERR_TOO_LONG;
+  DeviceInfo d;
+  const int st = device_info(&d);
+  if (st != ROWOP_OK) return st;
+  if (want && rows > 0 &&
+      (!ws || (reinterpret_cast<uintptr_t>(ws) & 15u) != 0 ||
+       ws_bytes < bwd_ws_bytes(op == kLayerNorm ? 2 : 1, cols, d.sm_count)))
+    return ROWOP_ERR_WORKSPACE;
+  BwdCall c;
+  c.dtype = dtype;
+  c.a = a;
+  c.dy = dy;
+  c.dx = dx;
+  c.gamma = gamma;
+  c.dgamma = dgamma;
+  c.dbeta = dbeta;
+  c.rows = rows;
+  c.cols = cols;
+  c.ld = ld;
+  c.eps = eps;
+  c.ws = ws;
+  c.stream = stream;
+  switch (op) {
+    case kSoftmax: return from_cuda(launch_bwd<kSoftmax>(c, d));
+    case kLogSoftmax: return from_cuda(launch_bwd<kLogSoftmax>(c, d));
+    case kLayerNorm: return from_cuda(launch_bwd<kLayerNorm>(c, d));
+    default: return from_cuda(launch_bwd<kRmsNorm>(c, d));
+  }
+}
+
+static size_t bwd_workspace_size(int nacc, int64_t cols) {
+  if (cols <= 0) return 0;
+  DeviceInfo d;
+  if (device_info(&d) != ROWOP_OK) return 0;
+  return bwd_ws_bytes(nacc, cols, d.sm_count);
+}
+
 // Waits on a barrier phase that only half of its expected arrivals reach, so
 // the bounded wait must run out; records the timeout and returns.
 __global__ void debug_wait_timeout_kernel(uint64_t limit_ns, unsigned int *status) {
@@ -309,6 +381,39 @@ int rowop_add_rmsnorm(const void *x, const void *r, void *sum_out, void *y, cons
   return run_dense(kRmsNorm, x, y, gamma, nullptr, rows, cols, ld, dtype, eps, stream, r,
                    sum_out);
 }
+
+int rowop_softmax_backward(const void *y, const void *dy, void *dx, int64_t rows, int64_t cols,
+                           int64_t ld, rowop_dtype_t dtype, cudaStream_t stream) {
+  return run_bwd(kSoftmax, y, dy, dx, nullptr, nullptr, nullptr, rows, cols, ld, dtype, 0.f,
+                 nullptr, 0, stream);
+}
+
+int rowop_logsoftmax_backward(const void *y, const void *dy, void *dx, int64_t rows,
+                              int64_t cols, int64_t ld, rowop_dtype_t dtype,
+                              cudaStream_t stream) {
+  return run_bwd(kLogSoftmax, y, dy, dx, nullptr, nullptr, nullptr, rows, cols, ld, dtype, 0.f,
+                 nullptr, 0, stream);
+}
+
+int rowop_layernorm_backward(const void *x, const void *dy, const void *gamma, void *dx,
+                             void *dgamma, void *dbeta, int64_t rows, int64_t cols, int64_t ld,
+                             rowop_dtype_t dtype, float eps, void *ws, size_t ws_bytes,
+                             cudaStream_t stream) {
+  return run_bwd(kLayerNorm, x, dy, dx, gamma, dgamma, dbeta, rows, cols, ld, dtype, eps, ws,
+                 ws_bytes, stream);
+}
+
+int rowop_rmsnorm_backward(const void *x, const void *dy, const void *gamma, void *dx,
+                           void *dgamma, int64_t rows, int64_t cols, int64_t ld,
+                           rowop_dtype_t dtype, float eps, void *ws, size_t ws_bytes,
+                           cudaStream_t stream) {
+  return run_bwd(kRmsNorm, x, dy, dx, gamma, dgamma, nullptr, rows, cols, ld, dtype, eps, ws,
+                 ws_bytes, stream);
+}
+
+size_t rowop_layernorm_backward_workspace_size(int64_t cols) { return bwd_workspace_size(2, cols); }
+
+size_t rowop_rmsnorm_backward_workspace_size(int64_t cols) { return bwd_workspace_size(1, cols); }
 
 size_t rowop_ragged_workspace_size(int64_t rows) {
   return rows <= 0 ? 256 : ragged_ws_bytes(rows);

@@ -60,6 +60,13 @@ SIGNATURES = {
     "rowop_layernorm_ragged_static": ([_P, _P, _P, _P, _P, _I64, _I64, _I, _F, _P], _I),
     "rowop_add_layernorm": ([_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _F, _P], _I),
     "rowop_add_rmsnorm": ([_P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _F, _P], _I),
+    "rowop_softmax_backward": ([_P, _P, _P, _I64, _I64, _I64, _I, _P], _I),
+    "rowop_logsoftmax_backward": ([_P, _P, _P, _I64, _I64, _I64, _I, _P], _I),
+    "rowop_layernorm_backward": ([_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _F, _P, _SZ,
+                                  _P], _I),
+    "rowop_rmsnorm_backward": ([_P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _F, _P, _SZ, _P], _I),
+    "rowop_layernorm_backward_workspace_size": ([_I64], _SZ),
+    "rowop_rmsnorm_backward_workspace_size": ([_I64], _SZ),
     "rowop_pad_scale": ([_P, _P, _I64, _I64, _I64, _I64, _I64, _F, _I, _P], _I),
     "rowop_moe_group_top2": ([_P, _P, _I64, _I64, _I64, _I, _P], _I),
     "rowop_select_bucket": ([_I64, _I], _I),
@@ -331,11 +338,90 @@ def moe_group_top2(scores, out=None, stream=None):
     return out
 
 
+def softmax_backward(y, dy, dx=None, stream=None):
+    """dx of softmax from its output y and the upstream gradient dy
+    (``rowop_softmax_backward``)."""
+    _check_cuda(y, dy, dx)
+    rows, cols, ld = _dense_layout(y)
+    dx = _out_like(y, dx)
+    _ok(rowop_softmax_backward(y.data_ptr(), dy.data_ptr(), dx.data_ptr(), rows, cols,  # noqa: F821
+                               ld, dtype_code(y.dtype), _stream(stream)),
+        "rowop_softmax_backward")
+    return dx
+
+
+def logsoftmax_backward(y, dy, dx=None, stream=None):
+    """dx of log-softmax from its output y and dy (``rowop_logsoftmax_backward``)."""
+    _check_cuda(y, dy, dx)
+    rows, cols, ld = _dense_layout(y)
+    dx = _out_like(y, dx)
+    _ok(rowop_logsoftmax_backward(y.data_ptr(), dy.data_ptr(), dx.data_ptr(), rows,  # noqa: F821
+                                  cols, ld, dtype_code(y.dtype), _stream(stream)),
+        "rowop_logsoftmax_backward")
+    return dx
+
+
+def _bwd_params(x, want, given, ws, size_fn):
+    torch = _torch()
+    cols = x.shape[1]
+    outs = [g if g is not None else (torch.empty(cols, dtype=x.dtype, device=x.device)
+                                     if w else None) for w, g in zip(want, given)]
+    if any(o is not None for o in outs) and ws is None:
+        ws = torch.empty(int(size_fn(cols)), dtype=torch.uint8, device=x.device)
+    return outs, ws
+
+
+def layernorm_backward(x, dy, gamma=None, eps=1e-5, want_dgamma=True, want_dbeta=True,
+                       dx=None, dgamma=None, dbeta=None, ws=None, stream=None):
+    """LayerNorm backward from the forward input x (``rowop_layernorm_backward``):
+    returns ``(dx, dgamma, dbeta)``, the last two None when not wanted (given
+    output tensors are used as they are)."""
+    _check_cuda(x, dy, gamma, dx, dgamma, dbeta, ws)
+    rows, cols, ld = _dense_layout(x)
+    dx = _out_like(x, dx)
+    (dg, db), ws = _bwd_params(x, (want_dgamma, want_dbeta), (dgamma, dbeta), ws,
+                               rowop_layernorm_backward_workspace_size)  # noqa: F821
+    _ok(rowop_layernorm_backward(x.data_ptr(), dy.data_ptr(), _ptr(gamma), dx.data_ptr(),  # noqa: F821
+                                 _ptr(dg), _ptr(db), rows, cols, ld, dtype_code(x.dtype),
+                                 float(eps), _ptr(ws), 0 if ws is None else ws.numel(),
+                                 _stream(stream)), "rowop_layernorm_backward")
+    return dx, dg, db
+
+
+def rmsnorm_backward(x, dy, gamma=None, eps=1e-6, want_dgamma=True, dx=None, dgamma=None,
+                     ws=None, stream=None):
+    """RMSNorm backward from the forward input x (``rowop_rmsnorm_backward``):
+    returns ``(dx, dgamma)``, dgamma None when not wanted."""
+    _check_cuda(x, dy, gamma, dx, dgamma, ws)
+    rows, cols, ld = _dense_layout(x)
+    dx = _out_like(x, dx)
+    (dg,), ws = _bwd_params(x, (want_dgamma,), (dgamma,), ws,
+                            rowop_rmsnorm_backward_workspace_size)  # noqa: F821
+    _ok(rowop_rmsnorm_backward(x.data_ptr(), dy.data_ptr(), _ptr(gamma), dx.data_ptr(),  # noqa: F821
+                               _ptr(dg), rows, cols, ld, dtype_code(x.dtype), float(eps),
+                               _ptr(ws), 0 if ws is None else ws.numel(), _stream(stream)),
+        "rowop_rmsnorm_backward")
+    return dx, dg
+
+
 def run(op: str, x, *, offsets=None, max_len=None, gamma=None, beta=None,
         eps=None, out=None, ws=None, stream=None, fft_size=None, scale=None, resid=None,
-        sum_out=None):
+        sum_out=None, dy=None, dgamma=None, dbeta=None):
     """One call of ``op`` on dense or ragged input (ragged when offsets is
-    given); returns the output tensor."""
+    given); returns the output tensor (dx for the backward passes, whose x is
+    the forward output for the softmax family and the forward input for the
+    norms)."""
+    if op == "softmax_backward":
+        return softmax_backward(x, dy, out, stream)
+    if op == "logsoftmax_backward":
+        return logsoftmax_backward(x, dy, out, stream)
+    if op == "layernorm_backward":
+        return layernorm_backward(x, dy, gamma, 1e-5 if eps is None else eps,
+                                  want_dgamma=True, want_dbeta=True, dx=out, dgamma=dgamma,
+                                  dbeta=dbeta, ws=ws, stream=stream)[0]
+    if op == "rmsnorm_backward":
+        return rmsnorm_backward(x, dy, gamma, 1e-6 if eps is None else eps, want_dgamma=True,
+                                dx=out, dgamma=dgamma, ws=ws, stream=stream)[0]
     if op == "pad_scale":
         return pad_scale(x, fft_size, scale, out, stream)
     if op == "add_layernorm":

@@ -30,7 +30,7 @@ from typing import Optional
 
 import torch
 
-ESIZE = {torch.float32: 4, torch.bfloat16: 2}
+ESIZE = {torch.float32: 4, torch.bfloat16: 2, torch.float16: 2}
 
 
 @dataclass
@@ -47,6 +47,7 @@ class Case:
     max_len: int = 0
     meta: dict = field(default_factory=dict)
     resid: Optional[torch.Tensor] = None     # fused residual add: the residual r
+    dy: Optional[torch.Tensor] = None        # backward passes: the upstream gradient
 
     @property
     def ragged(self) -> bool:
@@ -64,6 +65,16 @@ class Case:
         """Bytes the operator must move: read x once, write y once, read
         gamma/beta once, read the offsets once."""
         es = ESIZE[self.dtype]
+        if self.op.endswith("_backward"):
+            # read the forward input (norms) or output (softmax family) and dy,
+            # write dx; norms also read gamma and write dgamma (and dbeta)
+            b = 3 * self.elements * es
+            ncol = self.x.shape[1]
+            if self.op == "layernorm_backward":
+                b += 3 * ncol * es
+            elif self.op == "rmsnorm_backward":
+                b += 2 * ncol * es
+            return b
         if self.op == "pad_scale":  # read rows x seqlen, write rows x fft_size
             return self.x.numel() * es + self.x.shape[0] * self.meta["fft_size"] * es
         if self.op == "moe_group_top2":  # read the scores, write one float per group
@@ -198,6 +209,32 @@ def moe_group(tokens: int = 131072, experts: int = 256, seed: int = 6,
     return Case("moe_group_top2", "moe_group_top2", s.to(dtype), dtype)
 
 
+def norm_backward(op: str, rows: int = 8192, cols: int = 4096, seed: int = 8) -> Case:
+    """Backward of a workload-3 norm: bf16 x drawn as in workload 3, upstream
+    gradient dy = N(0,1), gamma as there; the gradients are dx, dgamma (and
+    dbeta for LayerNorm).  Not one of the five workloads."""
+    g = _gen(seed)
+    x = torch.randn(rows, cols, generator=g)
+    scale = 0.1 + 9.9 * torch.rand(rows, 1, generator=g)
+    x = (x * scale).to(torch.bfloat16)
+    dy = torch.randn(rows, cols, generator=g).to(torch.bfloat16)
+    gamma, _ = _affine(g, cols, torch.bfloat16)
+    return Case(f"medium_norm_backward_{op}", f"{op}_backward", x, torch.bfloat16, gamma=gamma,
+                eps=1e-5 if op == "layernorm" else 1e-6, dy=dy)
+
+
+def softmax_backward(op: str = "softmax", rows: int = 32768, cols: int = 1024,
+                     seed: int = 9) -> Case:
+    """Backward of softmax / log-softmax over fp32 rows of 1024 (attention-row
+    length): x = 4*N(0,1) is the FORWARD input -- the backward takes the
+    forward output y = op(x), which the caller forms -- and dy = N(0,1).  Not
+    one of the five workloads."""
+    g = _gen(seed)
+    x = 4.0 * torch.randn(rows, cols, generator=g)
+    dy = torch.randn(rows, cols, generator=g)
+    return Case(f"{op}_backward_{cols}", f"{op}_backward", x, torch.float32, dy=dy)
+
+
 def all_cases(scale_down: int = 1):
     """The five workloads as a flat list of cases.  ``scale_down`` > 1 divides
     every row count (not the row lengths) for quicker runs."""
@@ -214,11 +251,20 @@ def all_cases(scale_down: int = 1):
         out.append(medium_add_norm(op, rows=max(1, 8192 // s)))
     out.append(hyena_pad(rows=max(1, 16384 // s)))
     out.append(moe_group(tokens=max(1, 131072 // s)))
+    for op in ("layernorm", "rmsnorm"):
+        out.append(norm_backward(op, rows=max(1, 8192 // s)))
+    for op in ("softmax", "logsoftmax"):
+        out.append(softmax_backward(op, rows=max(1, 32768 // s)))
     return out
 
 
 def by_name(name: str) -> Case:
     """Builds one workload case from its name (as in all_cases())."""
+    if name.startswith("medium_norm_backward_"):
+        return norm_backward(name[len("medium_norm_backward_"):])
+    if name.startswith(("softmax_backward_", "logsoftmax_backward_")):
+        op, _, cols = name.split("_")
+        return softmax_backward(op, cols=int(cols))
     if name == "softmax_1k":
         return softmax_1k()
     if name.startswith("short_rows_"):

@@ -143,3 +143,41 @@ def test_pad_and_moe_validation(lib):
     assert lib.rowop_moe_group_top2(16, 16, 4, 64, 32, F32, None) == lib.ROWOP_ERR_INVALID_ARG
     assert lib.rowop_moe_group_top2(None, 16, 4, 64, 64, F32, None) == lib.ROWOP_ERR_INVALID_ARG
     assert lib.rowop_moe_group_top2(16, 18, 4, 64, 64, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+
+
+def test_backward_validation(lib):
+    """Backward entry points: bad arguments are refused before the device is
+    touched (the workspace size needs the device, so it is not checked
+    here)."""
+    F32, BF16 = lib.ROWOP_F32, lib.ROWOP_BF16
+    sb = lib.rowop_softmax_backward
+    assert sb(FAKE, FAKE, FAKE, 4, 8, 8, 7, None) == lib.ROWOP_ERR_UNSUPPORTED_DTYPE
+    assert sb(FAKE, FAKE, FAKE, -1, 8, 8, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert sb(None, None, None, 0, 8, 8, F32, None) == lib.ROWOP_OK
+    assert sb(FAKE, FAKE, FAKE, 4, 0, 8, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert sb(FAKE, FAKE, FAKE, 4, 8, 7, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert sb(FAKE, None, FAKE, 4, 8, 8, F32, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert sb(FAKE, FAKE, FAKE + 1, 4, 8, 8, BF16, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert sb(FAKE, FAKE, FAKE, 1, 262145, 262145, F32, None) == lib.ROWOP_ERR_TOO_LONG
+    ls = lib.rowop_logsoftmax_backward
+    assert ls(FAKE, FAKE, FAKE, 2, 8, 8, F32 + 9, None) == lib.ROWOP_ERR_UNSUPPORTED_DTYPE
+    ln = lib.rowop_layernorm_backward
+    assert ln(FAKE, FAKE, None, FAKE, None, None, 4, 8, 8, F32, -1.0, None, 0,
+              None) == lib.ROWOP_ERR_INVALID_ARG
+    assert ln(FAKE, FAKE, FAKE + 2, FAKE, None, None, 4, 8, 8, F32, 1e-5, None, 0,
+              None) == lib.ROWOP_ERR_INVALID_ARG
+    assert ln(FAKE, FAKE, None, FAKE, FAKE + 1, None, 4, 8, 8, BF16, 1e-5, None, 0,
+              None) == lib.ROWOP_ERR_INVALID_ARG
+    assert ln(None, None, None, None, None, None, 0, 0, 0, F32, 1e-5, None, 0,
+              None) == lib.ROWOP_OK  # no rows, no parameter gradients: a no-op
+    assert ln(None, None, None, None, FAKE, None, 0, 0, 0, F32, 1e-5, None, 0,
+              None) == lib.ROWOP_ERR_INVALID_ARG  # zeros of dgamma need cols
+    assert ln(FAKE, FAKE, None, FAKE, None, None, 1, 262145, 262145, F32, 1e-5, None, 0,
+              None) == lib.ROWOP_ERR_TOO_LONG
+    rms = lib.rowop_rmsnorm_backward
+    assert rms(FAKE, FAKE, None, FAKE, None, 4, 8, 8, F32, float("nan"), None, 0,
+               None) == lib.ROWOP_ERR_INVALID_ARG
+    assert rms(FAKE, FAKE, None, None, None, 4, 8, 8, F32, 1e-6, None, 0,
+               None) == lib.ROWOP_ERR_INVALID_ARG
+    assert lib.rowop_layernorm_backward_workspace_size(0) == 0
+    assert lib.rowop_rmsnorm_backward_workspace_size(-5) == 0
