@@ -220,10 +220,11 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
     }
   };
 
+  const bool accum = kNorm && p.part != nullptr;
   uint4 *gsm = reinterpret_cast<uint4 *>(bwd_dyn);
   float4 *acc = reinterpret_cast<float4 *>(bwd_dyn + (kNorm ? CPT * NT * 16 : 0));
-  float *red = reinterpret_cast<float *>(bwd_dyn + (kNorm ? CPT * NT * 16 + NA * S * NT * 4 : 0));
-  const bool accum = kNorm && p.part != nullptr;
+  float *red = reinterpret_cast<float *>(bwd_dyn + (kNorm ? CPT * NT * 16 : 0) +
+                                         (accum ? NA * S * NT * 4 : 0));
   if constexpr (kNorm) {
     // gamma at this thread's columns, once for all rows; the sums start at 0
     const T *gamma = static_cast<const T *>(p.gamma);
@@ -291,68 +292,75 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
       }
     }
 
-    // ---- row sums (masked elements load as zero and add nothing) ----
+    // ---- row sums, in packed pairs (masked elements load as zero and add
+    // nothing, but for LayerNorm's deviations, which are masked) ----
+    constexpr int NP = E / 2;
     float c0 = 0.f, c1 = 0.f, c2 = 0.f, mu = 0.f;
     bool ok = true;
     if constexpr (OP == kSoftmax || OP == kLogSoftmax) {
-      float v[1] = {0.f};
+      f2 s2 = f2_bcast(0.f);
 #pragma unroll
       for (int k = 0; k < CPT; ++k) {
-        float x[E], d[E];
-        unpack<T>(av[k], x);
-        unpack<T>(dv[k], d);
+        f2 x[NP], d[NP];
+        chunk_to_pairs<T>(av[k], x);
+        chunk_to_pairs<T>(dv[k], d);
 #pragma unroll
-        for (int e = 0; e < E; ++e)
-          v[0] = OP == kSoftmax ? __fmaf_rn(d[e], x[e], v[0]) : __fadd_rn(v[0], d[e]);
+        for (int i = 0; i < NP; ++i) s2 = OP == kSoftmax ? f2_fma(d[i], x[i], s2) : f2_add(s2, d[i]);
       }
+      float v[1] = {f2_total(s2)};
       ok = bwd_team_sum<1, CLUSTER>(v, sh, tm, p.timeout_ns, p.status);
       c0 = v[0];  // sum dy y, or sum dy
     } else if constexpr (OP == kRmsNorm) {
-      float v[2] = {0.f, 0.f};
+      f2 sxx = f2_bcast(0.f), sgx = f2_bcast(0.f);
 #pragma unroll
       for (int k = 0; k < CPT; ++k) {
-        float x[E], d[E], g[E];
-        unpack<T>(av[k], x);
-        unpack<T>(dv[k], d);
-        unpack<T>(gsm[k * NT + tid], g);
+        f2 x[NP], d[NP], g[NP];
+        chunk_to_pairs<T>(av[k], x);
+        chunk_to_pairs<T>(dv[k], d);
+        chunk_to_pairs<T>(gsm[k * NT + tid], g);
 #pragma unroll
-        for (int e = 0; e < E; ++e) {
-          v[0] = __fmaf_rn(x[e], x[e], v[0]);
-          v[1] = __fmaf_rn(__fmul_rn(d[e], g[e]), x[e], v[1]);
+        for (int i = 0; i < NP; ++i) {
+          sxx = f2_fma(x[i], x[i], sxx);
+          sgx = f2_fma(f2_mul(d[i], g[i]), x[i], sgx);
         }
       }
+      float v[2] = {f2_total(sxx), f2_total(sgx)};
       ok = bwd_team_sum<2, CLUSTER>(v, sh, tm, p.timeout_ns, p.status);
       c0 = rsqrtf(__fmaf_rn(v[0], inv_n, p.eps));      // rstd
       c1 = __fmul_rn(__fmul_rn(v[1], c0), inv_n);      // mean(g xhat)
     } else {
       // LayerNorm: the mean first, then the sums about it
-      float v1[1] = {0.f};
+      f2 sx = f2_bcast(0.f);
 #pragma unroll
       for (int k = 0; k < CPT; ++k) {
-        float x[E];
-        unpack<T>(av[k], x);
+        f2 x[NP];
+        chunk_to_pairs<T>(av[k], x);
 #pragma unroll
-        for (int e = 0; e < E; ++e) v1[0] = __fadd_rn(v1[0], x[e]);
+        for (int i = 0; i < NP; ++i) sx = f2_add(sx, x[i]);
       }
+      float v1[1] = {f2_total(sx)};
       ok = bwd_team_sum<1, CLUSTER>(v1, sh, tm, p.timeout_ns, p.status);
       mu = __fmul_rn(v1[0], inv_n);
-      float v[3] = {0.f, 0.f, 0.f};
+      const f2 nmu = f2_bcast(-mu);
+      f2 sdd = f2_bcast(0.f), sg = f2_bcast(0.f), sgd = f2_bcast(0.f);
 #pragma unroll
       for (int k = 0; k < CPT; ++k) {
-        float x[E], d[E], g[E];
-        unpack<T>(av[k], x);
-        unpack<T>(dv[k], d);
-        unpack<T>(gsm[k * NT + tid], g);
+        f2 x[NP], d[NP], g[NP];
+        chunk_to_pairs<T>(av[k], x);
+        chunk_to_pairs<T>(dv[k], d);
+        chunk_to_pairs<T>(gsm[k * NT + tid], g);
+        const bool full = msk[k] == (1u << E) - 1u;
 #pragma unroll
-        for (int e = 0; e < E; ++e) {
-          if (!((msk[k] >> e) & 1u)) continue;
-          const float dev = __fsub_rn(x[e], mu);
-          const float gg = __fmul_rn(d[e], g[e]);
-          v[0] = __fmaf_rn(dev, dev, v[0]);
-          v[1] = __fadd_rn(v[1], gg);
-          v[2] = __fmaf_rn(gg, dev, v[2]);
+        for (int i = 0; i < NP; ++i) {
+          f2 dev = f2_add(x[i], nmu);
+          if (!full) dev = f2_select(dev, (msk[k] >> (2 * i)) & 1u, (msk[k] >> (2 * i + 1)) & 1u, 0.f);
+          const f2 gg = f2_mul(d[i], g[i]);
+          sdd = f2_fma(dev, dev, sdd);
+          sg = f2_add(sg, gg);
+          sgd = f2_fma(gg, dev, sgd);
         }
       }
+      float v[3] = {f2_total(sdd), f2_total(sg), f2_total(sgd)};
       if (ok) ok = bwd_team_sum<3, CLUSTER>(v, sh, tm, p.timeout_ns, p.status);
       c0 = rsqrtf(__fadd_rn(__fmul_rn(v[0], inv_n), p.eps));   // rstd
       c1 = __fmul_rn(v[1], inv_n);                              // mean(g)
@@ -362,50 +370,57 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
 
     // ---- dx, and this thread's dgamma / dbeta sums ----
     if (!active) continue;
+    const f2 C0 = f2_bcast(c0), NC1 = f2_bcast(-c1), NC2 = f2_bcast(-c2);
+    const f2 NMC0 = f2_bcast(-__fmul_rn(mu, c0));  // xhat = x rstd - mu rstd
 #pragma unroll
     for (int k = 0; k < CPT; ++k) {
       if (msk[k] == 0u) continue;
-      float x[E], d[E], g[E], o[E], ag[E], ab[E];
-      unpack<T>(av[k], x);
-      unpack<T>(dv[k], d);
-      if constexpr (kNorm) unpack<T>(gsm[k * NT + tid], g);
+      f2 x[NP], d[NP], o[NP], ag[NP];
+      chunk_to_pairs<T>(av[k], x);
+      chunk_to_pairs<T>(dv[k], d);
+      if constexpr (OP == kSoftmax) {
+        const f2 ns = f2_bcast(-c0);
 #pragma unroll
-      for (int e = 0; e < E; ++e) {
-        if constexpr (OP == kSoftmax) {
-          o[e] = __fmul_rn(x[e], __fsub_rn(d[e], c0));
-        } else if constexpr (OP == kLogSoftmax) {
-          o[e] = __fsub_rn(d[e], __fmul_rn(exp_shifted(x[e], 0.f), c0));
-        } else if constexpr (OP == kRmsNorm) {
-          const float xh = __fmul_rn(x[e], c0);
-          o[e] = __fmul_rn(c0, __fsub_rn(__fmul_rn(d[e], g[e]), __fmul_rn(xh, c1)));
-          ag[e] = __fmul_rn(d[e], xh);
-        } else {
-          const float xh = __fmul_rn(__fsub_rn(x[e], mu), c0);
-          o[e] = __fmul_rn(c0, __fsub_rn(__fsub_rn(__fmul_rn(d[e], g[e]), c1), __fmul_rn(xh, c2)));
-          ag[e] = __fmul_rn(d[e], xh);
-          ab[e] = d[e];
+        for (int i = 0; i < NP; ++i) o[i] = f2_mul(x[i], f2_add(d[i], ns));
+      } else if constexpr (OP == kLogSoftmax) {
+        const f2 ns = f2_bcast(-c0);
+        const f2 l2e = f2_bcast(kLog2e);
+#pragma unroll
+        for (int i = 0; i < NP; ++i) {
+          const f2 u = f2_mul(x[i], l2e);
+          o[i] = f2_fma(f2_make(ex2_approx(u.x), ex2_approx(u.y)), ns, d[i]);
         }
-      }
-      if constexpr (kNorm) {
+      } else {
+        f2 g[NP];
+        chunk_to_pairs<T>(gsm[k * NT + tid], g);
+#pragma unroll
+        for (int i = 0; i < NP; ++i) {
+          f2 xh;
+          if constexpr (OP == kRmsNorm) {
+            xh = f2_mul(x[i], C0);
+          } else {
+            xh = f2_fma(x[i], C0, NMC0);
+          }
+          // rstd (g - mean(g) - xhat mean(g xhat)); RMSNorm has no mean(g)
+          f2 t = OP == kRmsNorm ? f2_mul(d[i], g[i]) : f2_fma(d[i], g[i], NC1);
+          t = f2_fma(xh, OP == kRmsNorm ? NC1 : NC2, t);
+          o[i] = f2_mul(C0, t);
+          ag[i] = f2_mul(d[i], xh);
+        }
         if (accum) {
           // masked elements have d = 0: they add exactly zero
+          float4 *ap = acc + (k * E / 4) * NT + tid;
 #pragma unroll
           for (int q = 0; q < E / 4; ++q) {
-            float4 &sg = acc[(k * E / 4 + q) * NT + tid];
-            float4 vg = sg;
-            vg.x = __fadd_rn(vg.x, ag[4 * q]);
-            vg.y = __fadd_rn(vg.y, ag[4 * q + 1]);
-            vg.z = __fadd_rn(vg.z, ag[4 * q + 2]);
-            vg.w = __fadd_rn(vg.w, ag[4 * q + 3]);
-            sg = vg;
+            float4 vg = ap[q * NT];
+            const f2 lo = f2_add(make_float2(vg.x, vg.y), ag[2 * q]);
+            const f2 hi = f2_add(make_float2(vg.z, vg.w), ag[2 * q + 1]);
+            ap[q * NT] = make_float4(lo.x, lo.y, hi.x, hi.y);
             if constexpr (NA == 2) {
-              float4 &sb = acc[((S + k * E) / 4 + q) * NT + tid];
-              float4 vb = sb;
-              vb.x = __fadd_rn(vb.x, ab[4 * q]);
-              vb.y = __fadd_rn(vb.y, ab[4 * q + 1]);
-              vb.z = __fadd_rn(vb.z, ab[4 * q + 2]);
-              vb.w = __fadd_rn(vb.w, ab[4 * q + 3]);
-              sb = vb;
+              float4 vb = ap[(S / 4 + q) * NT];
+              const f2 blo = f2_add(make_float2(vb.x, vb.y), d[2 * q]);
+              const f2 bhi = f2_add(make_float2(vb.z, vb.w), d[2 * q + 1]);
+              ap[(S / 4 + q) * NT] = make_float4(blo.x, blo.y, bhi.x, bhi.y);
             }
           }
         }
@@ -414,16 +429,17 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
         const int c = (k * cs + rank) * TPR + tt;
         if (msk[k] == (1u << E) - 1u) {
           stg_stream(reinterpret_cast<char *>(dxrow) - h * SZ + static_cast<int64_t>(c) * 16,
-                     pack<T>(o));
+                     pairs_to_chunk<T>(o));
         } else {
 #pragma unroll
           for (int e = 0; e < E; ++e)
-            if ((msk[k] >> e) & 1u) dxrow[static_cast<int64_t>(c) * E + e - h] = from_f32<T>(o[e]);
+            if ((msk[k] >> e) & 1u)
+              dxrow[static_cast<int64_t>(c) * E + e - h] = from_f32<T>(pair_elem(o, e));
         }
       } else {
 #pragma unroll
         for (int e = 0; e < E; ++e)
-          if ((msk[k] >> e) & 1u) dxrow[column(k, e)] = from_f32<T>(o[e]);
+          if ((msk[k] >> e) & 1u) dxrow[column(k, e)] = from_f32<T>(pair_elem(o, e));
       }
     }
   }
@@ -498,40 +514,64 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
 }
 
 // dgamma[j] (dbeta[j]) = sum over the partials q = 0, 1, ... of
-// part[q][0 (1)][j], in that order: warp w of the block adds q = w, w + 8, ...
-// for 32 consecutive columns, then the 8 warp sums are added in warp order.
-template <typename T>
-__global__ void __launch_bounds__(256) bwd_param_finalize_kernel(const float *part, int64_t nparts,
-                                                                 int64_t cols, int nacc,
-                                                                 T *dgamma, T *dbeta) {
-  __shared__ float sums[8][32];
+// part[q][0 (1)][j], in that order per warp: warp w of the block adds q = w,
+// w + 32, ... for its columns (V consecutive columns per lane, V = 4 when
+// every partial row is 16-byte aligned), U loads ahead, then the 32 warp sums
+// are added in warp order.
+constexpr int kFinThreads = 1024;
+constexpr int kFinWarps = kFinThreads / 32;
+template <typename T, int V>
+__global__ void __launch_bounds__(kFinThreads) bwd_param_finalize_kernel(const float *part,
+                                                                         int64_t nparts,
+                                                                         int64_t cols, int nacc,
+                                                                         T *dgamma, T *dbeta) {
+  __shared__ float sums[kFinWarps][32 * V];
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const int a = blockIdx.y;
   T *out = a == 0 ? dgamma : dbeta;
   if (out == nullptr) return;  // uniform over the block
-  const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + lane;
-  float s = 0.f;
-  if (j < cols) {
-    constexpr int U = 4;
-    for (int64_t q0 = warp; q0 < nparts; q0 += 8 * U) {
-      float v[U];
+  const int64_t j0 = (static_cast<int64_t>(blockIdx.x) * 32 + lane) * V;
+  float s[V];
+#pragma unroll
+  for (int v = 0; v < V; ++v) s[v] = 0.f;
+  if (j0 < cols) {
+    constexpr int U = 8;
+    for (int64_t q0 = warp; q0 < nparts; q0 += kFinWarps * U) {
+      float x[U][V];
 #pragma unroll
       for (int u = 0; u < U; ++u) {
-        const int64_t q = q0 + u * 8;
-        v[u] = q < nparts ? __ldcs(part + (q * nacc + a) * cols + j) : 0.f;
+        const int64_t q = q0 + u * kFinWarps;
+        const float *src = part + (q * nacc + a) * cols + j0;
+        if constexpr (V == 4) {
+          const float4 w = q < nparts ? __ldcs(reinterpret_cast<const float4 *>(src))
+                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+          x[u][0] = w.x;
+          x[u][1] = w.y;
+          x[u][2] = w.z;
+          x[u][3] = w.w;
+        } else {
+          x[u][0] = q < nparts ? __ldcs(src) : 0.f;
+        }
       }
 #pragma unroll
       for (int u = 0; u < U; ++u)
-        if (q0 + u * 8 < nparts) s = __fadd_rn(s, v[u]);
+        if (q0 + u * kFinWarps < nparts) {
+#pragma unroll
+          for (int v = 0; v < V; ++v) s[v] = __fadd_rn(s[v], x[u][v]);
+        }
     }
   }
-  sums[warp][lane] = s;
+#pragma unroll
+  for (int v = 0; v < V; ++v) sums[warp][lane * V + v] = s[v];
   __syncthreads();
-  if (warp == 0 && j < cols) {
-    float t = sums[0][lane];
-    for (int w = 1; w < 8; ++w) t = __fadd_rn(t, sums[w][lane]);
-    out[j] = from_f32<T>(t);
+  if (warp == 0 && j0 < cols) {
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+      float t = sums[0][lane * V + v];
+      for (int w = 1; w < kFinWarps; ++w) t = __fadd_rn(t, sums[w][lane * V + v]);
+      if (j0 + v < cols) out[j0 + v] = from_f32<T>(t);
+    }
   }
 }
 
