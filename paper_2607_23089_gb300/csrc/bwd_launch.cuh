@@ -54,16 +54,11 @@ inline bool bwd_shape(int64_t units, int cpt, int force_cs, int small_cta, BwdSh
 template <typename T>
 cudaError_t launch_bwd_finalize(const float *part, int64_t nparts, int64_t cols, int nacc,
                                 void *dgamma, void *dbeta, cudaStream_t stream) {
-  // four columns per lane when every partial row starts on 16 bytes
-  if (cols % 4 == 0) {
-    const dim3 grid(static_cast<unsigned>(ceil_div(cols, 128)), static_cast<unsigned>(nacc), 1);
-    bwd_param_finalize_kernel<T, 4><<<grid, kFinThreads, 0, stream>>>(
-        part, nparts, cols, nacc, static_cast<T *>(dgamma), static_cast<T *>(dbeta));
-  } else {
-    const dim3 grid(static_cast<unsigned>(ceil_div(cols, 32)), static_cast<unsigned>(nacc), 1);
-    bwd_param_finalize_kernel<T, 1><<<grid, kFinThreads, 0, stream>>>(
-        part, nparts, cols, nacc, static_cast<T *>(dgamma), static_cast<T *>(dbeta));
-  }
+  // a block per 32 columns, so many SMs share the reads, and 32 warps per
+  // block over the partials, so each warp's chain of loads is short
+  const dim3 grid(static_cast<unsigned>(ceil_div(cols, 32)), static_cast<unsigned>(nacc), 1);
+  bwd_param_finalize_kernel<T><<<grid, kFinThreads, 0, stream>>>(
+      part, nparts, cols, nacc, static_cast<T *>(dgamma), static_cast<T *>(dbeta));
   return cudaGetLastError();
 }
 

@@ -514,64 +514,44 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
 }
 
 // dgamma[j] (dbeta[j]) = sum over the partials q = 0, 1, ... of
-// part[q][0 (1)][j], in that order per warp: warp w of the block adds q = w,
-// w + 32, ... for its columns (V consecutive columns per lane, V = 4 when
-// every partial row is 16-byte aligned), U loads ahead, then the 32 warp sums
-// are added in warp order.
+// part[q][0 (1)][j]: a block per 32 columns, one column per lane; warp w adds
+// q = w, w + 32, ... in that order, U loads ahead, then the 32 warp sums are
+// added in warp order.
 constexpr int kFinThreads = 1024;
 constexpr int kFinWarps = kFinThreads / 32;
-template <typename T, int V>
+template <typename T>
 __global__ void __launch_bounds__(kFinThreads) bwd_param_finalize_kernel(const float *part,
                                                                          int64_t nparts,
                                                                          int64_t cols, int nacc,
                                                                          T *dgamma, T *dbeta) {
-  __shared__ float sums[kFinWarps][32 * V];
+  __shared__ float sums[kFinWarps][32];
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const int a = blockIdx.y;
   T *out = a == 0 ? dgamma : dbeta;
   if (out == nullptr) return;  // uniform over the block
-  const int64_t j0 = (static_cast<int64_t>(blockIdx.x) * 32 + lane) * V;
-  float s[V];
-#pragma unroll
-  for (int v = 0; v < V; ++v) s[v] = 0.f;
-  if (j0 < cols) {
+  const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + lane;
+  float s = 0.f;
+  if (j < cols) {
     constexpr int U = 8;
     for (int64_t q0 = warp; q0 < nparts; q0 += kFinWarps * U) {
-      float x[U][V];
+      float x[U];
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         const int64_t q = q0 + u * kFinWarps;
-        const float *src = part + (q * nacc + a) * cols + j0;
-        if constexpr (V == 4) {
-          const float4 w = q < nparts ? __ldcs(reinterpret_cast<const float4 *>(src))
-                                      : make_float4(0.f, 0.f, 0.f, 0.f);
-          x[u][0] = w.x;
-          x[u][1] = w.y;
-          x[u][2] = w.z;
-          x[u][3] = w.w;
-        } else {
-          x[u][0] = q < nparts ? __ldcs(src) : 0.f;
-        }
+        x[u] = q < nparts ? __ldcs(part + (q * nacc + a) * cols + j) : 0.f;
       }
 #pragma unroll
       for (int u = 0; u < U; ++u)
-        if (q0 + u * kFinWarps < nparts) {
-#pragma unroll
-          for (int v = 0; v < V; ++v) s[v] = __fadd_rn(s[v], x[u][v]);
-        }
+        if (q0 + u * kFinWarps < nparts) s = __fadd_rn(s, x[u]);
     }
   }
-#pragma unroll
-  for (int v = 0; v < V; ++v) sums[warp][lane * V + v] = s[v];
+  sums[warp][lane] = s;
   __syncthreads();
-  if (warp == 0 && j0 < cols) {
-#pragma unroll
-    for (int v = 0; v < V; ++v) {
-      float t = sums[0][lane * V + v];
-      for (int w = 1; w < kFinWarps; ++w) t = __fadd_rn(t, sums[w][lane * V + v]);
-      if (j0 + v < cols) out[j0 + v] = from_f32<T>(t);
-    }
+  if (warp == 0 && j < cols) {
+    float t = sums[0][lane];
+    for (int w = 1; w < kFinWarps; ++w) t = __fadd_rn(t, sums[w][lane]);
+    out[j] = from_f32<T>(t);
   }
 }
 
