@@ -278,27 +278,55 @@ def profile_traffic():
     return d.get("traffic_bytes_per_launch")
 
 
-def cpu_oracle_baseline(case, max_elems):
+def cpu_model():
+    """The host CPU's model name (lscpu, else /proc/cpuinfo), or None."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    return None
+
+
+def cpu_oracle_baseline(case, max_elems, single_elems=16_000_000):
     """The double-precision oracle on a bounded sample of the workload (its
-    first rows), on all host cores."""
+    first rows): on all host cores (OpenMP over rows), and single-threaded on
+    a smaller sample."""
     import numpy as np
     from oracle import rowop_oracle as orc
     off = case.offsets.numpy()
-    rows = int(np.searchsorted(off, max_elems, side="right") - 1)
-    rows = max(1, min(case.rows, rows))
-    n = int(off[rows])
-    x = case.x[:n].double().numpy()
     g = case.gamma.double().numpy()
     b = case.beta.double().numpy()
+
+    def run(elems, threads):
+        rows = max(1, min(case.rows, int(np.searchsorted(off, elems, side="right") - 1)))
+        n = int(off[rows])
+        x = case.x[:n].double().numpy()
+        t0 = time.perf_counter()
+        orc.layernorm_ragged(x, off[:rows + 1], g, b, eps=case.eps, nthreads=threads)
+        dt = time.perf_counter() - t0
+        nbytes = 2 * n * 2 + 2 * case.max_len * 2 + (rows + 1) * 8
+        return nbytes / dt / 1e9, dt, rows, n
+
     cores = os.cpu_count() or 1
-    t0 = time.perf_counter()
-    orc.layernorm_ragged(x, off[:rows + 1], g, b, eps=case.eps, nthreads=cores)
-    dt = time.perf_counter() - t0
-    nbytes = 2 * n * 2 + 2 * case.max_len * 2 + (rows + 1) * 8
-    return {"value": round(nbytes / dt / 1e9, 3), "unit": "GB/s", "cores": cores,
+    gbs, dt, rows, n = run(max_elems, cores)
+    gbs1, dt1, rows1, n1 = run(single_elems, 1)
+    return {"value": round(gbs, 3), "unit": "GB/s", "cores": cores,
             "kind": "oracle", "seconds": round(dt, 3),
             "sample": f"first {rows} of {case.rows} rows ({n} of {case.elements} elements), "
-                      "float64 C oracle, OpenMP over rows"}
+                      "float64 C oracle (gcc -O2, no fast-math), OpenMP over rows",
+            "single_thread": {"value": round(gbs1, 3), "unit": "GB/s", "seconds": round(dt1, 3),
+                              "sample": f"first {rows1} rows ({n1} elements), one thread"},
+            "cpu_model": cpu_model(), "precision": "double"}
 
 
 # ---------------------------------------------------------------------------

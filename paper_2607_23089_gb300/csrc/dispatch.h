@@ -149,9 +149,11 @@ inline int64_t max_row_len_elems(int esize) {
 //   ROWOP_STAGES        stage-ring depth of the tile kernel
 //   ROWOP_CTAS_PER_SM   upper bound on resident tile-kernel CTAs per SM
 //   ROWOP_GROUP_WARPS   consumer warps per item group of the tile kernel (1, 2, 4, 8)
-//   ROWOP_SOFTMAX_ONLINE 1 -> dense SMALL softmax / log-softmax use the online
-//                       one-pass statistics instead of the two-pass ones (a
-//                       comparison variant: its results differ by rounding)
+//   ROWOP_SOFTMAX_ONLINE 1 -> dense softmax / log-softmax use online one-pass
+//                       statistics instead of the two-pass ones: SMALL rows
+//                       a running maximum over the lane's chunks, MEDIUM /
+//                       LARGE tiles one sweep over the stage (a comparison
+//                       variant: its results differ by rounding)
 //   ROWOP_BWD_CLUSTER   backward passes: split every row over a cluster of
 //                       this many CTAs (2, 4, 8, 16); changes rounding order
 struct Knobs {

@@ -68,11 +68,12 @@ cudaError_t launch_small(const DenseCall &c, const DeviceInfo &d, bool exact, bo
 // group_warps: consumer warps per item group (W); the stage ring holds at
 // least one item per group.  min_stage_area: bytes the stages must span
 // together (ragged SMALL staging).
-template <int OP, typename T, bool EXACT, bool CLUSTER, bool RAGGED, bool RESID = false>
+template <int OP, typename T, bool EXACT, bool CLUSTER, bool RAGGED, bool RESID = false,
+          bool ONLINE = false>
 cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int group_warps,
                           int64_t items, const DeviceInfo &d, cudaStream_t stream,
                           uint32_t min_stage_area = 0) {
-  auto kern = tile_row_kernel<OP, T, EXACT, CLUSTER, RAGGED, RESID>;
+  auto kern = tile_row_kernel<OP, T, EXACT, CLUSTER, RAGGED, RESID, ONLINE>;
   const void *kp = reinterpret_cast<const void *>(kern);
   const int max_ctas_per_sm = read_knobs().ctas_per_sm;
   p.stage_bytes = static_cast<uint32_t>(stage_tiles) * kTileBytes;
@@ -213,6 +214,23 @@ cudaError_t launch_dense_impl(const DenseCall &c, const DeviceInfo &d) {
   if (st > kMaxPortionTiles) return cudaErrorInvalidValue;
   const int W = pick_group_warps(st, false, kn.group_warps);
   const int S = pick_stages(st, W, kn.stages);
+  if constexpr ((OP == kSoftmax || OP == kLogSoftmax) && !RESID) {
+    // the online one-pass tile statistics (a comparison variant, see Knobs)
+    if (kn.softmax_online) {
+      if (cs == 1) {
+        if (exact)
+          return launch_tile_k<OP, T, true, false, false, false, true>(p, 1, S, st, W, c.rows, d,
+                                                                       c.stream);
+        return launch_tile_k<OP, T, false, false, false, false, true>(p, 1, S, st, W, c.rows, d,
+                                                                      c.stream);
+      }
+      if (exact)
+        return launch_tile_k<OP, T, true, true, false, false, true>(p, cs, S, st, W, c.rows, d,
+                                                                    c.stream);
+      return launch_tile_k<OP, T, false, true, false, false, true>(p, cs, S, st, W, c.rows, d,
+                                                                   c.stream);
+    }
+  }
   if (cs == 1) {
     if (exact)
       return launch_tile_k<OP, T, true, false, false, RESID>(p, 1, S, st, W, c.rows, d, c.stream);

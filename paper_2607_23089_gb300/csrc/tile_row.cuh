@@ -266,7 +266,7 @@ __device__ __forceinline__ void residual_tile(unsigned char *tsm, int t, const I
   }
 }
 
-template <int OP, typename T, int B, bool FULL, bool RESID>
+template <int OP, typename T, int B, bool FULL, bool RESID, bool ONLINE = false>
 __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const ItemGeo &g, int lt0,
                                             int W, int lane, float4 *part, uint32_t piece_bar0,
                                             uint32_t par, uint64_t timeout_ns, int &waited,
@@ -274,6 +274,49 @@ __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const It
   constexpr int E = Elem<T>::kPerChunk;
   constexpr bool kMaxFirst = (OP == kSoftmax || OP == kLogSoftmax);
   float a[B], b[B];
+  static_assert(!(RESID && ONLINE), "the residual add serves the norms only");
+  if constexpr (kMaxFirst && ONLINE) {
+    // Online statistics: each lane reads its two chunks of the tile from the
+    // stage once, forms their maximum and the sum of exp about it from those
+    // registers, and the lanes merge their (m, s) pairs by the rescaling
+    // butterfly -- one sweep over shared memory instead of two.
+    constexpr int NP = E / 2;
+#pragma unroll
+    for (int q = 0; q < B; ++q) {
+      const int lt = lt0 + q * W;
+      const int pc = lt / kPieceTiles;
+      if (pc != waited) {
+        if (!mbar_wait_bounded(piece_bar0 + 8u * pc, par, timeout_ns)) return false;
+        waited = pc;
+      }
+      const int t = g.t0 + lt;
+      const TileMask m = FULL ? TileMask{0, E, 0, E} : tile_mask<T>(t, g, lane, tile_is_full(t, g));
+      const unsigned char *tsm = stage + lt * kTileBytes;
+      f2 p0[NP], p1[NP];
+      chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(tsm + lane * kChunkBytes), p0);
+      chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(tsm + (lane + 32) * kChunkBytes), p1);
+      a[q] = chunk_max<NP>(p1, chunk_max<NP>(p0, -INFINITY, m.lo0, m.hi0), m.lo1, m.hi1);
+      const f2 r2 = f2_bcast(a[q]);
+      b[q] = a[q] == -INFINITY
+                 ? 0.f
+                 : f2_total(chunk_sum_exp<NP>(p1, r2, chunk_sum_exp<NP>(p0, r2, f2_bcast(0.f), m.lo0, m.hi0),
+                                              m.lo1, m.hi1));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+      for (int q = 0; q < B; ++q) {
+        const float m2 = __shfl_xor_sync(kFullMask, a[q], o);
+        const float s2 = __shfl_xor_sync(kFullMask, b[q], o);
+        online_merge(a[q], b[q], m2, s2);
+      }
+    }
+    if (lane == 0) {
+#pragma unroll
+      for (int q = 0; q < B; ++q) part[lt0 + q * W] = make_float4(a[q], b[q], 0.f, 0.f);
+    }
+    return true;
+  }
 #pragma unroll
   for (int q = 0; q < B; ++q) {
     const int lt = lt0 + q * W;
@@ -345,7 +388,7 @@ __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const It
 // tiles lt = wig, wig + W, ..., taken PB at a time while that many remain,
 // then in a batch of two and one.  Each tile's arithmetic (and its butterfly
 // order) is the same whatever batch it falls in.
-template <int OP, typename T, int PB, bool RESID>
+template <int OP, typename T, int PB, bool RESID, bool ONLINE = false>
 __device__ __forceinline__ bool pass1_warp(const unsigned char *stage, const ItemGeo &g, int wig,
                                            int W, int lane, float4 *part, uint32_t piece_bar0,
                                            uint32_t par, uint64_t timeout_ns, const TileParams &p) {
@@ -362,19 +405,19 @@ __device__ __forceinline__ bool pass1_warp(const unsigned char *stage, const Ite
     const bool full = ta >= full0 && tb < full1;
     bool ok;
     if (PB > 2 && bsz == PB) {
-      ok = full ? pass1_batch<OP, T, PB, true, RESID>(stage, g, lt0, W, lane, part, piece_bar0, par,
+      ok = full ? pass1_batch<OP, T, PB, true, RESID, ONLINE>(stage, g, lt0, W, lane, part, piece_bar0, par,
                                                timeout_ns, waited, p)
-                : pass1_batch<OP, T, PB, false, RESID>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                : pass1_batch<OP, T, PB, false, RESID, ONLINE>(stage, g, lt0, W, lane, part, piece_bar0, par,
                                                 timeout_ns, waited, p);
     } else if (bsz == 2) {
-      ok = full ? pass1_batch<OP, T, 2, true, RESID>(stage, g, lt0, W, lane, part, piece_bar0, par,
+      ok = full ? pass1_batch<OP, T, 2, true, RESID, ONLINE>(stage, g, lt0, W, lane, part, piece_bar0, par,
                                               timeout_ns, waited, p)
-                : pass1_batch<OP, T, 2, false, RESID>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                : pass1_batch<OP, T, 2, false, RESID, ONLINE>(stage, g, lt0, W, lane, part, piece_bar0, par,
                                                timeout_ns, waited, p);
     } else {
-      ok = full ? pass1_batch<OP, T, 1, true, RESID>(stage, g, lt0, W, lane, part, piece_bar0, par,
+      ok = full ? pass1_batch<OP, T, 1, true, RESID, ONLINE>(stage, g, lt0, W, lane, part, piece_bar0, par,
                                               timeout_ns, waited, p)
-                : pass1_batch<OP, T, 1, false, RESID>(stage, g, lt0, W, lane, part, piece_bar0, par,
+                : pass1_batch<OP, T, 1, false, RESID, ONLINE>(stage, g, lt0, W, lane, part, piece_bar0, par,
                                                timeout_ns, waited, p);
     }
     if (!ok) return false;
@@ -901,7 +944,8 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
   }
 }
 
-template <int OP, typename T, bool EXACT, bool CLUSTER, bool RAGGED, bool RESID = false>
+template <int OP, typename T, bool EXACT, bool CLUSTER, bool RAGGED, bool RESID = false,
+          bool ONLINE = false>
 __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TileParams p) {
   constexpr int E = Elem<T>::kPerChunk;
   constexpr int SZ = Elem<T>::kSize;
@@ -1009,7 +1053,7 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
 
     // ---- pass 1 ----
     if (!bad && kind != kItemEnd)
-      bad = !pass1_warp<OP, T, kPass1Batch, RESID>(stage, g, wig, W, lane, part,
+      bad = !pass1_warp<OP, T, kPass1Batch, RESID, ONLINE>(stage, g, wig, W, lane, part,
                                                   sbase + L.bar_piece + 8u * (s * L.pieces), par,
                                                   p.timeout_ns, p);
     if (named_sync_or(gbar, gthreads, bad)) {

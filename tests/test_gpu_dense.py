@@ -195,11 +195,13 @@ def test_group_sizes_agree(rw, op, dtype, cols, ld, x_off):
 
 @pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
 @pytest.mark.parametrize("op", ["softmax", "logsoftmax"])
-@pytest.mark.parametrize("cols", [1, 5, 64, 255, 1000, 2047])
+@pytest.mark.parametrize("cols", [1, 5, 64, 255, 1000, 2047, 3000, 8192, 20000, 70001])
 def test_online_softmax_variant(rw, op, dtype, cols, monkeypatch):
-    """The one-pass (online) softmax statistics of the SMALL design, selected
-    by ROWOP_SOFTMAX_ONLINE, meet the same tolerance against the oracle,
-    also on rows whose maximum arrives late and rows with -inf entries."""
+    """The one-pass (online) softmax statistics, selected by
+    ROWOP_SOFTMAX_ONLINE -- a running maximum in the SMALL design, one sweep
+    over each staged tile in the MEDIUM / LARGE designs -- meet the same
+    tolerance against the oracle, also on rows whose maximum arrives late and
+    rows with -inf entries."""
     monkeypatch.setenv("ROWOP_SOFTMAX_ONLINE", "1")
     run_case(rw, op, dtype, 37, cols, seed=cols + 3)
     rows = 6
@@ -210,3 +212,14 @@ def test_online_softmax_variant(rw, op, dtype, cols, monkeypatch):
     y = rw.run(op, x.cuda()).cpu()
     ref = oracle_dense(op, x.double().numpy())
     assert_close(to_f64(y), ref, dtype, f"online {op}")
+
+
+@pytest.mark.parametrize("op", ["softmax", "logsoftmax"])
+@pytest.mark.parametrize("cs", [2, 8, 16])
+def test_online_softmax_cluster(rw, op, cs, monkeypatch):
+    """The online tile statistics across a cluster split of every size."""
+    monkeypatch.setenv("ROWOP_SOFTMAX_ONLINE", "1")
+    monkeypatch.setenv("ROWOP_FORCE_BUCKET", "2")
+    monkeypatch.setenv("ROWOP_CLUSTER", str(cs))
+    for dtype in (torch.float32, torch.bfloat16):
+        run_case(rw, op, dtype, 5, 50001, seed=cs)
