@@ -274,3 +274,34 @@ def test_ragged_bad_rows_in_several_blocks(rw):
         seg = r["y"][int(off[i]):int(off[i + 1])]
         ref = orc.softmax(r["x"][int(off[i]):int(off[i + 1])].double().numpy()[None])[0]
         assert_close(to_f64(seg), ref, dtype, f"row {i}")
+
+
+@pytest.mark.parametrize("op", ALL_OPS)
+def test_ragged_chunked_calls_equal_one_call(rw, op):
+    """Rows are independent: calls over contiguous chunks of rows, each given
+    its slice of the offsets (a first offset other than 0), write bitwise what
+    one call over all rows writes -- the decomposition the benchmark's
+    end-to-end pipeline uses."""
+    dtype = torch.bfloat16
+    max_len = 20000
+    lens = mixed_lengths(dtype, 90, 31, max_len)
+    whole = run_ragged(rw, op, dtype, lens, max_len, seed=31)
+    off = whole["off"]
+    offd = torch.from_numpy(off).cuda()
+    es = ESIZE[dtype]
+    G = whole["G"]
+    ybuf = canary_tensor(G + whole["total"] + G, dtype)
+    xbuf = canary_tensor(G + whole["total"] + G, dtype)
+    xbuf[G:G + whole["total"]] = whole["x"].cuda()
+    gd = whole["gam"].cuda() if op in ("layernorm", "rmsnorm") else None
+    bd = whole["bet"].cuda() if op == "layernorm" else None
+    bounds = [0, 1, 17, 40, 41, 90]
+    for r0, r1 in zip(bounds[:-1], bounds[1:]):
+        ws = rw.ragged_workspace(r1 - r0)
+        st = call_ragged(rw, op, xbuf.data_ptr() + G * es, ybuf.data_ptr() + G * es,
+                         offd.data_ptr() + 8 * r0, r1 - r0, max_len, gd, bd, dtype,
+                         whole["eps"], ws)
+        assert st == 0, rw.STATUS.get(st, st)
+    torch.cuda.synchronize()
+    got = ybuf[G:G + whole["total"]]
+    assert torch.equal(got.view(torch.int16), whole["y"].view(torch.int16))
