@@ -192,7 +192,9 @@ def per_config(torch, rw, wl, device, peak, steps):
         x = case.x.to(device)
         g = case.gamma.to(device) if case.gamma is not None else None
         b = case.beta.to(device) if case.beta is not None else None
-        if case.ragged:
+        if case.dy is not None:
+            fn, y = backward_call(torch, rw, case, x, device)
+        elif case.ragged:
             off = case.offsets.to(device)
             y = torch.empty_like(x)
             ws = rw.ragged_workspace(case.rows, device)
@@ -208,8 +210,6 @@ def per_config(torch, rw, wl, device, peak, steps):
             kw = dict(fft_size=case.meta.get("fft_size"), scale=case.meta.get("scale"))
             y = rw.run(case.op, x, **kw)
             fn = lambda: rw.run(case.op, x, out=y, **kw)  # noqa: E731
-        elif case.dy is not None:
-            fn, y = backward_call(torch, rw, case, x, device)
         else:
             y = torch.empty_like(x)
             fn = lambda: rw.run(case.op, x, gamma=g, beta=b, eps=case.eps, out=y)  # noqa: E731
@@ -246,6 +246,14 @@ def backward_call(torch, rw, case, x, device):
     once, outside the timed calls."""
     dy = case.dy.to(device)
     a = x
+    if case.ragged:  # softmax family over ragged rows
+        off = case.offsets.to(device)
+        ws = rw.ragged_workspace(case.rows, device)
+        a = rw.run(case.op[:-len("_backward")], x, offsets=off, max_len=case.max_len, ws=ws)
+        dx = torch.empty_like(a)
+        log = case.op.startswith("log")
+        return (lambda: rw.softmax_backward_ragged(a, dy, off, case.max_len, dx=dx, ws=ws,
+                                                   log=log)), dx
     if case.op in ("softmax_backward", "logsoftmax_backward"):
         a = rw.run(case.op[:-len("_backward")], x)
     dx = torch.empty_like(a)
@@ -613,7 +621,7 @@ def run_only(args, local):
         kw["out"] = rw.run(case.op, x, **kw)
     if case.resid is not None:
         kw.update(resid=case.resid.to(device), sum_out=torch.empty_like(x))
-    if case.ragged:
+    if case.ragged and case.dy is None:
         kw.update(offsets=case.offsets.to(device), max_len=case.max_len,
                   ws=rw.ragged_workspace(case.rows, device))
     fn = lambda: rw.run(case.op, x, **kw)  # noqa: E731

@@ -188,6 +188,24 @@ ROWOP_API int rowop_rmsnorm_backward(const void *x, const void *dy, const void *
                                      int64_t ld, rowop_dtype_t dtype, float eps, void *ws,
                                      size_t ws_bytes, cudaStream_t stream);
 
+/* Softmax / log-softmax backward over ragged rows: row i is elements
+ * [offsets[i], offsets[i+1]) of y, dy and dx alike (the ragged layout
+ * above), dx as the dense backward defines it.  ws is a ragged workspace of
+ * at least rowop_ragged_workspace_size(rows) bytes: the call runs the
+ * classify pass into it, then one launch per row bucket.  max_len <=
+ * ROWOP_BWD_MAX_COLS_SOFTMAX; rows longer than max_len or with decreasing
+ * offsets are skipped and flagged as in the forward ragged calls.  dx may be
+ * dy or y itself; partial overlap is undefined. */
+ROWOP_API int rowop_softmax_backward_ragged(const void *y, const void *dy, void *dx,
+                                            const int64_t *offsets, int64_t rows,
+                                            int64_t max_len, rowop_dtype_t dtype, void *ws,
+                                            size_t ws_bytes, cudaStream_t stream);
+
+ROWOP_API int rowop_logsoftmax_backward_ragged(const void *y, const void *dy, void *dx,
+                                               const int64_t *offsets, int64_t rows,
+                                               int64_t max_len, rowop_dtype_t dtype, void *ws,
+                                               size_t ws_bytes, cudaStream_t stream);
+
 /* Workspace bytes for dgamma (and dbeta) of rows of `cols` elements on the
  * current device; 0 if cols <= 0 or the device cannot be queried. */
 ROWOP_API size_t rowop_layernorm_backward_workspace_size(int64_t cols);

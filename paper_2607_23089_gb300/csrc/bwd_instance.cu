@@ -13,4 +13,6 @@
 namespace rowop {
 template cudaError_t launch_bwd_t<ROWOP_INST_OP, ROWOP_INST_T>(const BwdCall &,
                                                                const DeviceInfo &);
+template cudaError_t launch_bwd_ragged_t<ROWOP_INST_OP, ROWOP_INST_T>(const BwdRaggedCall &,
+                                                                      const DeviceInfo &);
 }  // namespace rowop

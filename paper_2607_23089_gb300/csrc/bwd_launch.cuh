@@ -62,10 +62,10 @@ cudaError_t launch_bwd_finalize(const float *part, int64_t nparts, int64_t cols,
   return cudaGetLastError();
 }
 
-template <int OP, typename T, int CPT, bool VEC, bool CLUSTER>
+template <int OP, typename T, int CPT, bool VEC, bool CLUSTER, bool RAGGED = false>
 cudaError_t launch_bwd_k(const BwdParams &p, const BwdShape &s, const BwdCall &c,
                          const DeviceInfo &d) {
-  auto kern = bwd_row_kernel<OP, T, CPT, VEC, CLUSTER>;
+  auto kern = bwd_row_kernel<OP, T, CPT, VEC, CLUSTER, RAGGED>;
   const void *kp = reinterpret_cast<const void *>(kern);
   constexpr bool kNorm = (OP == kLayerNorm || OP == kRmsNorm);
   const int teams_cta = s.nt / s.tpr;
@@ -179,6 +179,86 @@ cudaError_t launch_bwd_t(const BwdCall &c, const DeviceInfo &d) {
   }
   if (vec) return launch_bwd_k<OP, T, CPT, true, false>(p, s, c, d);
   return launch_bwd_k<OP, T, CPT, false, false>(p, s, c, d);
+}
+
+// Ragged backward (softmax family): the forward's classify pass sorts the
+// rows into three buckets by byte length; each bucket that max_len allows
+// gets one launch of the team kernel, shaped for the bucket's longest row,
+// which walks that bucket's list.  Rows are independent, so each row's
+// result depends only on its values, length and alignment and on the shape
+// of its bucket's teams.
+template <int OP, typename T>
+cudaError_t launch_bwd_ragged_t(const BwdRaggedCall &c, const DeviceInfo &d) {
+  if constexpr (OP == kLayerNorm || OP == kRmsNorm) {
+    return cudaErrorNotSupported;
+  } else {
+    constexpr int SZ = sizeof(T);
+    constexpr int E = 16 / SZ;
+    constexpr int CPT = kBwdSlots / E;
+    RaggedCall rc = {};
+    rc.dtype = c.dtype;
+    rc.offsets = c.offsets;
+    rc.rows = c.rows;
+    rc.max_len = c.max_len;
+    rc.ws = c.ws;
+    rc.stream = c.stream;
+    rc.classify = true;
+    cudaError_t e = launch_classify(rc, d);
+    if (e != cudaSuccess || c.max_len == 0) return e;
+    unsigned char *ws = static_cast<unsigned char *>(c.ws);
+    const RowRec *list0 = reinterpret_cast<const RowRec *>(ws + ragged_lists_offset(c.rows));
+    const bool vec = congruent16(c.a, c.dy) && congruent16(c.a, c.dx);
+    BwdParams p = {};
+    p.a = c.a;
+    p.dy = c.dy;
+    p.dx = c.dx;
+    p.rows = c.rows;  // an upper bound on every bucket's rows: sizes the grid
+    p.ld = 0;
+    p.eps = 0.f;
+    p.nacc = 1;
+    p.timeout_ns = kWaitLimitNs;
+    p.status = d.status;
+    p.block_counts = reinterpret_cast<const int32_t *>(ws + ragged_counts_offset(c.rows));
+    p.blocks = static_cast<int>(ragged_blocks(c.rows));
+    p.rows_per_block = ragged_rows_per_block(c.rows);
+    const int64_t max_bytes = c.max_len * SZ;
+    for (int b = kSmall; b <= kLarge; ++b) {
+      const int64_t lo = b == kSmall ? 0 : (b == kMedium ? kSmallMaxBytes : kMediumMaxBytes);
+      if (max_bytes <= lo && b != kSmall) break;  // no row can be this long
+      const int64_t hi = b == kSmall ? std::min(max_bytes, kSmallMaxBytes)
+                                     : (b == kMedium ? std::min(max_bytes, kMediumMaxBytes) : max_bytes);
+      const int64_t longest = std::max<int64_t>(1, hi / SZ);
+      bool bvec = vec;
+      BwdShape s;
+      if (!bwd_shape(bvec ? ceil_div(longest + E - 1, E) : ceil_div(longest, E), CPT, 0, 256, s)) {
+        // the longest row, starting mid-chunk, needs a chunk more than the
+        // largest cluster holds: this bucket takes the element path
+        bvec = false;
+        if (!bwd_shape(ceil_div(longest, E), CPT, 0, 256, s)) return cudaErrorInvalidValue;
+      }
+      p.list = list0 + static_cast<int64_t>(b) * c.rows;
+      p.bucket = b;
+      p.tpr = s.tpr;
+      p.cols = longest;
+      BwdCall bc = {};
+      bc.dtype = c.dtype;
+      bc.a = c.a;
+      bc.dy = c.dy;
+      bc.dx = c.dx;
+      bc.rows = c.rows;
+      bc.cols = longest;
+      bc.stream = c.stream;
+      if (s.cs > 1) {
+        e = bvec ? launch_bwd_k<OP, T, CPT, true, true, true>(p, s, bc, d)
+                 : launch_bwd_k<OP, T, CPT, false, true, true>(p, s, bc, d);
+      } else {
+        e = bvec ? launch_bwd_k<OP, T, CPT, true, false, true>(p, s, bc, d)
+                 : launch_bwd_k<OP, T, CPT, false, false, true>(p, s, bc, d);
+      }
+      if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+  }
 }
 
 }  // namespace rowop

@@ -50,6 +50,12 @@ struct BwdParams {
   int nacc;  // partial rows per partial index: 2 (dgamma, dbeta) or 1 (dgamma)
   uint64_t timeout_ns;
   unsigned int *status;
+  // ragged (softmax family): the rows of one bucket of a classify plan
+  const RowRec *list;           // that bucket's list: classify block b from entry b * rows_per_block
+  const int32_t *block_counts;  // [blocks][3] rows per bucket of each classify block
+  int blocks;
+  int64_t rows_per_block;
+  int bucket;
 };
 
 // Shared memory of the backward kernel (static part).
@@ -58,6 +64,7 @@ struct BwdShared {
   float cres[2][4];                    // this CTA's sums for the cluster peers
   uint64_t ready[2];                   // peers' sums published (cs arrivals)
   uint64_t released[2];                // peers done reading ours (cs * warps arrivals)
+  int pref[257];                       // ragged: list start of each classify block, then the total
 };
 
 // Where a thread stands in its team, and the state of the team reductions.
@@ -139,13 +146,14 @@ __device__ __forceinline__ bool bwd_team_sum(float (&v)[NV], BwdShared &sh, BwdT
   return true;
 }
 
-template <int OP, typename T, int CPT, bool VEC, bool CLUSTER>
+template <int OP, typename T, int CPT, bool VEC, bool CLUSTER, bool RAGGED = false>
 __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams p) {
   constexpr int E = Elem<T>::kPerChunk;
   constexpr int SZ = Elem<T>::kSize;
   constexpr int S = CPT * E;  // elements per thread per tensor
   constexpr bool kNorm = (OP == kLayerNorm || OP == kRmsNorm);
   constexpr int NA = OP == kLayerNorm ? 2 : 1;
+  static_assert(!(RAGGED && kNorm), "ragged backward rows: softmax family only");
   __shared__ BwdShared sh;
   // dynamic (norms): gamma at this thread's columns ([CPT][NT] chunks), the
   // thread's dgamma / dbeta sums ([NA][S/4][NT] float4) -- both private to
@@ -175,13 +183,36 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
     // team's row count, so shuffles always see every lane
     warp_team0 = static_cast<int64_t>(blockIdx.x) * teams_cta + (TPR < 32 ? (warp * 32) / TPR : team);
   }
-  const int64_t cols = p.cols;
-  const int h = VEC ? p.h : 0;
-  const int nc = VEC ? p.nc : 0;
-  const int cf = (VEC && h > 0) ? 1 : 0;                                 // first full chunk
-  const int cl = (VEC && ((h + cols) % E) != 0) ? nc - 1 : nc;          // end of full chunks
-  const int hn = h + static_cast<int>(cols);
-  const float inv_n = __frcp_rn(static_cast<float>(cols));
+  // row geometry: fixed for dense rows, set per row for ragged ones
+  int64_t cols = p.cols;
+  int h = VEC ? p.h : 0;
+  int nc = VEC ? p.nc : 0;
+  int cf = (VEC && h > 0) ? 1 : 0;                                 // first full chunk
+  int cl = (VEC && ((h + cols) % E) != 0) ? nc - 1 : nc;          // end of full chunks
+  int hn = h + static_cast<int>(cols);
+  float inv_n = __frcp_rn(static_cast<float>(cols));
+  int64_t nrows = p.rows;
+  if constexpr (RAGGED) {
+    // list position where each classify block's rows of this bucket start
+    if (warp == 0) {
+      int carry = 0;
+      for (int b0 = 0; b0 < p.blocks; b0 += 32) {
+        const int b = b0 + lane;
+        const int v = b < p.blocks ? p.block_counts[3 * b + p.bucket] : 0;
+        int x = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(kFullMask, x, o);
+          if (lane >= o) x += y;
+        }
+        if (b < p.blocks) sh.pref[b] = carry + x - v;
+        carry += __shfl_sync(kFullMask, x, 31);
+      }
+      if (lane == 0) sh.pref[p.blocks] = carry;
+    }
+    __syncthreads();
+    nrows = sh.pref[p.blocks];
+  }
 
   BwdTeam tm;
   tm.tpr = TPR;
@@ -248,12 +279,38 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
   const T *dybase = static_cast<const T *>(p.dy);
   T *dxbase = static_cast<T *>(p.dx);
 
-  for (int64_t r0 = warp_team0; r0 < p.rows; r0 += nteams) {
+  for (int64_t r0 = warp_team0; r0 < nrows; r0 += nteams) {
     const int64_t r = r0 + (gteam - warp_team0);
-    const bool active = r < p.rows;
-    const T *arow = abase + r * p.ld;
-    const T *dyrow = dybase + r * p.ld;
-    T *dxrow = dxbase + r * p.ld;
+    const bool active = r < nrows;
+    int64_t start = r * p.ld;
+    if constexpr (RAGGED) {
+      // record r of the bucket's list: classify block lo with pref[lo] <= r < pref[lo + 1]
+      start = 0;
+      cols = 0;
+      if (active) {
+        int lo = 0, hi = p.blocks;
+        while (hi - lo > 1) {
+          const int mid = (lo + hi) >> 1;
+          if (sh.pref[mid] <= r) {
+            lo = mid;
+          } else {
+            hi = mid;
+          }
+        }
+        const RowRec rec = p.list[static_cast<int64_t>(lo) * p.rows_per_block + (r - sh.pref[lo])];
+        start = rec.start;
+        cols = rec.n;
+      }
+      h = VEC ? static_cast<int>((reinterpret_cast<uintptr_t>(abase + start) & 15u) / SZ) : 0;
+      hn = h + static_cast<int>(cols);
+      nc = VEC ? (hn + E - 1) / E : 0;
+      cf = (VEC && h > 0) ? 1 : 0;
+      cl = (VEC && (hn % E) != 0) ? nc - 1 : nc;
+      inv_n = __frcp_rn(static_cast<float>(cols));
+    }
+    const T *arow = abase + start;
+    const T *dyrow = dybase + start;
+    T *dxrow = dxbase + start;
 
     // ---- loads: every chunk of both tensors in flight before any is used ----
     uint4 av[CPT], dv[CPT];

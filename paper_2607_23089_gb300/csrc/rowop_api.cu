@@ -25,6 +25,16 @@ cudaError_t launch_ragged_t(const RaggedCall &c, const DeviceInfo &d);
 template <int OP, typename T>
 cudaError_t launch_bwd_t(const BwdCall &c, const DeviceInfo &d);
 
+template <int OP, typename T>
+cudaError_t launch_bwd_ragged_t(const BwdRaggedCall &c, const DeviceInfo &d);
+
+template <int OP>
+static cudaError_t launch_bwd_ragged(const BwdRaggedCall &c, const DeviceInfo &d) {
+  if (c.dtype == ROWOP_F32) return launch_bwd_ragged_t<OP, float>(c, d);
+  if (c.dtype == ROWOP_F16) return launch_bwd_ragged_t<OP, __half>(c, d);
+  return launch_bwd_ragged_t<OP, __nv_bfloat16>(c, d);
+}
+
 template <int OP>
 static cudaError_t launch_bwd(const BwdCall &c, const DeviceInfo &d) {
   if (c.dtype == ROWOP_F32) return launch_bwd_t<OP, float>(c, d);
@@ -315,6 +325,37 @@ static int run_bwd(int op, const void *a, const void *dy, void *dx, const void *
   }
 }
 
+// Ragged backward passes (softmax family).  a = y.
+static int run_bwd_ragged(int op, const void *a, const void *dy, void *dx, const int64_t *offsets,
+                          int64_t rows, int64_t max_len, rowop_dtype_t dtype, void *ws,
+                          size_t ws_bytes, cudaStream_t stream) {
+  const int es = esize_of(dtype);
+  if (es == 0) return ROWOP_ERR_UNSUPPORTED_DTYPE;
+  if (rows < 0 || rows > INT32_MAX - 1 || max_len < 0) return ROWOP_ERR_INVALID_ARG;
+  if (rows == 0) return ROWOP_OK;
+  if (!offsets || !elem_aligned(offsets, 8)) return ROWOP_ERR_INVALID_ARG;
+  if (!a || !dy || !dx || !elem_aligned(a, es) || !elem_aligned(dy, es) || !elem_aligned(dx, es))
+    return ROWOP_ERR_INVALID_ARG;
+  if (max_len > kBwdMaxColsSoftmax) return ROWOP_ERR_TOO_LONG;
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < ragged_ws_bytes(rows))
+    return ROWOP_ERR_WORKSPACE;
+  DeviceInfo d;
+  const int st = device_info(&d);
+  if (st != ROWOP_OK) return st;
+  BwdRaggedCall c;
+  c.dtype = dtype;
+  c.a = a;
+  c.dy = dy;
+  c.dx = dx;
+  c.offsets = offsets;
+  c.rows = rows;
+  c.max_len = max_len;
+  c.ws = ws;
+  c.stream = stream;
+  if (op == kSoftmax) return from_cuda(launch_bwd_ragged<kSoftmax>(c, d));
+  return from_cuda(launch_bwd_ragged<kLogSoftmax>(c, d));
+}
+
 static size_t bwd_workspace_size(int nacc, int64_t cols) {
   if (cols <= 0) return 0;
   DeviceInfo d;
@@ -409,6 +450,20 @@ int rowop_rmsnorm_backward(const void *x, const void *dy, const void *gamma, voi
                            cudaStream_t stream) {
   return run_bwd(kRmsNorm, x, dy, dx, gamma, dgamma, nullptr, rows, cols, ld, dtype, eps, ws,
                  ws_bytes, stream);
+}
+
+int rowop_softmax_backward_ragged(const void *y, const void *dy, void *dx, const int64_t *offsets,
+                                  int64_t rows, int64_t max_len, rowop_dtype_t dtype, void *ws,
+                                  size_t ws_bytes, cudaStream_t stream) {
+  return run_bwd_ragged(kSoftmax, y, dy, dx, offsets, rows, max_len, dtype, ws, ws_bytes, stream);
+}
+
+int rowop_logsoftmax_backward_ragged(const void *y, const void *dy, void *dx,
+                                     const int64_t *offsets, int64_t rows, int64_t max_len,
+                                     rowop_dtype_t dtype, void *ws, size_t ws_bytes,
+                                     cudaStream_t stream) {
+  return run_bwd_ragged(kLogSoftmax, y, dy, dx, offsets, rows, max_len, dtype, ws, ws_bytes,
+                        stream);
 }
 
 size_t rowop_layernorm_backward_workspace_size(int64_t cols) { return bwd_workspace_size(2, cols); }

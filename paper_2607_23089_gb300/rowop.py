@@ -65,6 +65,8 @@ SIGNATURES = {
     "rowop_layernorm_backward": ([_P, _P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _F, _P, _SZ,
                                   _P], _I),
     "rowop_rmsnorm_backward": ([_P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _F, _P, _SZ, _P], _I),
+    "rowop_softmax_backward_ragged": ([_P, _P, _P, _P, _I64, _I64, _I, _P, _SZ, _P], _I),
+    "rowop_logsoftmax_backward_ragged": ([_P, _P, _P, _P, _I64, _I64, _I, _P, _SZ, _P], _I),
     "rowop_layernorm_backward_workspace_size": ([_I64], _SZ),
     "rowop_rmsnorm_backward_workspace_size": ([_I64], _SZ),
     "rowop_pad_scale": ([_P, _P, _I64, _I64, _I64, _I64, _I64, _F, _I, _P], _I),
@@ -358,6 +360,19 @@ def logsoftmax_backward(y, dy, dx=None, stream=None):
     _ok(rowop_logsoftmax_backward(y.data_ptr(), dy.data_ptr(), dx.data_ptr(), rows,  # noqa: F821
                                   cols, ld, dtype_code(y.dtype), _stream(stream)),
         "rowop_logsoftmax_backward")
+    return dx
+
+
+def softmax_backward_ragged(y, dy, offsets, max_len, dx=None, ws=None, stream=None,
+                            log=False):
+    """dx of softmax (log-softmax with ``log=True``) over ragged rows
+    (``rowop_{softmax,logsoftmax}_backward_ragged``)."""
+    rows, dx, ws = _ragged_args(y, offsets, ws, dx)
+    _check_cuda(dy)
+    fn = rowop_logsoftmax_backward_ragged if log else rowop_softmax_backward_ragged  # noqa: F821
+    _ok(fn(y.data_ptr(), dy.data_ptr(), dx.data_ptr(), offsets.data_ptr(), rows, int(max_len),
+           dtype_code(y.dtype), ws.data_ptr(), ws.numel(), _stream(stream)),
+        "rowop_softmax_backward_ragged")
     return dx
 
 

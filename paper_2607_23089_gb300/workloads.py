@@ -69,6 +69,8 @@ class Case:
             # read the forward input (norms) or output (softmax family) and dy,
             # write dx; norms also read gamma and write dgamma (and dbeta)
             b = 3 * self.elements * es
+            if self.ragged:
+                return b + self.offsets.numel() * 8
             ncol = self.x.shape[1]
             if self.op == "layernorm_backward":
                 b += 3 * ncol * es
@@ -235,6 +237,21 @@ def softmax_backward(op: str = "softmax", rows: int = 32768, cols: int = 1024,
     return Case(f"{op}_backward_{cols}", f"{op}_backward", x, torch.float32, dy=dy)
 
 
+def ragged_softmax_backward(rows: int = 32768, max_len: int = 4096, seed: int = 10) -> Case:
+    """Softmax backward over ragged fp32 rows (variable-length attention rows):
+    lengths uniform on {1..max_len} as int64 CSR offsets, x = 4*N(0,1) the
+    forward input (y = softmax(x) is formed by the caller), dy = N(0,1).  Not
+    one of the five workloads."""
+    g = _gen(seed)
+    lengths = ragged_lengths(rows, max_len, g)
+    off = offsets_from_lengths(lengths)
+    total = int(off[-1])
+    x = 4.0 * torch.randn(total, generator=g)
+    dy = torch.randn(total, generator=g)
+    return Case("ragged_softmax_backward", "softmax_backward", x, torch.float32, offsets=off,
+                max_len=max_len, dy=dy)
+
+
 def all_cases(scale_down: int = 1):
     """The five workloads as a flat list of cases.  ``scale_down`` > 1 divides
     every row count (not the row lengths) for quicker runs."""
@@ -255,6 +272,7 @@ def all_cases(scale_down: int = 1):
         out.append(norm_backward(op, rows=max(1, 8192 // s)))
     for op in ("softmax", "logsoftmax"):
         out.append(softmax_backward(op, rows=max(1, 32768 // s)))
+    out.append(ragged_softmax_backward(rows=max(1, 32768 // s)))
     return out
 
 
@@ -262,6 +280,8 @@ def by_name(name: str) -> Case:
     """Builds one workload case from its name (as in all_cases())."""
     if name.startswith("medium_norm_backward_"):
         return norm_backward(name[len("medium_norm_backward_"):])
+    if name == "ragged_softmax_backward":
+        return ragged_softmax_backward()
     if name.startswith(("softmax_backward_", "logsoftmax_backward_")):
         op, _, cols = name.split("_")
         return softmax_backward(op, cols=int(cols))

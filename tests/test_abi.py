@@ -181,3 +181,18 @@ def test_backward_validation(lib):
                None) == lib.ROWOP_ERR_INVALID_ARG
     assert lib.rowop_layernorm_backward_workspace_size(0) == 0
     assert lib.rowop_rmsnorm_backward_workspace_size(-5) == 0
+
+
+def test_backward_ragged_validation(lib):
+    F32 = lib.ROWOP_F32
+    f = lib.rowop_softmax_backward_ragged
+    ws_need = lib.rowop_ragged_workspace_size(10)
+    assert f(FAKE, FAKE, FAKE, FAKE, 10, 64, 7, FAKE, ws_need, None) == lib.ROWOP_ERR_UNSUPPORTED_DTYPE
+    assert f(FAKE, FAKE, FAKE, FAKE, -1, 64, F32, FAKE, ws_need, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert f(None, None, None, None, 0, 64, F32, None, 0, None) == lib.ROWOP_OK
+    assert f(FAKE, FAKE, FAKE, None, 10, 64, F32, FAKE, ws_need, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert f(FAKE, None, FAKE, FAKE, 10, 64, F32, FAKE, ws_need, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert f(FAKE, FAKE, FAKE, FAKE, 10, 262145, F32, FAKE, ws_need, None) == lib.ROWOP_ERR_TOO_LONG
+    assert f(FAKE, FAKE, FAKE, FAKE, 10, 64, F32, FAKE, ws_need - 1, None) == lib.ROWOP_ERR_WORKSPACE
+    g = lib.rowop_logsoftmax_backward_ragged
+    assert g(FAKE, FAKE, FAKE, FAKE, 10, -1, F32, FAKE, ws_need, None) == lib.ROWOP_ERR_INVALID_ARG

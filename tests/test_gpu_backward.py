@@ -369,3 +369,106 @@ def test_workload_softmax_backward(rw, op):
     ref = (orc.softmax_backward if op == "softmax" else orc.logsoftmax_backward)(a64, dy64)
     check(to_f64(dx[sel]), ref, scales(op, a64, dy64, None, 0)[0], case.dtype, R_COMP,
           f"{case.name} dx")
+
+
+def _ragged_lengths(dtype, rows, seed, max_len):
+    """Lengths over all three row buckets, with empty and length-1 rows."""
+    es = ESIZE[dtype]
+    g = np.random.default_rng(seed)
+    pools = [(0, 1), (1, 40), (41, 4096 // es), (4096 // es + 1, 32768 // es),
+             (32768 // es + 1, max_len)]
+    lens = [int(g.integers(lo, max(lo, min(hi, max_len)) + 1)) for lo, hi in
+            (pools[i % len(pools)] for i in range(rows))]
+    g.shuffle(lens)
+    return np.array(lens, dtype=np.int64)
+
+
+def run_bwd_ragged(rw, op, dtype, lens, max_len, seed, base_off=0, inplace=False):
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64) + base_off
+    total = int(off[-1])
+    rows = len(lens)
+    g = torch.Generator("cpu").manual_seed(seed)
+    y = torch.zeros(total, dtype=torch.float64)
+    for i in range(rows):
+        if lens[i]:
+            x = (3.0 * torch.randn(1, int(lens[i]), generator=g, dtype=torch.float64)).numpy()
+            y[off[i]:off[i + 1]] = torch.from_numpy(
+                (orc.softmax(x) if op == "softmax" else orc.logsoftmax(x))[0])
+    y = y.to(dtype)
+    dy = torch.randn(total, generator=g).to(dtype)
+    yb = canary_tensor(G + total + G, dtype)
+    yb[G:G + total] = y.cuda()
+    db = canary_tensor(G + total + G, dtype)
+    db[G:G + total] = dy.cuda()
+    xb = db if inplace else canary_tensor(G + total + G, dtype)
+    es = ESIZE[dtype]
+    offd = torch.from_numpy(off).cuda()
+    ws = rw.ragged_workspace(rows)
+    fn = rw.rowop_softmax_backward_ragged if op == "softmax" else rw.rowop_logsoftmax_backward_ragged
+    st = fn(yb.data_ptr() + G * es, db.data_ptr() + G * es, xb.data_ptr() + G * es,
+            offd.data_ptr(), rows, max_len, rw.dtype_code(dtype), ws.data_ptr(), ws.numel(),
+            torch.cuda.current_stream().cuda_stream)
+    assert st == 0, rw.STATUS.get(st, st)
+    return y, dy, xb, off, st
+
+
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
+@pytest.mark.parametrize("op", ["softmax", "logsoftmax"])
+@pytest.mark.parametrize("base_off", [0, 3])
+def test_backward_ragged(rw, op, dtype, base_off):
+    """Ragged softmax-family backward against the oracle row by row; rows of
+    every bucket (cluster-split ones included), empty and one-element rows,
+    rows at every alignment; nothing outside the rows is written."""
+    max_len = 70000
+    lens = _ragged_lengths(dtype, 60, 5, max_len)
+    y, dy, xb, off, _ = run_bwd_ragged(rw, op, dtype, lens, max_len, seed=9, base_off=base_off)
+    assert rw.check_status() == 0
+    dx = to_f64(xb[G:G + int(off[-1])])
+    for i, n in enumerate(lens):
+        if n == 0:
+            continue
+        a64 = y[off[i]:off[i + 1]].double().numpy()[None, :]
+        d64 = dy[off[i]:off[i + 1]].double().numpy()[None, :]
+        ref = (orc.softmax_backward if op == "softmax" else orc.logsoftmax_backward)(a64, d64)
+        check(dx[None, off[i]:off[i + 1]], ref, scales(op, a64, d64, None, 0)[0], dtype, R_COMP,
+              f"ragged {op} row {i} (len {n})")
+    assert is_canary(xb[:G + base_off]).all() and is_canary(xb[G + int(off[-1]):]).all()
+
+
+@pytest.mark.parametrize("op", ["softmax", "logsoftmax"])
+def test_backward_ragged_inplace_and_rejects(rw, op):
+    """dx written over dy; a row longer than max_len is skipped, left as it
+    was and flagged, while the other rows are still done."""
+    dtype = torch.float32
+    lens = np.array([5, 300, 2000, 9000, 40], dtype=np.int64)
+    y, dy, xb, off, _ = run_bwd_ragged(rw, op, dtype, lens, 8000, seed=2, inplace=True)
+    assert rw.check_status() == rw.ROWOP_ERR_BAD_OFFSETS
+    got = to_f64(xb[G:G + int(off[-1])])
+    # the 9000-element row is longer than max_len: its dy is untouched
+    assert np.array_equal(got[off[3]:off[4]], dy[off[3]:off[4]].double().numpy())
+    for i in (0, 1, 2, 4):
+        a64 = y[off[i]:off[i + 1]].double().numpy()[None, :]
+        d64 = dy[off[i]:off[i + 1]].double().numpy()[None, :]
+        ref = (orc.softmax_backward if op == "softmax" else orc.logsoftmax_backward)(a64, d64)
+        check(got[None, off[i]:off[i + 1]], ref, scales(op, a64, d64, None, 0)[0], dtype, R_COMP,
+              f"ragged {op} row {i}")
+
+
+def test_workload_ragged_softmax_backward(rw):
+    """The ragged softmax-backward workload at full size (32768 rows, lengths
+    up to 4096), y the oracle's forward of the workload's x rounded to fp32;
+    dx checked on every 64th row."""
+    from paper_2607_23089_gb300 import workloads as wl
+    case = wl.ragged_softmax_backward()
+    off = case.offsets.numpy()
+    y = torch.from_numpy(orc.softmax_ragged(case.x.double().numpy(), off, nthreads=8)).float()
+    offd = case.offsets.cuda()
+    dx = rw.softmax_backward_ragged(y.cuda(), case.dy.cuda(), offd, case.max_len)
+    assert rw.check_status() == 0
+    got = to_f64(dx)
+    for i in range(0, case.rows, 64):
+        a64 = y[off[i]:off[i + 1]].double().numpy()[None, :]
+        d64 = case.dy[off[i]:off[i + 1]].double().numpy()[None, :]
+        check(got[None, off[i]:off[i + 1]], orc.softmax_backward(a64, d64),
+              scales("softmax", a64, d64, None, 0)[0], torch.float32, R_COMP,
+              f"ragged softmax backward workload row {i}")
