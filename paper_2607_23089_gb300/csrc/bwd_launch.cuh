@@ -3,6 +3,7 @@
 // one translation unit per (operator, type) pair (bwd_instance.cu).
 #pragma once
 
+#include "bwd_call.h"
 #include "bwd_row.cuh"
 #include "launch_util.cuh"
 

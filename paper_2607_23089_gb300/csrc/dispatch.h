@@ -81,19 +81,6 @@ struct BwdCall {
   cudaStream_t stream;
 };
 
-// Backward pass of the softmax family over ragged rows (CSR offsets, the
-// same offsets index a = y, dy and dx); ws holds a classify plan.
-struct BwdRaggedCall {
-  int dtype;
-  const void *a;
-  const void *dy;
-  void *dx;
-  const int64_t *offsets;
-  int64_t rows, max_len;
-  void *ws;
-  cudaStream_t stream;
-};
-
 // Partial rows of dgamma / dbeta: the backward launch never runs more than
 // this many CTAs per SM (one partial row each).
 constexpr int kBwdMaxPartsPerSm = 8;

@@ -6,6 +6,7 @@
 #include <cstring>
 #include <mutex>
 
+#include "bwd_call.h"
 #include "classify.cuh"
 #include "common.cuh"
 #include "dispatch.h"
