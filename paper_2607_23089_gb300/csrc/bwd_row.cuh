@@ -16,14 +16,20 @@
 // statistics with a butterfly over its lanes, then (TPR > 32) through shared
 // memory in warp order, then (rows longer than one CTA holds) across the CTAs
 // of a thread-block cluster through distributed shared memory, in rank
-// order; every thread ends with the same row statistics.  The thread then
-// writes its dx chunks.  A thread owns the same columns in every row, so the
-// norms accumulate dgamma / dbeta in registers across all rows the team
-// processes; at the end the CTA sums its teams in team order and writes one
-// partial row per CTA (per cluster), and bwd_param_finalize_kernel sums the
-// partials in index order.  Nothing is atomic: the result is bitwise
-// reproducible for a given device (the number of partials follows the grid,
-// which follows the device's SM count).
+// order; every thread ends with the same row statistics (LayerNorm takes two
+// rounds: the mean, then the sums about it).  The thread then writes its dx
+// chunks.  A thread owns the same columns in every dense row, so the norms
+// keep gamma at those columns and the thread's dgamma / dbeta sums over all
+// rows the team processes in shared memory private to the thread; at the
+// end the CTA sums its teams in team order and writes one partial row per
+// CTA (per cluster), and bwd_param_finalize_kernel sums the partials in index
+// order.  Nothing is atomic: the result is bitwise reproducible for a given
+// device (the number of partials follows the grid, which follows the
+// device's SM count).
+//
+// Ragged rows (softmax family): the team walks one bucket's record list of a
+// classify plan, and each row's start, length and head offset are set per
+// row.
 #pragma once
 
 #include "common.cuh"
