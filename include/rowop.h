@@ -206,6 +206,49 @@ ROWOP_API int rowop_logsoftmax_backward_ragged(const void *y, const void *dy, vo
                                                int64_t max_len, rowop_dtype_t dtype, void *ws,
                                                size_t ws_bytes, cudaStream_t stream);
 
+/* LayerNorm / RMSNorm backward over ragged rows (§2.1's row-wise norms on
+ * the ragged layout above): row i is elements [offsets[i], offsets[i+1]) of
+ * x, dy and dx alike, and column j of every row uses gamma[j] (max_len
+ * elements, or NULL = ones).  dx of each row is the dense backward's, for a
+ * row of that length.  dgamma[j] (and, for LayerNorm, dbeta[j]) for
+ * j < max_len sums dy_j xhat_j (dy_j) over the rows longer than j: max_len
+ * elements of dtype each, or NULL when not wanted; rows == 0 sets them to
+ * zero.  Rows are read and written element by element, at any alignment.
+ *
+ * ws: device, 256-byte aligned, at least
+ * rowop_{layernorm,rmsnorm}_backward_ragged_workspace_size(rows, max_len,
+ * dtype) bytes on the current device: the classify plan, then one float32
+ * partial row per CTA for each row bucket, covering that bucket's longest
+ * row.  The partials of each bucket are added in index order, the buckets in
+ * order (SMALL, MEDIUM, LARGE), so the result is reproducible bit for bit on
+ * one device.  The workspace must not be shared by concurrent calls.
+ *
+ * max_len <= ROWOP_BWD_MAX_COLS_NORM (else ROWOP_ERR_TOO_LONG); rows longer
+ * than max_len or with decreasing offsets are skipped and flagged as in the
+ * forward ragged calls.  dx may be dy or x itself; partial overlap is
+ * undefined.  Errors: ROWOP_ERR_INVALID_ARG (NULL or misaligned pointer,
+ * rows < 0, max_len < 0, eps < 0), ROWOP_ERR_WORKSPACE,
+ * ROWOP_ERR_UNSUPPORTED_DTYPE, ROWOP_ERR_CUDA. */
+ROWOP_API int rowop_layernorm_backward_ragged(const void *x, const void *dy, const void *gamma,
+                                              void *dx, void *dgamma, void *dbeta,
+                                              const int64_t *offsets, int64_t rows,
+                                              int64_t max_len, rowop_dtype_t dtype, float eps,
+                                              void *ws, size_t ws_bytes, cudaStream_t stream);
+
+ROWOP_API int rowop_rmsnorm_backward_ragged(const void *x, const void *dy, const void *gamma,
+                                            void *dx, void *dgamma, const int64_t *offsets,
+                                            int64_t rows, int64_t max_len, rowop_dtype_t dtype,
+                                            float eps, void *ws, size_t ws_bytes,
+                                            cudaStream_t stream);
+
+/* Workspace bytes of a ragged norm backward call of `rows` rows up to
+ * max_len elements of dtype on the current device; 0 if an argument is
+ * invalid or the device cannot be queried. */
+ROWOP_API size_t rowop_layernorm_backward_ragged_workspace_size(int64_t rows, int64_t max_len,
+                                                                rowop_dtype_t dtype);
+ROWOP_API size_t rowop_rmsnorm_backward_ragged_workspace_size(int64_t rows, int64_t max_len,
+                                                              rowop_dtype_t dtype);
+
 /* Workspace bytes for dgamma (and dbeta) of rows of `cols` elements on the
  * current device; 0 if cols <= 0 or the device cannot be queried. */
 ROWOP_API size_t rowop_layernorm_backward_workspace_size(int64_t cols);

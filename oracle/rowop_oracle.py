@@ -343,3 +343,41 @@ def rmsnorm_backward(x, dy, gamma=None, eps=1e-6, nthreads=1):
     if rc != 0:
         raise MemoryError("oracle_rmsnorm_backward could not allocate its row statistics")
     return dx, dg
+
+
+def _ragged_norm_backward(dense_fn, x, dy, offsets, gamma, eps, nacc, nthreads):
+    """Row ``i`` of a ragged norm is the dense norm of ``x[off[i]:off[i+1]]``
+    with ``gamma[:len]``: its dx is the dense backward of that one row, and
+    the parameter gradients of column ``j`` add up, in row order, the rows
+    longer than ``j``.  Returns ``dx`` (packed like ``x``) and the ``nacc``
+    column sums, each of max_len entries."""
+    x = _f64(x).reshape(-1)
+    dy = _f64(dy).reshape(-1)
+    off = _offsets(offsets)
+    if x.shape != dy.shape or off[-1] > x.shape[0]:
+        raise ValueError("x and dy must be packed buffers of the same size holding every row")
+    n = _max_len(off)
+    g = _vec(gamma, max(n, 1), 1.0)
+    dx = np.zeros_like(x)
+    sums = [np.zeros(n, dtype=np.float64) for _ in range(nacc)]
+    for i in range(off.shape[0] - 1):
+        a, b = int(off[i]), int(off[i + 1])
+        if b == a:
+            continue
+        out = dense_fn(x[None, a:b], dy[None, a:b], g[:b - a], eps=eps, nthreads=nthreads)
+        dx[a:b] = out[0][0]
+        for s, part in zip(sums, out[1:]):
+            s[:b - a] += part
+    return (dx, *sums)
+
+
+def layernorm_backward_ragged(x, dy, offsets, gamma=None, eps=1e-5, nthreads=1):
+    """LayerNorm backward over ragged rows (gamma indexed by the column inside
+    the row).  Returns ``(dx, dgamma, dbeta)``, the last two of max_len
+    entries."""
+    return _ragged_norm_backward(layernorm_backward, x, dy, offsets, gamma, eps, 2, nthreads)
+
+
+def rmsnorm_backward_ragged(x, dy, offsets, gamma=None, eps=1e-6, nthreads=1):
+    """RMSNorm backward over ragged rows.  Returns ``(dx, dgamma)``."""
+    return _ragged_norm_backward(rmsnorm_backward, x, dy, offsets, gamma, eps, 1, nthreads)

@@ -53,19 +53,33 @@ inline bool bwd_shape(int64_t units, int cpt, int force_cs, int small_cta, BwdSh
 }
 
 template <typename T>
-cudaError_t launch_bwd_finalize(const float *part, int64_t nparts, int64_t cols, int nacc,
-                                void *dgamma, void *dbeta, cudaStream_t stream) {
+cudaError_t launch_bwd_finalize(const BwdSegments &sg, int64_t cols, int nacc, void *dgamma,
+                                void *dbeta, cudaStream_t stream) {
+  if (cols <= 0) return cudaSuccess;
   // a block per 32 columns, so many SMs share the reads, and 32 warps per
   // block over the partials, so each warp's chain of loads is short
   const dim3 grid(static_cast<unsigned>(ceil_div(cols, 32)), static_cast<unsigned>(nacc), 1);
   bwd_param_finalize_kernel<T><<<grid, kFinThreads, 0, stream>>>(
-      part, nparts, cols, nacc, static_cast<T *>(dgamma), static_cast<T *>(dbeta));
+      sg, cols, nacc, static_cast<T *>(dgamma), static_cast<T *>(dbeta));
   return cudaGetLastError();
 }
 
+// One segment of nparts partials covering all `cols` columns (a dense call).
+inline BwdSegments one_segment(const float *part, int64_t nparts, int64_t cols) {
+  BwdSegments sg = {};
+  sg.part[0] = part;
+  sg.nparts[0] = nparts;
+  sg.cover[0] = cols;
+  sg.n = 1;
+  return sg;
+}
+
+// Launches the team kernel; with partials wanted (p.part), either adds them
+// up into c.dgamma / c.dbeta (nparts_out NULL) or reports how many the
+// launch writes (nparts_out) for the caller to add up.
 template <int OP, typename T, int CPT, bool VEC, bool CLUSTER, bool RAGGED = false>
 cudaError_t launch_bwd_k(const BwdParams &p, const BwdShape &s, const BwdCall &c,
-                         const DeviceInfo &d) {
+                         const DeviceInfo &d, int64_t *nparts_out = nullptr) {
   auto kern = bwd_row_kernel<OP, T, CPT, VEC, CLUSTER, RAGGED>;
   const void *kp = reinterpret_cast<const void *>(kern);
   constexpr bool kNorm = (OP == kLayerNorm || OP == kRmsNorm);
@@ -129,7 +143,12 @@ cudaError_t launch_bwd_k(const BwdParams &p, const BwdShape &s, const BwdCall &c
   if (e != cudaSuccess) return e;
   e = cudaGetLastError();
   if (e != cudaSuccess || !p.part) return e;
-  return launch_bwd_finalize<T>(p.part, nparts, c.cols, p.nacc, c.dgamma, c.dbeta, c.stream);
+  if (nparts_out) {
+    *nparts_out = nparts;
+    return cudaSuccess;
+  }
+  return launch_bwd_finalize<T>(one_segment(p.part, nparts, c.cols), c.cols, p.nacc, c.dgamma,
+                                c.dbeta, c.stream);
 }
 
 template <int OP, typename T>
@@ -143,7 +162,8 @@ cudaError_t launch_bwd_t(const BwdCall &c, const DeviceInfo &d) {
   const bool want_params = kNorm && (c.dgamma || c.dbeta);
   if (c.rows == 0) {  // the parameter gradients of no rows are zero
     if (!want_params) return cudaSuccess;
-    return launch_bwd_finalize<T>(nullptr, 0, c.cols, nacc, c.dgamma, c.dbeta, c.stream);
+    return launch_bwd_finalize<T>(one_segment(nullptr, 0, c.cols), c.cols, nacc, c.dgamma,
+                                  c.dbeta, c.stream);
   }
   bool vec = ((c.ld * SZ) % 16 == 0) && congruent16(c.a, c.dy) && congruent16(c.a, c.dx);
   int h = vec ? static_cast<int>((reinterpret_cast<uintptr_t>(c.a) & 15u) / SZ) : 0;
@@ -182,20 +202,30 @@ cudaError_t launch_bwd_t(const BwdCall &c, const DeviceInfo &d) {
   return launch_bwd_k<OP, T, CPT, false, false>(p, s, c, d);
 }
 
-// Ragged backward (softmax family): the forward's classify pass sorts the
-// rows into three buckets by byte length; each bucket that max_len allows
-// gets one launch of the team kernel, shaped for the bucket's longest row,
-// which walks that bucket's list.  Rows are independent, so each row's
-// result depends only on its values, length and alignment and on the shape
-// of its bucket's teams.
+// Ragged backward: the forward's classify pass sorts the rows into three
+// buckets by byte length; each bucket that max_len allows gets one launch of
+// the team kernel, shaped for the bucket's longest row, which walks that
+// bucket's list.  Rows are independent, so each row's dx depends only on its
+// values, length and alignment and on the shape of its bucket's teams.  The
+// norms (element path) write each bucket's dgamma / dbeta partial rows into
+// that bucket's workspace segment, covering its longest row, and one
+// finalize adds the segments up in bucket order: the result depends on the
+// rows' lengths and the device, not on their order in memory.
 template <int OP, typename T>
 cudaError_t launch_bwd_ragged_t(const BwdRaggedCall &c, const DeviceInfo &d) {
-  if constexpr (OP == kLayerNorm || OP == kRmsNorm) {
-    return cudaErrorNotSupported;
-  } else {
-    constexpr int SZ = sizeof(T);
-    constexpr int E = 16 / SZ;
-    constexpr int CPT = kBwdSlots / E;
+  constexpr int SZ = sizeof(T);
+  constexpr int E = 16 / SZ;
+  constexpr int CPT = kBwdSlots / E;
+  constexpr bool kNorm = (OP == kLayerNorm || OP == kRmsNorm);
+  const int nacc = OP == kLayerNorm ? 2 : 1;
+  const bool want_params = kNorm && (c.dgamma || c.dbeta);
+  unsigned char *ws = static_cast<unsigned char *>(c.ws);
+  size_t seg_off[3] = {0, 0, 0};
+  if (kNorm) (void)bwd_ragged_layout(c.rows, c.max_len, SZ, nacc, d.sm_count, seg_off);
+  int64_t cover[3];
+  bwd_ragged_covers(c.max_len, SZ, cover);
+  BwdSegments sg = {};
+  if (c.rows > 0) {
     RaggedCall rc = {};
     rc.dtype = c.dtype;
     rc.offsets = c.offsets;
@@ -205,42 +235,43 @@ cudaError_t launch_bwd_ragged_t(const BwdRaggedCall &c, const DeviceInfo &d) {
     rc.stream = c.stream;
     rc.classify = true;
     cudaError_t e = launch_classify(rc, d);
-    if (e != cudaSuccess || c.max_len == 0) return e;
-    unsigned char *ws = static_cast<unsigned char *>(c.ws);
+    if (e != cudaSuccess) return e;
+  }
+  if (c.rows > 0 && c.max_len > 0) {
     const RowRec *list0 = reinterpret_cast<const RowRec *>(ws + ragged_lists_offset(c.rows));
-    const bool vec = congruent16(c.a, c.dy) && congruent16(c.a, c.dx);
+    const bool vec = !kNorm && congruent16(c.a, c.dy) && congruent16(c.a, c.dx);
     BwdParams p = {};
     p.a = c.a;
     p.dy = c.dy;
     p.dx = c.dx;
+    p.gamma = kNorm ? c.gamma : nullptr;
     p.rows = c.rows;  // an upper bound on every bucket's rows: sizes the grid
     p.ld = 0;
-    p.eps = 0.f;
-    p.nacc = 1;
+    p.eps = kNorm ? c.eps : 0.f;
+    p.nacc = nacc;
     p.timeout_ns = kWaitLimitNs;
     p.status = d.status;
     p.block_counts = reinterpret_cast<const int32_t *>(ws + ragged_counts_offset(c.rows));
     p.blocks = static_cast<int>(ragged_blocks(c.rows));
     p.rows_per_block = ragged_rows_per_block(c.rows);
-    const int64_t max_bytes = c.max_len * SZ;
+    const int small_cta = kNorm ? 128 : 256;
     for (int b = kSmall; b <= kLarge; ++b) {
-      const int64_t lo = b == kSmall ? 0 : (b == kMedium ? kSmallMaxBytes : kMediumMaxBytes);
-      if (max_bytes <= lo && b != kSmall) break;  // no row can be this long
-      const int64_t hi = b == kSmall ? std::min(max_bytes, kSmallMaxBytes)
-                                     : (b == kMedium ? std::min(max_bytes, kMediumMaxBytes) : max_bytes);
-      const int64_t longest = std::max<int64_t>(1, hi / SZ);
+      if (cover[b] == 0) continue;  // no row can be this long
+      const int64_t longest = cover[b];
       bool bvec = vec;
       BwdShape s;
-      if (!bwd_shape(bvec ? ceil_div(longest + E - 1, E) : ceil_div(longest, E), CPT, 0, 256, s)) {
+      if (!bwd_shape(bvec ? ceil_div(longest + E - 1, E) : ceil_div(longest, E), CPT, 0,
+                     small_cta, s)) {
         // the longest row, starting mid-chunk, needs a chunk more than the
         // largest cluster holds: this bucket takes the element path
         bvec = false;
-        if (!bwd_shape(ceil_div(longest, E), CPT, 0, 256, s)) return cudaErrorInvalidValue;
+        if (!bwd_shape(ceil_div(longest, E), CPT, 0, small_cta, s)) return cudaErrorInvalidValue;
       }
       p.list = list0 + static_cast<int64_t>(b) * c.rows;
       p.bucket = b;
       p.tpr = s.tpr;
       p.cols = longest;
+      p.part = want_params ? reinterpret_cast<float *>(ws + seg_off[b]) : nullptr;
       BwdCall bc = {};
       bc.dtype = c.dtype;
       bc.a = c.a;
@@ -249,7 +280,12 @@ cudaError_t launch_bwd_ragged_t(const BwdRaggedCall &c, const DeviceInfo &d) {
       bc.rows = c.rows;
       bc.cols = longest;
       bc.stream = c.stream;
-      if (s.cs > 1) {
+      int64_t np = 0;
+      cudaError_t e;
+      if constexpr (kNorm) {
+        e = s.cs > 1 ? launch_bwd_k<OP, T, CPT, false, true, true>(p, s, bc, d, &np)
+                     : launch_bwd_k<OP, T, CPT, false, false, true>(p, s, bc, d, &np);
+      } else if (s.cs > 1) {
         e = bvec ? launch_bwd_k<OP, T, CPT, true, true, true>(p, s, bc, d)
                  : launch_bwd_k<OP, T, CPT, false, true, true>(p, s, bc, d);
       } else {
@@ -257,9 +293,16 @@ cudaError_t launch_bwd_ragged_t(const BwdRaggedCall &c, const DeviceInfo &d) {
                  : launch_bwd_k<OP, T, CPT, false, false, true>(p, s, bc, d);
       }
       if (e != cudaSuccess) return e;
+      if (want_params) {
+        sg.part[sg.n] = p.part;
+        sg.nparts[sg.n] = np;
+        sg.cover[sg.n] = longest;
+        ++sg.n;
+      }
     }
-    return cudaSuccess;
   }
+  if (!want_params) return cudaSuccess;
+  return launch_bwd_finalize<T>(sg, c.max_len, nacc, c.dgamma, c.dbeta, c.stream);
 }
 
 }  // namespace rowop

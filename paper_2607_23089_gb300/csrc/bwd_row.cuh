@@ -27,9 +27,13 @@
 // device (the number of partials follows the grid, which follows the
 // device's SM count).
 //
-// Ragged rows (softmax family): the team walks one bucket's record list of a
-// classify plan, and each row's start, length and head offset are set per
-// row.
+// Ragged rows: the team walks one bucket's record list of a classify plan,
+// and each row's start, length and head offset are set per row.  The norms
+// take the element path there: a thread's columns are then counted from the
+// row's first element, whatever its alignment, so gamma and the dgamma /
+// dbeta sums stay at fixed columns across rows of any start.  The launch
+// covers the columns of its bucket's longest row (p.cols); a shorter row's
+// missing columns load as zero and add nothing.
 #pragma once
 
 #include "common.cuh"
@@ -48,7 +52,7 @@ struct BwdParams {
   void *dx;
   const void *gamma;  // norms; NULL = ones
   float *part;        // [nparts][nacc][cols] column partials (norms); NULL = not wanted
-  int64_t rows, cols, ld;
+  int64_t rows, cols, ld;  // ragged: cols = the columns the launch covers
   float eps;
   int tpr;   // threads of one CTA that share a row
   int h;     // VEC: head offset, in elements, of every row (a, dy and dx alike)
@@ -56,7 +60,7 @@ struct BwdParams {
   int nacc;  // partial rows per partial index: 2 (dgamma, dbeta) or 1 (dgamma)
   uint64_t timeout_ns;
   unsigned int *status;
-  // ragged (softmax family): the rows of one bucket of a classify plan
+  // ragged: the rows of one bucket of a classify plan
   const RowRec *list;           // that bucket's list: classify block b from entry b * rows_per_block
   const int32_t *block_counts;  // [blocks][3] rows per bucket of each classify block
   int blocks;
@@ -159,7 +163,7 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
   constexpr int S = CPT * E;  // elements per thread per tensor
   constexpr bool kNorm = (OP == kLayerNorm || OP == kRmsNorm);
   constexpr int NA = OP == kLayerNorm ? 2 : 1;
-  static_assert(!(RAGGED && kNorm), "ragged backward rows: softmax family only");
+  static_assert(!(RAGGED && kNorm && VEC), "ragged norm rows take the element path");
   __shared__ BwdShared sh;
   // dynamic (norms): gamma at this thread's columns ([CPT][NT] chunks), the
   // thread's dgamma / dbeta sums ([NA][S/4][NT] float4) -- both private to
@@ -189,8 +193,10 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
     // team's row count, so shuffles always see every lane
     warp_team0 = static_cast<int64_t>(blockIdx.x) * teams_cta + (TPR < 32 ? (warp * 32) / TPR : team);
   }
-  // row geometry: fixed for dense rows, set per row for ragged ones
-  int64_t cols = p.cols;
+  // row geometry: fixed for dense rows, set per row for ragged ones; pcols
+  // (the columns gamma and the partial rows cover) stays the launch's
+  const int64_t pcols = p.cols;
+  int64_t cols = pcols;
   int h = VEC ? p.h : 0;
   int nc = VEC ? p.nc : 0;
   int cf = (VEC && h > 0) ? 1 : 0;                                 // first full chunk
@@ -244,24 +250,28 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
     cluster_sync();  // every peer's barriers exist before any remote arrive
   }
 
-  // column of element e of this thread's chunk k, or -1 past the row
-  auto column = [&](int k, int e) -> int64_t {
+  // column of element e of this thread's chunk k, or -1 at or past `lim`:
+  // the row's length (column), or the launch's cover (pcolumn: gamma and the
+  // partial rows)
+  auto column_lim = [&](int k, int e, int64_t lim) -> int64_t {
     if constexpr (VEC) {
       const int c = (k * cs + rank) * TPR + tt;
       if (c >= nc) return -1;
       const int64_t j = static_cast<int64_t>(c) * E + e - h;
-      return (j >= 0 && j < cols) ? j : -1;
+      return (j >= 0 && j < lim) ? j : -1;
     } else {
       const int64_t j = (static_cast<int64_t>(k * E + e) * cs + rank) * TPR + tt;
-      return j < cols ? j : -1;
+      return j < lim ? j : -1;
     }
   };
+  auto column = [&](int k, int e) { return column_lim(k, e, cols); };
+  auto pcolumn = [&](int k, int e) { return column_lim(k, e, pcols); };
 
   const bool accum = kNorm && p.part != nullptr;
   uint4 *gsm = reinterpret_cast<uint4 *>(bwd_dyn);
   float4 *acc = reinterpret_cast<float4 *>(bwd_dyn + (kNorm ? CPT * NT * 16 : 0));
   float *red = reinterpret_cast<float *>(bwd_dyn + (kNorm ? CPT * NT * 16 : 0) +
-                                         (accum ? NA * S * NT * 4 : 0));
+                                         (accum ? NA * S * NT * 4 : 0));  // [NA][pcols]
   if constexpr (kNorm) {
     // gamma at this thread's columns, once for all rows; the sums start at 0
     const T *gamma = static_cast<const T *>(p.gamma);
@@ -270,7 +280,7 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
       float g[E];
 #pragma unroll
       for (int e = 0; e < E; ++e) {
-        const int64_t j = column(k, e);
+        const int64_t j = pcolumn(k, e);
         g[e] = (gamma && j >= 0) ? load_elem(gamma + j) : 1.f;
       }
       gsm[k * NT + tid] = pack<T>(g);
@@ -539,17 +549,17 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
     const int unit = TPR < 32 ? warp : team;
     const bool holder = TPR >= 32 || lane < TPR;
     const int64_t pidx = CLUSTER ? static_cast<int64_t>(cluster_id_x()) : static_cast<int64_t>(blockIdx.x);
-    float *prow = p.part + pidx * p.nacc * cols;
+    float *prow = p.part + pidx * p.nacc * pcols;
     if (units == 1) {
       if (holder) {
 #pragma unroll
         for (int k = 0; k < CPT; ++k)
 #pragma unroll
           for (int e = 0; e < E; ++e) {
-            const int64_t j = column(k, e);
+            const int64_t j = pcolumn(k, e);
             if (j < 0) continue;
 #pragma unroll
-            for (int a = 0; a < NA; ++a) prow[a * cols + j] = slot_sum(a, k * E + e);
+            for (int a = 0; a < NA; ++a) prow[a * pcols + j] = slot_sum(a, k * E + e);
           }
       }
       return;
@@ -561,30 +571,42 @@ __global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams
         for (int k = 0; k < CPT; ++k)
 #pragma unroll
           for (int e = 0; e < E; ++e) {
-            const int64_t j = column(k, e);
+            const int64_t j = pcolumn(k, e);
             if (j < 0) continue;
 #pragma unroll
             for (int a = 0; a < NA; ++a) {
               const float v = slot_sum(a, k * E + e);
-              red[a * cols + j] = u == 0 ? v : __fadd_rn(red[a * cols + j], v);
+              red[a * pcols + j] = u == 0 ? v : __fadd_rn(red[a * pcols + j], v);
             }
           }
       }
       __syncthreads();
     }
-    for (int64_t j = tid; j < NA * cols; j += NT) prow[j] = red[j];
+    for (int64_t j = tid; j < NA * pcols; j += NT) prow[j] = red[j];
   }
 }
 
-// dgamma[j] (dbeta[j]) = sum over the partials q = 0, 1, ... of
-// part[q][0 (1)][j]: a block per 32 columns, one column per lane; warp w adds
-// q = w, w + 32, ... in that order, U loads ahead, then the 32 warp sums are
-// added in warp order.
+// Partial rows to be summed into dgamma / dbeta: segment i holds nparts[i]
+// partials of nacc rows of cover[i] floats each (a dense call has one
+// segment; a ragged call one per row bucket, covering that bucket's longest
+// row).
+constexpr int kMaxBwdSegments = 3;
+struct BwdSegments {
+  const float *part[kMaxBwdSegments];
+  int64_t nparts[kMaxBwdSegments];
+  int64_t cover[kMaxBwdSegments];
+  int n;
+};
+
+// dgamma[j] (dbeta[j]) for j < cols = the sum over the segments in order of
+// each segment's sum over its partials q = 0, 1, ... of part[q][0 (1)][j]
+// (zero where j is past the segment's cover): a block per 32 columns, one
+// column per lane; warp w adds q = w, w + 32, ... in that order, U loads
+// ahead, then the 32 warp sums are added in warp order.
 constexpr int kFinThreads = 1024;
 constexpr int kFinWarps = kFinThreads / 32;
 template <typename T>
-__global__ void __launch_bounds__(kFinThreads) bwd_param_finalize_kernel(const float *part,
-                                                                         int64_t nparts,
+__global__ void __launch_bounds__(kFinThreads) bwd_param_finalize_kernel(const BwdSegments sg,
                                                                          int64_t cols, int nacc,
                                                                          T *dgamma, T *dbeta) {
   __shared__ float sums[kFinWarps][32];
@@ -594,28 +616,39 @@ __global__ void __launch_bounds__(kFinThreads) bwd_param_finalize_kernel(const f
   T *out = a == 0 ? dgamma : dbeta;
   if (out == nullptr) return;  // uniform over the block
   const int64_t j = static_cast<int64_t>(blockIdx.x) * 32 + lane;
-  float s = 0.f;
-  if (j < cols) {
-    constexpr int U = 8;
-    for (int64_t q0 = warp; q0 < nparts; q0 += kFinWarps * U) {
-      float x[U];
+  float total = 0.f;
+  bool first = true;
+  for (int i = 0; i < sg.n; ++i) {
+    const int64_t cover = sg.cover[i];
+    if (static_cast<int64_t>(blockIdx.x) * 32 >= cover) continue;  // uniform over the block
+    const float *part = sg.part[i];
+    const int64_t nparts = sg.nparts[i];
+    float s = 0.f;
+    if (j < cover) {
+      constexpr int U = 8;
+      for (int64_t q0 = warp; q0 < nparts; q0 += kFinWarps * U) {
+        float x[U];
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int64_t q = q0 + u * kFinWarps;
-        x[u] = q < nparts ? __ldcs(part + (q * nacc + a) * cols + j) : 0.f;
+        for (int u = 0; u < U; ++u) {
+          const int64_t q = q0 + u * kFinWarps;
+          x[u] = q < nparts ? __ldcs(part + (q * nacc + a) * cover + j) : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+          if (q0 + u * kFinWarps < nparts) s = __fadd_rn(s, x[u]);
       }
-#pragma unroll
-      for (int u = 0; u < U; ++u)
-        if (q0 + u * kFinWarps < nparts) s = __fadd_rn(s, x[u]);
+    }
+    __syncthreads();  // the previous segment's sums have been read
+    sums[warp][lane] = s;
+    __syncthreads();
+    if (warp == 0) {
+      float t = sums[0][lane];
+      for (int w = 1; w < kFinWarps; ++w) t = __fadd_rn(t, sums[w][lane]);
+      total = first ? t : __fadd_rn(total, t);
+      first = false;
     }
   }
-  sums[warp][lane] = s;
-  __syncthreads();
-  if (warp == 0 && j < cols) {
-    float t = sums[0][lane];
-    for (int w = 1; w < kFinWarps; ++w) t = __fadd_rn(t, sums[w][lane]);
-    out[j] = from_f32<T>(t);
-  }
+  if (warp == 0 && j < cols) out[j] = from_f32<T>(total);
 }
 
 }  // namespace rowop

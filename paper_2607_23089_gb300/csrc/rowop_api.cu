@@ -326,35 +326,67 @@ static int run_bwd(int op, const void *a, const void *dy, void *dx, const void *
   }
 }
 
-// Ragged backward passes (softmax family).  a = y.
-static int run_bwd_ragged(int op, const void *a, const void *dy, void *dx, const int64_t *offsets,
-                          int64_t rows, int64_t max_len, rowop_dtype_t dtype, void *ws,
+// Ragged backward passes.  a = y (softmax family) or x (norms).
+static int run_bwd_ragged(int op, const void *a, const void *dy, void *dx, const void *gamma,
+                          void *dgamma, void *dbeta, const int64_t *offsets, int64_t rows,
+                          int64_t max_len, rowop_dtype_t dtype, float eps, void *ws,
                           size_t ws_bytes, cudaStream_t stream) {
   const int es = esize_of(dtype);
+  const bool norm = (op == kLayerNorm || op == kRmsNorm);
   if (es == 0) return ROWOP_ERR_UNSUPPORTED_DTYPE;
   if (rows < 0 || rows > INT32_MAX - 1 || max_len < 0) return ROWOP_ERR_INVALID_ARG;
-  if (rows == 0) return ROWOP_OK;
-  if (!offsets || !elem_aligned(offsets, 8)) return ROWOP_ERR_INVALID_ARG;
-  if (!a || !dy || !dx || !elem_aligned(a, es) || !elem_aligned(dy, es) || !elem_aligned(dx, es))
+  if (norm && !eps_ok(eps)) return ROWOP_ERR_INVALID_ARG;
+  const bool want = norm && (dgamma || dbeta) && max_len > 0;
+  if (rows == 0 && !want) return ROWOP_OK;
+  if ((gamma && !elem_aligned(gamma, es)) || (dgamma && !elem_aligned(dgamma, es)) ||
+      (dbeta && !elem_aligned(dbeta, es)))
     return ROWOP_ERR_INVALID_ARG;
-  if (max_len > kBwdMaxColsSoftmax) return ROWOP_ERR_TOO_LONG;
+  if (rows > 0) {
+    if (!offsets || !elem_aligned(offsets, 8)) return ROWOP_ERR_INVALID_ARG;
+    if (!a || !dy || !dx || !elem_aligned(a, es) || !elem_aligned(dy, es) ||
+        !elem_aligned(dx, es))
+      return ROWOP_ERR_INVALID_ARG;
+  }
+  if (max_len > (norm ? kBwdMaxColsNorm : kBwdMaxColsSoftmax)) return ROWOP_ERR_TOO_LONG;
+  // every call holds at least the classify plan; the norms' partial rows
+  // follow it, sized by the device's SM count
   if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < ragged_ws_bytes(rows))
     return ROWOP_ERR_WORKSPACE;
   DeviceInfo d;
   const int st = device_info(&d);
   if (st != ROWOP_OK) return st;
+  if (norm && ws_bytes < bwd_ragged_layout(rows, max_len, es, op == kLayerNorm ? 2 : 1,
+                                           d.sm_count, nullptr))
+    return ROWOP_ERR_WORKSPACE;
   BwdRaggedCall c;
   c.dtype = dtype;
   c.a = a;
   c.dy = dy;
   c.dx = dx;
+  c.gamma = norm ? gamma : nullptr;
+  c.dgamma = norm ? dgamma : nullptr;
+  c.dbeta = op == kLayerNorm ? dbeta : nullptr;
+  c.eps = eps;
   c.offsets = offsets;
   c.rows = rows;
   c.max_len = max_len;
   c.ws = ws;
   c.stream = stream;
-  if (op == kSoftmax) return from_cuda(launch_bwd_ragged<kSoftmax>(c, d));
-  return from_cuda(launch_bwd_ragged<kLogSoftmax>(c, d));
+  switch (op) {
+    case kSoftmax: return from_cuda(launch_bwd_ragged<kSoftmax>(c, d));
+    case kLogSoftmax: return from_cuda(launch_bwd_ragged<kLogSoftmax>(c, d));
+    case kLayerNorm: return from_cuda(launch_bwd_ragged<kLayerNorm>(c, d));
+    default: return from_cuda(launch_bwd_ragged<kRmsNorm>(c, d));
+  }
+}
+
+static size_t bwd_ragged_workspace_size(int nacc, int64_t rows, int64_t max_len,
+                                        rowop_dtype_t dtype) {
+  const int es = esize_of(dtype);
+  if (es == 0 || rows < 0 || max_len < 0) return 0;
+  DeviceInfo d;
+  if (device_info(&d) != ROWOP_OK) return 0;
+  return bwd_ragged_layout(rows, max_len, es, nacc, d.sm_count, nullptr);
 }
 
 static size_t bwd_workspace_size(int nacc, int64_t cols) {
@@ -456,15 +488,42 @@ int rowop_rmsnorm_backward(const void *x, const void *dy, const void *gamma, voi
 int rowop_softmax_backward_ragged(const void *y, const void *dy, void *dx, const int64_t *offsets,
                                   int64_t rows, int64_t max_len, rowop_dtype_t dtype, void *ws,
                                   size_t ws_bytes, cudaStream_t stream) {
-  return run_bwd_ragged(kSoftmax, y, dy, dx, offsets, rows, max_len, dtype, ws, ws_bytes, stream);
+  return run_bwd_ragged(kSoftmax, y, dy, dx, nullptr, nullptr, nullptr, offsets, rows, max_len,
+                        dtype, 0.f, ws, ws_bytes, stream);
 }
 
 int rowop_logsoftmax_backward_ragged(const void *y, const void *dy, void *dx,
                                      const int64_t *offsets, int64_t rows, int64_t max_len,
                                      rowop_dtype_t dtype, void *ws, size_t ws_bytes,
                                      cudaStream_t stream) {
-  return run_bwd_ragged(kLogSoftmax, y, dy, dx, offsets, rows, max_len, dtype, ws, ws_bytes,
-                        stream);
+  return run_bwd_ragged(kLogSoftmax, y, dy, dx, nullptr, nullptr, nullptr, offsets, rows,
+                        max_len, dtype, 0.f, ws, ws_bytes, stream);
+}
+
+int rowop_layernorm_backward_ragged(const void *x, const void *dy, const void *gamma, void *dx,
+                                    void *dgamma, void *dbeta, const int64_t *offsets,
+                                    int64_t rows, int64_t max_len, rowop_dtype_t dtype,
+                                    float eps, void *ws, size_t ws_bytes, cudaStream_t stream) {
+  return run_bwd_ragged(kLayerNorm, x, dy, dx, gamma, dgamma, dbeta, offsets, rows, max_len,
+                        dtype, eps, ws, ws_bytes, stream);
+}
+
+int rowop_rmsnorm_backward_ragged(const void *x, const void *dy, const void *gamma, void *dx,
+                                  void *dgamma, const int64_t *offsets, int64_t rows,
+                                  int64_t max_len, rowop_dtype_t dtype, float eps, void *ws,
+                                  size_t ws_bytes, cudaStream_t stream) {
+  return run_bwd_ragged(kRmsNorm, x, dy, dx, gamma, dgamma, nullptr, offsets, rows, max_len,
+                        dtype, eps, ws, ws_bytes, stream);
+}
+
+size_t rowop_layernorm_backward_ragged_workspace_size(int64_t rows, int64_t max_len,
+                                                      rowop_dtype_t dtype) {
+  return bwd_ragged_workspace_size(2, rows, max_len, dtype);
+}
+
+size_t rowop_rmsnorm_backward_ragged_workspace_size(int64_t rows, int64_t max_len,
+                                                    rowop_dtype_t dtype) {
+  return bwd_ragged_workspace_size(1, rows, max_len, dtype);
 }
 
 size_t rowop_layernorm_backward_workspace_size(int64_t cols) { return bwd_workspace_size(2, cols); }

@@ -67,6 +67,12 @@ SIGNATURES = {
     "rowop_rmsnorm_backward": ([_P, _P, _P, _P, _P, _I64, _I64, _I64, _I, _F, _P, _SZ, _P], _I),
     "rowop_softmax_backward_ragged": ([_P, _P, _P, _P, _I64, _I64, _I, _P, _SZ, _P], _I),
     "rowop_logsoftmax_backward_ragged": ([_P, _P, _P, _P, _I64, _I64, _I, _P, _SZ, _P], _I),
+    "rowop_layernorm_backward_ragged": ([_P, _P, _P, _P, _P, _P, _P, _I64, _I64, _I, _F, _P,
+                                         _SZ, _P], _I),
+    "rowop_rmsnorm_backward_ragged": ([_P, _P, _P, _P, _P, _P, _I64, _I64, _I, _F, _P, _SZ, _P],
+                                      _I),
+    "rowop_layernorm_backward_ragged_workspace_size": ([_I64, _I64, _I], _SZ),
+    "rowop_rmsnorm_backward_ragged_workspace_size": ([_I64, _I64, _I], _SZ),
     "rowop_layernorm_backward_workspace_size": ([_I64], _SZ),
     "rowop_rmsnorm_backward_workspace_size": ([_I64], _SZ),
     "rowop_pad_scale": ([_P, _P, _I64, _I64, _I64, _I64, _I64, _F, _I, _P], _I),
@@ -417,6 +423,46 @@ def rmsnorm_backward(x, dy, gamma=None, eps=1e-6, want_dgamma=True, dx=None, dga
                                _ptr(ws), 0 if ws is None else ws.numel(), _stream(stream)),
         "rowop_rmsnorm_backward")
     return dx, dg
+
+
+def _ragged_norm_backward(x, dy, offsets, max_len, gamma, eps, want, given, dx, ws, stream,
+                          size_fn, call, name):
+    torch = _torch()
+    _check_cuda(x, dy, offsets, gamma, dx, ws, *given)
+    rows = offsets.numel() - 1
+    max_len = int(max_len)
+    dx = torch.empty_like(x) if dx is None else dx
+    outs = [g if g is not None else (torch.empty(max_len, dtype=x.dtype, device=x.device)
+                                     if w else None) for w, g in zip(want, given)]
+    code = dtype_code(x.dtype)
+    if ws is None:
+        ws = torch.empty(int(size_fn(rows, max_len, code)), dtype=torch.uint8, device=x.device)
+    _ok(call(x.data_ptr(), dy.data_ptr(), _ptr(gamma), dx.data_ptr(), *[_ptr(o) for o in outs],
+             offsets.data_ptr(), rows, max_len, code, float(eps), ws.data_ptr(), ws.numel(),
+             _stream(stream)), name)
+    return (dx, *outs)
+
+
+def layernorm_backward_ragged(x, dy, offsets, max_len, gamma=None, eps=1e-5, want_dgamma=True,
+                              want_dbeta=True, dx=None, dgamma=None, dbeta=None, ws=None,
+                              stream=None):
+    """LayerNorm backward over ragged rows (``rowop_layernorm_backward_ragged``):
+    returns ``(dx, dgamma, dbeta)``, dgamma / dbeta of max_len elements or
+    None when not wanted."""
+    return _ragged_norm_backward(
+        x, dy, offsets, max_len, gamma, eps, (want_dgamma, want_dbeta), (dgamma, dbeta), dx, ws,
+        stream, rowop_layernorm_backward_ragged_workspace_size,  # noqa: F821
+        rowop_layernorm_backward_ragged, "rowop_layernorm_backward_ragged")  # noqa: F821
+
+
+def rmsnorm_backward_ragged(x, dy, offsets, max_len, gamma=None, eps=1e-6, want_dgamma=True,
+                            dx=None, dgamma=None, ws=None, stream=None):
+    """RMSNorm backward over ragged rows (``rowop_rmsnorm_backward_ragged``):
+    returns ``(dx, dgamma)``."""
+    return _ragged_norm_backward(
+        x, dy, offsets, max_len, gamma, eps, (want_dgamma,), (dgamma,), dx, ws, stream,
+        rowop_rmsnorm_backward_ragged_workspace_size,  # noqa: F821
+        rowop_rmsnorm_backward_ragged, "rowop_rmsnorm_backward_ragged")  # noqa: F821
 
 
 def run(op: str, x, *, offsets=None, max_len=None, gamma=None, beta=None,

@@ -69,9 +69,9 @@ class Case:
             # read the forward input (norms) or output (softmax family) and dy,
             # write dx; norms also read gamma and write dgamma (and dbeta)
             b = 3 * self.elements * es
+            ncol = self.max_len if self.ragged else self.x.shape[1]
             if self.ragged:
-                return b + self.offsets.numel() * 8
-            ncol = self.x.shape[1]
+                b += self.offsets.numel() * 8
             if self.op == "layernorm_backward":
                 b += 3 * ncol * es
             elif self.op == "rmsnorm_backward":
@@ -252,6 +252,25 @@ def ragged_softmax_backward(rows: int = 32768, max_len: int = 4096, seed: int = 
                 max_len=max_len, dy=dy)
 
 
+def ragged_norm_backward(op: str = "layernorm", rows: int = 16384, max_len: int = 32768,
+                         seed: int = 11) -> Case:
+    """Backward of a norm over the ragged rows of workload 5: bf16 x drawn as
+    there (lengths uniform on {1..max_len}, a scale per row), dy = N(0,1),
+    gamma of max_len; the gradients are dx, dgamma (and dbeta for LayerNorm)
+    of max_len columns.  Not one of the five workloads."""
+    g = _gen(seed)
+    lengths = ragged_lengths(rows, max_len, g)
+    off = offsets_from_lengths(lengths)
+    total = int(off[-1])
+    x = torch.randn(total, generator=g)
+    scale = 0.1 + 9.9 * torch.rand(rows, generator=g)
+    x = (x * torch.repeat_interleave(scale, lengths)).to(torch.bfloat16)
+    dy = torch.randn(total, generator=g).to(torch.bfloat16)
+    gamma, _ = _affine(g, max_len, torch.bfloat16)
+    return Case(f"ragged_{op}_backward", f"{op}_backward", x, torch.bfloat16, offsets=off,
+                gamma=gamma, eps=1e-5 if op == "layernorm" else 1e-6, max_len=max_len, dy=dy)
+
+
 def all_cases(scale_down: int = 1):
     """The five workloads as a flat list of cases.  ``scale_down`` > 1 divides
     every row count (not the row lengths) for quicker runs."""
@@ -273,6 +292,8 @@ def all_cases(scale_down: int = 1):
     for op in ("softmax", "logsoftmax"):
         out.append(softmax_backward(op, rows=max(1, 32768 // s)))
     out.append(ragged_softmax_backward(rows=max(1, 32768 // s)))
+    for op in ("layernorm", "rmsnorm"):
+        out.append(ragged_norm_backward(op, rows=max(1, 16384 // s)))
     return out
 
 
@@ -282,6 +303,8 @@ def by_name(name: str) -> Case:
         return norm_backward(name[len("medium_norm_backward_"):])
     if name == "ragged_softmax_backward":
         return ragged_softmax_backward()
+    if name in ("ragged_layernorm_backward", "ragged_rmsnorm_backward"):
+        return ragged_norm_backward(name.split("_")[1])
     if name.startswith(("softmax_backward_", "logsoftmax_backward_")):
         op, _, cols = name.split("_")
         return softmax_backward(op, cols=int(cols))

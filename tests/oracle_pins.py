@@ -381,6 +381,43 @@ def pin_backward_finite_difference(orc):
     _close(dg, _fd_grad(lambda a: np.sum(dy * orc.rmsnorm(x, a, eps=eps)), g), **tol)
 
 
+def pin_backward_ragged_norms(orc):
+    """The ragged norm backward passes against central differences of the
+    (separately pinned) ragged forward oracle, on rows of lengths 4, 0, 7, 1
+    and 5 (an empty row, a one-element row, gamma columns reached by some rows
+    only): dx, and dgamma / dbeta of max_len entries, of the loss
+    sum(dy * f(x, gamma, beta)); then rows of one length, which must agree
+    with the dense backward."""
+    rng = np.random.default_rng(33)
+    lens = np.array([4, 0, 7, 1, 5])
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    total, n = int(off[-1]), int(lens.max())
+    x = rng.normal(0.4, 1.5, total)
+    dy = rng.normal(0.0, 1.0, total)
+    g = rng.normal(1.0, 0.3, n)
+    b = rng.normal(0.0, 0.3, n)
+    tol = dict(rtol=1e-6, atol=1e-8)
+    eps = float(np.float32(1e-5))
+    dx, dg, db = orc.layernorm_backward_ragged(x, dy, off, g, eps=eps)
+    ln = lambda xx, gg, bb: np.sum(dy * orc.layernorm_ragged(xx, off, gg, bb, eps=eps))  # noqa: E731
+    _close(dx, _fd_grad(lambda a: ln(a, g, b), x), **tol)
+    _close(dg, _fd_grad(lambda a: ln(x, a, b), g), **tol)
+    _close(db, _fd_grad(lambda a: ln(x, g, a), b), **tol)
+    eps = float(np.float32(1e-6))
+    dx, dg = orc.rmsnorm_backward_ragged(x, dy, off, g, eps=eps)
+    rms = lambda xx, gg: np.sum(dy * orc.rmsnorm_ragged(xx, off, gg, eps=eps))  # noqa: E731
+    _close(dx, _fd_grad(lambda a: rms(a, g), x), **tol)
+    _close(dg, _fd_grad(lambda a: rms(x, a), g), **tol)
+    # equal lengths: the dense backward of the same rows
+    xe = rng.normal(0.0, 2.0, (3, 6))
+    de = rng.normal(0.0, 1.0, (3, 6))
+    ge = rng.normal(1.0, 0.3, 6)
+    offe = np.arange(0, 19, 6, dtype=np.int64)
+    for got, exp in zip(orc.layernorm_backward_ragged(xe.reshape(-1), de.reshape(-1), offe, ge),
+                        orc.layernorm_backward(xe, de, ge)):
+        _close(got, exp.reshape(-1), rtol=1e-14, atol=1e-15)
+
+
 def pin_backward_invariants(orc):
     """Properties any correct backward pass has: softmax-family gradients sum
     to zero over a row; a constant upstream gradient gives no softmax
@@ -471,4 +508,4 @@ ALL_PINS = [pin_hand_cases, pin_softmax_invariants, pin_layernorm_invariants,
             pin_rmsnorm_invariants, pin_brute_force, pin_torch_float64,
             pin_ragged, pin_bucket_rule, pin_pad_scale, pin_moe_group_top2,
             pin_residual_norm, pin_backward_finite_difference, pin_backward_invariants,
-            pin_backward_torch]
+            pin_backward_torch, pin_backward_ragged_norms]

@@ -183,6 +183,61 @@ def test_backward_validation(lib):
     assert lib.rowop_rmsnorm_backward_workspace_size(-5) == 0
 
 
+def test_backward_ragged_norm_validation(lib):
+    """Argument checks of the ragged norm backward calls that come before any
+    device query (this host has no GPU)."""
+    F32, BF16 = lib.ROWOP_F32, lib.ROWOP_BF16
+    ln = lib.rowop_layernorm_backward_ragged
+    rms = lib.rowop_rmsnorm_backward_ragged
+    plan = lib.rowop_ragged_workspace_size(10)
+    # x, dy, gamma, dx, dgamma, dbeta, offsets, rows, max_len, dtype, eps, ws, ws_bytes, stream
+    assert ln(FAKE, FAKE, None, FAKE, FAKE, FAKE, FAKE, 10, 64, 7, 1e-5, FAKE, plan,
+              None) == lib.ROWOP_ERR_UNSUPPORTED_DTYPE
+    assert ln(FAKE, FAKE, None, FAKE, FAKE, FAKE, FAKE, -1, 64, F32, 1e-5, FAKE, plan,
+              None) == lib.ROWOP_ERR_INVALID_ARG
+    assert ln(FAKE, FAKE, None, FAKE, FAKE, FAKE, FAKE, 10, -1, F32, 1e-5, FAKE, plan,
+              None) == lib.ROWOP_ERR_INVALID_ARG
+    assert ln(FAKE, FAKE, None, FAKE, FAKE, FAKE, FAKE, 10, 64, F32, -1.0, FAKE, plan,
+              None) == lib.ROWOP_ERR_INVALID_ARG
+    # nothing to do: no rows and no parameter gradients (or none of any length)
+    assert ln(None, None, None, None, None, None, None, 0, 64, F32, 1e-5, None, 0,
+              None) == lib.ROWOP_OK
+    assert ln(None, None, None, None, FAKE, FAKE, None, 0, 0, F32, 1e-5, None, 0,
+              None) == lib.ROWOP_OK
+    # rows, or dgamma / dbeta to zero, need their pointers and a workspace
+    assert ln(FAKE, FAKE, None, FAKE, FAKE, FAKE, None, 10, 64, F32, 1e-5, FAKE, plan,
+              None) == lib.ROWOP_ERR_INVALID_ARG
+    assert ln(FAKE, None, None, FAKE, None, None, FAKE, 10, 64, F32, 1e-5, FAKE, plan,
+              None) == lib.ROWOP_ERR_INVALID_ARG
+    assert ln(FAKE + 1, FAKE, None, FAKE, None, None, FAKE, 10, 64, BF16, 1e-5, FAKE, plan,
+              None) == lib.ROWOP_ERR_INVALID_ARG
+    assert ln(FAKE, FAKE, FAKE + 2, FAKE, None, None, FAKE, 10, 64, F32, 1e-5, FAKE, plan,
+              None) == lib.ROWOP_ERR_INVALID_ARG
+    assert ln(FAKE, FAKE, None, FAKE, FAKE + 1, None, FAKE, 10, 64, BF16, 1e-5, FAKE, plan,
+              None) == lib.ROWOP_ERR_INVALID_ARG
+    assert ln(FAKE, FAKE, None, FAKE, FAKE, FAKE, FAKE, 10, 262145, F32, 1e-5, FAKE, plan,
+              None) == lib.ROWOP_ERR_TOO_LONG
+    assert ln(FAKE, FAKE, None, FAKE, FAKE, FAKE, FAKE, 10, 64, F32, 1e-5, FAKE, plan - 1,
+              None) == lib.ROWOP_ERR_WORKSPACE
+    assert ln(FAKE, FAKE, None, FAKE, FAKE, FAKE, FAKE, 10, 64, F32, 1e-5, FAKE + 16, plan,
+              None) == lib.ROWOP_ERR_WORKSPACE
+    assert ln(None, None, None, None, FAKE, FAKE, None, 0, 64, F32, 1e-5, None, 0,
+              None) == lib.ROWOP_ERR_WORKSPACE
+    # x, dy, gamma, dx, dgamma, offsets, rows, max_len, dtype, eps, ws, ws_bytes, stream
+    assert rms(FAKE, FAKE, None, FAKE, FAKE, FAKE, 10, 64, 9, 1e-6, FAKE, plan,
+               None) == lib.ROWOP_ERR_UNSUPPORTED_DTYPE
+    assert rms(FAKE, FAKE, None, FAKE, FAKE, None, 10, 64, F32, 1e-6, FAKE, plan,
+               None) == lib.ROWOP_ERR_INVALID_ARG
+    assert rms(FAKE, FAKE, None, FAKE, FAKE, FAKE, 10, 300000, F32, 1e-6, FAKE, plan,
+               None) == lib.ROWOP_ERR_TOO_LONG
+    assert rms(FAKE, FAKE, None, FAKE, FAKE, FAKE, 10, 64, F32, 1e-6, None, plan,
+               None) == lib.ROWOP_ERR_WORKSPACE
+    # the size queries reject bad arguments without a device
+    assert lib.rowop_layernorm_backward_ragged_workspace_size(-1, 64, F32) == 0
+    assert lib.rowop_rmsnorm_backward_ragged_workspace_size(10, -1, F32) == 0
+    assert lib.rowop_rmsnorm_backward_ragged_workspace_size(10, 64, 7) == 0
+
+
 def test_backward_ragged_validation(lib):
     F32 = lib.ROWOP_F32
     f = lib.rowop_softmax_backward_ragged
