@@ -246,6 +246,23 @@ def backward_call(torch, rw, case, x, device):
     once, outside the timed calls."""
     dy = case.dy.to(device)
     a = x
+    if case.ragged and case.op in ("layernorm_backward", "rmsnorm_backward"):
+        off = case.offsets.to(device)
+        g = case.gamma.to(device)
+        n = case.max_len
+        code = rw.dtype_code(x.dtype)
+        dx = torch.empty_like(x)
+        dg = torch.empty(n, dtype=x.dtype, device=device)
+        if case.op == "layernorm_backward":
+            db = torch.empty(n, dtype=x.dtype, device=device)
+            ws = torch.empty(rw.rowop_layernorm_backward_ragged_workspace_size(case.rows, n, code),
+                             dtype=torch.uint8, device=device)
+            return (lambda: rw.layernorm_backward_ragged(x, dy, off, n, g, case.eps, dx=dx,
+                                                         dgamma=dg, dbeta=db, ws=ws)), dx
+        ws = torch.empty(rw.rowop_rmsnorm_backward_ragged_workspace_size(case.rows, n, code),
+                         dtype=torch.uint8, device=device)
+        return (lambda: rw.rmsnorm_backward_ragged(x, dy, off, n, g, case.eps, dx=dx, dgamma=dg,
+                                                   ws=ws)), dx
     if case.ragged:  # softmax family over ragged rows
         off = case.offsets.to(device)
         ws = rw.ragged_workspace(case.rows, device)
@@ -288,7 +305,10 @@ def headline_kernel_stamp():
         with open(os.path.join(bld.CSRC, name), "rb") as f:
             h.update(name.encode())
             h.update(f.read())
-    h.update(" ".join(bld.NVCC_FLAGS).encode())
+    # include paths relative to the repository, so a checkout at another
+    # path (or on another machine) gives the same stamp
+    flags = [os.path.relpath(f, bld.ROOT) if os.path.isabs(f) else f for f in bld.NVCC_FLAGS]
+    h.update(" ".join(flags).encode())
     return h.hexdigest()
 
 
