@@ -217,6 +217,9 @@ cudaError_t launch_bwd_ragged_t(const BwdRaggedCall &c, const DeviceInfo &d) {
   constexpr int E = 16 / SZ;
   constexpr int CPT = kBwdSlots / E;
   constexpr bool kNorm = (OP == kLayerNorm || OP == kRmsNorm);
+  // the norms' element path holds half the slots: one register per element
+  // in flight (not one per two, as 16-byte chunks of 16-bit types take)
+  constexpr int kCptN = CPT / 2;
   const int nacc = OP == kLayerNorm ? 2 : 1;
   const bool want_params = kNorm && (c.dgamma || c.dbeta);
   unsigned char *ws = static_cast<unsigned char *>(c.ws);
@@ -260,12 +263,13 @@ cudaError_t launch_bwd_ragged_t(const BwdRaggedCall &c, const DeviceInfo &d) {
       const int64_t longest = cover[b];
       bool bvec = vec;
       BwdShape s;
-      if (!bwd_shape(bvec ? ceil_div(longest + E - 1, E) : ceil_div(longest, E), CPT, 0,
+      const int cpt = kNorm ? kCptN : CPT;
+      if (!bwd_shape(bvec ? ceil_div(longest + E - 1, E) : ceil_div(longest, E), cpt, 0,
                      small_cta, s)) {
         // the longest row, starting mid-chunk, needs a chunk more than the
         // largest cluster holds: this bucket takes the element path
         bvec = false;
-        if (!bwd_shape(ceil_div(longest, E), CPT, 0, small_cta, s)) return cudaErrorInvalidValue;
+        if (!bwd_shape(ceil_div(longest, E), cpt, 0, small_cta, s)) return cudaErrorInvalidValue;
       }
       p.list = list0 + static_cast<int64_t>(b) * c.rows;
       p.bucket = b;
@@ -283,8 +287,8 @@ cudaError_t launch_bwd_ragged_t(const BwdRaggedCall &c, const DeviceInfo &d) {
       int64_t np = 0;
       cudaError_t e;
       if constexpr (kNorm) {
-        e = s.cs > 1 ? launch_bwd_k<OP, T, CPT, false, true, true>(p, s, bc, d, &np)
-                     : launch_bwd_k<OP, T, CPT, false, false, true>(p, s, bc, d, &np);
+        e = s.cs > 1 ? launch_bwd_k<OP, T, kCptN, false, true, true>(p, s, bc, d, &np)
+                     : launch_bwd_k<OP, T, kCptN, false, false, true>(p, s, bc, d, &np);
       } else if (s.cs > 1) {
         e = bvec ? launch_bwd_k<OP, T, CPT, true, true, true>(p, s, bc, d)
                  : launch_bwd_k<OP, T, CPT, false, true, true>(p, s, bc, d);

@@ -156,8 +156,16 @@ __device__ __forceinline__ bool bwd_team_sum(float (&v)[NV], BwdShared &sh, BwdT
   return true;
 }
 
+// Ragged norm rows (element path, half the slots) are compiled for two
+// 512-thread CTAs per SM: twice the rows in flight per SM.
+template <int OP, bool RAGGED>
+constexpr int bwd_min_blocks() {
+  return (RAGGED && (OP == kLayerNorm || OP == kRmsNorm)) ? 2 : 1;
+}
+
 template <int OP, typename T, int CPT, bool VEC, bool CLUSTER, bool RAGGED = false>
-__global__ void __launch_bounds__(kBwdMaxThreads) bwd_row_kernel(const BwdParams p) {
+__global__ void __launch_bounds__(kBwdMaxThreads, bwd_min_blocks<OP, RAGGED>())
+    bwd_row_kernel(const BwdParams p) {
   constexpr int E = Elem<T>::kPerChunk;
   constexpr int SZ = Elem<T>::kSize;
   constexpr int S = CPT * E;  // elements per thread per tensor
