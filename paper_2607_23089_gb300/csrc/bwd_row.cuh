@@ -452,7 +452,9 @@ __global__ void __launch_bounds__(kBwdMaxThreads, bwd_min_blocks<OP, RAGGED>())
     // ---- dx, and this thread's dgamma / dbeta sums ----
     if (!active) continue;
     const f2 C0 = f2_bcast(c0), NC1 = f2_bcast(-c1), NC2 = f2_bcast(-c2);
-    const f2 NMC0 = f2_bcast(-__fmul_rn(mu, c0));  // xhat = x rstd - mu rstd
+    // xhat = (x - mu) rstd: x - mu is exact for x near mu, where x rstd -
+    // mu rstd would carry the rounding of mu rstd (large for |mu| >> std)
+    const f2 NMU = f2_bcast(-mu);
 #pragma unroll
     for (int k = 0; k < CPT; ++k) {
       if (msk[k] == 0u) continue;
@@ -480,7 +482,7 @@ __global__ void __launch_bounds__(kBwdMaxThreads, bwd_min_blocks<OP, RAGGED>())
           if constexpr (OP == kRmsNorm) {
             xh = f2_mul(x[i], C0);
           } else {
-            xh = f2_fma(x[i], C0, NMC0);
+            xh = f2_mul(f2_add(x[i], NMU), C0);
           }
           // rstd (g - mean(g) - xhat mean(g xhat)); RMSNorm has no mean(g)
           f2 t = OP == kRmsNorm ? f2_mul(d[i], g[i]) : f2_fma(d[i], g[i], NC1);

@@ -298,6 +298,32 @@ def test_backward_forced_cluster(rw, op, cs, monkeypatch):
         run_bwd(rw, op, torch.bfloat16, rows, cols, offs=(1, 1, 1), seed=cols + cs)
 
 
+@pytest.mark.parametrize("cols", [100, 4096, 40000])
+@pytest.mark.parametrize("mean,std", [(100.0, 1.0), (-5.0, 0.05)])
+def test_layernorm_backward_far_from_zero(rw, cols, mean, std):
+    """fp32 LayerNorm backward of rows whose mean is 100 times their spread
+    (several teams per CTA, one team per CTA, cluster-split rows): the row
+    statistics, merged pairwise from each thread's own, keep the full
+    tolerance (a one-pass E[x^2] - mean^2 would lose about 100^2 * 2^-24 of
+    the variance).  Far larger ratios are bounded by the fp32 mean itself,
+    whose rounding shifts every xhat by up to ulp(mean) / (2 std)."""
+    dtype = torch.float32
+    g = torch.Generator("cpu").manual_seed(cols)
+    x = (mean + std * torch.randn(6, cols, generator=g, dtype=torch.float64)).float()
+    dy = torch.randn(6, cols, generator=g)
+    gam = 1.0 + 0.2 * torch.randn(cols, generator=g)
+    dx, dg, db = rw.layernorm_backward(x.cuda(), dy.cuda(), gam.cuda(), 1e-5)
+    assert rw.check_status() == 0
+    a64, d64, g64 = x.double().numpy(), dy.double().numpy(), gam.double().numpy()
+    eps = float(np.float32(1e-5))
+    rdx, rdg, rdb = oracle("layernorm", a64, d64, g64, eps)
+    sdx, sdg, sdb = scales("layernorm", a64, d64, g64, eps)
+    what = f"layernorm far from zero (mean {mean}, std {std}, {cols} cols)"
+    check(to_f64(dx), rdx, sdx, dtype, R_COMP, what + " dx")
+    check(to_f64(dg), rdg, sdg, dtype, R_COMP_PARAM, what + " dgamma")
+    check(to_f64(db), rdb, sdb, dtype, R_COMP_PARAM, what + " dbeta")
+
+
 @pytest.mark.parametrize("op", OPS)
 def test_backward_deterministic(rw, op):
     outs = [run_bwd(rw, op, torch.bfloat16, 700, 5000, seed=5, compare=(i == 0)) for i in range(2)]
