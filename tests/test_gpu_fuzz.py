@@ -1,7 +1,7 @@
 """Randomised parity sweep through the C ABI: seeded random shapes, row
 strides, element offsets (16-byte congruent or not), dtypes, in-place calls
 and operators -- forward (dense and ragged, with a first offset other than 0)
-and the backward passes -- each checked against the double-precision oracle
+and the backward passes, dense and ragged -- each checked against the double-precision oracle
 with the tolerance its own tests use.  Every case is a pure function of its seed, so a
 failure names a reproducible case."""
 import numpy as np
@@ -195,6 +195,32 @@ def bwd_case(rw, seed):
         check(to_f64(dbt), rdb, sdb, dtype, R_COMP_PARAM, what + " dbeta")
 
 
+def ragged_bwd_case(rw, seed):
+    """Ragged LayerNorm / RMSNorm backward: random row count, lengths
+    log-uniform up to 70000 (empty rows included), a random first offset,
+    dtype, gamma present or not, which gradients are wanted, dx in place."""
+    from tests.test_gpu_backward_ragged_norm import call, make_inputs, reference, verify
+    g = np.random.default_rng(30_000 + seed)
+    op = ("layernorm", "rmsnorm")[seed % 2]
+    dtype = DTYPES[(seed // 2) % 3]
+    rows = int(g.integers(1, 40))
+    top = int(np.exp(g.uniform(0, np.log(70000))))
+    lens = np.minimum(top, np.exp(g.uniform(0, np.log(top + 1), rows)).astype(np.int64))
+    lens[g.random(rows) < 0.1] = 0
+    max_len = int(lens.max()) + int(g.integers(0, 50))
+    affine = g.random() < 0.8
+    x, dy, gam, off = make_inputs(dtype, lens, max_len, seed=seed, base_off=int(g.integers(0, 9)),
+                                  affine=affine)
+    want = (bool(g.random() < 0.8), bool(g.random() < 0.8))
+    inplace = (None, None, "dy", "x")[int(g.integers(0, 4))]
+    st, dxb, dgb, dbb = call(rw, op, dtype, x, dy, gam, off, max_len, inplace, want)
+    assert st == 0, (seed, rw.STATUS.get(st, st))
+    assert rw.check_status() == 0
+    dx_rows, params, ps = reference(op, x, dy, gam, off, max_len)
+    verify(op, dtype, dx_rows, params, ps, off, dxb, dgb, dbb, max_len,
+           f"seed {seed}: ragged {op} backward {dtype} rows {rows} max_len {max_len}")
+
+
 BATCH = 12
 
 
@@ -214,3 +240,9 @@ def test_fuzz_ragged_forward(rw, batch):
 def test_fuzz_backward(rw, batch):
     for seed in range(batch * BATCH, (batch + 1) * BATCH):
         bwd_case(rw, seed)
+
+
+@pytest.mark.parametrize("batch", range(8))
+def test_fuzz_ragged_norm_backward(rw, batch):
+    for seed in range(batch * BATCH, (batch + 1) * BATCH):
+        ragged_bwd_case(rw, seed)
