@@ -135,3 +135,47 @@ def test_pins_catch_mutant(tmp_path, func, old, new, what):
         except (AssertionError, ValueError, FloatingPointError) as e:
             caught.append(pin.__name__)
     assert caught, f"no pin caught the planted mistake: {what}"
+
+
+# Mistakes planted in the Python composition of the ragged norm backward
+# (rowop_oracle.py, _ragged_norm_backward): (text, replacement, what).
+RAGGED_BWD_MUTANTS = [
+    ("g[:b - a]", "g[1:b - a + 1]", "gamma taken one column late"),
+    ("s[:b - a] += part", "s[-(b - a):] += part", "column sums aligned to the row end"),
+    ("range(off.shape[0] - 1)", "range(off.shape[0] - 2)", "last row left out"),
+    ("zip(sums, out[1:])", "zip(sums, out[1:2])", "dbeta never summed"),
+    ("dx[a:b] = out[0][0]", "dx[a:b] = out[0][0][::-1]", "dx of a row reversed"),
+    ("if b == a:\n            continue", "if b - a < 2:\n            continue",
+     "one-element rows skipped"),
+]
+
+
+@pytest.mark.parametrize("old,new,what", RAGGED_BWD_MUTANTS,
+                         ids=[m[2].replace(" ", "_") for m in RAGGED_BWD_MUTANTS])
+def test_pins_catch_ragged_backward_mutant(tmp_path, old, new, what):
+    """The composition is Python, so the mutant is an edited copy of the
+    wrapper that loads the real (unmodified) compiled oracle."""
+    from oracle import rowop_oracle as real
+    real.build()
+    with open(WRAPPER) as f:
+        text = f.read()
+    start = text.index("def _ragged_norm_backward(")
+    end = text.index("\ndef ", start + 1)
+    body = text[start:end]
+    assert old in body, old
+    path = tmp_path / "oracle_ragged_mutant.py"
+    path.write_text(text[:start] + body.replace(old, new, 1) + text[end:])
+    spec = importlib.util.spec_from_file_location("oracle_ragged_mutant", str(path))
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    mod._SRCS = real._SRCS
+    mod._BUILD_DIR = real._BUILD_DIR
+    mod._LIB_PATH = real._LIB_PATH
+    mod._lib = None
+    caught = []
+    for pin in ALL_PINS:
+        try:
+            pin(mod)
+        except (AssertionError, ValueError, FloatingPointError):
+            caught.append(pin.__name__)
+    assert caught, f"no pin caught the planted mistake: {what}"
