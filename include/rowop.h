@@ -169,6 +169,7 @@ ROWOP_API int rowop_add_rmsnorm(const void *x, const void *r, void *sum_out, voi
  * ROWOP_ERR_WORKSPACE, ROWOP_ERR_UNSUPPORTED_DTYPE, ROWOP_ERR_CUDA.        */
 #define ROWOP_BWD_MAX_COLS_SOFTMAX 262144
 #define ROWOP_BWD_MAX_COLS_NORM 262144
+#define ROWOP_BWD_MAX_COLS_NORM_RAGGED 131072
 
 ROWOP_API int rowop_softmax_backward(const void *y, const void *dy, void *dx, int64_t rows,
                                      int64_t cols, int64_t ld, rowop_dtype_t dtype,
@@ -223,7 +224,7 @@ ROWOP_API int rowop_logsoftmax_backward_ragged(const void *y, const void *dy, vo
  * order (SMALL, MEDIUM, LARGE), so the result is reproducible bit for bit on
  * one device.  The workspace must not be shared by concurrent calls.
  *
- * max_len <= ROWOP_BWD_MAX_COLS_NORM (else ROWOP_ERR_TOO_LONG); rows longer
+ * max_len <= ROWOP_BWD_MAX_COLS_NORM_RAGGED (else ROWOP_ERR_TOO_LONG); rows longer
  * than max_len or with decreasing offsets are skipped and flagged as in the
  * forward ragged calls.  dx may be dy or x itself; partial overlap is
  * undefined.  Errors: ROWOP_ERR_INVALID_ARG (NULL or misaligned pointer,

@@ -28,6 +28,11 @@ struct BwdRaggedCall {
   cudaStream_t stream;
 };
 
+// Longest ragged row of the norms' backward: the element path holds 16
+// elements per thread per tensor, in teams of up to 16 CTAs of 512 threads
+// (checked against those constants in bwd_launch.cuh).
+constexpr int64_t kBwdMaxColsNormRagged = 131072;
+
 // Columns covered by the launch of each row bucket (SMALL, MEDIUM, LARGE) of
 // rows up to max_len elements of esize bytes: the bucket's longest row, or 0
 // when no row can fall in the bucket.

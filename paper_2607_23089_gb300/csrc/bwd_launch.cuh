@@ -220,6 +220,9 @@ cudaError_t launch_bwd_ragged_t(const BwdRaggedCall &c, const DeviceInfo &d) {
   // the norms' element path holds half the slots: one register per element
   // in flight (not one per two, as 16-byte chunks of 16-bit types take)
   constexpr int kCptN = CPT / 2;
+  static_assert(static_cast<int64_t>(kCptN) * E * kBwdMaxThreads * kMaxCluster ==
+                    kBwdMaxColsNormRagged,
+                "the longest ragged norm row one team can hold");
   const int nacc = OP == kLayerNorm ? 2 : 1;
   const bool want_params = kNorm && (c.dgamma || c.dbeta);
   unsigned char *ws = static_cast<unsigned char *>(c.ws);

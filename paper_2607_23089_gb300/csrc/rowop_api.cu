@@ -347,7 +347,7 @@ static int run_bwd_ragged(int op, const void *a, const void *dy, void *dx, const
         !elem_aligned(dx, es))
       return ROWOP_ERR_INVALID_ARG;
   }
-  if (max_len > (norm ? kBwdMaxColsNorm : kBwdMaxColsSoftmax)) return ROWOP_ERR_TOO_LONG;
+  if (max_len > (norm ? kBwdMaxColsNormRagged : kBwdMaxColsSoftmax)) return ROWOP_ERR_TOO_LONG;
   // every call holds at least the classify plan; the norms' partial rows
   // follow it, sized by the device's SM count
   if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < ragged_ws_bytes(rows))

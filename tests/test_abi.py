@@ -230,6 +230,12 @@ def test_backward_ragged_norm_validation(lib):
                None) == lib.ROWOP_ERR_INVALID_ARG
     assert rms(FAKE, FAKE, None, FAKE, FAKE, FAKE, 10, 300000, F32, 1e-6, FAKE, plan,
                None) == lib.ROWOP_ERR_TOO_LONG
+    # one team holds at most 131072 elements of a ragged norm row
+    for dtype in (F32, BF16):
+        assert ln(FAKE, FAKE, None, FAKE, FAKE, FAKE, FAKE, 10, 131073, dtype, 1e-5, FAKE, plan,
+                  None) == lib.ROWOP_ERR_TOO_LONG
+        assert ln(FAKE, FAKE, None, FAKE, FAKE, FAKE, FAKE, 10, 131072, dtype, 1e-5, FAKE,
+                  plan - 1, None) == lib.ROWOP_ERR_WORKSPACE
     assert rms(FAKE, FAKE, None, FAKE, FAKE, FAKE, 10, 64, F32, 1e-6, None, plan,
                None) == lib.ROWOP_ERR_WORKSPACE
     # the size queries reject bad arguments without a device

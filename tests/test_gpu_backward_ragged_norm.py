@@ -142,10 +142,11 @@ def test_ragged_norm_backward(rw, op, dtype, base_off):
 
 
 @pytest.mark.parametrize("op", ["layernorm", "rmsnorm"])
-@pytest.mark.parametrize("max_len", [1, 40, 2048, 2049, 16384, 16385, 100000])
+@pytest.mark.parametrize("max_len", [1, 40, 2048, 2049, 16384, 16385, 100000, 131072])
 def test_ragged_norm_backward_bucket_edges(rw, op, max_len):
     """max_len at and around the bucket edges of bf16 (launch covers of one,
-    two or three buckets), rows up to max_len."""
+    two or three buckets) and at the longest ragged norm row, rows up to
+    max_len."""
     dtype = torch.bfloat16
     g = np.random.default_rng(max_len)
     lens = np.minimum(max_len, g.integers(0, max_len + 1, 24)).astype(np.int64)
