@@ -3,7 +3,7 @@
  * operators the paper traces: the Hyena FFT-size padding operator and the
  * MoE group score.
  *
- * TEST INFRASTRUCTURE ONLY.  This file is part of the checker, not the
+ * TEST INFRASTRUCTURE ONLY.  This file is part of the oracle, not the
  * product: only the test suite, the smoke check and the benchmark's
  * CPU-baseline leg may load it.  It shares no code, header, table or constant
  * with the CUDA library, and it never includes anything from it.

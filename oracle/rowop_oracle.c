@@ -3,7 +3,7 @@
  * reduce-then-normalise operator family (softmax, log-softmax, LayerNorm,
  * RMSNorm) over dense rows and over ragged rows given by CSR offsets.
  *
- * TEST INFRASTRUCTURE ONLY.  This file is the checker, not the product: only
+ * TEST INFRASTRUCTURE ONLY.  This file is the oracle, not the product: only
  * the test suite, the smoke check and the benchmark's CPU-baseline leg may
  * load it.  It shares no code, header, table or constant with the CUDA
  * library, and it never includes anything from it.

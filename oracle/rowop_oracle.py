@@ -1,6 +1,6 @@
 """Python face of the double-precision CPU oracle (``rowop_oracle.c``).
 
-TEST INFRASTRUCTURE ONLY.  This module is the checker the CUDA library is
+TEST INFRASTRUCTURE ONLY.  This module is the oracle the CUDA library is
 compared against.  Only the test suite, ``__graft_entry__.smoke()`` and the
 benchmark's CPU-baseline / reference leg may import it; the product path
 (``paper_2607_23089_gb300``) never does, and this module never imports the
