@@ -257,3 +257,46 @@ def test_backward_ragged_validation(lib):
     assert f(FAKE, FAKE, FAKE, FAKE, 10, 64, F32, FAKE, ws_need - 1, None) == lib.ROWOP_ERR_WORKSPACE
     g = lib.rowop_logsoftmax_backward_ragged
     assert g(FAKE, FAKE, FAKE, FAKE, 10, -1, F32, FAKE, ws_need, None) == lib.ROWOP_ERR_INVALID_ARG
+
+
+C_CLIENT = r"""
+#include <stdio.h>
+#include <string.h>
+#include "rowop.h"
+
+/* A plain C99 client of the ABI: only calls that need no device. */
+int main(void) {
+    if (rowop_select_bucket(1024, ROWOP_F32) != ROWOP_SMALL) return 1;
+    if (rowop_select_bucket(1025, ROWOP_F32) != ROWOP_MEDIUM) return 2;
+    if (rowop_select_bucket(16385, ROWOP_BF16) != ROWOP_LARGE) return 3;
+    if (rowop_max_row_len(ROWOP_BF16) < 2 * (int64_t)262144 - 8) return 4;
+    if (strlen(rowop_status_string(ROWOP_ERR_TOO_LONG)) == 0) return 5;
+    if (rowop_softmax(NULL, NULL, -1, 8, 8, ROWOP_F32, NULL) != ROWOP_ERR_INVALID_ARG) return 6;
+    if (rowop_layernorm(NULL, NULL, NULL, NULL, 4, 8, 8, (rowop_dtype_t)9, 1e-5f, NULL) !=
+        ROWOP_ERR_UNSUPPORTED_DTYPE)
+        return 7;
+    if (rowop_softmax(NULL, NULL, 0, 8, 8, ROWOP_F32, NULL) != ROWOP_OK) return 8;
+    puts("ok");
+    return 0;
+}
+"""
+
+
+def test_plain_c_client(tmp_path, lib):
+    """include/rowop.h compiles as strict C99 and a C program links
+    librowop.so and gets the documented answers from the device-free calls."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "client.c"
+    src.write_text(C_CLIENT)
+    exe = tmp_path / "client"
+    libdir = os.path.dirname(lib.LIB_PATH)
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-I", inc,
+                    str(src), "-o", str(exe), "-L", libdir, "-l:librowop.so",
+                    f"-Wl,-rpath,{libdir}"], check=True)
+    r = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
+    assert r.returncode == 0 and r.stdout.strip() == "ok", (r.returncode, r.stdout, r.stderr)
