@@ -1,0 +1,135 @@
+// host_rules.cu -- the launch code's host-side rules, checked exhaustively on
+// the CPU (no device is touched): the backward team shapes, the ragged
+// workspace offsets, the ragged norm backward's bucket covers and partial-row
+// segments, and the longest ragged norm row.  Built and run by
+// tests/test_host_rules.py; prints "ok" and exits 0 when every check holds.
+#include <cstdio>
+#include <initializer_list>
+
+#include "bwd_launch.cuh"
+
+using namespace rowop;
+
+static int g_fails = 0;
+#define CHECK(cond, fmt, ...)                                                   \
+  do {                                                                          \
+    if (!(cond)) {                                                              \
+      if (g_fails++ < 20)                                                       \
+        std::printf("FAIL line %d: %s | " fmt "\n", __LINE__, #cond, __VA_ARGS__); \
+    }                                                                           \
+  } while (0)
+
+static bool pow2(int64_t v) { return v > 0 && (v & (v - 1)) == 0; }
+
+// Team shapes: a team (tpr threads of each of cs CTAs, cpt slots a thread)
+// covers the row's units; lane groups are powers of two filling a CTA of
+// small_cta threads; warp teams are whole warps; CTAs stay within 512
+// threads; clusters are powers of two up to 16; a forced split is honoured
+// whenever its CTAs fit; the rule refuses only rows no 16-CTA team can hold.
+static void check_shapes() {
+  for (int cpt : {2, 4, 8})
+    for (int small : {128, 256})
+      for (int force : {0, 2, 4, 8, 16})
+        for (int64_t units = 1; units <= 8192LL * cpt + 64; units += units < 4096 ? 1 : 29) {
+          BwdShape s{};
+          const bool ok = bwd_shape(units, cpt, force, small, s);
+          const int64_t need = (units + cpt - 1) / cpt;
+          CHECK(ok == (need <= 8192), "units %lld cpt %d force %d", (long long)units, cpt, force);
+          if (!ok) continue;
+          CHECK(s.cs >= 1 && s.cs <= kMaxCluster && pow2(s.cs), "cs %d", s.cs);
+          CHECK(s.nt >= 1 && s.nt <= kBwdMaxThreads && s.nt % s.tpr == 0, "nt %d tpr %d", s.nt,
+                s.tpr);
+          if (s.tpr < 32) {
+            CHECK(pow2(s.tpr) && s.nt == small && s.cs == 1, "tpr %d nt %d cs %d", s.tpr, s.nt,
+                  s.cs);
+          } else {
+            CHECK(s.tpr % 32 == 0 && s.tpr <= kBwdMaxThreads, "tpr %d", s.tpr);
+          }
+          if (s.cs > 1) CHECK(s.nt == s.tpr, "a cluster CTA is one team: nt %d tpr %d", s.nt, s.tpr);
+          CHECK(static_cast<int64_t>(s.tpr) * s.cs * cpt >= units, "units %lld tpr %d cs %d",
+                (long long)units, s.tpr, s.cs);
+          const int64_t per = (need + force - 1) / (force > 0 ? force : 1);
+          if (force >= 2 && per <= kBwdMaxThreads)
+            CHECK(s.cs == force, "forced %d got %d", force, s.cs);
+        }
+}
+
+// Ragged workspace: the regions follow each other, 256-byte aligned, each
+// large enough; the classify blocks cover every row.
+static void check_ragged_workspace() {
+  for (int64_t rows : {0LL, 1LL, 7LL, 1023LL, 1024LL, 1025LL, 16384LL, 262144LL, 262145LL,
+                       1000000LL, 2147483646LL}) {
+    const int64_t blocks = ragged_blocks(rows), rpb = ragged_rows_per_block(rows);
+    CHECK(blocks >= 1 && blocks <= kClassifyMaxBlocks, "rows %lld blocks %lld", (long long)rows,
+          (long long)blocks);
+    CHECK(blocks * rpb >= rows, "rows %lld", (long long)rows);
+    const size_t co = ragged_counts_offset(rows), lo = ragged_lists_offset(rows);
+    CHECK(co % 256 == 0 && co >= kWsBuckets + static_cast<size_t>(rows), "rows %lld",
+          (long long)rows);
+    CHECK(lo % 256 == 0 && lo >= co + 12 * static_cast<size_t>(blocks), "rows %lld",
+          (long long)rows);
+    CHECK(ragged_ws_bytes(rows) >= lo + 3 * kWsRecordBytes * static_cast<size_t>(rows),
+          "rows %lld", (long long)rows);
+  }
+}
+
+// Ragged norm backward: every row of every bucket fits its bucket's cover;
+// the covers' segments follow the classify plan, 256-byte aligned, disjoint,
+// each with room for the partial rows the launch may write.
+static void check_ragged_norm_layout() {
+  for (int es : {2, 4})
+    for (int64_t max_len : {0LL, 1LL, 40LL, 1024LL, 1025LL, 2048LL, 2049LL, 8192LL, 8193LL,
+                            16384LL, 16385LL, 70000LL, 131072LL})
+      for (int nacc : {1, 2})
+        for (int sm : {1, 148, 152}) {
+          int64_t cover[3];
+          bwd_ragged_covers(max_len, es, cover);
+          CHECK(cover[kSmall] >= 1, "max_len %lld", (long long)max_len);
+          for (int64_t n : std::initializer_list<int64_t>{1, max_len / 3, max_len / 2, max_len - 1,
+                                                          max_len}) {
+            if (n < 1 || n > max_len) continue;
+            CHECK(cover[bucket_of(n, es)] >= n, "row %lld of max_len %lld es %d", (long long)n,
+                  (long long)max_len, es);
+          }
+          CHECK(cover[kLarge] == (max_len * es > kMediumMaxBytes ? max_len : 0), "max_len %lld",
+                (long long)max_len);
+          for (int64_t rows : {1LL, 1000LL, 16384LL}) {
+            size_t seg[3];
+            const size_t total = bwd_ragged_layout(rows, max_len, es, nacc, sm, seg);
+            CHECK(seg[0] >= ragged_ws_bytes(rows), "rows %lld", (long long)rows);
+            for (int b = 0; b < 3; ++b) {
+              const size_t need = static_cast<size_t>(kBwdMaxPartsPerSm) * sm * nacc *
+                                  static_cast<size_t>(cover[b]) * sizeof(float);
+              const size_t next = b < 2 ? seg[b + 1] : total;
+              CHECK(seg[b] % 256 == 0 && seg[b] + need <= next, "bucket %d rows %lld", b,
+                    (long long)rows);
+            }
+            CHECK(total == bwd_ragged_layout(rows, max_len, es, nacc, sm, nullptr), "%s", "");
+          }
+        }
+}
+
+// The longest ragged norm row is the longest row a team of half-slot
+// threads can hold; one element more is refused by the shape rule.
+static void check_ragged_norm_limit() {
+  for (int es : {2, 4}) {
+    const int e = 16 / es;
+    const int cpt = kBwdSlots / e / 2;
+    BwdShape s{};
+    CHECK(bwd_shape((kBwdMaxColsNormRagged + e - 1) / e, cpt, 0, 128, s), "es %d", es);
+    CHECK(!bwd_shape((kBwdMaxColsNormRagged + 1 + e - 1) / e, cpt, 0, 128, s), "es %d", es);
+  }
+}
+
+int main() {
+  check_shapes();
+  check_ragged_workspace();
+  check_ragged_norm_layout();
+  check_ragged_norm_limit();
+  if (g_fails) {
+    std::printf("%d checks failed\n", g_fails);
+    return 1;
+  }
+  std::printf("ok\n");
+  return 0;
+}
