@@ -7,6 +7,7 @@
 #include <initializer_list>
 
 #include "bwd_launch.cuh"
+#include "launchers.cuh"
 
 using namespace rowop;
 
@@ -121,7 +122,43 @@ static void check_ragged_norm_limit() {
   }
 }
 
+// Forward tile design: the longest accepted row fits the largest cluster's
+// portions at every head offset (one element more does not at the last
+// offset), and the cluster chosen for a K-tile row is the smallest power of
+// two whose portions hold at most `cap` tiles.
+static void check_forward_rules() {
+  for (int es : {2, 4}) {
+    const int64_t e = 16 / es;
+    const int64_t n = max_row_len_elems(es);
+    const int64_t capacity = static_cast<int64_t>(kMaxPortionTiles) * kMaxCluster;
+    for (int64_t h = 0; h < e; ++h) {
+      const int64_t k = ((h + n + e - 1) / e + kTileChunks - 1) / kTileChunks;
+      CHECK(k <= capacity, "es %d head %lld tiles %lld", es, (long long)h, (long long)k);
+    }
+    const int64_t k1 = ((e - 1 + n + 1 + e - 1) / e + kTileChunks - 1) / kTileChunks;
+    CHECK(k1 > capacity, "es %d: one element more still fits", es);
+  }
+  for (int64_t cap : {1LL, 12LL, 96LL, 192LL})
+    for (int64_t k = 1; k <= cap * kMaxCluster; ++k) {
+      const int cs = pick_cluster(k, cap, 0);
+      CHECK(pow2(cs) && cs >= 2 && cs <= kMaxCluster, "cs %d", cs);
+      CHECK(ceil_div(k, cs) <= cap, "k %lld cap %lld cs %d", (long long)k, (long long)cap, cs);
+      CHECK(cs == 2 || ceil_div(k, cs / 2) > cap, "k %lld cap %lld cs %d not smallest",
+            (long long)k, (long long)cap, cs);
+    }
+  for (int w : {1, 2, 4, 8})
+    for (int64_t tiles : {1LL, 4LL, 16LL, 17LL, 32LL, 64LL, 72LL, 192LL}) {
+      const int g = kConsumerWarps / w;
+      const int st = pick_stages(tiles, w, 0);
+      CHECK(st >= g, "stages %d for %d groups", st, g);
+      if (static_cast<int64_t>(g) * tiles * kTileBytes <= kStageBudgetBytes)
+        CHECK(static_cast<int64_t>(st) * tiles * kTileBytes <= kStageBudgetBytes,
+              "stages %d of %lld tiles over the budget", st, (long long)tiles);
+    }
+}
+
 int main() {
+  check_forward_rules();
   check_shapes();
   check_ragged_workspace();
   check_ragged_norm_layout();
