@@ -472,6 +472,18 @@ def run(op: str, x, *, offsets=None, max_len=None, gamma=None, beta=None,
     given); returns the output tensor (dx for the backward passes, whose x is
     the forward output for the softmax family and the forward input for the
     norms)."""
+    if offsets is not None and op.endswith("_backward"):
+        if op in ("softmax_backward", "logsoftmax_backward"):
+            return softmax_backward_ragged(x, dy, offsets, max_len, dx=out, ws=ws, stream=stream,
+                                           log=op.startswith("log"))
+        if op == "layernorm_backward":
+            return layernorm_backward_ragged(x, dy, offsets, max_len, gamma,
+                                             1e-5 if eps is None else eps, dx=out, dgamma=dgamma,
+                                             dbeta=dbeta, ws=ws, stream=stream)[0]
+        if op == "rmsnorm_backward":
+            return rmsnorm_backward_ragged(x, dy, offsets, max_len, gamma,
+                                           1e-6 if eps is None else eps, dx=out, dgamma=dgamma,
+                                           ws=ws, stream=stream)[0]
     if op == "softmax_backward":
         return softmax_backward(x, dy, out, stream)
     if op == "logsoftmax_backward":
