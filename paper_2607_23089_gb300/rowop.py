@@ -472,6 +472,9 @@ def run(op: str, x, *, offsets=None, max_len=None, gamma=None, beta=None,
     given); returns the output tensor (dx for the backward passes, whose x is
     the forward output for the softmax family and the forward input for the
     norms)."""
+    if offsets is not None and op in ("pad_scale", "add_layernorm", "add_rmsnorm",
+                                      "moe_group_top2"):
+        raise ValueError(f"{op} has no ragged form")
     if offsets is not None and op.endswith("_backward"):
         if op in ("softmax_backward", "logsoftmax_backward"):
             return softmax_backward_ragged(x, dy, offsets, max_len, dx=out, ws=ws, stream=stream,

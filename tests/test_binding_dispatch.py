@@ -42,3 +42,9 @@ def test_backward_ops_follow_the_layout(calls, op, dense, ragged):
         assert kwargs.get("log") is True
     elif op == "softmax_backward":
         assert kwargs.get("log") is False
+
+
+@pytest.mark.parametrize("op", ["pad_scale", "add_layernorm", "add_rmsnorm", "moe_group_top2"])
+def test_dense_only_ops_refuse_offsets(op):
+    with pytest.raises(ValueError, match="no ragged form"):
+        rowop.run(op, "x", offsets="off", max_len=8)
