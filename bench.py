@@ -239,6 +239,32 @@ def per_config(torch, rw, wl, device, peak, steps):
     return out
 
 
+# The five workloads of the benchmark specification by case name; configs 3
+# and 4 carry the bandwidth target (>= 0.80 of the HBM peak).
+TARGET_CASES = (("cfg1_softmax_1k", "softmax_1k"),
+                ("cfg2_softmax_64", "short_rows_softmax_64"),
+                ("cfg2_softmax_512", "short_rows_softmax_512"),
+                ("cfg2_logsoftmax_512", "short_rows_logsoftmax_512"),
+                ("cfg3_rmsnorm", "medium_norm_rmsnorm"),
+                ("cfg3_layernorm", "medium_norm_layernorm"),
+                ("cfg4_logsoftmax", "long_rows_logsoftmax"),
+                ("cfg5_ragged_layernorm", "ragged_layernorm"))
+
+
+def targets(per, headline_frac):
+    """Compact figures of the five workloads from per_config: GB/s (median
+    call) and the fraction of the measured copy peak."""
+    by = {e["name"]: e for e in per}
+    out = {}
+    for key, name in TARGET_CASES:
+        e = by.get(name)
+        if e is not None:
+            out[key] = [e["gbs_median"], round(e["pct_of_measured"] / 100, 3)]
+    out["fields"] = "[GB/s median call, fraction of measured peak]"
+    out["headline_frac"] = headline_frac
+    return out
+
+
 def backward_call(torch, rw, case, x, device):
     """A backward-pass case on device buffers: returns (fn, dx).  The softmax
     family's forward output y is formed once, by the library's forward, from
@@ -611,6 +637,10 @@ def run_rowop(args, rank, world, local):
         result["per_config"] = per_config(torch, rw, wl, device, peak, args.config_steps)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_oracle_baseline(case, args.cpu_sample_elems)
+    if rank == 0 and "per_config" in result:
+        # last key of the line, so that a reader that keeps only the end of
+        # the output still has the five workloads' figures
+        result["targets"] = targets(result["per_config"], result["roofline"]["frac"])
     if rank == 0:
         print(json.dumps(result), flush=True)
     return 0

@@ -396,13 +396,45 @@ ROWOP_API int rowop_select_bucket(int64_t len, rowop_dtype_t dtype);
 /* Longest row (elements) the library accepts for dtype, dense or ragged. */
 ROWOP_API int64_t rowop_max_row_len(rowop_dtype_t dtype);
 
+/* The library's dispatch thresholds and limits, as this build uses them.
+ * None of them depends on the device or on the environment.  The bucket
+ * rule (launch_by_rows, §2.1) is: SMALL if len * esize <= small_max_bytes,
+ * MEDIUM if <= medium_max_bytes, else LARGE. */
+typedef struct rowop_config {
+    uint32_t size;                  /* bytes of this struct the library filled */
+    uint32_t chunk_bytes;           /* 16: the unit of every vector load / store */
+    uint32_t tile_bytes;            /* 1024: a warp's unit of a MEDIUM / LARGE row */
+    uint32_t max_cluster;           /* largest thread-block cluster a row is split over */
+    int64_t small_max_bytes;        /* 4096 */
+    int64_t medium_max_bytes;       /* 32768 */
+    int64_t max_row_len[3];         /* rowop_max_row_len() per rowop_dtype_t */
+    int64_t resident_max_tiles[2];  /* longest row portion (tiles) a CTA holds in
+                                       registers: [0] float32, [1] 16-bit types */
+    int64_t staged_max_tiles;       /* longest portion a CTA holds staged in shared memory */
+    int64_t stage_budget_bytes[2];  /* shared memory for stages per CTA: [0] resident
+                                       design (two CTAs an SM), [1] staged (three) */
+    int64_t wait_limit_ns;          /* a bounded device wait gives up after this long */
+    int64_t static_max_rows;        /* ROWOP_STATIC_MAX_ROWS */
+} rowop_config_t;
+
+/* Fills *cfg (which must not be NULL; ROWOP_ERR_INVALID_ARG otherwise) and
+ * returns ROWOP_OK.  Pure host function. */
+ROWOP_API int rowop_get_config(rowop_config_t *cfg);
+
 /* Human-readable name of a status code (static storage, never NULL). */
 ROWOP_API const char *rowop_status_string(int status);
 
-/* Synchronises `stream`, then reads and clears the device status word of the
- * current device: returns ROWOP_OK, ROWOP_ERR_TIMEOUT if any bounded device
- * wait ran out, ROWOP_ERR_BAD_OFFSETS if ragged rows were rejected (timeout
- * wins when both are set), or ROWOP_ERR_CUDA if the synchronisation failed. */
+/* Synchronises `stream` (the host waits until all work queued on it has
+ * finished), then reads and clears the device status word of the current
+ * device: returns ROWOP_OK, ROWOP_ERR_TIMEOUT if any bounded device wait ran
+ * out, ROWOP_ERR_BAD_OFFSETS if ragged rows were rejected (timeout wins when
+ * both are set), or ROWOP_ERR_CUDA if the synchronisation failed.
+ * The status word belongs to the device, not to a call or a stream: every
+ * call on the device, on any stream (rowop_layernorm_ragged_static
+ * included), sets its bits, and the first rowop_check_status to run reads
+ * and clears them.  Work still running on other streams may set bits after
+ * the read.  To attribute a condition to one call, run it alone on its
+ * stream, or synchronise the other streams first. */
 ROWOP_API int rowop_check_status(cudaStream_t stream);
 
 /* Test hook for the bounded-wait path, launching one tiny kernel that waits

@@ -131,6 +131,21 @@ constexpr size_t ragged_ws_bytes(int64_t rows) {
   return ragged_lists_offset(rows) + 3 * kWsRecordBytes * static_cast<size_t>(rows) + 256;
 }
 
+// Every bounded device wait gives up after this long.
+constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
+// Shared memory one CTA of the staged tile design spends on stages, so that
+// three CTAs fit an SM.
+constexpr int64_t kStageBudgetBytes = 72 * 1024;
+// Shared memory one CTA of the register-resident design spends on stages, so
+// that two CTAs share an SM (a stage is refilled as soon as its rows are in
+// registers, so a few stages keep enough bytes in flight).
+constexpr int64_t kResStageBudgetBytes = 96 * 1024;
+// Longest row portion (tiles) one CTA of the register-resident design holds:
+// 64 fp32 values of row data per thread, 8 warps of 32 lanes, two 16-byte
+// chunks a lane per tile.
+constexpr int kResMaxTilesF32 = 64;
+constexpr int kResMaxTiles16 = 32;
+
 // Tile budget of one CTA portion: the longest row the resident split-row
 // design takes is this many 1 KiB tiles per CTA times the largest cluster.
 constexpr int kMaxPortionTiles = 192;
@@ -156,6 +171,9 @@ inline int64_t max_row_len_elems(int esize) {
 //                       variant: its results differ by rounding)
 //   ROWOP_BWD_CLUSTER   backward passes: split every row over a cluster of
 //                       this many CTAs (2, 4, 8, 16); changes rounding order
+//   ROWOP_RESIDENT      0 -> MEDIUM / LARGE rows use the staged tile design
+//                       even where the register-resident one can hold them
+//                       (the two give the same bits)
 struct Knobs {
   int force_bucket = -1;
   int cluster = 0;
@@ -164,6 +182,7 @@ struct Knobs {
   int group_warps = 0;
   int softmax_online = 0;
   int bwd_cluster = 0;
+  int resident = 1;
 };
 Knobs read_knobs();
 

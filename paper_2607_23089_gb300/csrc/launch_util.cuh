@@ -11,7 +11,6 @@
 
 namespace rowop {
 
-constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s per bounded wait
 
 inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 inline bool congruent16(const void *a, const void *b) {

@@ -75,6 +75,7 @@ Knobs read_knobs() {
   k.group_warps = env_int("ROWOP_GROUP_WARPS", 0);
   k.softmax_online = env_int("ROWOP_SOFTMAX_ONLINE", 0);
   k.bwd_cluster = env_int("ROWOP_BWD_CLUSTER", 0);
+  k.resident = env_int("ROWOP_RESIDENT", 1);
   return k;
 }
 
@@ -230,10 +231,11 @@ static int run_dense(int op, const void *in, void *out, const void *gamma, const
 }
 
 // op < 0: only the classify pass (rowop_ragged_plan)
-static int run_ragged(int op, const void *in, void *out, const void *gamma, const void *beta,
-                      const int64_t *offsets, int64_t rows, int64_t max_len,
-                      rowop_dtype_t dtype, float eps, void *ws, size_t ws_bytes,
-                      cudaStream_t stream, bool classify) {
+// Argument checks of a ragged call, everything but the workspace: the
+// status the call returns for them, or ROWOP_OK.
+static int check_ragged_args(int op, const void *in, const void *out, const void *gamma,
+                             const void *beta, const int64_t *offsets, int64_t rows,
+                             int64_t max_len, rowop_dtype_t dtype, float eps) {
   const int es = esize_of(dtype);
   const bool norm = (op == kLayerNorm || op == kRmsNorm);
   if (es == 0) return ROWOP_ERR_UNSUPPORTED_DTYPE;
@@ -246,6 +248,15 @@ static int run_ragged(int op, const void *in, void *out, const void *gamma, cons
   if ((gamma && !elem_aligned(gamma, es)) || (beta && !elem_aligned(beta, es)))
     return ROWOP_ERR_INVALID_ARG;
   if (max_len > max_row_len_elems(es)) return ROWOP_ERR_TOO_LONG;
+  return ROWOP_OK;
+}
+
+static int run_ragged(int op, const void *in, void *out, const void *gamma, const void *beta,
+                      const int64_t *offsets, int64_t rows, int64_t max_len,
+                      rowop_dtype_t dtype, float eps, void *ws, size_t ws_bytes,
+                      cudaStream_t stream, bool classify) {
+  const int chk = check_ragged_args(op, in, out, gamma, beta, offsets, rows, max_len, dtype, eps);
+  if (chk != ROWOP_OK || rows == 0) return chk;
   if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0 ||
       ws_bytes < ragged_ws_bytes(rows))
     return ROWOP_ERR_WORKSPACE;
@@ -603,10 +614,12 @@ int rowop_layernorm_ragged_static(const void *in, void *out, const void *gamma,
                                   const void *beta, const int64_t *offsets, int64_t rows,
                                   int64_t max_len, rowop_dtype_t dtype, float eps,
                                   cudaStream_t stream) {
+  // argument errors first, as the caller-workspace call reports them; only a
+  // call that is otherwise valid is refused for its row count
+  const int chk = check_ragged_args(kLayerNorm, in, out, gamma, beta, offsets, rows, max_len,
+                                    dtype, eps);
+  if (chk != ROWOP_OK || rows == 0) return chk;
   if (rows > ROWOP_STATIC_MAX_ROWS) return ROWOP_ERR_WORKSPACE;
-  if (rows <= 0)  // nothing to stage: same checks and result as the caller-workspace call
-    return run_ragged(kLayerNorm, in, out, gamma, beta, offsets, rows, max_len, dtype, eps,
-                      nullptr, 0, stream, true);
   void *ws = nullptr;
   const int st = static_workspace(&ws);
   if (st != ROWOP_OK) return st;
@@ -691,6 +704,30 @@ const char *rowop_status_string(int status) {
     case ROWOP_ERR_TOO_LONG: return "ROWOP_ERR_TOO_LONG: row longer than rowop_max_row_len()";
     default: return "ROWOP: unknown status";
   }
+}
+
+int rowop_get_config(rowop_config_t *cfg) {
+  if (!cfg) return ROWOP_ERR_INVALID_ARG;
+  rowop_config_t c;
+  std::memset(&c, 0, sizeof(c));
+  c.size = sizeof(rowop_config_t);
+  c.chunk_bytes = kChunkBytes;
+  c.tile_bytes = kTileBytes;
+  c.max_cluster = kMaxCluster;
+  c.small_max_bytes = kSmallMaxBytes;
+  c.medium_max_bytes = kMediumMaxBytes;
+  c.max_row_len[ROWOP_F32] = max_row_len_elems(4);
+  c.max_row_len[ROWOP_BF16] = max_row_len_elems(2);
+  c.max_row_len[ROWOP_F16] = max_row_len_elems(2);
+  c.resident_max_tiles[0] = kResMaxTilesF32;
+  c.resident_max_tiles[1] = kResMaxTiles16;
+  c.staged_max_tiles = kMaxPortionTiles;
+  c.stage_budget_bytes[0] = kResStageBudgetBytes;
+  c.stage_budget_bytes[1] = kStageBudgetBytes;
+  c.wait_limit_ns = static_cast<int64_t>(kWaitLimitNs);
+  c.static_max_rows = ROWOP_STATIC_MAX_ROWS;
+  *cfg = c;
+  return ROWOP_OK;
 }
 
 int rowop_check_status(cudaStream_t stream) {

@@ -790,6 +790,17 @@ __device__ __forceinline__ RowRec ragged_record(const TileParams &p, const int *
   return list[static_cast<int64_t>(lo) * p.rows_per_block + (idx - pref[lo])];
 }
 
+// A record taken from bucket b's list fits the call that uses it: a row of
+// at least one and at most glen elements whose bucket, for this call's
+// element type, is b.  A plan made by rowop_ragged_plan for another element
+// type or a longer max_len than the planned call's fails this for some rows;
+// they are skipped (left untouched) and flagged as rejected rows, and never
+// staged past a buffer sized for this call.
+template <typename T>
+__device__ __forceinline__ bool ragged_record_fits(const RowRec &r, int b, int64_t glen) {
+  return r.n >= 1 && r.n <= glen && bucket_of(r.n, Elem<T>::kSize) == b;
+}
+
 template <typename T, bool EXACT, bool CLUSTER, bool RAGGED>
 __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSmemLayout &L,
                                               unsigned char *smem, int cs, int rank, int64_t cid,
@@ -817,26 +828,34 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
     start = 0;
     n = 0;
     if (RAGGED) {
-      if (!medium_phase) {
-        const int64_t li = cid + k_large * ncl;
-        if (li < pref[2 * nb1 + p.blocks]) {
-          const RowRec r = ragged_record(p, pref + 2 * nb1, p.rec_large, li);
-          ++k_large;
-          kind = kItemLarge;
-          start = r.start;
-          n = r.n;
-        } else {
+      for (;;) {
+        if (!medium_phase) {
+          const int64_t li = cid + k_large * ncl;
+          if (li < pref[2 * nb1 + p.blocks]) {
+            const RowRec r = ragged_record(p, pref + 2 * nb1, p.rec_large, li);
+            ++k_large;
+            if (!ragged_record_fits<T>(r, kLarge, p.glen)) {
+              atomicOr(p.status, kStatusBadOffsets);
+              continue;
+            }
+            kind = kItemLarge;
+            start = r.start;
+            n = r.n;
+            return;
+          }
           medium_phase = true;
         }
-      }
-      if (medium_phase) {
         const unsigned int m = atomicAdd(&p.counters[0], 1u);
-        if (m < static_cast<unsigned int>(pref[nb1 + p.blocks])) {
-          const RowRec r = ragged_record(p, pref + nb1, p.rec_medium, m);
-          kind = kItemMedium;
-          start = r.start;
-          n = r.n;
+        if (m >= static_cast<unsigned int>(pref[nb1 + p.blocks])) return;
+        const RowRec r = ragged_record(p, pref + nb1, p.rec_medium, m);
+        if (!ragged_record_fits<T>(r, kMedium, p.glen)) {
+          atomicOr(p.status, kStatusBadOffsets);
+          continue;
         }
+        kind = kItemMedium;
+        start = r.start;
+        n = r.n;
+        return;
       }
     } else {
       const int64_t r = cid + k_dense * ncl;
@@ -1151,6 +1170,10 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
       const int *pref = reinterpret_cast<const int *>(smem + L.pref);  // SMALL: bucket 0
       if (idx >= static_cast<unsigned int>(pref[p.blocks])) break;
       const RowRec rec = ragged_record(p, pref, p.rec_small, idx);
+      if (!ragged_record_fits<T>(rec, kSmall, p.glen)) {
+        if (lane == 0) atomicOr(p.status, kStatusBadOffsets);
+        continue;
+      }
       const T *in_row = in + rec.start;
       const uintptr_t ia = reinterpret_cast<uintptr_t>(in_row);
       const int h = static_cast<int>((ia & 15) / SZ);

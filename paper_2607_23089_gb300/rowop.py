@@ -40,6 +40,16 @@ _I = ctypes.c_int
 _F = ctypes.c_float
 _SZ = ctypes.c_size_t
 
+class RowopConfig(ctypes.Structure):
+    """rowop_config_t of include/rowop.h."""
+    _fields_ = [("size", ctypes.c_uint32), ("chunk_bytes", ctypes.c_uint32),
+                ("tile_bytes", ctypes.c_uint32), ("max_cluster", ctypes.c_uint32),
+                ("small_max_bytes", _I64), ("medium_max_bytes", _I64),
+                ("max_row_len", _I64 * 3), ("resident_max_tiles", _I64 * 2),
+                ("staged_max_tiles", _I64), ("stage_budget_bytes", _I64 * 2),
+                ("wait_limit_ns", _I64), ("static_max_rows", _I64)]
+
+
 # C signatures (argument types, return type), in header order.
 SIGNATURES = {
     "rowop_softmax": ([_P, _P, _I64, _I64, _I64, _I, _P], _I),
@@ -79,6 +89,7 @@ SIGNATURES = {
     "rowop_moe_group_top2": ([_P, _P, _I64, _I64, _I64, _I, _P], _I),
     "rowop_select_bucket": ([_I64, _I], _I),
     "rowop_max_row_len": ([_I], _I64),
+    "rowop_get_config": ([ctypes.POINTER(RowopConfig)], _I),
     "rowop_status_string": ([_I], ctypes.c_char_p),
     "rowop_check_status": ([_P], _I),
     "rowop_debug_wait_timeout": ([_I64, _P], _I),
@@ -122,6 +133,19 @@ def _c(name):
 
 for _name in SIGNATURES:
     globals()[_name] = _c(_name)
+
+
+def get_config() -> dict:
+    """rowop_get_config() as a dict."""
+    cfg = RowopConfig()
+    st = rowop_get_config(ctypes.byref(cfg))  # noqa: F821 (defined above)
+    if st != 0:
+        raise RowopError(st, "rowop_get_config")
+    out = {}
+    for name, _ in RowopConfig._fields_:
+        v = getattr(cfg, name)
+        out[name] = list(v) if hasattr(v, "__len__") else int(v)
+    return out
 
 
 # ---------------------------------------------------------------------------

@@ -68,6 +68,31 @@ def test_limits_and_strings(lib):
     assert ws >= 256 + n + 3 * 4 * n
 
 
+def test_get_config(lib):
+    """rowop_get_config reports the rule rowop_select_bucket applies and the
+    limits the entry points enforce."""
+    import ctypes as _ct
+    cfg = lib.get_config()
+    assert cfg["size"] == _ct.sizeof(lib.RowopConfig)
+    assert cfg["chunk_bytes"] == 16 and cfg["tile_bytes"] == 1024
+    for dtype, es in ((lib.ROWOP_F32, 4), (lib.ROWOP_BF16, 2), (lib.ROWOP_F16, 2)):
+        s_el = cfg["small_max_bytes"] // es
+        m_el = cfg["medium_max_bytes"] // es
+        assert lib.rowop_select_bucket(s_el, dtype) == 0
+        assert lib.rowop_select_bucket(s_el + 1, dtype) == 1
+        assert lib.rowop_select_bucket(m_el, dtype) == 1
+        assert lib.rowop_select_bucket(m_el + 1, dtype) == 2
+        assert cfg["max_row_len"][dtype] == lib.rowop_max_row_len(dtype)
+    assert cfg["small_max_bytes"] == 4096 and cfg["medium_max_bytes"] == 32768
+    assert cfg["max_cluster"] == 16
+    assert cfg["resident_max_tiles"] == [64, 32]
+    assert cfg["wait_limit_ns"] == 2 * 10**9
+    text = open(HEADER).read()
+    assert cfg["static_max_rows"] == int(
+        re.search(r"#define\s+ROWOP_STATIC_MAX_ROWS\s+(\d+)", text).group(1))
+    assert lib.rowop_get_config(None) == lib.ROWOP_ERR_INVALID_ARG
+
+
 FAKE = 1 << 20  # a non-NULL, 16-byte aligned address that is never touched
 
 
@@ -114,6 +139,28 @@ def test_ragged_validation(lib):
     ln = lib.rowop_layernorm_ragged
     assert ln(FAKE, FAKE, None, None, FAKE, 10, 64, F32, -0.5, FAKE, ws_need,
               None) == lib.ROWOP_ERR_INVALID_ARG
+
+
+def test_static_ragged_validation_order(lib):
+    """The library-workspace ragged LayerNorm reports argument errors exactly
+    as the caller-workspace call does, before its row limit: only an
+    otherwise valid call is refused for having too many rows."""
+    import re as _re
+    text = open(HEADER).read()
+    nmax = int(_re.search(r"#define\s+ROWOP_STATIC_MAX_ROWS\s+(\d+)", text).group(1))
+    F32 = lib.ROWOP_F32
+    st = lib.rowop_layernorm_ragged_static
+    big = nmax + 1
+    assert st(FAKE, FAKE, None, None, FAKE, big, 64, 9, 1e-5, None) == \
+        lib.ROWOP_ERR_UNSUPPORTED_DTYPE
+    assert st(FAKE, FAKE, None, None, None, big, 64, F32, 1e-5, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert st(FAKE, FAKE, None, None, FAKE, big, 64, F32, -1.0, None) == lib.ROWOP_ERR_INVALID_ARG
+    assert st(FAKE, None, None, None, FAKE, big, 64, F32, 1e-5, None) == lib.ROWOP_ERR_INVALID_ARG
+    too_long = lib.rowop_max_row_len(F32) + 1
+    assert st(FAKE, FAKE, None, None, FAKE, big, too_long, F32, 1e-5, None) == \
+        lib.ROWOP_ERR_TOO_LONG
+    assert st(FAKE, FAKE, None, None, FAKE, big, 64, F32, 1e-5, None) == lib.ROWOP_ERR_WORKSPACE
+    assert st(None, None, None, None, None, 0, 64, F32, 1e-5, None) == lib.ROWOP_OK
 
 
 def test_debug_timeout_rejects_bad_limits(lib):
