@@ -412,7 +412,7 @@ typedef struct rowop_config {
                                        registers: [0] float32, [1] 16-bit types */
     int64_t staged_max_tiles;       /* longest portion a CTA holds staged in shared memory */
     int64_t stage_budget_bytes[2];  /* shared memory for stages per CTA: [0] resident
-                                       design (two CTAs an SM), [1] staged (three) */
+                                       design at two CTAs an SM, [1] staged (three) */
     int64_t wait_limit_ns;          /* a bounded device wait gives up after this long */
     int64_t static_max_rows;        /* ROWOP_STATIC_MAX_ROWS */
 } rowop_config_t;

@@ -136,10 +136,10 @@ constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
 // Shared memory one CTA of the staged tile design spends on stages, so that
 // three CTAs fit an SM.
 constexpr int64_t kStageBudgetBytes = 72 * 1024;
-// Shared memory one CTA of the register-resident design spends on stages, so
-// that two CTAs share an SM (a stage is refilled as soon as its rows are in
-// registers, so a few stages keep enough bytes in flight).
-constexpr int64_t kResStageBudgetBytes = 96 * 1024;
+// Shared memory one CTA of the register-resident design spends on stages
+// when `ctas` CTAs share an SM's 228 KiB (a stage is refilled as soon as its
+// row is in registers, so a few stages keep enough bytes in flight).
+constexpr int64_t res_stage_budget(int ctas) { return (228 * 1024) / ctas - 8 * 1024; }
 // Longest row portion (tiles) one CTA of the register-resident design holds:
 // 64 fp32 values of row data per thread, 8 warps of 32 lanes, two 16-byte
 // chunks a lane per tile.
@@ -171,9 +171,9 @@ inline int64_t max_row_len_elems(int esize) {
 //                       variant: its results differ by rounding)
 //   ROWOP_BWD_CLUSTER   backward passes: split every row over a cluster of
 //                       this many CTAs (2, 4, 8, 16); changes rounding order
-//   ROWOP_RESIDENT      0 -> MEDIUM / LARGE rows use the staged tile design
-//                       even where the register-resident one can hold them
-//                       (the two give the same bits)
+//   ROWOP_RESIDENT      0 -> MEDIUM / LARGE rows (dense and ragged) use the
+//                       staged tile design even where a register-resident
+//                       one can hold them (they give the same bits)
 struct Knobs {
   int force_bucket = -1;
   int cluster = 0;

@@ -136,93 +136,29 @@ cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int
 }
 
 // ---------------------------------------------------------------------------
-// MEDIUM / LARGE / ragged: the register-resident tile kernel
+// MEDIUM / LARGE dense rows of whole tiles: the register-resident tile kernel
 // ---------------------------------------------------------------------------
-// Tiles a consumer warp keeps in registers: 64 fp32 values of row data per
-// lane (eight 1 KiB tiles of fp32, four of 16-bit elements).
+// Tiles a warp keeps in registers: 64 fp32 values of row data per lane
+// (eight 1 KiB tiles of fp32, four of 16-bit elements).
 template <typename T>
 constexpr int res_max_r() {
   return (sizeof(T) == 4 ? kResMaxTilesF32 : kResMaxTiles16) / kResWarps;
 }
-// Resident tiles per warp for an item of `tiles` tiles (8 consumer warps).
-inline int res_r_for(int64_t tiles) {
-  return tiles <= 8 ? 1 : (tiles <= 16 ? 2 : (tiles <= 32 ? 4 : 8));
-}
-
-template <int OP, typename T, int R, bool CLUSTER, bool RAGGED, bool GC>
-cudaError_t launch_res_k(TileParams p, int cs, int stage_tiles, int64_t items, const DeviceInfo &d,
-                         cudaStream_t stream, uint32_t min_stage_area = 0) {
-  auto kern = resident_row_kernel<OP, T, R, CLUSTER, RAGGED, GC>;
-  const void *kp = reinterpret_cast<const void *>(kern);
-  const Knobs kn = read_knobs();
-  p.stage_bytes = static_cast<uint32_t>(stage_tiles) * kTileBytes;
-  p.max_tiles = stage_tiles;
-  p.group_warps = kResWarps;
-  int stages = kn.stages > 0 ? std::min(kn.stages, 32)
-                             : static_cast<int>(std::max<int64_t>(
-                                   1, std::min<int64_t>(16, kResStageBudgetBytes / p.stage_bytes)));
-  while (static_cast<uint64_t>(stages) * p.stage_bytes < min_stage_area) ++stages;
-  // ragged item records travel through the stage's record slot, which needs
-  // two stages (a record is read one item barrier after it is written)
-  if (RAGGED) stages = std::max(stages, 2);
-  const auto total = [&](int s) {
-    return ResSmemLayout(p.stage_bytes, s, stage_tiles, CLUSTER, RAGGED ? p.blocks : 0).total;
-  };
-  const uint32_t optin = static_cast<uint32_t>(d.max_smem_optin);
-  while (stages > (RAGGED ? 2 : 1) && total(stages) > optin) --stages;
-  if (total(stages) > optin || static_cast<uint64_t>(stages) * p.stage_bytes < min_stage_area)
-    return cudaErrorInvalidConfiguration;
-  p.stages = stages;
-  const size_t smem = total(stages);
-  cudaError_t e = prepare_kernel(kp, d, CLUSTER);
-  if (e != cudaSuccess) return e;
-
-  cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
-  cfg.blockDim = dim3(kResThreads, 1, 1);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = stream;
-  const int max_ctas_per_sm = kn.ctas_per_sm;
-  int grid;
-  if (CLUSTER) {
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = cs;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    cfg.gridDim = dim3(cs * std::max(1, d.sm_count / cs), 1, 1);
-    int ncl = cached_occupancy(kp, kResThreads, smem, cs, &cfg);
-    if (max_ctas_per_sm > 0) ncl = std::min(ncl, max_ctas_per_sm * d.sm_count / cs);
-    if (ncl < 1) ncl = 1;
-    grid = static_cast<int>(cs * std::max<int64_t>(1, std::min<int64_t>(items, ncl)));
-  } else {
-    int bps = std::max(1, cached_occupancy(kp, kResThreads, smem, 1, nullptr));
-    if (max_ctas_per_sm > 0) bps = std::min(bps, max_ctas_per_sm);
-    grid = static_cast<int>(std::max<int64_t>(
-        1, std::min<int64_t>(items, static_cast<int64_t>(bps) * d.sm_count)));
-  }
-  cfg.gridDim = dim3(grid, 1, 1);
-  e = cudaLaunchKernelEx(&cfg, kern, p);
-  if (e != cudaSuccess) return e;
-  return cudaGetLastError();
-}
-
-// Whole-tile dense rows on the specialised resident kernel: every warp owns
-// exactly R tiles of each row (or of this CTA's portion of it).  R = 1 is
-// compiled for three CTAs an SM, larger R for two.
-template <int OP, typename T, int R, bool CLUSTER, bool GC>
+// Whole-tile dense rows on the specialised resident kernel: each of the NW
+// warps of a CTA owns exactly R tiles of each row (or of this CTA's portion
+// of it).  4-warp CTAs are compiled for four CTAs an SM, 8-warp CTAs with one
+// tile a warp for three, the others for two.
+template <int OP, typename T, int R, int NW, bool CLUSTER, bool GC>
 cudaError_t launch_res_full_k(TileParams p, int cs, const DenseCall &c, const DeviceInfo &d) {
-  constexpr int MINB = R == 1 ? 3 : 2;
-  auto kern = resident_full_kernel<OP, T, R, CLUSTER, GC, MINB>;
+  constexpr int MINB = NW == 4 ? 4 : (R == 1 ? 3 : 2);
+  auto kern = resident_full_kernel<OP, T, R, NW, CLUSTER, GC, MINB>;
   const void *kp = reinterpret_cast<const void *>(kern);
   const Knobs kn = read_knobs();
-  const int stage_tiles = kResWarps * R;
+  const int stage_tiles = NW * R;
   p.stage_bytes = static_cast<uint32_t>(stage_tiles) * kTileBytes;
   p.max_tiles = stage_tiles;
-  p.group_warps = kResWarps;
-  // shared memory per CTA so that MINB CTAs share an SM's 228 KiB
-  const int64_t budget = (228 * 1024) / MINB - 8 * 1024;
+  p.group_warps = NW;
+  const int64_t budget = res_stage_budget(MINB);
   int stages = kn.stages > 0 ? std::min(kn.stages, 32)
                              : static_cast<int>(std::max<int64_t>(
                                    1, std::min<int64_t>(16, budget / p.stage_bytes)));
@@ -238,7 +174,7 @@ cudaError_t launch_res_full_k(TileParams p, int cs, const DenseCall &c, const De
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
-  cfg.blockDim = dim3(kResThreads, 1, 1);
+  cfg.blockDim = dim3(NW * 32, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = c.stream;
   int grid;
@@ -250,12 +186,12 @@ cudaError_t launch_res_full_k(TileParams p, int cs, const DenseCall &c, const De
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     cfg.gridDim = dim3(cs * std::max(1, d.sm_count / cs), 1, 1);
-    int ncl = cached_occupancy(kp, kResThreads, smem, cs, &cfg);
+    int ncl = cached_occupancy(kp, NW * 32, smem, cs, &cfg);
     if (kn.ctas_per_sm > 0) ncl = std::min(ncl, kn.ctas_per_sm * d.sm_count / cs);
     if (ncl < 1) ncl = 1;
     grid = static_cast<int>(cs * std::max<int64_t>(1, std::min<int64_t>(c.rows, ncl)));
   } else {
-    int bps = std::max(1, cached_occupancy(kp, kResThreads, smem, 1, nullptr));
+    int bps = std::max(1, cached_occupancy(kp, NW * 32, smem, 1, nullptr));
     if (kn.ctas_per_sm > 0) bps = std::min(bps, kn.ctas_per_sm);
     grid = static_cast<int>(std::max<int64_t>(
         1, std::min<int64_t>(c.rows, static_cast<int64_t>(bps) * d.sm_count)));
@@ -283,21 +219,21 @@ bool try_res_full(const TileParams &p, const DenseCall &c, const DeviceInfo &d, 
   const int64_t K = c.cols / (kTileChunks * E);
   if (bucket == kMedium) {
     if (kn.cluster > 1) return false;
-    if (K == 8) {
-      *err = kAffine ? launch_res_full_k<OP, T, 1, false, kAffine>(p, 1, c, d)
-                     : launch_res_full_k<OP, T, 1, false, false>(p, 1, c, d);
+    if (K == 8) {  // four warps of two tiles: more of each row per lane
+      *err = kAffine ? launch_res_full_k<OP, T, 2, 4, false, kAffine>(p, 1, c, d)
+                     : launch_res_full_k<OP, T, 2, 4, false, false>(p, 1, c, d);
       return true;
     }
     if (K == 16) {
       if constexpr (kAffine && SZ == 4) {
-        *err = launch_res_full_k<OP, T, 2, false, true>(p, 1, c, d);
+        *err = launch_res_full_k<OP, T, 2, 8, false, true>(p, 1, c, d);
       } else {
-        *err = launch_res_full_k<OP, T, 2, false, false>(p, 1, c, d);
+        *err = launch_res_full_k<OP, T, 2, 8, false, false>(p, 1, c, d);
       }
       return true;
     }
     if (K == 32) {
-      *err = launch_res_full_k<OP, T, 4, false, false>(p, 1, c, d);
+      *err = launch_res_full_k<OP, T, 4, 8, false, false>(p, 1, c, d);
       return true;
     }
     return false;
@@ -309,39 +245,15 @@ bool try_res_full(const TileParams &p, const DenseCall &c, const DeviceInfo &d, 
     if (cs < 2 || cs > kMaxCluster || (cs & (cs - 1)) != 0) continue;
     if (kn.cluster > 0 && kn.cluster != cs) continue;
     if (R == 2) {
-      *err = launch_res_full_k<OP, T, 2, true, false>(p, static_cast<int>(cs), c, d);
+      *err = launch_res_full_k<OP, T, 2, 8, true, false>(p, static_cast<int>(cs), c, d);
     } else if (R == 4) {
-      *err = launch_res_full_k<OP, T, 4, true, false>(p, static_cast<int>(cs), c, d);
+      *err = launch_res_full_k<OP, T, 4, 8, true, false>(p, static_cast<int>(cs), c, d);
     } else {
-      if constexpr (SZ == 4) *err = launch_res_full_k<OP, T, 8, true, false>(p, static_cast<int>(cs), c, d);
+      if constexpr (SZ == 4) *err = launch_res_full_k<OP, T, 8, 8, true, false>(p, static_cast<int>(cs), c, d);
     }
     return true;
   }
   return false;
-}
-
-// Dense rows on the resident kernel: R from the portion's tiles; gamma/beta
-// cached in registers when every row starts at the same offset modulo 16
-// bytes and the lane's share fits (one tile of 16-bit elements, two of fp32).
-template <int OP, typename T, bool CLUSTER>
-cudaError_t launch_res_dense(const TileParams &p, int cs, int st, bool hconst,
-                             const DenseCall &c, const DeviceInfo &d) {
-  constexpr bool kAffine = (OP == kLayerNorm || OP == kRmsNorm);
-  const int R = res_r_for(st);
-  if constexpr (kAffine && !CLUSTER) {
-    if (hconst && R == 1) return launch_res_k<OP, T, 1, false, false, true>(p, 1, st, c.rows, d, c.stream);
-    if constexpr (sizeof(T) == 4) {
-      if (hconst && R == 2) return launch_res_k<OP, T, 2, false, false, true>(p, 1, st, c.rows, d, c.stream);
-    }
-  }
-  if constexpr (CLUSTER) {
-    if (R <= 2) return launch_res_k<OP, T, 2, true, false, false>(p, cs, st, c.rows, d, c.stream);
-    return launch_res_k<OP, T, res_max_r<T>(), true, false, false>(p, cs, st, c.rows, d, c.stream);
-  } else {
-    if (R == 1) return launch_res_k<OP, T, 1, false, false, false>(p, 1, st, c.rows, d, c.stream);
-    if (R == 2) return launch_res_k<OP, T, 2, false, false, false>(p, 1, st, c.rows, d, c.stream);
-    return launch_res_k<OP, T, 4, false, false, false>(p, 1, st, c.rows, d, c.stream);
-  }
 }
 
 // Consumer warps per item group.  Items of a few tiles (dense rows of up to
@@ -446,18 +358,6 @@ cudaError_t launch_dense_impl(const DenseCall &c, const DeviceInfo &d) {
     cudaError_t err = cudaSuccess;
     if (try_res_full<OP, T>(p, c, d, bucket, kn, &err)) return err;
   }
-  // the general resident kernel (rows that are not whole tiles): measured
-  // slower than the staged design, so only on request
-  if (!RESID && kn.resident == 2 && out_vec) {
-    constexpr int kCap = 8 * res_max_r<T>();
-    const int csr = bucket == kMedium ? 1 : pick_cluster(K, kCap, kn.cluster);
-    const int64_t str = ceil_div(K, csr);
-    const bool hconst = (c.ld * SZ) % 16 == 0;  // every row at the same offset mod 16 bytes
-    if (csr == 1 && str <= 32)
-      return launch_res_dense<OP, T, false>(p, 1, static_cast<int>(str), hconst, c, d);
-    if (csr > 1 && str <= kCap)
-      return launch_res_dense<OP, T, true>(p, csr, static_cast<int>(str), hconst, c, d);
-  }
   if (cs == 1) {
     if (exact)
       return launch_tile_k<OP, T, true, false, false, RESID>(p, 1, S, st, W, c.rows, d, c.stream);
@@ -527,10 +427,10 @@ cudaError_t launch_ragged_t(const RaggedCall &c, const DeviceInfo &d) {
                                               : pick_cluster(kmax, std::max(kmed, budget), kn.cluster);
     st = std::max<int64_t>(st, ceil_div(kmax, cs));
   }
+  const uint32_t small_area = kConsumerWarps * kSmallSliceBytes;
   if (st > kMaxPortionTiles) return cudaErrorInvalidValue;
   const int W = pick_group_warps(st, true, kn.group_warps);
   const int S = pick_stages(st, W, kn.stages);
-  const uint32_t small_area = kConsumerWarps * kSmallSliceBytes;
   if (cs > 1)
     return launch_tile_k<OP, T, false, true, true>(p, cs, S, static_cast<int>(st), W, c.rows, d,
                                                    c.stream, small_area);

@@ -722,7 +722,7 @@ int rowop_get_config(rowop_config_t *cfg) {
   c.resident_max_tiles[0] = kResMaxTilesF32;
   c.resident_max_tiles[1] = kResMaxTiles16;
   c.staged_max_tiles = kMaxPortionTiles;
-  c.stage_budget_bytes[0] = kResStageBudgetBytes;
+  c.stage_budget_bytes[0] = res_stage_budget(2);
   c.stage_budget_bytes[1] = kStageBudgetBytes;
   c.wait_limit_ns = static_cast<int64_t>(kWaitLimitNs);
   c.static_max_rows = ROWOP_STATIC_MAX_ROWS;

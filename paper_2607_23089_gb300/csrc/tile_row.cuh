@@ -90,7 +90,8 @@ struct ItemMeta {
 // Per consumer group: tile partials of split items (part_c) and of items a
 // CTA handles alone (part_m), both double-buffered by the parity of the
 // group's item count; the two halves of the cooperative combine's scratch
-// (xw); the partials of a short split row gathered from the peers (gather);
+// (blk: the block partials of a long row); the partials of a short split row
+// gathered from the peers (gather);
 // the cluster barriers ready / released, one per buffer.
 struct TileSmemLayout {
   uint32_t part_c, part_m, gather, meta, xw, pref, bar_meta, bar_piece, bar_empty, bar_ready,
@@ -110,7 +111,7 @@ struct TileSmemLayout {
     meta = off;
     off += stages * 32u;
     xw = off;
-    off += static_cast<uint32_t>(groups) * 2u * kConsumerWarps * 4u;
+    off += static_cast<uint32_t>(groups) * kShortCombineTiles * 16u;
     pref = off;  // ragged: [3][blocks + 1] list position where each classify block starts
     off += (3u * (blocks + 1) * 4u + 15u) & ~15u;
     bar_meta = off;
@@ -431,9 +432,9 @@ __device__ __forceinline__ bool pass1_warp(const unsigned char *stage, const Ite
 // order that depends on K only.
 //   K <= 64: lane l of a warp takes t = l, l+32 in turn, then a 5-level
 //            butterfly; every warp computes it, so nothing is broadcast.
-//   K > 64:  thread v of the 256 consumer threads takes t = v, v+256, ... in
-//            turn, a butterfly per warp, then the 8 warp results in warp
-//            order; the warps cooperate through `xw` and named barriers.
+//   K > 64:  blocks of 64 consecutive tiles: each block's partial as for
+//            K <= 64 (the group's warps share the blocks), then the block
+//            partials the same way (combine_blocks).
 // (s0, s1): softmax (M, 1/S), log-softmax (M, log S), LayerNorm (mu, rstd),
 // RMSNorm (-, rstd).
 // ---------------------------------------------------------------------------
@@ -491,60 +492,71 @@ __device__ __forceinline__ void combine_short(Get get, int K, float inv_n, float
   finish_stats<OP>(first, second, inv_n, eps, s0, s1);
 }
 
-// The 256 virtual lanes of the long combine are spread over the group's W
-// warps: warp `wig` plays virtual warps wig, wig + W, ...; the group meets at
-// its named barrier `bar` and shares the 8 virtual-warp results through xw.
-template <int OP, class Get>
-__device__ __forceinline__ void combine_long(Get get, int K, float inv_n, float eps, int lane,
-                                             int wig, int W, uint32_t bar, volatile float *xw,
-                                             float &s0, float &s1) {
+// Rows of more than 64 tiles: the tiles fall into blocks of 64 consecutive
+// tiles.  Level 1: each block's partial is formed from its tile partials the
+// way a short row's statistics are (lane l takes the block's tiles l and
+// l+32, then butterflies): softmax (M_b, S_b), LayerNorm (sum_b, mean_b, Q_b,
+// n_b) with Q_b = sum over the block's tiles of Q_t + n_t (mu_t - mean_b)^2
+// (Chan's merge), RMSNorm the block's sum of squares.  The W warps of the
+// group take blocks wig, wig + W, ... (two at a time, so their partials are
+// fetched together) and leave the block partials in blk[].  Level 2: after
+// the group's named barrier `bar`, every warp combines the block partials as
+// combine_short combines tile partials.  The order depends on K only.
+template <int OP>
+__device__ __forceinline__ float4 block_partial(const float4 &p0, const float4 &p1, bool h0,
+                                                bool h1) {
   constexpr bool kMax = (OP == kSoftmax || OP == kLogSoftmax);
-  constexpr int kAhead = 4;  // partials a lane fetches before folding them (in order)
-  const uint32_t nthreads = static_cast<uint32_t>(W) * 32u;
-  const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int vw = wig; vw < kConsumerWarps; vw += W) {
-    float v = kMax ? -INFINITY : 0.f;
-    for (int t0 = vw * 32 + lane; t0 < K; t0 += kAhead * kConsumerThreads) {
-      float4 q[kAhead];
-#pragma unroll
-      for (int i = 0; i < kAhead; ++i) {
-        const int t = t0 + i * kConsumerThreads;
-        q[i] = t < K ? get(t) : z;
-      }
-#pragma unroll
-      for (int i = 0; i < kAhead; ++i)
-        if (t0 + i * kConsumerThreads < K) v = kMax ? fmaxf(v, q[i].x) : __fadd_rn(v, q[i].x);
-    }
-    v = kMax ? warp_max(v) : warp_sum(v);
-    if (lane == 0) xw[vw] = v;
+  float first;
+  if constexpr (kMax) {
+    first = warp_max(fmaxf(p0.x, p1.x));
+  } else {
+    first = warp_sum(__fadd_rn(p0.x, p1.x));
   }
-  named_sync(bar, nthreads);
-  float first = xw[0];
-  for (int w = 1; w < kConsumerWarps; ++w) first = kMax ? fmaxf(first, xw[w]) : __fadd_rn(first, xw[w]);
-  if constexpr (OP == kLayerNorm) first = __fmul_rn(first, inv_n);
-  float second = 0.f;
-  if constexpr (OP != kRmsNorm) {
-    for (int vw = wig; vw < kConsumerWarps; vw += W) {
-      float u = 0.f;
-      for (int t0 = vw * 32 + lane; t0 < K; t0 += kAhead * kConsumerThreads) {
-        float4 q[kAhead];
-#pragma unroll
-        for (int i = 0; i < kAhead; ++i) {
-          const int t = t0 + i * kConsumerThreads;
-          q[i] = t < K ? get(t) : z;
-        }
-#pragma unroll
-        for (int i = 0; i < kAhead; ++i)
-          if (t0 + i * kConsumerThreads < K) u = __fadd_rn(u, second_term<OP>(q[i], first));
-      }
-      u = warp_sum(u);
-      if (lane == 0) xw[kConsumerWarps + vw] = u;
-    }
-    named_sync(bar, nthreads);
-    second = xw[kConsumerWarps];
-    for (int w = 1; w < kConsumerWarps; ++w) second = __fadd_rn(second, xw[kConsumerWarps + w]);
+  if constexpr (OP == kRmsNorm) {
+    return make_float4(first, 0.f, 0.f, 0.f);
+  } else if constexpr (OP == kLayerNorm) {
+    const float nb = warp_sum(__fadd_rn(p0.w, p1.w));  // element count: exact
+    const float mean = nb > 0.f ? __fdiv_rn(first, nb) : 0.f;
+    float v = h0 ? second_term<OP>(p0, mean) : 0.f;
+    if (h1) v = __fadd_rn(v, second_term<OP>(p1, mean));
+    return make_float4(first, mean, warp_sum(v), nb);
+  } else {
+    float v = h0 ? second_term<OP>(p0, first) : 0.f;
+    if (h1) v = __fadd_rn(v, second_term<OP>(p1, first));
+    return make_float4(first, warp_sum(v), 0.f, 0.f);
   }
-  finish_stats<OP>(first, second, inv_n, eps, s0, s1);
+}
+
+template <int OP, class Get>
+__device__ __forceinline__ void combine_blocks(Get get, int K, float inv_n, float eps, int lane,
+                                               int wig, int W, uint32_t bar, float4 *blk,
+                                               float &s0, float &s1) {
+  constexpr bool kMax = (OP == kSoftmax || OP == kLogSoftmax);
+  const float4 z = make_float4(kMax ? -INFINITY : 0.f, 0.f, 0.f, 0.f);
+  const int nb = (K + kShortCombineTiles - 1) / kShortCombineTiles;
+  for (int b0 = wig; b0 < nb; b0 += 2 * W) {
+    float4 q[2][2];
+    bool h[2][2];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int bb = b0 + u * W;
+      const int kb = bb < nb ? min(kShortCombineTiles, K - kShortCombineTiles * bb) : 0;
+      h[u][0] = lane < kb;
+      h[u][1] = lane + 32 < kb;
+      q[u][0] = h[u][0] ? get(kShortCombineTiles * bb + lane) : z;
+      q[u][1] = h[u][1] ? get(kShortCombineTiles * bb + lane + 32) : z;
+    }
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int bb = b0 + u * W;
+      if (bb < nb) {  // the same for every lane of the warp
+        const float4 r = block_partial<OP>(q[u][0], q[u][1], h[u][0], h[u][1]);
+        if (lane == 0) blk[bb] = r;
+      }
+    }
+  }
+  named_sync(bar, static_cast<uint32_t>(W) * 32u);
+  combine_short<OP>([&](int t) { return blk[t]; }, nb, inv_n, eps, lane, s0, s1);
 }
 
 // gamma/beta chunk for window chunk c of a row with compile-time head offset
@@ -1038,7 +1050,7 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
   const uint32_t gbar = kBarGroup0 + static_cast<uint32_t>(grp);
   float4 *part_c = reinterpret_cast<float4 *>(smem + L.part_c) + static_cast<size_t>(grp) * 2 * p.max_tiles;
   float4 *part_m = reinterpret_cast<float4 *>(smem + L.part_m) + static_cast<size_t>(grp) * 2 * p.max_tiles;
-  volatile float *xw = reinterpret_cast<volatile float *>(smem + L.xw) + grp * 2 * kConsumerWarps;
+  float4 *blk = reinterpret_cast<float4 *>(smem + L.xw) + grp * kShortCombineTiles;
   float4 *gather = reinterpret_cast<float4 *>(smem + L.gather) + grp * kShortCombineTiles;
   const uint32_t bar_ready = sbase + L.bar_ready + 16u * grp;        // + 8 b
   const uint32_t bar_released = sbase + L.bar_released + 16u * grp;  // + 8 b
@@ -1120,7 +1132,7 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
         if (lane < cs) mbar_arrive_remote(bar_released + 8u * b, static_cast<uint32_t>(lane));
         combine_short<OP>([&](int t) { return gather[t]; }, g.K, inv_n, p.eps, lane, s0, s1);
       } else {
-        combine_long<OP>(peer, g.K, inv_n, p.eps, lane, wig, W, gbar, xw, s0, s1);
+        combine_blocks<OP>(peer, g.K, inv_n, p.eps, lane, wig, W, gbar, blk, s0, s1);
         // this warp has read every peer partial it needs: let the peers reuse them
         __syncwarp();
         if (lane < cs) mbar_arrive_remote(bar_released + 8u * b, static_cast<uint32_t>(lane));
@@ -1135,7 +1147,7 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
       if (g.K <= kShortCombineTiles) {
         combine_short<OP>(local, g.K, inv_n, p.eps, lane, s0, s1);
       } else {
-        combine_long<OP>(local, g.K, inv_n, p.eps, lane, wig, W, gbar, xw, s0, s1);
+        combine_blocks<OP>(local, g.K, inv_n, p.eps, lane, wig, W, gbar, blk, s0, s1);
       }
     }
 

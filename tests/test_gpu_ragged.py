@@ -305,3 +305,96 @@ def test_ragged_chunked_calls_equal_one_call(rw, op):
     torch.cuda.synchronize()
     got = ybuf[G:G + whole["total"]]
     assert torch.equal(got.view(torch.int16), whole["y"].view(torch.int16))
+
+
+@pytest.mark.parametrize("op", ["softmax", "layernorm"])
+def test_planned_call_refuses_a_mismatched_plan(rw, op):
+    """A plan made for another element type, or for a longer max_len, than the
+    planned call that reuses it: the rows whose record does not fit the call
+    (another bucket for the call's element size, or longer than its max_len)
+    are skipped, left untouched, and flagged as rejected rows; the others are
+    computed as usual."""
+    s = torch.cuda.current_stream().cuda_stream
+    # lengths as a bf16 plan sorts them: SMALL, SMALL (a MEDIUM row in fp32),
+    # MEDIUM, MEDIUM (a LARGE row in fp32), LARGE, LARGE
+    lens = np.array([100, 1500, 3000, 10000, 20000, 25000], dtype=np.int64)
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    rows, total = len(lens), int(off[-1])
+    offd = torch.from_numpy(off).cuda()
+    gx = torch.Generator("cpu").manual_seed(61)
+    x = (3.0 * torch.randn(total, generator=gx)).float()
+    gam, bet = gen_affine(30000, torch.float32, 61)
+    gd, bd = gam.cuda(), bet.cuda()
+    eps = eps_for(op)
+    ws = rw.ragged_workspace(rows)
+
+    params = {torch.float32: (gd, bd), torch.bfloat16: (gd.bfloat16(), bd.bfloat16())}
+
+    def planned(dtype, max_len):
+        xd = x.to(dtype).cuda()
+        y = canary_tensor(total, dtype)
+        code = rw.dtype_code(dtype)
+        gp, bp = params[dtype]  # kept alive until the call has run
+        if op == "softmax":
+            st = rw.rowop_softmax_ragged_planned(xd.data_ptr(), y.data_ptr(), offd.data_ptr(),
+                                                 rows, max_len, code, ws.data_ptr(), ws.numel(), s)
+        else:
+            st = rw.rowop_layernorm_ragged_planned(xd.data_ptr(), y.data_ptr(), gp.data_ptr(),
+                                                   bp.data_ptr(), offd.data_ptr(), rows, max_len,
+                                                   code, eps, ws.data_ptr(), ws.numel(), s)
+        assert st == rw.ROWOP_OK
+        torch.cuda.synchronize()
+        return xd, y
+
+    def check(dtype, xd, y, skipped):
+        assert rw.check_status() == rw.ROWOP_ERR_BAD_OFFSETS
+        ref = oracle_ragged(op, xd.double().cpu().numpy(), off,
+                            gam.to(dtype).double().numpy(), bet.to(dtype).double().numpy(), eps)
+        for i in range(rows):
+            seg = slice(int(off[i]), int(off[i + 1]))
+            if i in skipped:
+                assert is_canary(y[seg]).all(), f"row {i} written"
+            else:
+                assert_close(to_f64(y[seg]), ref[seg], dtype, f"row {i}")
+
+    # a bf16 plan reused by an fp32 call
+    st = rw.rowop_ragged_plan(offd.data_ptr(), rows, 30000, rw.ROWOP_BF16, ws.data_ptr(),
+                              ws.numel(), s)
+    assert st == rw.ROWOP_OK
+    xd, y = planned(torch.float32, 30000)
+    check(torch.float32, xd, y, {1, 3})
+    # a plan for max_len 30000 reused by a call whose max_len is 22000
+    xd, y = planned(torch.bfloat16, 22000)
+    check(torch.bfloat16, xd, y, {5})
+    # the matching call still works on the same plan
+    xd, y = planned(torch.bfloat16, 30000)
+    assert rw.check_status() == rw.ROWOP_OK
+    ref = oracle_ragged(op, xd.double().cpu().numpy(), off,
+                        gam.to(torch.bfloat16).double().numpy(),
+                        bet.to(torch.bfloat16).double().numpy(), eps)
+    assert_close(to_f64(y), ref, torch.bfloat16, "matching plan")
+
+
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
+@pytest.mark.parametrize("op", ALL_OPS)
+@pytest.mark.parametrize("base_off", [0, 1, 5])
+def test_ragged_longest_and_boundary_rows(rw, op, dtype, base_off):
+    """Rows at the bucket boundaries (+-1 element), the longest rows the call
+    allows at several head offsets (so their last chunk may start a tile of
+    its own), one- to three-element rows, among rows of every bucket."""
+    es = ESIZE[dtype]
+    max_len = 32768 if es == 2 else 40000
+    med = 32768 // es
+    special = [max_len, max_len - 1, max_len - 7, med, med + 1, med - 1, med + 9, 4096 // es,
+               4096 // es + 1, 1, 2, 3, 512 * 16 // es, 512 * 16 // es + 1]
+    lens = np.concatenate([np.array(special, dtype=np.int64),
+                           mixed_lengths(dtype, 120, seed=base_off + 101, max_len=max_len)])
+    np.random.default_rng(7).shuffle(lens)
+    got = run_ragged(rw, op, dtype, lens, max_len, seed=77, base_off=base_off)
+    assert rw.check_status() == 0
+    ref = oracle_ragged(op, got["x"].double().numpy(), got["off"], got["gam"].double().numpy(),
+                        got["bet"].double().numpy(), got["eps"])
+    assert_close(to_f64(got["y"]), ref, dtype, f"{op} boundary rows")
+    G, b = got["G"], got["base_off"]
+    assert is_canary(got["ybuf"][:G + b]).all()
+    assert is_canary(got["ybuf"][G + b + got["total"]:]).all()

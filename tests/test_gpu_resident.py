@@ -8,10 +8,9 @@ they can take:
   * the whole-tile kernel (the default for dense rows that are a whole
     number of tiles): one CTA per row of 8, 16 or 32 tiles, and cluster
     splits of LARGE rows into equal portions;
-  * the general resident kernel (ROWOP_RESIDENT=2): any row, one CTA or a
-    cluster split of any size, rows at one head offset (gamma/beta cached in
-    registers) and rows whose head offset moves from row to row, with and
-    without gamma/beta.
+  * the general resident kernel serves ragged rows; test_gpu_ragged.py holds
+    it to the staged design (ROWOP_RESIDENT=0, and the knobs that select the
+    staged design) bit for bit.
 Parity of every design against the oracle is checked here as well.
 """
 import os
@@ -61,14 +60,6 @@ def _bits(t):
     return t.view(torch.int32) if t.dtype == torch.float32 else t.view(torch.int16)
 
 
-# (cols, ld, x_off): MEDIUM rows of one to four tiles per warp, aligned, at a
-# fixed head offset (x_off) and at a head offset that moves from row to row
-# (ld not a multiple of 16 bytes); a row that ends mid-chunk
-SHAPES = [(1500, None, 0), (2100, None, 0), (3000, None, 0), (4096, None, 0), (4096, None, 3),
-          (4099, 4103, 1), (6000, None, 0), (8192, None, 0), (8191, 8195, 5), (12000, None, 2),
-          (16384, None, 0), (16383, None, 1)]
-
-
 # whole-tile rows: (cols per dtype size, design): MEDIUM rows of 8, 16 and 32
 # tiles on one CTA; LARGE rows split into equal portions
 FULL_MEDIUM = {4: (2048, 4096, 8192), 2: (4096, 8192, 16384)}
@@ -116,48 +107,4 @@ def test_whole_tile_stage_counts(rw, stages):
     for op in ("layernorm", "softmax"):
         a = _run(rw, op, torch.bfloat16, 301, 4096, 1, stages=stages, check=True)
         b = _run(rw, op, torch.bfloat16, 301, 4096, 0)
-        assert torch.equal(_bits(a), _bits(b))
-
-
-@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
-@pytest.mark.parametrize("op", ALL_OPS)
-@pytest.mark.parametrize("cols,ld,x_off", SHAPES)
-def test_resident_medium_equals_staged(rw, op, dtype, cols, ld, x_off):
-    if cols * ESIZE[dtype] <= 4096:
-        pytest.skip("SMALL bucket")
-    rows = 37
-    a = _run(rw, op, dtype, rows, cols, 2, ld=ld, x_off=x_off, check=True)
-    b = _run(rw, op, dtype, rows, cols, 0, ld=ld, x_off=x_off)
-    assert torch.equal(_bits(a), _bits(b))
-
-
-@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
-@pytest.mark.parametrize("op", ("layernorm", "rmsnorm"))
-def test_resident_without_affine(rw, op, dtype):
-    """NULL gamma / beta: ones and zeros, cached or not."""
-    for cols, x_off in ((4096, 0), (3000, 1)):
-        a = _run(rw, op, dtype, 9, cols, 2, x_off=x_off, affine=False, check=True)
-        b = _run(rw, op, dtype, 9, cols, 0, x_off=x_off, affine=False)
-        assert torch.equal(_bits(a), _bits(b))
-
-
-@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
-@pytest.mark.parametrize("op", ALL_OPS)
-@pytest.mark.parametrize("cols,ld,x_off", [(40000, None, 0), (40001, 40005, 3),
-                                          (70000, None, 0)])
-def test_resident_cluster_equals_staged(rw, op, dtype, cols, ld, x_off):
-    """LARGE rows split over clusters: the general resident design at every
-    cluster size it can hold the portions at equals the staged design."""
-    rows = 5
-    ref = _run(rw, op, dtype, rows, cols, 0, ld=ld, x_off=x_off, check=True)
-    for cs in (None, 2, 4, 8, 16):
-        got = _run(rw, op, dtype, rows, cols, 2, ld=ld, x_off=x_off, bucket=2, cluster=cs)
-        assert torch.equal(_bits(ref), _bits(got)), f"cluster {cs}"
-
-
-@pytest.mark.parametrize("stages", [1, 2, 5])
-def test_resident_stage_counts(rw, stages):
-    for op in ("layernorm", "softmax"):
-        a = _run(rw, op, torch.bfloat16, 301, 3000, 2, stages=stages, check=True)
-        b = _run(rw, op, torch.bfloat16, 301, 3000, 0)
         assert torch.equal(_bits(a), _bits(b))
