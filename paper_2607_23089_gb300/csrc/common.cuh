@@ -390,6 +390,11 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
 // A waiting thread is suspended until the phase completes or this many
 // nanoseconds pass, whichever comes first, instead of re-polling.
 constexpr uint32_t kWaitSuspendNs = 1000000;
+// pause between two polls of a barrier that is not yet complete
+#ifndef ROWOP_WAIT_BACKOFF_NS
+#define ROWOP_WAIT_BACKOFF_NS 64
+#endif
+constexpr uint32_t kWaitBackoffNs = ROWOP_WAIT_BACKOFF_NS;
 
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
@@ -409,6 +414,9 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   for (;;) {
+    // a retry only after a pause, so that a waiting warp leaves the issue
+    // slots to the warps that have work
+    __nanosleep(kWaitBackoffNs);
     if (mbar_try_wait(bar, parity)) return true;
     if (global_timer_ns() - t0 > limit_ns) return false;
   }

@@ -171,9 +171,13 @@ inline int64_t max_row_len_elems(int esize) {
 //                       variant: its results differ by rounding)
 //   ROWOP_BWD_CLUSTER   backward passes: split every row over a cluster of
 //                       this many CTAs (2, 4, 8, 16); changes rounding order
-//   ROWOP_RESIDENT      0 -> MEDIUM / LARGE rows (dense and ragged) use the
-//                       staged tile design even where a register-resident
-//                       one can hold them (they give the same bits)
+//   ROWOP_RESIDENT      0 -> dense MEDIUM rows of whole tiles use the staged
+//                       tile design instead of the register-resident one;
+//                       2 -> LARGE rows of whole tiles use the resident one
+//                       too, split over a cluster (all give the same bits)
+//   ROWOP_RESIDENT_GC   0 -> the register-resident design reads gamma/beta
+//                       per row instead of keeping them in registers (fewer
+//                       registers, more CTAs an SM; the same bits)
 struct Knobs {
   int force_bucket = -1;
   int cluster = 0;
@@ -183,6 +187,7 @@ struct Knobs {
   int softmax_online = 0;
   int bwd_cluster = 0;
   int resident = 1;
+  int res_gc = 1;
 };
 Knobs read_knobs();
 

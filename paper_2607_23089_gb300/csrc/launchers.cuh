@@ -146,11 +146,12 @@ constexpr int res_max_r() {
 }
 // Whole-tile dense rows on the specialised resident kernel: each of the NW
 // warps of a CTA owns exactly R tiles of each row (or of this CTA's portion
-// of it).  4-warp CTAs are compiled for four CTAs an SM, 8-warp CTAs with one
-// tile a warp for three, the others for two.
+// of it).  4-warp CTAs are compiled for four CTAs an SM when they cache
+// gamma/beta in registers and six when they do not, 8-warp CTAs with one tile
+// a warp for three, the others for two.
 template <int OP, typename T, int R, int NW, bool CLUSTER, bool GC>
 cudaError_t launch_res_full_k(TileParams p, int cs, const DenseCall &c, const DeviceInfo &d) {
-  constexpr int MINB = NW == 4 ? 4 : (R == 1 ? 3 : 2);
+  constexpr int MINB = NW == 4 ? (GC ? 4 : 6) : (R == 1 ? 3 : 2);
   auto kern = resident_full_kernel<OP, T, R, NW, CLUSTER, GC, MINB>;
   const void *kp = reinterpret_cast<const void *>(kern);
   const Knobs kn = read_knobs();
@@ -220,8 +221,8 @@ bool try_res_full(const TileParams &p, const DenseCall &c, const DeviceInfo &d, 
   if (bucket == kMedium) {
     if (kn.cluster > 1) return false;
     if (K == 8) {  // four warps of two tiles: more of each row per lane
-      *err = kAffine ? launch_res_full_k<OP, T, 2, 4, false, kAffine>(p, 1, c, d)
-                     : launch_res_full_k<OP, T, 2, 4, false, false>(p, 1, c, d);
+      *err = (kAffine && kn.res_gc) ? launch_res_full_k<OP, T, 2, 4, false, kAffine>(p, 1, c, d)
+                                    : launch_res_full_k<OP, T, 2, 4, false, false>(p, 1, c, d);
       return true;
     }
     if (K == 16) {
@@ -238,7 +239,10 @@ bool try_res_full(const TileParams &p, const DenseCall &c, const DeviceInfo &d, 
     }
     return false;
   }
-  // LARGE: equal portions of R tiles a warp over a cluster of 2..16 CTAs
+  // LARGE: equal portions of R tiles a warp over a cluster of 2..16 CTAs --
+  // on request only: two CTAs an SM fit fewer 16-CTA clusters than the
+  // staged design's three (1 MiB fp32 rows: 155 us against 148 us)
+  if (kn.resident < 2) return false;
   for (int R = res_max_r<T>(); R >= 2; R /= 2) {
     if (K % (kResWarps * R) != 0) continue;
     const int64_t cs = K / (kResWarps * R);

@@ -246,6 +246,11 @@ __global__ void __launch_bounds__(NW * 32, MINB) resident_full_kernel(const Tile
     }
   }
   const float inv_n = __frcp_rn(static_cast<float>(p.cols));
+  // gamma/beta read as vectors: present, 16-byte aligned (the row's columns
+  // are whole chunks, all below glen)
+  const bool pvec = kAffine && p.gvec && p.gamma && (OP == kRmsNorm || p.beta != nullptr);
+  const uint4 *gv = reinterpret_cast<const uint4 *>(p.gamma) + t0 * kTileChunks;
+  const uint4 *bv = reinterpret_cast<const uint4 *>(p.beta) + t0 * kTileChunks;
 
   uint32_t uses0 = 0, uses1 = 0;
   int s = 0;
@@ -344,6 +349,10 @@ __global__ void __launch_bounds__(NW * 32, MINB) resident_full_kernel(const Tile
             gp[i] = gc[k][i];
             bp[i] = bc[k][i];
           }
+        } else if (pvec) {
+          // aligned gamma/beta covering the row: one vector load each
+          chunk_to_pairs<T>(__ldg(gv + off[k] / kChunkBytes), gp);
+          if constexpr (OP == kLayerNorm) chunk_to_pairs<T>(__ldg(bv + off[k] / kChunkBytes), bp);
         } else {
           const int c = t0 * kTileChunks + static_cast<int>(off[k] / kChunkBytes);
           load_param_pairs<T>(static_cast<const T *>(p.gamma), p.gamma ? p.glen : 0, c, 0,

@@ -76,6 +76,7 @@ Knobs read_knobs() {
   k.softmax_online = env_int("ROWOP_SOFTMAX_ONLINE", 0);
   k.bwd_cluster = env_int("ROWOP_BWD_CLUSTER", 0);
   k.resident = env_int("ROWOP_RESIDENT", 1);
+  k.res_gc = env_int("ROWOP_RESIDENT_GC", 1);
   return k;
 }
 

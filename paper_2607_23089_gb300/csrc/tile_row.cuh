@@ -197,15 +197,12 @@ __device__ __forceinline__ TileMask tile_mask(int t, const ItemGeo &g, int lane,
   return m;
 }
 
-// first lane-level statistic of a tile: max (softmax family), sum
-// (LayerNorm), sum of squares (RMSNorm)
-template <int OP, typename T>
-__device__ __forceinline__ float tile_lane_first(const unsigned char *tsm, const TileMask &m,
-                                                 int lane) {
-  constexpr int NP = Elem<T>::kPerChunk / 2;
-  f2 p0[NP], p1[NP];
-  chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(tsm + lane * kChunkBytes), p0);
-  chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(tsm + (lane + 32) * kChunkBytes), p1);
+// first lane-level statistic of a tile from the lane's two chunks (chunk l,
+// then chunk l+32) as fp32 pairs: max (softmax family), sum (LayerNorm), sum
+// of squares (RMSNorm)
+template <int OP, int NP>
+__device__ __forceinline__ float tile_pairs_first(const f2 (&p0)[NP], const f2 (&p1)[NP],
+                                                  const TileMask &m) {
   if constexpr (OP == kSoftmax || OP == kLogSoftmax) {
     return chunk_max<NP>(p1, chunk_max<NP>(p0, -INFINITY, m.lo0, m.hi0), m.lo1, m.hi1);
   } else if constexpr (OP == kLayerNorm) {
@@ -218,13 +215,9 @@ __device__ __forceinline__ float tile_lane_first(const unsigned char *tsm, const
 
 // second lane-level statistic: sum exp(x - ref) (softmax family, ref = m_t)
 // or sum (x - ref)^2 (LayerNorm, ref = mean_t)
-template <int OP, typename T>
-__device__ __forceinline__ float tile_lane_second(const unsigned char *tsm, const TileMask &m,
-                                                  int lane, float ref) {
-  constexpr int NP = Elem<T>::kPerChunk / 2;
-  f2 p0[NP], p1[NP];
-  chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(tsm + lane * kChunkBytes), p0);
-  chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(tsm + (lane + 32) * kChunkBytes), p1);
+template <int OP, int NP>
+__device__ __forceinline__ float tile_pairs_second(const f2 (&p0)[NP], const f2 (&p1)[NP],
+                                                   const TileMask &m, float ref) {
   const f2 r2 = f2_bcast(ref);
   if constexpr (OP == kSoftmax || OP == kLogSoftmax) {
     if (ref == -INFINITY) return 0.f;  // no element of the tile is above -inf
@@ -234,6 +227,33 @@ __device__ __forceinline__ float tile_lane_second(const unsigned char *tsm, cons
     return f2_total(chunk_sum_sqdev<NP>(p1, r2, chunk_sum_sqdev<NP>(p0, r2, f2_bcast(0.f), m.lo0, m.hi0),
                                         m.lo1, m.hi1));
   }
+}
+
+// The lane's two chunks of a staged tile as fp32 pairs.
+template <typename T>
+__device__ __forceinline__ void tile_lane_pairs(const unsigned char *tsm, int lane,
+                                                f2 (&p0)[Elem<T>::kPerChunk / 2],
+                                                f2 (&p1)[Elem<T>::kPerChunk / 2]) {
+  chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(tsm + lane * kChunkBytes), p0);
+  chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(tsm + (lane + 32) * kChunkBytes), p1);
+}
+
+template <int OP, typename T>
+__device__ __forceinline__ float tile_lane_first(const unsigned char *tsm, const TileMask &m,
+                                                 int lane) {
+  constexpr int NP = Elem<T>::kPerChunk / 2;
+  f2 p0[NP], p1[NP];
+  tile_lane_pairs<T>(tsm, lane, p0, p1);
+  return tile_pairs_first<OP, NP>(p0, p1, m);
+}
+
+template <int OP, typename T>
+__device__ __forceinline__ float tile_lane_second(const unsigned char *tsm, const TileMask &m,
+                                                  int lane, float ref) {
+  constexpr int NP = Elem<T>::kPerChunk / 2;
+  f2 p0[NP], p1[NP];
+  tile_lane_pairs<T>(tsm, lane, p0, p1);
+  return tile_pairs_second<OP, NP>(p0, p1, m, ref);
 }
 
 // B tiles of one warp, lt0, lt0 + W, ..., lt0 + W(B-1), all below the item's
@@ -318,6 +338,12 @@ __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const It
     }
     return true;
   }
+  // one tile at a time (the fused ragged kernel): the lane's pairs stay in
+  // registers for the second sweep; larger batches read the stage again
+  // (keeping them would spill)
+  constexpr int NP = E / 2;
+  constexpr bool kKeep = (OP != kRmsNorm) && B == 1;
+  f2 kp0[kKeep ? B : 1][NP], kp1[kKeep ? B : 1][NP];
 #pragma unroll
   for (int q = 0; q < B; ++q) {
     const int lt = lt0 + q * W;
@@ -330,7 +356,12 @@ __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const It
     if constexpr (RESID)
       residual_tile<T>(const_cast<unsigned char *>(stage) + lt * kTileBytes, t, g, lane, p);
     const TileMask m = FULL ? TileMask{0, E, 0, E} : tile_mask<T>(t, g, lane, tile_is_full(t, g));
-    a[q] = tile_lane_first<OP, T>(stage + lt * kTileBytes, m, lane);
+    if constexpr (kKeep) {
+      tile_lane_pairs<T>(stage + lt * kTileBytes, lane, kp0[q], kp1[q]);
+      a[q] = tile_pairs_first<OP, NP>(kp0[q], kp1[q], m);
+    } else {
+      a[q] = tile_lane_first<OP, T>(stage + lt * kTileBytes, m, lane);
+    }
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -368,14 +399,18 @@ __device__ __forceinline__ bool pass1_batch(const unsigned char *stage, const It
         }
       }
       const TileMask m = FULL ? TileMask{0, E, 0, E} : tile_mask<T>(t, g, lane, full);
-      b[q] = tile_lane_second<OP, T>(stage + lt * kTileBytes, m, lane, ref[q]);
+      if constexpr (kKeep) {
+        b[q] = tile_pairs_second<OP, NP>(kp0[q], kp1[q], m, ref[q]);
+      } else {
+        b[q] = tile_lane_second<OP, T>(stage + lt * kTileBytes, m, lane, ref[q]);
+      }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
 #pragma unroll
       for (int q = 0; q < B; ++q) b[q] = __fadd_rn(b[q], __shfl_xor_sync(kFullMask, b[q], o));
     }
-    if (lane == 0) {
+  if (lane == 0) {
 #pragma unroll
       for (int q = 0; q < B; ++q)
         part[lt0 + q * W] = (OP == kLayerNorm) ? make_float4(a[q], ref[q], b[q], ntf[q])
@@ -400,7 +435,7 @@ __device__ __forceinline__ bool pass1_warp(const unsigned char *stage, const Ite
   int waited = -1;
   int lt0 = wig;
   while (lt0 < ntl) {
-    const int left = (ntl - lt0 + W - 1) / W;
+    const int left = (ntl - lt0 + W - 1) >> (31 - __clz(W));  // W is a power of two
     const int bsz = left >= PB ? PB : (left >= 2 ? 2 : 1);
     const int ta = g.t0 + lt0, tb = ta + (bsz - 1) * W;
     const bool full = ta >= full0 && tb < full1;
@@ -651,6 +686,53 @@ __device__ __forceinline__ void chunk_store_edge(const unsigned char *csm, int c
   store_chunk<T>(v, owin, out_row, c, g.h, lo, hi, p.out_vec != 0);
 }
 
+// gamma/beta chunk at v (16-byte aligned vectors, v = chunk c of the
+// parameter array) realigned for head offset H: columns c E - H .. c E - H +
+// E - 1, from chunks c - 1 and c.
+template <typename T, int H>
+__device__ __forceinline__ uint4 param_chunk_at(const uint4 *__restrict__ v) {
+  constexpr int E = Elem<T>::kPerChunk;
+  if constexpr (H == 0) {
+    return __ldg(v);
+  } else {
+    const uint4 A = __ldg(v - 1);
+    const uint4 B = __ldg(v);
+    if constexpr (E == 4) {
+      return shift_words<H>(A, B);
+    } else if constexpr ((H & 1) == 0) {
+      return shift_words<H / 2>(A, B);
+    } else {
+      return shift_half<(H + 1) / 2>(A, B);
+    }
+  }
+}
+
+// Both chunks of a lane in a tile made only of fast chunks (see
+// chunk_store_fast), c0 the lane's first chunk: every address is formed once
+// for the tile and the second chunk (c0 + 32) is reached by a fixed offset.
+template <int OP, typename T, int H>
+__device__ __forceinline__ void tile_store_fast(const unsigned char *lsm, int c0, float s0,
+                                                float s1, const T *gamma, const T *beta,
+                                                char *owin) {
+  constexpr int NP = Elem<T>::kPerChunk / 2;
+  const uint4 *gv = reinterpret_cast<const uint4 *>(gamma) + c0;
+  const uint4 *bv = reinterpret_cast<const uint4 *>(beta) + c0;
+  uint4 *ov = reinterpret_cast<uint4 *>(owin) + c0;
+  f2 v[2][NP], g[2][NP], b[2][NP];
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(lsm + 32 * u * kChunkBytes), v[u]);
+    if constexpr (OP == kLayerNorm || OP == kRmsNorm)
+      chunk_to_pairs<T>(param_chunk_at<T, H>(gv + 32 * u), g[u]);
+    if constexpr (OP == kLayerNorm) chunk_to_pairs<T>(param_chunk_at<T, H>(bv + 32 * u), b[u]);
+  }
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    normalize_pairs<OP, NP>(v[u], s0, s1, g[u], b[u]);
+    stg_stream(ov + 32 * u, pairs_to_chunk<T>(v[u]));
+  }
+}
+
 // pass 2 over this warp's tiles (wig, wig + W, ...) of an item whose head
 // offset is H.  Chunks [g.cf, cfast) take the fast path, the row's other
 // chunks the general one: tiles made only of fast chunks (all but the row's
@@ -670,10 +752,8 @@ __device__ __forceinline__ void pass2_tiles(const unsigned char *stage, const It
   for (int lt = wig; lt < ntl; lt += W) {
     const int t = g.t0 + lt;
     if (t < fa || t >= fb) continue;
-#pragma unroll
-    for (int u = 0; u < 2; ++u)
-      chunk_store_fast<OP, T, H>(stage + lt * kTileBytes + (lane + 32 * u) * kChunkBytes,
-                                 t * kTileChunks + lane + 32 * u, s0, s1, gamma, beta, owin);
+    tile_store_fast<OP, T, H>(stage + lt * kTileBytes + lane * kChunkBytes,
+                              t * kTileChunks + lane, s0, s1, gamma, beta, owin);
   }
   for (int lt = wig; lt < ntl; lt += W) {
     const int t = g.t0 + lt;
