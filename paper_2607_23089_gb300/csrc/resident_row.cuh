@@ -227,17 +227,17 @@ __global__ void __launch_bounds__(NW * 32, MINB) resident_full_kernel(const Tile
   const uint32_t bar_ready = sbase + L.bar_ready;
   const uint32_t bar_released = sbase + L.bar_released;
 
-  // byte offset of each slot in the portion (stage and row alike)
-  uint32_t off[NS];
-#pragma unroll
-  for (int k = 0; k < NS; ++k)
-    off[k] = static_cast<uint32_t>(((w + NW * (k >> 1)) * kTileChunks + lane + 32 * (k & 1)) *
-                                   kChunkBytes);
+  // byte offset of each slot in the portion (stage and row alike): the
+  // lane's base plus a compile-time offset per slot
+  const uint32_t obase = static_cast<uint32_t>((w * kTileChunks + lane) * kChunkBytes);
+  auto off = [&](int k) -> uint32_t {
+    return obase + static_cast<uint32_t>((NW * (k >> 1) * kTileChunks + 32 * (k & 1)) * kChunkBytes);
+  };
   f2 gc[GC ? NS : 1][NP], bc[GC ? NS : 1][NP];
   if constexpr (GC) {
 #pragma unroll
     for (int k = 0; k < NS; ++k) {
-      const int c = t0 * kTileChunks + static_cast<int>(off[k] / kChunkBytes);
+      const int c = t0 * kTileChunks + static_cast<int>(off(k) / kChunkBytes);
       load_param_pairs<T>(static_cast<const T *>(p.gamma), p.gamma ? p.glen : 0, c, 0,
                           p.gvec != 0, 1.f, gc[k]);
       if constexpr (OP == kLayerNorm)
@@ -270,7 +270,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) resident_full_kernel(const Tile
       const unsigned char *stage = smem + static_cast<size_t>(s) * p.stage_bytes;
 #pragma unroll
       for (int k = 0; k < NS; ++k)
-        chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(stage + off[k]), x[k]);
+        chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(stage + off(k)), x[k]);
       full_pass1<OP, T, R, NW>(x, w, lane, part);
     }
     // every warp has its chunks of row r in registers past this barrier
@@ -351,10 +351,10 @@ __global__ void __launch_bounds__(NW * 32, MINB) resident_full_kernel(const Tile
           }
         } else if (pvec) {
           // aligned gamma/beta covering the row: one vector load each
-          chunk_to_pairs<T>(__ldg(gv + off[k] / kChunkBytes), gp);
-          if constexpr (OP == kLayerNorm) chunk_to_pairs<T>(__ldg(bv + off[k] / kChunkBytes), bp);
+          chunk_to_pairs<T>(__ldg(gv + off(k) / kChunkBytes), gp);
+          if constexpr (OP == kLayerNorm) chunk_to_pairs<T>(__ldg(bv + off(k) / kChunkBytes), bp);
         } else {
-          const int c = t0 * kTileChunks + static_cast<int>(off[k] / kChunkBytes);
+          const int c = t0 * kTileChunks + static_cast<int>(off(k) / kChunkBytes);
           load_param_pairs<T>(static_cast<const T *>(p.gamma), p.gamma ? p.glen : 0, c, 0,
                               p.gvec != 0, 1.f, gp);
           if constexpr (OP == kLayerNorm)
@@ -363,7 +363,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) resident_full_kernel(const Tile
         }
       }
       normalize_pairs<OP, NP>(x[k], s0, s1, gp, bp);
-      stg_stream(orow + off[k], pairs_to_chunk<T>(x[k]));
+      stg_stream(orow + off(k), pairs_to_chunk<T>(x[k]));
     }
   }
 
