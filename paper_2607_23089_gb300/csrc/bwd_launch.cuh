@@ -5,6 +5,7 @@
 
 #include "bwd_call.h"
 #include "bwd_row.cuh"
+#include "bwd_tile.cuh"
 #include "launch_util.cuh"
 
 namespace rowop {
@@ -151,6 +152,74 @@ cudaError_t launch_bwd_k(const BwdParams &p, const BwdShape &s, const BwdCall &c
                                 c.dbeta, c.stream);
 }
 
+// The whole-tile norm kernel (bwd_tile.cuh) on rows of NW R tiles: compiled
+// for 16 warps an SM, as many stages as the CTA's share of shared memory
+// holds (up to kBwdTileMaxStages), a grid of at most the resident CTAs and
+// at most one CTA per row, and the finalize over the grid's partial rows.
+template <int OP, typename T, int R, int NW>
+cudaError_t launch_bwd_tile_k(const BwdCall &c, const DeviceInfo &d) {
+  constexpr int MINB = 16 / NW;
+  auto kern = bwd_tile_kernel<OP, T, R, NW, MINB>;
+  const void *kp = reinterpret_cast<const void *>(kern);
+  cudaError_t e = prepare_kernel(kp, d, false);
+  if (e != cudaSuccess) return e;
+  constexpr uint32_t stage_bytes = 2u * NW * R * kTileBytes;
+  const int stages = static_cast<int>(std::max<int64_t>(
+      1, std::min<int64_t>(kBwdTileMaxStages, res_stage_budget(MINB) / stage_bytes)));
+  const BwdTileSmem L(stage_bytes, stages, NW);
+  const int occ = std::max(1, cached_occupancy(kp, NW * 32, L.total, 1, nullptr));
+  const int64_t grid = std::max<int64_t>(
+      1, std::min<int64_t>({c.rows, static_cast<int64_t>(occ) * d.sm_count,
+                            static_cast<int64_t>(kBwdMaxPartsPerSm) * d.sm_count}));
+  const bool want_params = c.dgamma || c.dbeta;
+  BwdTileParams p = {};
+  p.x = c.a;
+  p.dy = c.dy;
+  p.dx = c.dx;
+  p.gamma = c.gamma;
+  p.part = want_params ? static_cast<float *>(c.ws) : nullptr;
+  p.rows = c.rows;
+  p.cols = c.cols;
+  p.ld = c.ld;
+  p.eps = c.eps;
+  p.stages = stages;
+  p.stage_bytes = stage_bytes;
+  p.timeout_ns = kWaitLimitNs;
+  p.status = d.status;
+  kern<<<static_cast<unsigned>(grid), NW * 32, L.total, c.stream>>>(p);
+  e = cudaGetLastError();
+  if (e != cudaSuccess || !want_params) return e;
+  return launch_bwd_finalize<T>(one_segment(p.part, grid, c.cols), c.cols,
+                                OP == kLayerNorm ? 2 : 1, c.dgamma, c.dbeta, c.stream);
+}
+
+// Dense norm rows the whole-tile kernel takes: x, dy and dx 16-byte aligned,
+// a row stride of whole chunks, and rows of 4, 8 or 16 warps' tiles (one
+// tile a warp for 16-bit types, two for fp32: 16 elements a lane per
+// tensor).  Returns false, launching nothing, for any other shape.
+template <int OP, typename T>
+bool try_bwd_tile(const BwdCall &c, const DeviceInfo &d, cudaError_t *err) {
+  constexpr int SZ = sizeof(T);
+  constexpr int E = 16 / SZ;
+  constexpr int R = SZ == 4 ? 2 : 1;
+  if (c.rows <= 0 || !aligned16(c.a) || !aligned16(c.dy) || !aligned16(c.dx) ||
+      (c.ld * SZ) % 16 != 0 || c.cols % (kTileChunks * E * R) != 0)
+    return false;
+  switch (c.cols / (kTileChunks * E * R)) {
+    case 4:
+      *err = launch_bwd_tile_k<OP, T, R, 4>(c, d);
+      return true;
+    case 8:
+      *err = launch_bwd_tile_k<OP, T, R, 8>(c, d);
+      return true;
+    case 16:
+      *err = launch_bwd_tile_k<OP, T, R, 16>(c, d);
+      return true;
+    default:
+      return false;
+  }
+}
+
 template <int OP, typename T>
 cudaError_t launch_bwd_t(const BwdCall &c, const DeviceInfo &d) {
   constexpr int SZ = sizeof(T);
@@ -165,10 +234,15 @@ cudaError_t launch_bwd_t(const BwdCall &c, const DeviceInfo &d) {
     return launch_bwd_finalize<T>(one_segment(nullptr, 0, c.cols), c.cols, nacc, c.dgamma,
                                   c.dbeta, c.stream);
   }
+  const Knobs kn = read_knobs();
+  const int force_cs = kn.bwd_cluster;
+  if constexpr (kNorm) {
+    cudaError_t err = cudaSuccess;
+    if (kn.bwd_tile != 0 && force_cs == 0 && try_bwd_tile<OP, T>(c, d, &err)) return err;
+  }
   bool vec = ((c.ld * SZ) % 16 == 0) && congruent16(c.a, c.dy) && congruent16(c.a, c.dx);
   int h = vec ? static_cast<int>((reinterpret_cast<uintptr_t>(c.a) & 15u) / SZ) : 0;
   int64_t units = vec ? ceil_div(h + c.cols, E) : ceil_div(c.cols, E);
-  const int force_cs = read_knobs().bwd_cluster;
   BwdShape s;
   if (!bwd_shape(units, CPT, force_cs, small_cta, s)) {
     // a row of the longest length that starts mid-chunk needs one window

@@ -156,8 +156,8 @@ inline int64_t max_row_len_elems(int esize) {
 }
 
 // Test-and-tuning knobs read from the environment (none changes results but
-// ROWOP_SOFTMAX_ONLINE and ROWOP_BWD_CLUSTER, which select another way to
-// round):
+// ROWOP_SOFTMAX_ONLINE, ROWOP_BWD_CLUSTER and ROWOP_BWD_TILE, which select
+// another way to round):
 //   ROWOP_FORCE_BUCKET  0/1/2 -> dense rows use that design when it can hold
 //                       the row (SMALL only for rows of <= 288 chunks)
 //   ROWOP_CLUSTER       cluster size for split rows (1, 2, 4, 8, 16)
@@ -178,6 +178,9 @@ inline int64_t max_row_len_elems(int esize) {
 //   ROWOP_RESIDENT_GC   0 -> the register-resident design reads gamma/beta
 //                       per row instead of keeping them in registers (fewer
 //                       registers, more CTAs an SM; the same bits)
+//   ROWOP_BWD_TILE      0 -> dense norm backward rows of whole tiles use the
+//                       team design instead of the whole-tile one (another
+//                       summation order)
 struct Knobs {
   int force_bucket = -1;
   int cluster = 0;
@@ -188,6 +191,7 @@ struct Knobs {
   int bwd_cluster = 0;
   int resident = 1;
   int res_gc = 1;
+  int bwd_tile = 1;
 };
 Knobs read_knobs();
 

@@ -77,6 +77,7 @@ Knobs read_knobs() {
   k.bwd_cluster = env_int("ROWOP_BWD_CLUSTER", 0);
   k.resident = env_int("ROWOP_RESIDENT", 1);
   k.res_gc = env_int("ROWOP_RESIDENT_GC", 1);
+  k.bwd_tile = env_int("ROWOP_BWD_TILE", 1);
   return k;
 }
 

@@ -498,3 +498,47 @@ def test_workload_ragged_softmax_backward(rw):
         check(got[None, off[i]:off[i + 1]], orc.softmax_backward(a64, d64),
               scales("softmax", a64, d64, None, 0)[0], torch.float32, R_COMP,
               f"ragged softmax backward workload row {i}")
+
+
+# rows of whole 1 KiB tiles that the whole-tile norm kernel takes: 4, 8 and
+# 16 warps of one tile (16-bit types) or two tiles (fp32) each
+WHOLE_TILE_COLS = {4: (2048, 4096, 8192), 2: (2048, 4096, 8192)}
+
+
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
+@pytest.mark.parametrize("op", NORMS)
+def test_backward_whole_tile_rows(rw, op, dtype, monkeypatch):
+    """The whole-tile design (x and dy staged by bulk copies, gamma and the
+    dgamma / dbeta sums in registers) and the team design both hold the
+    oracle's tolerance: few rows (fewer than the stages), many rows per CTA
+    (the stage ring wraps many times), a row stride wider than the row, and
+    no gamma."""
+    es = ESIZE[dtype]
+    for cols in WHOLE_TILE_COLS[es]:
+        for tile in ("1", "0"):
+            monkeypatch.setenv("ROWOP_BWD_TILE", tile)
+            run_bwd(rw, op, dtype, 3, cols, seed=cols + 1)
+            run_bwd(rw, op, dtype, 1500 if cols < 8192 else 700, cols, seed=cols + 2)
+            run_bwd(rw, op, dtype, 37, cols, ld=cols + 64, seed=cols + 3)
+            run_bwd(rw, op, dtype, 37, cols, affine=False, seed=cols + 4)
+
+
+@pytest.mark.parametrize("op", NORMS)
+def test_backward_whole_tile_options(rw, op):
+    """dgamma / dbeta each optional, in place over x or dy, and rows that are
+    not 16-byte aligned (the team design takes those) on the same shape."""
+    for want in ((True, False), (False, True), (False, False)):
+        run_bwd(rw, op, torch.bfloat16, 300, 4096, want=want, seed=21)
+    for where in ("dy", "a"):
+        run_bwd(rw, op, torch.bfloat16, 300, 4096, inplace=where, seed=22)
+    run_bwd(rw, op, torch.bfloat16, 30, 4096, offs=(8, 8, 8), seed=23)
+    run_bwd(rw, op, torch.bfloat16, 30, 4096, offs=(1, 1, 1), seed=24)
+
+
+@pytest.mark.parametrize("op", NORMS)
+def test_backward_whole_tile_deterministic(rw, op):
+    outs = [run_bwd(rw, op, torch.bfloat16, 2000, 4096, seed=5, compare=(i == 0))
+            for i in range(2)]
+    for k in (0, 1, 2):
+        if outs[0][k] is not None:
+            assert torch.equal(_bits(outs[0][k]), _bits(outs[1][k]))
