@@ -619,16 +619,24 @@ __device__ __forceinline__ uint4 param_chunk_fixed(const T *__restrict__ g, int 
 // pass 2 fast path for one chunk: entirely the row's, output 16-byte
 // congruent to the input, gamma/beta aligned and covering its columns.  Same
 // arithmetic as chunk_store_edge.
-template <int OP, typename T, int H>
+template <int OP, typename T, int H, bool P>
 __device__ __forceinline__ void chunk_store_fast(const unsigned char *csm, int c, float s0,
                                                  float s1, const T *gamma, const T *beta,
                                                  char *owin) {
   constexpr int NP = Elem<T>::kPerChunk / 2;
   f2 v[NP], g[NP], b[NP];
   chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(csm), v);
-  if constexpr (OP == kLayerNorm || OP == kRmsNorm)
-    chunk_to_pairs<T>(param_chunk_fixed<T, H>(gamma, c), g);
-  if constexpr (OP == kLayerNorm) chunk_to_pairs<T>(param_chunk_fixed<T, H>(beta, c), b);
+  if constexpr (!P) {
+#pragma unroll
+    for (int i = 0; i < NP; ++i) {
+      g[i] = f2_bcast(1.f);
+      b[i] = f2_bcast(0.f);
+    }
+  } else {
+    if constexpr (OP == kLayerNorm || OP == kRmsNorm)
+      chunk_to_pairs<T>(param_chunk_fixed<T, H>(gamma, c), g);
+    if constexpr (OP == kLayerNorm) chunk_to_pairs<T>(param_chunk_fixed<T, H>(beta, c), b);
+  }
   normalize_pairs<OP, NP>(v, s0, s1, g, b);
   stg_stream(owin + static_cast<int64_t>(c) * kChunkBytes, pairs_to_chunk<T>(v));
 }
@@ -710,7 +718,9 @@ __device__ __forceinline__ uint4 param_chunk_at(const uint4 *__restrict__ v) {
 // Both chunks of a lane in a tile made only of fast chunks (see
 // chunk_store_fast), c0 the lane's first chunk: every address is formed once
 // for the tile and the second chunk (c0 + 32) is reached by a fixed offset.
-template <int OP, typename T, int H>
+// P: gamma (and beta) are present; without them (P false) the norms take
+// gamma = 1 and beta = 0, as the general path does.
+template <int OP, typename T, int H, bool P>
 __device__ __forceinline__ void tile_store_fast(const unsigned char *lsm, int c0, float s0,
                                                 float s1, const T *gamma, const T *beta,
                                                 char *owin) {
@@ -722,9 +732,17 @@ __device__ __forceinline__ void tile_store_fast(const unsigned char *lsm, int c0
 #pragma unroll
   for (int u = 0; u < 2; ++u) {
     chunk_to_pairs<T>(*reinterpret_cast<const uint4 *>(lsm + 32 * u * kChunkBytes), v[u]);
-    if constexpr (OP == kLayerNorm || OP == kRmsNorm)
-      chunk_to_pairs<T>(param_chunk_at<T, H>(gv + 32 * u), g[u]);
-    if constexpr (OP == kLayerNorm) chunk_to_pairs<T>(param_chunk_at<T, H>(bv + 32 * u), b[u]);
+    if constexpr (!P) {
+#pragma unroll
+      for (int i = 0; i < NP; ++i) {
+        g[u][i] = f2_bcast(1.f);
+        b[u][i] = f2_bcast(0.f);
+      }
+    } else {
+      if constexpr (OP == kLayerNorm || OP == kRmsNorm)
+        chunk_to_pairs<T>(param_chunk_at<T, H>(gv + 32 * u), g[u]);
+      if constexpr (OP == kLayerNorm) chunk_to_pairs<T>(param_chunk_at<T, H>(bv + 32 * u), b[u]);
+    }
   }
 #pragma unroll
   for (int u = 0; u < 2; ++u) {
@@ -738,7 +756,7 @@ __device__ __forceinline__ void tile_store_fast(const unsigned char *lsm, int c0
 // chunks the general one: tiles made only of fast chunks (all but the row's
 // ends, as a rule) run first with both chunks of a lane issued together, then
 // the remaining tiles chunk by chunk.
-template <int OP, typename T, int H>
+template <int OP, typename T, int H, bool P>
 __device__ __forceinline__ void pass2_tiles(const unsigned char *stage, const ItemGeo &g, int wig,
                                             int W, int lane, float s0, float s1,
                                             const TileParams &p, char *owin, T *out_row,
@@ -752,8 +770,8 @@ __device__ __forceinline__ void pass2_tiles(const unsigned char *stage, const It
   for (int lt = wig; lt < ntl; lt += W) {
     const int t = g.t0 + lt;
     if (t < fa || t >= fb) continue;
-    tile_store_fast<OP, T, H>(stage + lt * kTileBytes + lane * kChunkBytes,
-                              t * kTileChunks + lane, s0, s1, gamma, beta, owin);
+    tile_store_fast<OP, T, H, P>(stage + lt * kTileBytes + lane * kChunkBytes,
+                                 t * kTileChunks + lane, s0, s1, gamma, beta, owin);
   }
   for (int lt = wig; lt < ntl; lt += W) {
     const int t = g.t0 + lt;
@@ -762,7 +780,7 @@ __device__ __forceinline__ void pass2_tiles(const unsigned char *stage, const It
       const int c = t * kTileChunks + lane + 32 * u;
       const unsigned char *csm = stage + lt * kTileBytes + (lane + 32 * u) * kChunkBytes;
       if (c >= g.cf && c < cfast) {
-        chunk_store_fast<OP, T, H>(csm, c, s0, s1, gamma, beta, owin);
+        chunk_store_fast<OP, T, H, P>(csm, c, s0, s1, gamma, beta, owin);
       } else if (c < g.nc) {
         chunk_store_edge<OP, T, H>(csm, c, g, s0, s1, p, owin, out_row);
       }
@@ -778,29 +796,34 @@ __device__ __forceinline__ void pass2_item(const unsigned char *stage, const Ite
                                            const TileParams &p, char *owin, T *out_row) {
   constexpr int E = Elem<T>::kPerChunk;
   constexpr bool kAffine = (OP == kLayerNorm || OP == kRmsNorm);
+  // no parameters at all: gamma = 1 and beta = 0 without loads
+  const bool none = kAffine && !p.gamma && !p.beta;
   const bool params_ok =
-      !kAffine || (p.gvec && p.gamma && (OP == kRmsNorm || p.beta != nullptr));
+      !kAffine || none || (p.gvec && p.gamma && (OP == kRmsNorm || p.beta != nullptr));
   // fast chunks end where the row's full chunks end, or where the vector
   // parameter loads would reach past gamma/beta (they read up to column
   // (c + 1) * E - 1 for chunk c)
   int cfast = g.cf;
   if (p.out_vec && params_ok)
-    cfast = kAffine ? static_cast<int>(min(static_cast<int64_t>(g.cl), p.glen / E)) : g.cl;
-  if constexpr (EXACT || !kAffine) {
-    pass2_tiles<OP, T, 0>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast);
+    cfast = (kAffine && !none) ? static_cast<int>(min(static_cast<int64_t>(g.cl), p.glen / E))
+                               : g.cl;
+  if (!kAffine || none) {
+    pass2_tiles<OP, T, 0, false>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast);
+  } else if constexpr (EXACT) {
+    pass2_tiles<OP, T, 0, true>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast);
   } else {
     switch (g.h) {
-      case 0: pass2_tiles<OP, T, 0>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
-      case 1: pass2_tiles<OP, T, 1>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
-      case 2: pass2_tiles<OP, T, 2>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
-      case 3: pass2_tiles<OP, T, 3>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+      case 0: pass2_tiles<OP, T, 0, true>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+      case 1: pass2_tiles<OP, T, 1, true>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+      case 2: pass2_tiles<OP, T, 2, true>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+      case 3: pass2_tiles<OP, T, 3, true>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
       default:
         if constexpr (E == 8) {
           switch (g.h) {
-            case 4: pass2_tiles<OP, T, 4>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
-            case 5: pass2_tiles<OP, T, 5>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
-            case 6: pass2_tiles<OP, T, 6>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
-            default: pass2_tiles<OP, T, 7>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+            case 4: pass2_tiles<OP, T, 4, true>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+            case 5: pass2_tiles<OP, T, 5, true>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+            case 6: pass2_tiles<OP, T, 6, true>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
+            default: pass2_tiles<OP, T, 7, true>(stage, g, wig, W, lane, s0, s1, p, owin, out_row, cfast); break;
           }
         }
         break;
@@ -809,61 +832,19 @@ __device__ __forceinline__ void pass2_item(const unsigned char *stage, const Ite
 }
 
 // ---------------------------------------------------------------------------
-// producer: edge chunks loaded now, written into the stage one item later
+// producer: one warp.  Lane 0 owns the ring (stage barriers, item records);
+// the lanes share the per-item work so that no step waits on another:
+//   * ragged records are claimed in batches and looked up one per lane (the
+//     LARGE rows of this CTA up to 32 at a time, the MEDIUM rows
+//     kFetchBatch per work-counter step), so one round trip serves several
+//     items;
+//   * lane pc issues piece pc's bulk copy;
+//   * the at most two 16-byte chunks a row only partly covers are read one
+//     element per lane (all loads in flight together) and written into the
+//     stage after the next item's record is in hand, so their latency
+//     overlaps that lookup.
 // ---------------------------------------------------------------------------
-// The head chunk (window chunk 0) and the tail chunk (the last) of an item,
-// in fixed fields so nothing is indexed at run time.
-struct PendingEdges {
-  bool active;        // an item's edges still have to be written
-  bool head, tail;    // which edge chunks it has
-  bool tail_own_bar;  // the tail chunk lies in another piece than the head
-  uint32_t head_dst, tail_dst, head_bar, tail_bar;
-  uint4 head_val, tail_val;
-};
-
-__device__ __forceinline__ void st_shared_u4(uint32_t dst, const uint4 &v) {
-  asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(v.x), "r"(v.y),
-               "r"(v.z), "r"(v.w)
-               : "memory");
-}
-
-__device__ __forceinline__ uint32_t ld_u16_issue(const void *p) {
-  unsigned short v;
-  asm volatile("ld.global.u16 %0, [%1];" : "=h"(v) : "l"(p));
-  return v;
-}
-__device__ __forceinline__ uint32_t ld_u32_issue(const void *p) {
-  uint32_t v;
-  asm volatile("ld.global.u32 %0, [%1];" : "=r"(v) : "l"(p));
-  return v;
-}
-// Chunk image of window chunk c with only the row's elements (issued loads).
-template <typename T>
-__device__ __forceinline__ uint4 issue_edge_chunk(const T *in_row, int64_t c, int h, int64_t n) {
-  constexpr int E = Elem<T>::kPerChunk;
-  uint32_t w[4] = {0u, 0u, 0u, 0u};
-#pragma unroll
-  for (int e = 0; e < E; ++e) {
-    const int64_t j = c * E + e - h;
-    if (j >= 0 && j < n) {
-      if (sizeof(T) == 2) {
-        w[e >> 1] |= ld_u16_issue(in_row + j) << ((e & 1) * 16);
-      } else {
-        w[e] = ld_u32_issue(in_row + j);
-      }
-    }
-  }
-  return make_uint4(w[0], w[1], w[2], w[3]);
-}
-
-__device__ __forceinline__ void complete_pending(PendingEdges &pe) {
-  if (!pe.active) return;
-  if (pe.head) st_shared_u4(pe.head_dst, pe.head_val);
-  if (pe.tail) st_shared_u4(pe.tail_dst, pe.tail_val);
-  if (pe.head) mbar_arrive(pe.head_bar);
-  if (pe.tail && (pe.tail_own_bar || !pe.head)) mbar_arrive(pe.tail_bar);
-  pe.active = false;
-}
+constexpr int kFetchBatch = 4;  // MEDIUM rows one work-counter step claims
 
 // Record `idx` of a bucket's list: the classify block b with
 // pref[b] <= idx < pref[b + 1] wrote it at entry b * rows_per_block +
@@ -893,10 +874,44 @@ __device__ __forceinline__ bool ragged_record_fits(const RowRec &r, int b, int64
   return r.n >= 1 && r.n <= glen && bucket_of(r.n, Elem<T>::kSize) == b;
 }
 
+// The edge elements of an item, one per lane: lanes [0, E) the head chunk
+// (window chunk 0), lanes [E, 2E) the tail chunk (the last one), each
+// element read only when it lies in the row (zero otherwise), written into
+// the stage later.  The chunks' pieces are complete when lane 0 arrives on
+// their barriers after the writes.
+struct EdgeLanes {
+  bool active;              // (uniform) an item's edges are still to be written
+  bool mine;                // this lane writes an element
+  bool head, tail, tail_own_bar;  // (uniform)
+  uint32_t dst;             // this lane's element in the stage
+  uint32_t val;             // its bits
+  uint32_t head_bar, tail_bar;    // (uniform)
+};
+
+template <typename T>
+__device__ __forceinline__ void edges_write(EdgeLanes &e, int lane) {
+  if (!e.active) return;
+  if (e.mine) {
+    if constexpr (sizeof(T) == 2) {
+      asm volatile("st.shared.u16 [%0], %1;" ::"r"(e.dst), "h"(static_cast<unsigned short>(e.val))
+                   : "memory");
+    } else {
+      asm volatile("st.shared.u32 [%0], %1;" ::"r"(e.dst), "r"(e.val) : "memory");
+    }
+  }
+  __syncwarp();
+  if (lane == 0) {
+    if (e.head) mbar_arrive(e.head_bar);
+    if (e.tail && (e.tail_own_bar || !e.head)) mbar_arrive(e.tail_bar);
+  }
+  e.active = false;
+}
+
 template <typename T, bool EXACT, bool CLUSTER, bool RAGGED>
 __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSmemLayout &L,
                                               unsigned char *smem, int cs, int rank, int64_t cid,
-                                              int64_t ncl) {
+                                              int64_t ncl, int lane) {
+  constexpr int E = Elem<T>::kPerChunk;
   constexpr int SZ = Elem<T>::kSize;
   const int S = p.stages;
   const int G = kConsumerWarps / p.group_warps;  // every group gets an end-of-work item
@@ -909,42 +924,61 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
   const int nb1 = p.blocks + 1;
   int64_t k_large = 0, k_dense = 0;
   bool medium_phase = false;
-  PendingEdges pend;
-  pend.active = false;
+  EdgeLanes edges;
+  edges.active = false;
   uint32_t fill_mask = 0, fill_parity = 0;
 
-  // The next item of this CTA: its record is fetched one step ahead, so the
-  // load (and the work-counter round trip) overlaps the wait for a free stage.
+  // the current batch of ragged records: lane k holds record k
+  RowRec mine;
+  mine.start = 0;
+  mine.n = 0;
+  int qn = 0, qi = 0, qkind = kItemEnd;
+  auto refill = [&]() {
+    qn = 0;
+    qi = 0;
+    if (!medium_phase) {
+      const int64_t nl = pref[2 * nb1 + p.blocks];
+      const int64_t li0 = cid + k_large * ncl;
+      if (li0 < nl) {
+        const int cnt = static_cast<int>(min(static_cast<int64_t>(32), (nl - li0 + ncl - 1) / ncl));
+        if (lane < cnt) mine = ragged_record(p, pref + 2 * nb1, p.rec_large, li0 + lane * ncl);
+        k_large += cnt;
+        qn = cnt;
+        qkind = kItemLarge;
+        return;
+      }
+      medium_phase = true;
+    }
+    const int64_t nm = pref[nb1 + p.blocks];
+    unsigned int m = 0;
+    if (lane == 0) m = atomicAdd(&p.counters[0], static_cast<unsigned int>(kFetchBatch));
+    const int64_t m0 = __shfl_sync(kFullMask, m, 0);
+    if (m0 >= nm) return;  // no rows left: the end of this CTA's work
+    const int cnt = static_cast<int>(min(static_cast<int64_t>(kFetchBatch), nm - m0));
+    if (lane < cnt) mine = ragged_record(p, pref + nb1, p.rec_medium, m0 + lane);
+    qn = cnt;
+    qkind = kItemMedium;
+  };
+  // The next item of this CTA (the same on every lane).
   auto fetch = [&](int &kind, int64_t &start, int64_t &n) {
     kind = kItemEnd;
     start = 0;
     n = 0;
     if (RAGGED) {
       for (;;) {
-        if (!medium_phase) {
-          const int64_t li = cid + k_large * ncl;
-          if (li < pref[2 * nb1 + p.blocks]) {
-            const RowRec r = ragged_record(p, pref + 2 * nb1, p.rec_large, li);
-            ++k_large;
-            if (!ragged_record_fits<T>(r, kLarge, p.glen)) {
-              atomicOr(p.status, kStatusBadOffsets);
-              continue;
-            }
-            kind = kItemLarge;
-            start = r.start;
-            n = r.n;
-            return;
-          }
-          medium_phase = true;
+        if (qi == qn) {
+          refill();
+          if (qn == 0) return;
         }
-        const unsigned int m = atomicAdd(&p.counters[0], 1u);
-        if (m >= static_cast<unsigned int>(pref[nb1 + p.blocks])) return;
-        const RowRec r = ragged_record(p, pref + nb1, p.rec_medium, m);
-        if (!ragged_record_fits<T>(r, kMedium, p.glen)) {
-          atomicOr(p.status, kStatusBadOffsets);
+        RowRec r;
+        r.start = __shfl_sync(kFullMask, mine.start, qi);
+        r.n = __shfl_sync(kFullMask, mine.n, qi);
+        ++qi;
+        if (!ragged_record_fits<T>(r, qkind == kItemLarge ? kLarge : kMedium, p.glen)) {
+          if (lane == 0) atomicOr(p.status, kStatusBadOffsets);
           continue;
         }
-        kind = kItemMedium;
+        kind = qkind;
         start = r.start;
         n = r.n;
         return;
@@ -967,23 +1001,28 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
     const int s = static_cast<int>(it % S);
     const int kind = next_kind;
     const int64_t start = next_start, n = next_n;
-    if (kind != kItemEnd) fetch(next_kind, next_start, next_n);
-    if (it >= S) {
-      if (!mbar_wait_bounded(sbase + L.bar_empty + 8u * s,
+    bool stop = false;
+    if (lane == 0) {
+      if (it >= S &&
+          !mbar_wait_bounded(sbase + L.bar_empty + 8u * s,
                              static_cast<uint32_t>(((it / S) - 1) & 1), p.timeout_ns)) {
         atomicOr(p.status, kStatusTimeout);
         flags[0] = 1;
-        break;
       }
-      fill_mask &= ~(1u << s);
+      stop = flags[0] != 0;
     }
-    if (flags[0]) break;
-    complete_pending(pend);
+    if (__shfl_sync(kFullMask, stop ? 1 : 0, 0)) break;
+    if (it >= S) fill_mask &= ~(1u << s);
+    // (dense, several stages) the previous item's edges, whose loads had the
+    // wait above to land
+    edges_write<T>(edges, lane);
 
-    meta[s].start = start;
-    meta[s].n = n;
-    meta[s].kind = kind;
-    mbar_arrive(sbase + L.bar_meta + 8u * s);
+    if (lane == 0) {
+      meta[s].start = start;
+      meta[s].n = n;
+      meta[s].kind = kind;
+      mbar_arrive(sbase + L.bar_meta + 8u * s);
+    }
     if (kind == kItemEnd) {
       if (++ends == G) break;
       continue;
@@ -1000,8 +1039,13 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
     const bool tail = c0 < c1 && g.cl < g.nc && c1 == g.nc && !(head && g.nc == 1);
     const int head_pc = 0;
     const int tail_pc = tail ? static_cast<int>((g.nc - 1 - c0) / (kPieceTiles * kTileChunks)) : -1;
-    bool any_copy = false;
-    for (int pc = 0; pc < L.pieces; ++pc) {
+    // generic writes of this lane into the stage (an earlier item's edges)
+    // are ordered before the bulk copies that overwrite it
+    fence_proxy_async_smem();
+    __syncwarp();
+    bool copied = false;
+    if (lane < L.pieces) {
+      const int pc = lane;
       const uint32_t bar = sbase + L.bar_piece + 8u * (s * L.pieces + pc);
       const int64_t q0 = c0 + static_cast<int64_t>(pc) * kPieceTiles * kTileChunks;
       const int64_t q1 = min(c1, q0 + kPieceTiles * kTileChunks);
@@ -1018,35 +1062,50 @@ __device__ __forceinline__ void tile_producer(const TileParams &p, const TileSme
         mbar_arrive(bar);
       }
       if (bytes) {
-        fence_proxy_async_smem();
         bulk_g2s(stage + static_cast<uint32_t>((b0 - c0) * kChunkBytes), win + b0 * kChunkBytes,
                  bytes, bar, pol);
-        any_copy = true;
+        copied = true;
       }
     }
-    if (any_copy) {
+    if (__any_sync(kFullMask, copied)) {
       fill_mask |= 1u << s;
       fill_parity = (fill_parity & ~(1u << s)) | (static_cast<uint32_t>((it / S) & 1) << s);
     }
     if (head || tail) {
-      PendingEdges pe;
-      pe.active = true;
-      pe.head = head;
-      pe.tail = tail;
-      pe.tail_own_bar = tail && !(head && tail_pc == head_pc);
-      pe.head_dst = stage;
-      pe.head_bar = sbase + L.bar_piece + 8u * (s * L.pieces + head_pc);
-      pe.tail_dst = stage + static_cast<uint32_t>((g.nc - 1 - c0) * kChunkBytes);
-      pe.tail_bar = sbase + L.bar_piece + 8u * (s * L.pieces + (tail ? tail_pc : 0));
-      pe.head_val = head ? issue_edge_chunk<T>(in_row, 0, g.h, g.n) : make_uint4(0, 0, 0, 0);
-      pe.tail_val = tail ? issue_edge_chunk<T>(in_row, g.nc - 1, g.h, g.n) : make_uint4(0, 0, 0, 0);
-      pend = pe;
-      if (S == 1) complete_pending(pend);
+      // lane l < E: element l of the head chunk; E <= l < 2E: element l - E
+      // of the tail chunk
+      edges.active = true;
+      edges.head = head;
+      edges.tail = tail;
+      edges.tail_own_bar = tail && !(head && tail_pc == head_pc);
+      edges.head_bar = sbase + L.bar_piece + 8u * (s * L.pieces + head_pc);
+      edges.tail_bar = sbase + L.bar_piece + 8u * (s * L.pieces + (tail ? tail_pc : 0));
+      const bool is_tail = lane >= E;
+      const int e = is_tail ? lane - E : lane;
+      const int64_t c = is_tail ? g.nc - 1 : 0;
+      edges.mine = lane < 2 * E && (is_tail ? tail : head);
+      edges.dst = stage + static_cast<uint32_t>((c - c0) * kChunkBytes) + static_cast<uint32_t>(e * SZ);
+      edges.val = 0u;
+      if (edges.mine) {
+        const int64_t j = c * E + e - g.h;
+        if (j >= 0 && j < g.n) {
+          if constexpr (SZ == 2) {
+            edges.val = *reinterpret_cast<const volatile unsigned short *>(in_row + j);
+          } else {
+            edges.val = *reinterpret_cast<const volatile uint32_t *>(in_row + j);
+          }
+        }
+      }
     }
+    // the next item while this one's edge loads are in flight; then its
+    // edges (ragged, whose lookups take the round trips, or one stage), or
+    // (dense) after the next stage's wait
+    fetch(next_kind, next_start, next_n);
+    if (RAGGED || S == 1) edges_write<T>(edges, lane);
   }
-  complete_pending(pend);
+  edges_write<T>(edges, lane);
   // a producer that gave up must not leave copies in flight into its stages
-  if (flags[0]) {
+  if (lane == 0 && flags[0]) {
     for (int s = 0; s < S; ++s)
       if (fill_mask >> s & 1u)
         for (int pc = 0; pc < L.pieces; ++pc)
@@ -1118,7 +1177,7 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
   if (CLUSTER) cluster_sync();  // every peer's barriers exist before any remote arrive
 
   if (warp == kConsumerWarps) {
-    if (lane == 0) tile_producer<T, EXACT, CLUSTER, RAGGED>(p, L, smem, cs, rank, cid, ncl);
+    tile_producer<T, EXACT, CLUSTER, RAGGED>(p, L, smem, cs, rank, cid, ncl, lane);
     return;
   }
 
