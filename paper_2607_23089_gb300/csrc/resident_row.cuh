@@ -300,8 +300,21 @@ __global__ void __launch_bounds__(NW * 32, MINB) resident_full_kernel(const Tile
 
     // ---- combine ----
     float s0, s1;
+    // portions of whole 64-tile blocks: each CTA forms its own blocks'
+    // partials (combine_blocks' level 1) and publishes those in place of its
+    // blocks' first tile partials
+    constexpr bool kOwnBlocks = kPortionTiles % kShortCombineTiles == 0;
     if (CLUSTER) {
       const uint32_t ready = bar_ready + 8u * b;
+      if (kOwnBlocks && K > kShortCombineTiles) {
+        for (int lb = w; lb * kShortCombineTiles < kPortionTiles; lb += NW) {
+          const float4 r = block_partial<OP>(part[kShortCombineTiles * lb + lane],
+                                             part[kShortCombineTiles * lb + lane + 32], true, true);
+          __syncwarp();
+          if (lane == 0) part[kShortCombineTiles * lb] = r;
+        }
+        named_sync(kResBar, kThreads);
+      }
       if (tid < cs) mbar_arrive_remote(ready, static_cast<uint32_t>(tid));
       const bool ok = mbar_wait_cluster_bounded(ready, uses_b & 1, p.timeout_ns);
       if (named_sync_or(kResBar, kThreads, !ok)) {
@@ -317,7 +330,18 @@ __global__ void __launch_bounds__(NW * 32, MINB) resident_full_kernel(const Tile
         return ld_dsmem_f4(map_to_rank(mine + static_cast<uint32_t>((t - rk * kPortionTiles) * 16),
                                        static_cast<uint32_t>(rk)));
       };
-      if (K <= kShortCombineTiles) {
+      if (kOwnBlocks && K > kShortCombineTiles) {
+        constexpr int bpc = kPortionTiles / kShortCombineTiles;
+        auto peer_block = [&](int t) {
+          const int rk = t / bpc;
+          return ld_dsmem_f4(map_to_rank(
+              mine + static_cast<uint32_t>((t - rk * bpc) * kShortCombineTiles * 16),
+              static_cast<uint32_t>(rk)));
+        };
+        combine_short<OP>(peer_block, K / kShortCombineTiles, inv_n, p.eps, lane, s0, s1);
+        __syncwarp();
+        if (lane < cs) mbar_arrive_remote(bar_released + 8u * b, static_cast<uint32_t>(lane));
+      } else if (K <= kShortCombineTiles) {
         for (int t = tid; t < K; t += static_cast<int>(kThreads)) gather[t] = peer(t);
         named_sync(kResBar, kThreads);
         __syncwarp();

@@ -1243,6 +1243,24 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
     const float inv_n = __frcp_rn(static_cast<float>(g.n));
     if (split) {
       const uint32_t ready = bar_ready + 8u * b;
+      const int tpc = (g.K + cs - 1) / cs;
+      // portions of whole 64-tile blocks: each CTA forms its own blocks'
+      // partials (the same arithmetic as combine_blocks' level 1) and
+      // publishes those, in place of its blocks' first tile partials
+      const bool own_blocks = g.K > kShortCombineTiles && tpc % kShortCombineTiles == 0;
+      if (own_blocks) {
+        const int ntl = g.t1 - g.t0;
+        for (int lb = wig; lb * kShortCombineTiles < ntl; lb += W) {
+          const int kb = min(kShortCombineTiles, ntl - kShortCombineTiles * lb);
+          const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+          const float4 q0 = lane < kb ? part[kShortCombineTiles * lb + lane] : z;
+          const float4 q1 = lane + 32 < kb ? part[kShortCombineTiles * lb + lane + 32] : z;
+          const float4 r = block_partial<OP>(q0, q1, lane < kb, lane + 32 < kb);
+          __syncwarp();
+          if (lane == 0) part[kShortCombineTiles * lb] = r;
+        }
+        named_sync(gbar, gthreads);
+      }
       // thread r signals rank r; the named barrier above already ordered
       // every warp's partial writes before these releases
       if (gtid < cs) mbar_arrive_remote(ready, static_cast<uint32_t>(gtid));
@@ -1255,14 +1273,26 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
         break;
       }
       // partial t lives in rank t / tpc at the same offset of its part_c
-      const int tpc = (g.K + cs - 1) / cs;
       const uint32_t mine = smem_addr(part);
       auto peer = [&](int t) {
         const int r = t / tpc;
         return ld_dsmem_f4(map_to_rank(mine + static_cast<uint32_t>((t - r * tpc) * 16),
                                        static_cast<uint32_t>(r)));
       };
-      if (g.K <= kShortCombineTiles) {
+      if (own_blocks) {
+        // block partial t: rank t / (tpc / 64), first slot of its block there
+        const int bpc = tpc / kShortCombineTiles;
+        const int nb = (g.K + kShortCombineTiles - 1) / kShortCombineTiles;
+        auto peer_block = [&](int t) {
+          const int r = t / bpc;
+          return ld_dsmem_f4(map_to_rank(
+              mine + static_cast<uint32_t>((t - r * bpc) * kShortCombineTiles * 16),
+              static_cast<uint32_t>(r)));
+        };
+        combine_short<OP>(peer_block, nb, inv_n, p.eps, lane, s0, s1);
+        __syncwarp();
+        if (lane < cs) mbar_arrive_remote(bar_released + 8u * b, static_cast<uint32_t>(lane));
+      } else if (g.K <= kShortCombineTiles) {
         // every warp combines all K partials: copy them here once, then
         // combine from local shared memory
         for (int t = gtid; t < g.K; t += static_cast<int>(gthreads)) gather[t] = peer(t);
