@@ -138,13 +138,20 @@ class ClockSampler:
 # GPU timing helpers
 # ---------------------------------------------------------------------------
 class L2Flusher:
+    """Evicts the timed call's data from L2 before each timed call: writes a
+    buffer twice the size of L2, then reads another one as large, so that
+    the lines the write left dirty are written back before the timed region
+    instead of during it."""
+
     def __init__(self, torch, device):
         l2 = torch.cuda.get_device_properties(device).L2_cache_size
-        self.buf = torch.empty(max(2 * l2, 256 << 20) // 4, dtype=torch.int32,
-                               device=device)
+        n = max(2 * l2, 256 << 20) // 4
+        self.buf = torch.empty(n, dtype=torch.int32, device=device)
+        self.rd = torch.ones(n, dtype=torch.int32, device=device)
 
     def __call__(self):
         self.buf.fill_(1)
+        self.rd.sum()
 
 
 def time_calls(torch, fn, steps, warmup, flush=None):
@@ -233,7 +240,8 @@ def per_config(torch, rw, wl, device, peak, steps):
             "pct_of_8TBs": round(100 * gbs / NOMINAL_HBM_GBS, 1),
             "pct_of_measured": round(100 * gbs / peak, 1),
             "rows_per_s": round(case.rows / (med * 1e-3), 1),
-            "l2": "flushed" if use_flush else "inputs larger than L2",
+            "l2": ("flushed (2x L2 written, then 2x L2 read)" if use_flush
+                   else "inputs larger than L2"),
         })
         del x, y, g, b
     return out
