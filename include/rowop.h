@@ -424,6 +424,11 @@ ROWOP_API int rowop_get_config(rowop_config_t *cfg);
 /* Human-readable name of a status code (static storage, never NULL). */
 ROWOP_API const char *rowop_status_string(int status);
 
+/* The CUDA runtime's description of the last CUDA error that made a call of
+ * this thread return ROWOP_ERR_CUDA ("no error" if none has; static storage,
+ * never NULL).  Pure host function. */
+ROWOP_API const char *rowop_last_cuda_error(void);
+
 /* Synchronises `stream` (the host waits until all work queued on it has
  * finished), then reads and clears the device status word of the current
  * device: returns ROWOP_OK, ROWOP_ERR_TIMEOUT if any bounded device wait ran

@@ -5,7 +5,7 @@
 #pragma once
 
 #include "launch_util.cuh"
-#include "resident_row.cuh"
+#include "stream_row.cuh"
 #include "small_row.cuh"
 #include "tile_row.cuh"
 
@@ -209,6 +209,73 @@ cudaError_t launch_res_full_k(TileParams p, int cs, const DenseCall &c, const De
 // cluster of cs CTAs of R tiles a warp (the largest R that splits the row
 // into 2..16 equal portions) when it is LARGE.  Returns false when the call
 // does not qualify (the caller takes another design).
+// LARGE dense rows whose cluster portions are whole 64-tile blocks: the
+// streamed split (stream_row.cuh).  Portions of at most 256 tiles (the
+// smallest such cluster), a ring of 8 pieces (ROWOP_STAGES: another depth);
+// returns false, launching nothing, for any other shape.
+template <int OP, typename T>
+bool try_stream(const DenseCall &c, const DeviceInfo &d, const Knobs &kn, cudaError_t *err) {
+  constexpr int SZ = sizeof(T);
+  constexpr int E = 16 / SZ;
+  constexpr bool kAffine = (OP == kLayerNorm || OP == kRmsNorm);
+  if (kn.stream == 0 || c.rows <= 0) return false;
+  if (!aligned16(c.in) || !aligned16(c.out) || (c.ld * SZ) % 16 != 0) return false;
+  if (c.cols % (kTileChunks * E) != 0) return false;
+  const int64_t K = c.cols / (kTileChunks * E);
+  int cs = 2;
+  if (kn.cluster > 1) {
+    cs = kn.cluster;
+  } else {
+    while (cs < kMaxCluster && K / cs > 256) cs <<= 1;
+  }
+  if (K % (static_cast<int64_t>(cs) * kShortCombineTiles) != 0) return false;
+  const int PT = static_cast<int>(K / cs);
+  const int NP = kn.stages > 0 ? std::min(kn.stages, 16) : 8;
+  const StreamSmem L(NP, PT);
+  if (L.total > static_cast<uint32_t>(d.max_smem_optin)) return false;
+  auto kern = stream_row_kernel<OP, T>;
+  const void *kp = reinterpret_cast<const void *>(kern);
+  cudaError_t e = prepare_kernel(kp, d, true);
+  if (e != cudaSuccess) {
+    *err = e;
+    return true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cs;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cfg.blockDim = dim3(kStreamThreads, 1, 1);
+  cfg.dynamicSmemBytes = L.total;
+  cfg.stream = c.stream;
+  cfg.gridDim = dim3(cs * std::max(1, d.sm_count / cs), 1, 1);
+  int ncl = cached_occupancy(kp, kStreamThreads, L.total, cs, &cfg);
+  if (kn.ctas_per_sm > 0) ncl = std::min(ncl, kn.ctas_per_sm * d.sm_count / cs);
+  ncl = std::max(1, ncl);
+  cfg.gridDim = dim3(static_cast<unsigned>(cs * std::min<int64_t>(c.rows, ncl)), 1, 1);
+  StreamParams sp = {};
+  sp.in = c.in;
+  sp.out = c.out;
+  sp.gamma = c.gamma;
+  sp.beta = c.beta;
+  sp.rows = c.rows;
+  sp.cols = c.cols;
+  sp.ld = c.ld;
+  sp.eps = c.eps;
+  sp.pieces = NP;
+  sp.portion = PT;
+  sp.gvec = kAffine && c.gamma && aligned16(c.gamma) &&
+            (OP == kRmsNorm || (c.beta && aligned16(c.beta)));
+  sp.timeout_ns = kWaitLimitNs;
+  sp.status = d.status;
+  e = cudaLaunchKernelEx(&cfg, kern, sp);
+  *err = e != cudaSuccess ? e : cudaGetLastError();
+  return true;
+}
+
 template <int OP, typename T>
 bool try_res_full(const TileParams &p, const DenseCall &c, const DeviceInfo &d, int bucket,
                   const Knobs &kn, cudaError_t *err) {
@@ -312,6 +379,13 @@ cudaError_t launch_dense_impl(const DenseCall &c, const DeviceInfo &d) {
   if (bucket == kMedium && K > kMaxPortionTiles) bucket = kLarge;
 
   if (bucket == kSmall) return launch_small<OP, T, RESID>(c, d, exact, out_vec, gvec);
+  // LARGE rows of whole 64-tile blocks per cluster CTA: the streamed split
+  // (not the online softmax statistics, another arithmetic)
+  if (!RESID && out_vec && bucket == kLarge &&
+      !((OP == kSoftmax || OP == kLogSoftmax) && kn.softmax_online)) {
+    cudaError_t err = cudaSuccess;
+    if (try_stream<OP, T>(c, d, kn, &err)) return err;
+  }
 
   TileParams p = {};
   p.in = c.in;

@@ -78,6 +78,7 @@ Knobs read_knobs() {
   k.resident = env_int("ROWOP_RESIDENT", 1);
   k.res_gc = env_int("ROWOP_RESIDENT_GC", 1);
   k.bwd_tile = env_int("ROWOP_BWD_TILE", 1);
+  k.stream = env_int("ROWOP_STREAM", 0);
   return k;
 }
 
@@ -172,8 +173,12 @@ static bool elem_aligned(const void *p, int esize) {
 
 static bool eps_ok(float eps) { return std::isfinite(eps) && eps >= 0.f; }
 
+// the last CUDA error that a call of this thread turned into ROWOP_ERR_CUDA
+static thread_local cudaError_t t_last_cuda_error = cudaSuccess;
+
 static int from_cuda(cudaError_t e) {
   if (e == cudaSuccess) return ROWOP_OK;
+  t_last_cuda_error = e;
   cudaGetLastError();
   return ROWOP_ERR_CUDA;
 }
@@ -693,6 +698,8 @@ int64_t rowop_max_row_len(rowop_dtype_t dtype) {
   const int es = esize_of(dtype);
   return es == 0 ? 0 : max_row_len_elems(es);
 }
+
+const char *rowop_last_cuda_error(void) { return cudaGetErrorString(t_last_cuda_error); }
 
 const char *rowop_status_string(int status) {
   switch (status) {

@@ -91,6 +91,7 @@ SIGNATURES = {
     "rowop_max_row_len": ([_I], _I64),
     "rowop_get_config": ([ctypes.POINTER(RowopConfig)], _I),
     "rowop_status_string": ([_I], ctypes.c_char_p),
+    "rowop_last_cuda_error": ([], ctypes.c_char_p),
     "rowop_check_status": ([_P], _I),
     "rowop_debug_wait_timeout": ([_I64, _P], _I),
 }
@@ -185,6 +186,8 @@ def _check_cuda(*ts):
 
 def _ok(st, what):
     if st != 0:
+        if st == ROWOP_ERR_CUDA:
+            what = f"{what} ({_lib.rowop_last_cuda_error().decode()})"
         raise RowopError(st, what)
 
 

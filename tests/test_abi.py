@@ -31,7 +31,8 @@ def test_header_declares_the_abi():
     for n in ("rowop_softmax", "rowop_logsoftmax", "rowop_layernorm", "rowop_rmsnorm",
               "rowop_softmax_ragged", "rowop_logsoftmax_ragged", "rowop_layernorm_ragged",
               "rowop_rmsnorm_ragged", "rowop_ragged_workspace_size",
-              "rowop_select_bucket", "rowop_status_string", "rowop_check_status"):
+              "rowop_select_bucket", "rowop_status_string", "rowop_check_status",
+              "rowop_last_cuda_error"):
         assert n in names
 
 

@@ -108,3 +108,50 @@ def test_whole_tile_stage_counts(rw, stages):
         a = _run(rw, op, torch.bfloat16, 301, 4096, 1, stages=stages, check=True)
         b = _run(rw, op, torch.bfloat16, 301, 4096, 0)
         assert torch.equal(_bits(a), _bits(b))
+
+
+# LARGE rows whose cluster portions are whole 64-tile blocks: (cols per dtype
+# size, rows) -- the streamed split against the staged split
+STREAM_LARGE = {4: ((32768, 5), (262144, 3)), 2: ((65536, 5), (131072, 3))}
+
+
+def _run_knobs(rw, op, dtype, rows, cols, knobs, check=False):
+    names = ("ROWOP_STREAM", "ROWOP_CLUSTER", "ROWOP_STAGES", "ROWOP_CTAS_PER_SM", "ROWOP_RESIDENT")
+    old = {k: os.environ.get(k) for k in names}
+    try:
+        for k in names:
+            os.environ.pop(k, None)
+        os.environ.update({k: str(v) for k, v in knobs.items()})
+        return run_case(rw, op, dtype, rows, cols, seed=cols + rows, check=check).clone()
+    finally:
+        for k, v in old.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+
+
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
+@pytest.mark.parametrize("op", ALL_OPS)
+def test_streamed_split_equals_staged(rw, op, dtype):
+    """The streamed split (each portion read twice through a ring of pieces)
+    forms the same tile partials, block partials and combine as the staged
+    split, so the two agree bit for bit; checked against the oracle too."""
+    for cols, rows in STREAM_LARGE[ESIZE[dtype]]:
+        a = _run_knobs(rw, op, dtype, rows, cols, {"ROWOP_STREAM": 1}, check=True)
+        b = _run_knobs(rw, op, dtype, rows, cols, {"ROWOP_STREAM": 0, "ROWOP_RESIDENT": 0})
+        assert torch.equal(_bits(a), _bits(b)), cols
+
+
+@pytest.mark.parametrize("knobs", [{"ROWOP_CLUSTER": 2}, {"ROWOP_CLUSTER": 8},
+                                   {"ROWOP_CLUSTER": 16}, {"ROWOP_STAGES": 2},
+                                   {"ROWOP_STAGES": 3}, {"ROWOP_CTAS_PER_SM": 1}],
+                         ids=["cs2", "cs8", "cs16", "ring2", "ring3", "one_cta_sm"])
+def test_streamed_split_shapes(rw, knobs):
+    """Cluster sizes, ring depths (one that does not divide the pieces of a
+    pass) and many rows per cluster (one CTA an SM): the same bits."""
+    cols, rows = 262144, 40
+    for op in ("logsoftmax", "layernorm"):
+        a = _run_knobs(rw, op, torch.float32, rows, cols, dict(knobs, ROWOP_STREAM=1))
+        b = _run_knobs(rw, op, torch.float32, rows, cols, {"ROWOP_STREAM": 0, "ROWOP_RESIDENT": 0})
+        assert torch.equal(_bits(a), _bits(b)), knobs
