@@ -178,9 +178,10 @@ inline int64_t max_row_len_elems(int esize) {
 //   ROWOP_RESIDENT_GC   0 -> the register-resident design reads gamma/beta
 //                       per row instead of keeping them in registers (fewer
 //                       registers, more CTAs an SM; the same bits)
-//   ROWOP_STREAM        1 -> LARGE dense rows whose cluster portions are whole
-//                       64-tile blocks are streamed twice through a ring
-//                       instead of held in shared memory (the same bits)
+//   ROWOP_STREAM        0 -> LARGE dense rows whose cluster portions are whole
+//                       64-tile blocks are held in shared memory (the staged
+//                       split) instead of streamed twice through a ring
+//                       (the same bits)
 //   ROWOP_BWD_TILE      0 -> dense norm backward rows of whole tiles use the
 //                       team design instead of the whole-tile one (another
 //                       summation order)
@@ -195,7 +196,7 @@ struct Knobs {
   int resident = 1;
   int res_gc = 1;
   int bwd_tile = 1;
-  int stream = 0;
+  int stream = 1;
 };
 Knobs read_knobs();
 

@@ -210,9 +210,12 @@ cudaError_t launch_res_full_k(TileParams p, int cs, const DenseCall &c, const De
 // into 2..16 equal portions) when it is LARGE.  Returns false when the call
 // does not qualify (the caller takes another design).
 // LARGE dense rows whose cluster portions are whole 64-tile blocks: the
-// streamed split (stream_row.cuh).  Portions of at most 256 tiles (the
-// smallest such cluster), a ring of 8 pieces (ROWOP_STAGES: another depth);
-// returns false, launching nothing, for any other shape.
+// streamed split (stream_row.cuh).  Portions of at most 128 tiles (the
+// smallest such cluster) and a ring of 4 pieces, so three CTAs share an SM
+// (measured on 256 x 262144 fp32 log-softmax: clusters of 8 with 4 pieces
+// 106 us; 3 / 6 pieces 108 / 114 us; clusters of 4 / 16 118 / 132 us);
+// ROWOP_CLUSTER and ROWOP_STAGES override.  Returns false, launching
+// nothing, for any other shape.
 template <int OP, typename T>
 bool try_stream(const DenseCall &c, const DeviceInfo &d, const Knobs &kn, cudaError_t *err) {
   constexpr int SZ = sizeof(T);
@@ -226,11 +229,11 @@ bool try_stream(const DenseCall &c, const DeviceInfo &d, const Knobs &kn, cudaEr
   if (kn.cluster > 1) {
     cs = kn.cluster;
   } else {
-    while (cs < kMaxCluster && K / cs > 256) cs <<= 1;
+    while (cs < kMaxCluster && K / cs > 128) cs <<= 1;
   }
   if (K % (static_cast<int64_t>(cs) * kShortCombineTiles) != 0) return false;
   const int PT = static_cast<int>(K / cs);
-  const int NP = kn.stages > 0 ? std::min(kn.stages, 16) : 8;
+  const int NP = kn.stages > 0 ? std::min(kn.stages, 16) : 4;
   const StreamSmem L(NP, PT);
   if (L.total > static_cast<uint32_t>(d.max_smem_optin)) return false;
   auto kern = stream_row_kernel<OP, T>;

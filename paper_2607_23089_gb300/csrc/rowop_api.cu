@@ -78,7 +78,7 @@ Knobs read_knobs() {
   k.resident = env_int("ROWOP_RESIDENT", 1);
   k.res_gc = env_int("ROWOP_RESIDENT_GC", 1);
   k.bwd_tile = env_int("ROWOP_BWD_TILE", 1);
-  k.stream = env_int("ROWOP_STREAM", 0);
+  k.stream = env_int("ROWOP_STREAM", 1);
   return k;
 }
 

@@ -8,9 +8,8 @@ they can take:
   * the whole-tile kernel (the default for dense MEDIUM rows that are a
     whole number of tiles): one CTA per row of 8, 16 or 32 tiles, and, with
     ROWOP_RESIDENT=2, cluster splits of LARGE rows into equal portions;
-  * the general resident kernel serves ragged rows; test_gpu_ragged.py holds
-    it to the staged design (ROWOP_RESIDENT=0, and the knobs that select the
-    staged design) bit for bit.
+  * the streamed split of LARGE rows (each cluster portion read twice
+    through a ring of pieces, the default for whole-block portions).
 Parity of every design against the oracle is checked here as well.
 """
 import os
@@ -23,7 +22,7 @@ from tests.test_gpu_dense import run_case
 
 pytestmark = pytest.mark.gpu
 
-KNOBS = ("ROWOP_RESIDENT", "ROWOP_FORCE_BUCKET", "ROWOP_CLUSTER", "ROWOP_STAGES")
+KNOBS = ("ROWOP_RESIDENT", "ROWOP_FORCE_BUCKET", "ROWOP_CLUSTER", "ROWOP_STAGES", "ROWOP_STREAM")
 
 
 @pytest.fixture(scope="module")
@@ -40,6 +39,7 @@ def _run(rw, op, dtype, rows, cols, resident, ld=None, x_off=0, bucket=None, clu
     old = {k: os.environ.get(k) for k in KNOBS}
     try:
         os.environ["ROWOP_RESIDENT"] = str(int(resident))
+        os.environ["ROWOP_STREAM"] = "0"  # the streamed split has its own tests below
         for k, v in (("ROWOP_FORCE_BUCKET", bucket), ("ROWOP_CLUSTER", cluster),
                      ("ROWOP_STAGES", stages)):
             if v is not None:
