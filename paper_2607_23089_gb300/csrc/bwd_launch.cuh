@@ -59,9 +59,20 @@ cudaError_t launch_bwd_finalize(const BwdSegments &sg, int64_t cols, int nacc, v
   if (cols <= 0) return cudaSuccess;
   // a block per 32 columns, so many SMs share the reads, and 32 warps per
   // block over the partials, so each warp's chain of loads is short
-  const dim3 grid(static_cast<unsigned>(ceil_div(cols, 32)), static_cast<unsigned>(nacc), 1);
-  bwd_param_finalize_kernel<T><<<grid, kFinThreads, 0, stream>>>(
-      sg, cols, nacc, static_cast<T *>(dgamma), static_cast<T *>(dbeta));
+  // a programmatic dependent launch: the finalize's launch overlaps the
+  // tail of the kernel before it, whose results it waits for on the device
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cfg.gridDim = dim3(static_cast<unsigned>(ceil_div(cols, 32)), static_cast<unsigned>(nacc), 1);
+  cfg.blockDim = dim3(kFinThreads, 1, 1);
+  cfg.stream = stream;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, bwd_param_finalize_kernel<T>, sg, cols, nacc,
+                                     static_cast<T *>(dgamma), static_cast<T *>(dbeta));
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -620,6 +620,10 @@ __global__ void __launch_bounds__(kFinThreads) bwd_param_finalize_kernel(const B
                                                                          int64_t cols, int nacc,
                                                                          T *dgamma, T *dbeta) {
   __shared__ float sums[kFinWarps][32];
+  // launched as a programmatic dependent of the kernel that wrote the
+  // partials: its blocks may start while that kernel drains, and wait here
+  // until it has finished and its writes are visible (a no-op otherwise)
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const int a = blockIdx.y;

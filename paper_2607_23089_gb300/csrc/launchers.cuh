@@ -106,17 +106,18 @@ cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int
   if (e != cudaSuccess) return e;
 
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   cfg.blockDim = dim3(kTileThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   int grid;
+  cfg.attrs = attr;
+  cfg.numAttrs = 0;
   if (CLUSTER) {
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = cs;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
     cfg.numAttrs = 1;
     cfg.gridDim = dim3(cs * std::max(1, d.sm_count / cs), 1, 1);
     int ncl = cached_occupancy(kp, kTileThreads, smem, cs, &cfg);
@@ -130,6 +131,14 @@ cudaError_t launch_tile_k(TileParams p, int cs, int stages, int stage_tiles, int
         1, std::min<int64_t>(items, static_cast<int64_t>(bps) * d.sm_count)));
   }
   cfg.gridDim = dim3(grid, 1, 1);
+  if (RAGGED) {
+    // a programmatic dependent of the classify launch before it: the fused
+    // kernel's launch and set-up overlap the classify tail, and its threads
+    // wait on the device for the classify results
+    attr[cfg.numAttrs].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[cfg.numAttrs].val.programmaticStreamSerializationAllowed = 1;
+    ++cfg.numAttrs;
+  }
   e = cudaLaunchKernelEx(&cfg, kern, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();

@@ -1155,6 +1155,10 @@ __global__ void __launch_bounds__(kTileThreads, 3) tile_row_kernel(const TilePar
     flags[0] = 0;
     fence_mbar_init();
   }
+  // (ragged) launched as a programmatic dependent of the classify kernel:
+  // the barriers above were set up meanwhile; the plan is read below, once
+  // that kernel has finished and its writes are visible (a no-op otherwise)
+  if constexpr (RAGGED) asm volatile("griddepcontrol.wait;" ::: "memory");
   if (RAGGED && warp < 3) {
     // warp k: exclusive scan of bucket k's row counts over the classify blocks
     int *pref = reinterpret_cast<int *>(smem + L.pref) + warp * (p.blocks + 1);
