@@ -62,4 +62,58 @@ inline size_t bwd_ragged_layout(int64_t rows, int64_t max_len, int esize, int na
   return off;
 }
 
+// The striped ragged norm backward (bwd_stripe.cuh): column stripes of
+// each kernel, in elements of esize bytes.  A stripe is one 16-byte window
+// chunk narrower than the chunk slots of the kernel's CTA, so the stripe of
+// a row that starts mid-chunk still fits.
+constexpr int kStatThreads = 256;  // threads of a stats CTA
+constexpr int kStatChunks = 2;     // window chunks a stats lane holds per row
+constexpr int kStatRows = 64;      // rows of a stats CTA
+constexpr int kDxThreads = 256;    // threads of a dx CTA (one chunk a lane per row)
+constexpr int kDxBatch = 256;      // rows a dx CTA sorts at a time
+constexpr int kDxMaxGroups = 128;  // dgamma / dbeta partial rows at most
+constexpr int kDxMinGroupRows = 32;
+// max_len from which the ragged norm backward takes the striped design by
+// default (ROWOP_BWD_STRIPE=1; 2 takes it for every max_len, 0 never)
+constexpr int64_t kStripeMinCols = 2048;
+
+inline int64_t stripe_stat_width(int esize) {
+  return static_cast<int64_t>(16 / esize) * (kStatThreads * kStatChunks - 1);
+}
+inline int64_t stripe_dx_width(int esize) {
+  return static_cast<int64_t>(16 / esize) * (kDxThreads - 1);
+}
+
+// Workspace of the striped design, all 256-byte aligned: each row's first
+// element (LayerNorm's shift), the per-stripe row sums [rows][ns1] float4,
+// and the dgamma / dbeta partial rows [ng2][nacc][max_len] float32.
+struct StripeLayout {
+  int64_t ns1, ng1, ns2, ng2, g2;  // stripes and row groups of the two kernels
+  size_t shift, psum, part, total;
+};
+
+inline StripeLayout stripe_layout(int64_t rows, int64_t max_len, int esize, int nacc) {
+  StripeLayout L = {};
+  const auto up = [](size_t v) { return (v + 255) & ~static_cast<size_t>(255); };
+  L.ns1 = max_len > 0 ? (max_len + stripe_stat_width(esize) - 1) / stripe_stat_width(esize) : 0;
+  L.ns2 = max_len > 0 ? (max_len + stripe_dx_width(esize) - 1) / stripe_dx_width(esize) : 0;
+  L.ng1 = (rows + kStatRows - 1) / kStatRows;
+  L.ng2 = std::max<int64_t>(
+      1, std::min<int64_t>((rows + kDxMinGroupRows - 1) / kDxMinGroupRows, kDxMaxGroups));
+  L.g2 = (rows + L.ng2 - 1) / L.ng2;
+  const size_t r = static_cast<size_t>(std::max<int64_t>(rows, 0));
+  L.shift = 0;
+  L.psum = up(r * sizeof(float));
+  L.part = L.psum + up(r * static_cast<size_t>(L.ns1) * 16u);
+  L.total = L.part + up(static_cast<size_t>(L.ng2) * static_cast<size_t>(nacc) *
+                        static_cast<size_t>(max_len) * sizeof(float));
+  return L;
+}
+
+// Workspace bytes of a ragged norm backward call: enough for either design.
+inline size_t bwd_ragged_norm_ws(int64_t rows, int64_t max_len, int esize, int nacc, int sm) {
+  return std::max(bwd_ragged_layout(rows, max_len, esize, nacc, sm, nullptr),
+                  stripe_layout(rows, max_len, esize, nacc).total);
+}
+
 }  // namespace rowop

@@ -5,6 +5,7 @@
 
 #include "bwd_call.h"
 #include "bwd_row.cuh"
+#include "bwd_stripe.cuh"
 #include "bwd_tile.cuh"
 #include "launch_util.cuh"
 
@@ -287,6 +288,62 @@ cudaError_t launch_bwd_t(const BwdCall &c, const DeviceInfo &d) {
   return launch_bwd_k<OP, T, CPT, false, false>(p, s, c, d);
 }
 
+// Ragged norm rows by column stripes (bwd_stripe.cuh): x, dy and dx
+// congruent modulo 16 bytes and, unless forced (mode 2), max_len of at
+// least kStripeMinCols.  Returns false, launching nothing, otherwise.
+template <int OP, typename T>
+bool try_bwd_stripe(const BwdRaggedCall &c, const DeviceInfo &d, int mode, cudaError_t *err) {
+  constexpr int SZ = sizeof(T);
+  if (mode == 0 || c.rows <= 0 || c.max_len <= 0) return false;
+  if (mode != 2 && c.max_len < kStripeMinCols) return false;
+  if (!congruent16(c.a, c.dy) || !congruent16(c.a, c.dx)) return false;
+  const int nacc = OP == kLayerNorm ? 2 : 1;
+  const bool want_params = c.dgamma || c.dbeta;
+  const StripeLayout L = stripe_layout(c.rows, c.max_len, SZ, nacc);
+  unsigned char *ws = static_cast<unsigned char *>(c.ws);
+  StripeParams p = {};
+  p.x = c.a;
+  p.dy = c.dy;
+  p.dx = c.dx;
+  p.gamma = c.gamma;
+  p.offsets = c.offsets;
+  p.rows = c.rows;
+  p.max_len = c.max_len;
+  p.eps = c.eps;
+  p.hb = static_cast<int>((reinterpret_cast<uintptr_t>(c.a) & 15u) / SZ);
+  p.shift = reinterpret_cast<float *>(ws + L.shift);
+  p.psum = reinterpret_cast<float4 *>(ws + L.psum);
+  p.part = want_params ? reinterpret_cast<float *>(ws + L.part) : nullptr;
+  p.ns1 = L.ns1;
+  p.ng1 = L.ng1;
+  p.ng2 = L.ng2;
+  p.g2 = L.g2;
+  p.status = d.status;
+  bwd_stripe_stats_kernel<OP, T>
+      <<<static_cast<unsigned>(L.ns1 * L.ng1), kStatThreads, 0, c.stream>>>(p);
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) {
+    // a programmatic dependent launch: the dx kernel's CTAs sort their rows
+    // while the stats kernel drains, and wait for it on the device
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cfg.gridDim = dim3(static_cast<unsigned>(L.ns2 * L.ng2), 1, 1);
+    cfg.blockDim = dim3(kDxThreads, 1, 1);
+    cfg.stream = c.stream;
+    e = cudaLaunchKernelEx(&cfg, bwd_stripe_dx_kernel<OP, T>, p);
+    if (e == cudaSuccess) e = cudaGetLastError();
+  }
+  if (e == cudaSuccess && want_params)
+    e = launch_bwd_finalize<T>(one_segment(p.part, L.ng2, c.max_len), c.max_len, nacc,
+                               c.dgamma, c.dbeta, c.stream);
+  *err = e;
+  return true;
+}
+
 // Ragged backward: the forward's classify pass sorts the rows into three
 // buckets by byte length; each bucket that max_len allows gets one launch of
 // the team kernel, shaped for the bucket's longest row, which walks that
@@ -310,6 +367,10 @@ cudaError_t launch_bwd_ragged_t(const BwdRaggedCall &c, const DeviceInfo &d) {
                 "the longest ragged norm row one team can hold");
   const int nacc = OP == kLayerNorm ? 2 : 1;
   const bool want_params = kNorm && (c.dgamma || c.dbeta);
+  if constexpr (kNorm) {
+    cudaError_t err = cudaSuccess;
+    if (try_bwd_stripe<OP, T>(c, d, read_knobs().bwd_stripe, &err)) return err;
+  }
   unsigned char *ws = static_cast<unsigned char *>(c.ws);
   size_t seg_off[3] = {0, 0, 0};
   if (kNorm) (void)bwd_ragged_layout(c.rows, c.max_len, SZ, nacc, d.sm_count, seg_off);

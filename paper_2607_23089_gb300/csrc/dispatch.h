@@ -185,6 +185,10 @@ inline int64_t max_row_len_elems(int esize) {
 //   ROWOP_BWD_TILE      0 -> dense norm backward rows of whole tiles use the
 //                       team design instead of the whole-tile one (another
 //                       summation order)
+//   ROWOP_BWD_STRIPE    ragged norm backward: 0 -> the bucket launches of the
+//                       team design for every max_len; 2 -> the column-stripe
+//                       design for every max_len (default 1: from
+//                       kStripeMinCols); another summation order
 struct Knobs {
   int force_bucket = -1;
   int cluster = 0;
@@ -197,6 +201,7 @@ struct Knobs {
   int res_gc = 1;
   int bwd_tile = 1;
   int stream = 1;
+  int bwd_stripe = 1;
 };
 Knobs read_knobs();
 

@@ -79,6 +79,7 @@ Knobs read_knobs() {
   k.res_gc = env_int("ROWOP_RESIDENT_GC", 1);
   k.bwd_tile = env_int("ROWOP_BWD_TILE", 1);
   k.stream = env_int("ROWOP_STREAM", 1);
+  k.bwd_stripe = env_int("ROWOP_BWD_STRIPE", 1);
   return k;
 }
 
@@ -373,8 +374,8 @@ static int run_bwd_ragged(int op, const void *a, const void *dy, void *dx, const
   DeviceInfo d;
   const int st = device_info(&d);
   if (st != ROWOP_OK) return st;
-  if (norm && ws_bytes < bwd_ragged_layout(rows, max_len, es, op == kLayerNorm ? 2 : 1,
-                                           d.sm_count, nullptr))
+  if (norm && ws_bytes < bwd_ragged_norm_ws(rows, max_len, es, op == kLayerNorm ? 2 : 1,
+                                            d.sm_count))
     return ROWOP_ERR_WORKSPACE;
   BwdRaggedCall c;
   c.dtype = dtype;
@@ -404,7 +405,7 @@ static size_t bwd_ragged_workspace_size(int nacc, int64_t rows, int64_t max_len,
   if (es == 0 || rows < 0 || max_len < 0) return 0;
   DeviceInfo d;
   if (device_info(&d) != ROWOP_OK) return 0;
-  return bwd_ragged_layout(rows, max_len, es, nacc, d.sm_count, nullptr);
+  return bwd_ragged_norm_ws(rows, max_len, es, nacc, d.sm_count);
 }
 
 static size_t bwd_workspace_size(int nacc, int64_t cols) {

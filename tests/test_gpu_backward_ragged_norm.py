@@ -42,22 +42,24 @@ def make_inputs(dtype, lens, max_len, seed, base_off=0, affine=True):
     return x.to(dtype), dy.to(dtype), None if gam is None else gam.to(dtype), off
 
 
-def call(rw, op, dtype, x, dy, gam, off, max_len, inplace=None, want=(True, True)):
+def call(rw, op, dtype, x, dy, gam, off, max_len, inplace=None, want=(True, True), shift=0):
     """One call on canary-guarded buffers; returns (status, dx buffer, dgamma
-    buffer, dbeta buffer) -- the data sits at [G, G + n) of each."""
+    buffer, dbeta buffer) -- the data sits at [G, G + n) of each.  x, dy and
+    dx start `shift` elements past G of their allocations (the returned dx
+    buffer is the view from `shift`)."""
     total = int(off[-1])
     rows = len(off) - 1
     es = ESIZE[dtype]
-    xb = canary_tensor(G + total + G, dtype)
+    xb = canary_tensor(shift + G + total + G, dtype)[shift:]
     xb[G:G + total] = x.cuda()
-    db = canary_tensor(G + total + G, dtype)
+    db = canary_tensor(shift + G + total + G, dtype)[shift:]
     db[G:G + total] = dy.cuda()
     if inplace == "dy":
         dxb = db
     elif inplace == "x":
         dxb = xb
     else:
-        dxb = canary_tensor(G + total + G, dtype)
+        dxb = canary_tensor(shift + G + total + G, dtype)[shift:]
     n = max(max_len, 1)
     dgb = canary_tensor(G + n + G, dtype) if want[0] else None
     dbb = canary_tensor(G + n + G, dtype) if (op == "layernorm" and want[1]) else None
@@ -124,11 +126,14 @@ def verify(op, dtype, dx_rows, params, pscales, off, dxb, dgb, dbb, max_len, wha
 @pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
 @pytest.mark.parametrize("op", ["layernorm", "rmsnorm"])
 @pytest.mark.parametrize("base_off", [0, 5])
-def test_ragged_norm_backward(rw, op, dtype, base_off):
+@pytest.mark.parametrize("design", ["team", "stripe"])
+def test_ragged_norm_backward(rw, monkeypatch, op, dtype, base_off, design):
     """Rows of every bucket (cluster-split ones included), empty and
     one-element rows, every alignment; dgamma / dbeta over max_len columns,
     the last ones past every row (zero); nothing outside the outputs
-    written."""
+    written.  Both designs: the bucket launches of the team kernel and the
+    column stripes."""
+    monkeypatch.setenv("ROWOP_BWD_STRIPE", "0" if design == "team" else "1")
     lens = _ragged_lengths(dtype, 60, 6, 70000)
     max_len = int(lens.max()) + 37
     x, dy, gam, off = make_inputs(dtype, lens, max_len, seed=11, base_off=base_off)
@@ -295,3 +300,101 @@ def test_workload_ragged_norm_backward(rw, op):
                       f"workload {op} dx row {i}")
     for k, name in enumerate(("dgamma", "dbeta")[:len(sums)]):
         check(to_f64(out[1 + k]), sums[k], ssum[k], case.dtype, R_COMP_PARAM, f"workload {name}")
+
+
+def _stripe_widths(dtype):
+    """Columns of a stripe of the stats and dx kernels: 511 and 255 window
+    chunks of 16 bytes."""
+    e = 16 // ESIZE[dtype]
+    return e * 511, e * 255
+
+
+@pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
+@pytest.mark.parametrize("op", ["layernorm", "rmsnorm"])
+@pytest.mark.parametrize("base_off", [0, 3])
+def test_ragged_norm_backward_stripe_edges(rw, monkeypatch, op, dtype, base_off):
+    """The column-stripe design, taken for every max_len: rows that end at,
+    one before and one past the stripe edges of both kernels, rows shorter
+    than a chunk, empty and one-element rows, at every head class (the
+    lengths repeat, so each length lands at several starts); against the
+    oracle, with nothing outside the outputs written."""
+    monkeypatch.setenv("ROWOP_BWD_STRIPE", "2")
+    w1, w2 = _stripe_widths(dtype)
+    base = [0, 1, 2, 3, 5, 7, 8, 9, 15, 17, w2 - 1, w2, w2 + 1, 2 * w2 + 3, w1 - 1, w1,
+            w1 + 1, w1 + w2, 2 * w1 + 5]
+    lens = np.array(base * 3, dtype=np.int64)
+    np.random.default_rng(base_off).shuffle(lens)
+    max_len = int(lens.max()) + 11
+    x, dy, gam, off = make_inputs(dtype, lens, max_len, seed=21, base_off=base_off)
+    st, dxb, dgb, dbb = call(rw, op, dtype, x, dy, gam, off, max_len)
+    assert st == 0 and rw.check_status() == 0
+    dx_rows, params, ps = reference(op, x, dy, gam, off, max_len)
+    verify(op, dtype, dx_rows, params, ps, off, dxb, dgb, dbb, max_len, f"stripe {op} {dtype}")
+    assert is_canary(dxb[:G + base_off]).all() and is_canary(dxb[G + int(off[-1]):]).all()
+
+
+@pytest.mark.parametrize("op", ["layernorm", "rmsnorm"])
+@pytest.mark.parametrize("max_len", [1, 9, 300])
+def test_ragged_norm_backward_stripe_short(rw, monkeypatch, op, max_len):
+    """The column-stripe design on short rows (one stripe, mostly idle lanes),
+    the options of the call (gamma NULL, dgamma only, no parameter
+    gradients, dx over dy and over x) and a rejected row."""
+    monkeypatch.setenv("ROWOP_BWD_STRIPE", "2")
+    dtype = torch.float32
+    g = np.random.default_rng(max_len)
+    lens = g.integers(0, max_len + 1, 70).astype(np.int64)
+    x, dy, gam, off = make_inputs(dtype, lens, max_len, seed=22, affine=False)
+    dx_rows, params, ps = reference(op, x, dy, None, off, max_len)
+    for inplace, want in ((None, (True, True)), (None, (True, False)), ("dy", (False, False)),
+                          ("x", (True, True))):
+        st, dxb, dgb, dbb = call(rw, op, dtype, x, dy, None, off, max_len, inplace, want)
+        assert st == 0 and rw.check_status() == 0
+        verify(op, dtype, dx_rows, params, ps, off, dxb, dgb, dbb, max_len,
+               f"stripe short {op} max_len {max_len} inplace {inplace} want {want}")
+    lens2 = lens.copy()
+    lens2[3] = max_len + 1
+    x, dy, gam, off = make_inputs(dtype, lens2, max_len, seed=23)
+    st, dxb, dgb, dbb = call(rw, op, dtype, x, dy, gam, off, max_len, inplace="dy")
+    assert st == 0
+    assert rw.check_status() == rw.ROWOP_ERR_BAD_OFFSETS
+    got = to_f64(dxb[G:G + int(off[-1])])
+    assert np.array_equal(got[off[3]:off[4]], dy[off[3]:off[4]].double().numpy())
+    dx_rows, params, ps = reference(op, x, dy, gam, off, max_len, skip=(3,))
+    verify(op, dtype, dx_rows, params, ps, off, dxb, dgb, dbb, max_len, f"stripe rejects {op}")
+
+
+def test_ragged_norm_backward_stripe_many_rows(rw, monkeypatch):
+    """More rows than the dx kernel's groups take in one sorted batch (33000
+    rows: 128 groups of 258), in both designs, against the oracle."""
+    dtype = torch.bfloat16
+    g = np.random.default_rng(24)
+    lens = g.integers(0, 13, 33000).astype(np.int64)
+    max_len = 12
+    x, dy, gam, off = make_inputs(dtype, lens, max_len, seed=24, base_off=1)
+    dx_rows, params, ps = reference("layernorm", x, dy, gam, off, max_len)
+    for mode in ("2", "0"):
+        monkeypatch.setenv("ROWOP_BWD_STRIPE", mode)
+        st, dxb, dgb, dbb = call(rw, "layernorm", dtype, x, dy, gam, off, max_len)
+        assert st == 0 and rw.check_status() == 0
+        verify("layernorm", dtype, dx_rows, params, ps, off, dxb, dgb, dbb, max_len,
+               f"many rows mode {mode}")
+
+
+@pytest.mark.parametrize("op", ["layernorm", "rmsnorm"])
+def test_ragged_norm_backward_stripe_congruent(rw, monkeypatch, op):
+    """x, dy and dx that start past a 16-byte boundary (all by the same
+    amount) take the column-stripe design too: head classes count from the
+    boundary before x."""
+    monkeypatch.setenv("ROWOP_BWD_STRIPE", "2")
+    dtype = torch.bfloat16
+    lens = _ragged_lengths(dtype, 40, 25, 9000)
+    max_len = int(lens.max())
+    x, dy, gam, off = make_inputs(dtype, lens, max_len, seed=25)
+    for shift in (3, 5):  # 6 and 10 bytes past a boundary
+        st, dxb, dgb, dbb = call(rw, op, dtype, x, dy, gam, off, max_len, shift=shift)
+        assert st == 0 and rw.check_status() == 0
+        dx_rows, params, ps = reference(op, x, dy, gam, off, max_len)
+        verify(op, dtype, dx_rows, params, ps, off, dxb, dgb, dbb, max_len,
+               f"congruent {op} shift {shift}")
+        assert is_canary(dxb[:G]).all() and is_canary(dxb[G + int(off[-1]):]).all()
+
