@@ -288,7 +288,8 @@ cudaError_t launch_bwd_t(const BwdCall &c, const DeviceInfo &d) {
   return launch_bwd_k<OP, T, CPT, false, false>(p, s, c, d);
 }
 
-// Ragged norm rows by column stripes (bwd_stripe.cuh): x, dy and dx
+// Ragged norm rows by column stripes (bwd_stripe.cuh: the stats kernel, the
+// dx kernel, then its own finalize over the group partial rows): x, dy and dx
 // congruent modulo 16 bytes and, unless forced (mode 2), max_len of at
 // least kStripeMinCols.  Returns false, launching nothing, otherwise.
 template <int OP, typename T>
@@ -319,9 +320,17 @@ bool try_bwd_stripe(const BwdRaggedCall &c, const DeviceInfo &d, int mode, cudaE
   p.ng2 = L.ng2;
   p.g2 = L.g2;
   p.status = d.status;
+  const void *k1 = reinterpret_cast<const void *>(bwd_stripe_stats_kernel<OP, T>);
+  const void *k2 = reinterpret_cast<const void *>(bwd_stripe_dx_kernel<OP, T>);
+  cudaError_t e = reserve_dynamic_smem(k1, d, kStatRingBytes);
+  if (e == cudaSuccess) e = reserve_dynamic_smem(k2, d, kDxRingBytes);
+  if (e != cudaSuccess) {
+    *err = e;
+    return true;
+  }
   bwd_stripe_stats_kernel<OP, T>
-      <<<static_cast<unsigned>(L.ns1 * L.ng1), kStatThreads, 0, c.stream>>>(p);
-  cudaError_t e = cudaGetLastError();
+      <<<static_cast<unsigned>(L.ns1 * L.ng1), kStatThreads, kStatRingBytes, c.stream>>>(p);
+  e = cudaGetLastError();
   if (e == cudaSuccess) {
     // a programmatic dependent launch: the dx kernel's CTAs sort their rows
     // while the stats kernel drains, and wait for it on the device
@@ -333,13 +342,26 @@ bool try_bwd_stripe(const BwdRaggedCall &c, const DeviceInfo &d, int mode, cudaE
     cfg.numAttrs = 1;
     cfg.gridDim = dim3(static_cast<unsigned>(L.ns2 * L.ng2), 1, 1);
     cfg.blockDim = dim3(kDxThreads, 1, 1);
+    cfg.dynamicSmemBytes = kDxRingBytes;
     cfg.stream = c.stream;
     e = cudaLaunchKernelEx(&cfg, bwd_stripe_dx_kernel<OP, T>, p);
     if (e == cudaSuccess) e = cudaGetLastError();
   }
-  if (e == cudaSuccess && want_params)
-    e = launch_bwd_finalize<T>(one_segment(p.part, L.ng2, c.max_len), c.max_len, nacc,
-                               c.dgamma, c.dbeta, c.stream);
+  if (e == cudaSuccess && want_params) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cfg.gridDim = dim3(static_cast<unsigned>(ceil_div(c.max_len, 64)), static_cast<unsigned>(nacc), 1);
+    cfg.blockDim = dim3(kStripeFinThreads, 1, 1);
+    cfg.stream = c.stream;
+    e = cudaLaunchKernelEx(&cfg, bwd_stripe_finalize_kernel<T>, static_cast<const float *>(p.part),
+                           L.ng2, c.max_len, nacc, static_cast<T *>(c.dgamma),
+                           static_cast<T *>(c.dbeta));
+    if (e == cudaSuccess) e = cudaGetLastError();
+  }
   *err = e;
   return true;
 }

@@ -64,6 +64,7 @@ struct StripeRows {
   int64_t off[N];
   int len[N];
   int row[N];
+  int cls[N];
   int seg[10];
   int wcnt[9][kDxThreads / 32];
 };
@@ -122,6 +123,7 @@ __device__ __forceinline__ bool stripe_sort(StripeRows<N> &L, const int64_t *off
     L.off[pos] = o;
     L.len[pos] = len;
     L.row[pos] = static_cast<int>(r0 + tid);
+    L.cls[pos] = key;
     if (first) first_out[pos] = k;
   }
   __syncthreads();
@@ -163,19 +165,42 @@ __device__ __forceinline__ void stripe_pairs(const uint4 &raw, int lo, int hi, f
   }
 }
 
-// gamma at the columns of a lane's M window chunks for head class h: chunk
-// m is window chunk tid + NT m of the stripe at column `from`; columns
-// outside [from, lim) read as 1 (their data is masked out).
-template <typename T, int M, int NT>
+// Asynchronous 16-byte copy global -> shared through L2 (cp.async, a lane's
+// own copy): only the first `bytes` (0..16) bytes are read, the rest of the
+// 16 bytes written as zero.  Groups commit in order; wait_group N returns
+// once at most N of the lane's latest groups are pending.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(addr));
+  return v;
+}
+
+// gamma at the columns of a lane's M window chunks for head class h: the
+// lane's chunk m starts at column dc[m] (window chunk q: from + E q - h);
+// columns outside [from, lim) read as 1 (their data is masked out).
+template <typename T, int M>
 __device__ __forceinline__ void stripe_gamma(f2 (&gam)[M][Elem<T>::kPerChunk / 2], const T *gamma,
-                                             int64_t from, int64_t lim, int h, int tid) {
+                                             int from, int lim, const int (&dc)[M]) {
   constexpr int E = Elem<T>::kPerChunk;
 #pragma unroll
   for (int m = 0; m < M; ++m) {
     float g[E];
 #pragma unroll
     for (int e = 0; e < E; ++e) {
-      const int64_t col = from + static_cast<int64_t>(E) * (tid + NT * m) + e - h;
+      const int col = dc[m] + e;
       g[e] = (gamma && col >= from && col < lim) ? load_elem(gamma + col) : 1.f;
     }
 #pragma unroll
@@ -206,48 +231,90 @@ __device__ __forceinline__ float warp_reduce_scatter(float (&v)[NV], int lane) {
   return t;
 }
 
-// Position of the chunk a lane owns within one row: element index of the
-// chunk, the column of its element 0, and its valid elements [lo, hi).
-struct StripeChunk {
-  int64_t elem;
-  bool whole;
-  int lo, hi;
-};
+// A lane's sums over its M chunks of one row (raw, from the ring): LayerNorm
+// sum (x - k), sum (x - k)^2, sum t, sum t (x - k) (t = dy gamma); RMSNorm
+// sum x^2, sum t x.  MASK: elements outside a chunk's valid range [lo, hi)
+// read as k (x) and 0 (dy).
+template <typename T, bool kLN, int M, bool MASK>
+__device__ __forceinline__ void stat_sums(const uint4 (&xr)[M], const uint4 (&dr)[M],
+                                          const int (&lo)[M], const int (&hi)[M], float k,
+                                          const f2 (&gam)[M][Elem<T>::kPerChunk / 2],
+                                          float (&v)[kLN ? 4 : 2]) {
+  constexpr int NP = Elem<T>::kPerChunk / 2;
+  const f2 nk = f2_bcast(-k);
+  f2 s1 = f2_bcast(0.f), s2 = f2_bcast(0.f), s3 = f2_bcast(0.f), s4 = f2_bcast(0.f);
+#pragma unroll
+  for (int m = 0; m < M; ++m) {
+    f2 xv[NP], dv[NP];
+    if constexpr (MASK) {
+      stripe_pairs<T>(xr[m], lo[m], hi[m], k, xv);
+      stripe_pairs<T>(dr[m], lo[m], hi[m], 0.f, dv);
+    } else {
+      chunk_to_pairs<T>(xr[m], xv);
+      chunk_to_pairs<T>(dr[m], dv);
+    }
+#pragma unroll
+    for (int i = 0; i < NP; ++i) {
+      const f2 xs = kLN ? f2_add(xv[i], nk) : xv[i];
+      const f2 t = f2_mul(dv[i], gam[m][i]);
+      if constexpr (kLN) {
+        s1 = f2_add(s1, xs);
+        s3 = f2_add(s3, t);
+      }
+      s2 = f2_fma(xs, xs, s2);
+      s4 = f2_fma(t, xs, s4);
+    }
+  }
+  if constexpr (kLN) {
+    v[0] = f2_total(s1);
+    v[1] = f2_total(s2);
+    v[2] = f2_total(s3);
+    v[3] = f2_total(s4);
+  } else {
+    v[0] = f2_total(s2);
+    v[1] = f2_total(s4);
+  }
+}
 
-template <int E>
-__device__ __forceinline__ StripeChunk stripe_chunk(int64_t o, int len, int h, int64_t from,
-                                                    int64_t width, int q) {
-  StripeChunk c;
-  const int64_t d0 = from + static_cast<int64_t>(E) * q - h;  // column of element 0
-  c.elem = o + d0;
-  c.lo = (q == 0) ? h : 0;
-  const int64_t lim = min(from + width, static_cast<int64_t>(len));
-  c.hi = static_cast<int>(max(static_cast<int64_t>(0), min(static_cast<int64_t>(E), lim - d0)));
-  c.whole = d0 >= 0 && d0 + E <= len;
-  return c;
+// Bytes of a lane's chunk that starting at column dc lie before the end of a
+// row of len elements of SZ bytes (0..16): a copy reads no byte past the row.
+template <int SZ>
+__device__ __forceinline__ uint32_t stripe_bytes(int dc, int len) {
+  return static_cast<uint32_t>(max(0, min(16, SZ * (len - dc))));
 }
 
 // ---------------------------------------------------------------------------
-// Row sums per stripe.  Every warp walks the CTA's sorted rows two at a time;
-// a lane reads its two window chunks of x and dy of both rows before using
-// them, then the warp's eight (LayerNorm) or four (RMSNorm) sums are reduced
-// by recursive halving into shared memory; the warps are added in warp order
-// at the end.
+// Row sums per stripe.  Warp w owns the stripe's window chunks
+// [64 w, 64 w + 64), lane l chunks 64 w + l and 64 w + l + 32.  The lanes
+// walk the CTA's sorted rows with their chunks of x and dy of the next
+// kStatDepth - 1 rows in flight (cp.async into the lane's own slots of a
+// shared-memory ring); per row the warp's four (LayerNorm) or two (RMSNorm)
+// sums are reduced by recursive halving into shared memory, and the warps
+// are added in warp order at the end.  A row whose chunks in the warp are
+// all whole and inside the stripe takes a path without masks; a warp with
+// no element of the row skips it (its sums stay zero).
 // ---------------------------------------------------------------------------
+constexpr int kStatDepth = 4;
+constexpr size_t kStatRingBytes = static_cast<size_t>(kStatDepth) * kStatChunks * 2 * kStatThreads * 16;
+
 template <int OP, typename T>
 __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const StripeParams p) {
   static_assert(OP == kLayerNorm || OP == kRmsNorm, "norm backward passes");
+  static_assert(kStatChunks == 2, "two chunks a lane: 64 a warp");
   constexpr int E = Elem<T>::kPerChunk;
+  constexpr int SZ = Elem<T>::kSize;
   constexpr int NP = E / 2;
   constexpr int M = kStatChunks;
   constexpr int NT = kStatThreads;
   constexpr int NW = NT / 32;
-  constexpr int64_t W = static_cast<int64_t>(E) * (NT * M - 1);
+  constexpr int D = kStatDepth;
+  constexpr int W = E * (NT * M - 1);
   constexpr bool kLN = OP == kLayerNorm;
-  constexpr int NV = kLN ? 8 : 4;  // sums of two rows
+  constexpr int NV = kLN ? 4 : 2;  // sums of a row
   __shared__ StripeRows<kStatRows> L;
   __shared__ float kfirst[kStatRows];
   __shared__ float4 wsum[kStatRows][NW];
+  extern __shared__ __align__(16) unsigned char ring[];
   // the dx kernel may be scheduled once every CTA of this one has started;
   // it waits for this grid's completion before it reads what this one writes
   asm volatile("griddepcontrol.launch_dependents;");
@@ -258,11 +325,20 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
   const int64_t g = static_cast<int64_t>(blockIdx.x) % p.ng1;
   const int64_t r0 = g * kStatRows;
   const int n = static_cast<int>(min(static_cast<int64_t>(kStatRows), p.rows - r0));
-  const int64_t from = s * W;
-  const int64_t lim = min(from + W, p.max_len);
+  const int from = static_cast<int>(s) * W;
+  const int lim = static_cast<int>(min(static_cast<int64_t>(from) + W, p.max_len));
   const T *x = static_cast<const T *>(p.x);
   const T *dy = static_cast<const T *>(p.dy);
   const T *gamma = static_cast<const T *>(p.gamma);
+  const uint32_t rbase = smem_addr(ring) + 16u * tid;
+  // the lane's slot of chunk m of tensor t (0 x, 1 dy) for list entry j
+  const auto slot = [&](int j, int m, int t) -> uint32_t {
+    return rbase + static_cast<uint32_t>((((j % D) * M + m) * 2 + t) * NT * 16);
+  };
+  int q[M];
+#pragma unroll
+  for (int m = 0; m < M; ++m) q[m] = 64 * w + lane + 32 * m;
+  for (int i = tid; i < kStatRows * NW; i += NT) (&wsum[0][0])[i] = make_float4(0.f, 0.f, 0.f, 0.f);
 
   const bool bad = stripe_sort<T, NT>(L, p.offsets, r0, n, from, p.max_len, p.hb,
                                       kLN ? x : nullptr, kfirst);
@@ -271,83 +347,91 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
     if (kLN && tid < L.seg[E]) p.shift[L.row[tid]] = kfirst[tid];
   }
   const int cnt = L.seg[E];
-  for (int c = 0; c < E; ++c) {
-    const int j0 = L.seg[c], j1 = L.seg[c + 1];
-    if (j0 == j1) continue;
-    f2 gam[M][NP];
-    stripe_gamma<T, M, NT>(gam, gamma, from, lim, c, tid);
-    for (int j = j0; j < j1; j += 2) {
-      const bool two = j + 1 < j1;
-      uint4 xr[2][M], dr[2][M];
-      int lo[2][M], hi[2][M];
-      float kk[2];
+  // list entry j's chunks into the ring (a group per entry, empty or not)
+  const auto issue = [&](int j) {
+    if (j < cnt) {
+      const int c = L.cls[j];
+      const int len = L.len[j];
+      const int64_t o = L.off[j];
+      const int rl = min(lim, len);
 #pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int jj = (u == 1 && !two) ? j : j + u;
-        kk[u] = kLN ? kfirst[jj] : 0.f;
-        const int64_t o = L.off[jj];
-        const int len = (u == 1 && !two) ? 0 : L.len[jj];
-#pragma unroll
-        for (int m = 0; m < M; ++m) {
-          const StripeChunk ch = stripe_chunk<E>(o, len, c, from, W, tid + NT * m);
-          lo[u][m] = ch.lo;
-          hi[u][m] = ch.hi;
-          xr[u][m] = dr[u][m] = make_uint4(0u, 0u, 0u, 0u);
-          if (ch.lo < ch.hi) {
-            xr[u][m] = stripe_load<T>(x + ch.elem, ch.whole, ch.lo, ch.hi);
-            dr[u][m] = stripe_load<T>(dy + ch.elem, ch.whole, ch.lo, ch.hi);
-          }
+      for (int m = 0; m < M; ++m) {
+        const int dc = from + E * q[m] - c;
+        const int lo = q[m] == 0 ? c : 0;
+        if (lo < min(E, rl - dc)) {
+          const uint32_t nb = stripe_bytes<SZ>(dc, len);
+          cp_async16(slot(j, m, 0), x + o + dc, nb);
+          cp_async16(slot(j, m, 1), dy + o + dc, nb);
         }
-      }
-      float v[NV];
-#pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const f2 nk = f2_bcast(-kk[u]);
-        f2 s1 = f2_bcast(0.f), s2 = f2_bcast(0.f), s3 = f2_bcast(0.f), s4 = f2_bcast(0.f);
-#pragma unroll
-        for (int m = 0; m < M; ++m) {
-          // elements outside the chunk's valid range read as k (x) and 0 (dy)
-          f2 xv[NP], dv[NP];
-          stripe_pairs<T>(xr[u][m], lo[u][m], hi[u][m], kk[u], xv);
-          stripe_pairs<T>(dr[u][m], lo[u][m], hi[u][m], 0.f, dv);
-#pragma unroll
-          for (int i = 0; i < NP; ++i) {
-            const f2 xs = kLN ? f2_add(xv[i], nk) : xv[i];
-            const f2 t = f2_mul(dv[i], gam[m][i]);
-            if constexpr (kLN) {
-              s1 = f2_add(s1, xs);
-              s3 = f2_add(s3, t);
-            }
-            s2 = f2_fma(xs, xs, s2);
-            s4 = f2_fma(t, xs, s4);
-          }
-        }
-        if constexpr (kLN) {
-          v[4 * u + 0] = f2_total(s1);
-          v[4 * u + 1] = f2_total(s2);
-          v[4 * u + 2] = f2_total(s3);
-          v[4 * u + 3] = f2_total(s4);
-        } else {
-          v[2 * u + 0] = f2_total(s2);
-          v[2 * u + 1] = f2_total(s4);
-        }
-      }
-      const float t = warp_reduce_scatter<NV>(v, lane);
-      constexpr int kStride = 32 / NV;
-      if ((lane & (kStride - 1)) == 0) {
-        const int i = lane / kStride;  // value index
-        const int u = kLN ? (i >> 2) : (i >> 1);
-        const int comp = kLN ? (i & 3) : 1 + 2 * (i & 1);  // RMSNorm: .y, .w
-        if (u == 0 || two) reinterpret_cast<float *>(&wsum[j + u][w])[comp] = t;
       }
     }
+    cp_async_commit();
+  };
+#pragma unroll
+  for (int j = 0; j < D - 1; ++j) issue(j);
+  int cur = -1;
+  int dc[M], lo[M];
+  f2 gam[M][NP];
+  for (int j = 0; j < cnt; ++j) {
+    issue(j + D - 1);
+    const int c = L.cls[j];
+    if (c != cur) {  // a new head class: the lane's columns and gamma there
+      cur = c;
+#pragma unroll
+      for (int m = 0; m < M; ++m) {
+        dc[m] = from + E * q[m] - c;
+        lo[m] = q[m] == 0 ? c : 0;
+      }
+      stripe_gamma<T, M>(gam, gamma, from, lim, dc);
+    }
+    const int rl = min(lim, L.len[j]);
+    const float k = kLN ? kfirst[j] : 0.f;
+    int hi[M];
+    bool full = true, any = false;
+#pragma unroll
+    for (int m = 0; m < M; ++m) {
+      hi[m] = min(E, rl - dc[m]);
+      full = full && hi[m] == E && lo[m] == 0;
+      any = any || hi[m] > lo[m];
+    }
+    cp_async_wait<D - 1>();  // entry j's copies have landed
+    float v[NV];
+    uint4 xr[M], dr[M];
+    if (__all_sync(kFullMask, full)) {
+#pragma unroll
+      for (int m = 0; m < M; ++m) {
+        xr[m] = lds128(slot(j, m, 0));
+        dr[m] = lds128(slot(j, m, 1));
+      }
+      stat_sums<T, kLN, M, false>(xr, dr, lo, hi, k, gam, v);
+    } else if (__any_sync(kFullMask, any)) {
+#pragma unroll
+      for (int m = 0; m < M; ++m) {
+        xr[m] = dr[m] = make_uint4(0u, 0u, 0u, 0u);
+        if (lo[m] < hi[m]) {
+          xr[m] = lds128(slot(j, m, 0));
+          dr[m] = lds128(slot(j, m, 1));
+        }
+      }
+      stat_sums<T, kLN, M, true>(xr, dr, lo, hi, k, gam, v);
+    } else {
+      continue;  // no element of the row in this warp's chunks
+    }
+    const float t = warp_reduce_scatter<NV>(v, lane);
+    constexpr int kStride = 32 / NV;
+    if ((lane & (kStride - 1)) == 0) {
+      const int i = lane / kStride;                   // value index
+      const int comp = kLN ? i : 1 + 2 * i;           // RMSNorm: .y, .w
+      reinterpret_cast<float *>(&wsum[j][w])[comp] = t;
+    }
   }
+  cp_async_wait<0>();
   __syncthreads();
   for (int j = tid; j < cnt; j += NT) {
     float4 t = wsum[j][0];
 #pragma unroll
-    for (int q = 1; q < NW; ++q) {
-      const float4 u = wsum[j][q];
+    for (int qq = 1; qq < NW; ++qq) {
+      const float4 u = wsum[j][qq];
       t.y = __fadd_rn(t.y, u.y);
       t.w = __fadd_rn(t.w, u.w);
       if constexpr (kLN) {
@@ -364,45 +448,96 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
 // word of padding every 32, so that lanes E columns apart hit distinct banks.
 __device__ __forceinline__ int stripe_pad(int local) { return local + (local >> 5); }
 
+// dx of one chunk from its pairs and the row's coefficients {rstd,
+// -mean rstd, -mean(t) rstd, -mean(t xhat) rstd} (t = dy gamma), adding
+// dy xhat (and dy) to the lane's column sums when wanted.
+template <bool kLN, int NP>
+__device__ __forceinline__ void stripe_dx(const f2 (&xv)[NP], const f2 (&dv)[NP],
+                                          const f2 (&gam)[NP], const float4 &cf, bool want,
+                                          f2 (&o)[NP], f2 (&accg)[NP], f2 (&accb)[NP]) {
+  const f2 C0 = f2_bcast(cf.x), C1 = f2_bcast(cf.y), NA = f2_bcast(cf.z), NB = f2_bcast(cf.w);
+#pragma unroll
+  for (int i = 0; i < NP; ++i) {
+    const f2 xh = f2_fma(xv[i], C0, C1);
+    const f2 t = f2_mul(dv[i], gam[i]);
+    o[i] = f2_fma(t, C0, f2_fma(xh, NB, NA));
+    if (want) {
+      accg[i] = f2_fma(dv[i], xh, accg[i]);
+      if constexpr (kLN) accb[i] = f2_add(accb[i], dv[i]);
+    }
+  }
+}
+
 // ---------------------------------------------------------------------------
-// dx and the column sums.  Per batch of up to 256 rows of the group: sort,
-// then each listed row's statistics from the stats kernel's stripe sums (in
-// stripe order), then per head class the rows four at a time: a lane reads
-// its window chunk of x and dy of the four rows, then writes its dx chunks
-// and adds dy xhat (and dy) to its register sums; at the class's end the
-// lane adds those sums into the CTA's partial row in shared memory.  The
-// CTA writes its partial row (its stripe of group g's row) at the end.
+// dx and the column sums.  Lane t owns window chunk t of the stripe.  Per
+// batch of up to 256 rows of the group: sort, then each listed row's
+// statistics from the stats kernel's stripe sums (in stripe order), then the
+// rows in list order with the lane's chunks of x and dy of the next
+// kDxDepth - 1 rows in flight (cp.async into the lane's own ring slots): the
+// lane writes its dx chunk and adds dy xhat (and dy) to its register sums.
+// When the head class changes the lane adds those sums into the CTA's
+// partial row in shared memory at their columns.  A row whose chunks in the
+// warp are all whole and inside the stripe takes a path without masks; a
+// warp with no element of the row skips it.  The CTA writes its partial row
+// (its stripe of group g's row) at the end.
 // ---------------------------------------------------------------------------
+constexpr int kDxDepth = 5;
+constexpr size_t kDxRingBytes = static_cast<size_t>(kDxDepth) * 2 * kDxThreads * 16;
+
 template <int OP, typename T>
 __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const StripeParams p) {
   static_assert(OP == kLayerNorm || OP == kRmsNorm, "norm backward passes");
   constexpr int E = Elem<T>::kPerChunk;
+  constexpr int SZ = Elem<T>::kSize;
   constexpr int NP = E / 2;
   constexpr int NT = kDxThreads;
-  constexpr int64_t W = static_cast<int64_t>(E) * (NT - 1);
-  constexpr int64_t W1 = static_cast<int64_t>(E) * (kStatThreads * kStatChunks - 1);
+  constexpr int D = kDxDepth;
+  constexpr int W = E * (NT - 1);
+  constexpr int W1 = E * (kStatThreads * kStatChunks - 1);
   constexpr bool kLN = OP == kLayerNorm;
   constexpr int NA = kLN ? 2 : 1;
-  constexpr int kPadW = static_cast<int>(W + W / 32 + 1);
-  constexpr int U = 3;
+  constexpr int kPadW = W + W / 32 + 1;
   __shared__ StripeRows<kDxBatch> L;
   __shared__ float4 coef[kDxBatch];
   __shared__ float spart[NA][kPadW];
+  extern __shared__ __align__(16) unsigned char ring[];
   const int tid = threadIdx.x;
   const int64_t s = static_cast<int64_t>(blockIdx.x) / p.ng2;  // heavy stripes first
   const int64_t g = static_cast<int64_t>(blockIdx.x) % p.ng2;
-  const int64_t from = s * W;
-  const int64_t lim = min(from + W, p.max_len);
+  const int from = static_cast<int>(s) * W;
+  const int lim = static_cast<int>(min(static_cast<int64_t>(from) + W, p.max_len));
   const T *x = static_cast<const T *>(p.x);
   const T *dy = static_cast<const T *>(p.dy);
   T *dx = static_cast<T *>(p.dx);
   const T *gamma = static_cast<const T *>(p.gamma);
   const bool want = p.part != nullptr;
+  const uint32_t rbase = smem_addr(ring) + 16u * tid;
+  // the lane's slot of tensor t (0 x, 1 dy) for list entry j
+  const auto slot = [&](int j, int t) -> uint32_t {
+    return rbase + static_cast<uint32_t>(((j % D) * 2 + t) * NT * 16);
+  };
   for (int i = tid; i < NA * kPadW; i += NT) (&spart[0][0])[i] = 0.f;
 
   f2 accg[NP], accb[NP];
 #pragma unroll
   for (int i = 0; i < NP; ++i) accg[i] = accb[i] = f2_bcast(0.f);
+  // the class's sums into the partial row at their columns (class c)
+  const auto flush = [&](int c) {
+    if (want) {
+#pragma unroll
+      for (int e = 0; e < E; ++e) {
+        const int local = E * tid + e - c;
+        if (local >= 0 && local < W) {
+          const int qq = stripe_pad(local);
+          spart[0][qq] = __fadd_rn(spart[0][qq], pair_elem(accg, e));
+          if constexpr (kLN) spart[NA - 1][qq] = __fadd_rn(spart[NA - 1][qq], pair_elem(accb, e));
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < NP; ++i) accg[i] = accb[i] = f2_bcast(0.f);
+    }
+    __syncthreads();  // the next flush may add to the same columns
+  };
   const int64_t gr0 = g * p.g2;
   const int64_t gr1 = min(gr0 + p.g2, p.rows);
   bool waited = false;
@@ -417,15 +552,33 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
       waited = true;
     }
     const int cnt = L.seg[E];
+    // list entry j's chunk into the ring (a group per entry, empty or not)
+    const auto issue = [&](int j) {
+      if (j < cnt) {
+        const int c = L.cls[j];
+        const int len = L.len[j];
+        const int dc = from + E * tid - c;
+        const int lo = tid == 0 ? c : 0;
+        if (lo < min(E, min(lim, len) - dc)) {
+          const int64_t o = L.off[j];
+          const uint32_t nb = stripe_bytes<SZ>(dc, len);
+          cp_async16(slot(j, 0), x + o + dc, nb);
+          cp_async16(slot(j, 1), dy + o + dc, nb);
+        }
+      }
+      cp_async_commit();
+    };
+#pragma unroll
+    for (int j = 0; j < D - 1; ++j) issue(j);
     if (tid < cnt) {
       const int64_t r = L.row[tid];
       const int len = L.len[tid];
-      const int nst = static_cast<int>((len + W1 - 1) / W1);
+      const int nst = (len + W1 - 1) / W1;
       const float4 *ps = p.psum + r * p.ns1;
       float4 t = ps[0];
 #pragma unroll 4
-      for (int q = 1; q < nst; ++q) {
-        const float4 u = ps[q];
+      for (int qq = 1; qq < nst; ++qq) {
+        const float4 u = ps[qq];
         t.x = __fadd_rn(t.x, u.x);
         t.y = __fadd_rn(t.y, u.y);
         t.z = __fadd_rn(t.z, u.z);
@@ -449,78 +602,101 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
       coef[tid] = cf;
     }
     __syncthreads();
-    for (int c = 0; c < E; ++c) {
-      const int j0 = L.seg[c], j1 = L.seg[c + 1];
-      if (j0 == j1) continue;
-      f2 gam[1][NP];
-      stripe_gamma<T, 1, NT>(gam, gamma, from, lim, c, tid);
-      for (int j = j0; j < j1; j += U) {
-        uint4 xr[U], dr[U];
-        StripeChunk ch[U];
+    int cur = -1, dc = 0, lo = 0;
+    f2 gam[1][NP];
+    for (int j = 0; j < cnt; ++j) {
+      issue(j + D - 1);
+      const int c = L.cls[j];
+      if (c != cur) {  // a new head class: the lane's columns and gamma there
+        if (cur >= 0) flush(cur);
+        cur = c;
+        dc = from + E * tid - c;
+        lo = tid == 0 ? c : 0;
+        const int dc1[1] = {dc};
+        stripe_gamma<T, 1>(gam, gamma, from, lim, dc1);
+      }
+      const int len = L.len[j];
+      const int hi = min(E, min(lim, len) - dc);
+      const bool full = hi == E && lo == 0;
+      cp_async_wait<D - 1>();  // entry j's copies have landed
+      if (__all_sync(kFullMask, full)) {
+        f2 xv[NP], dv[NP], ov[NP];
+        chunk_to_pairs<T>(lds128(slot(j, 0)), xv);
+        chunk_to_pairs<T>(lds128(slot(j, 1)), dv);
+        stripe_dx<kLN, NP>(xv, dv, gam[0], coef[j], want, ov, accg, accb);
+        stg_stream(dx + L.off[j] + dc, pairs_to_chunk<T>(ov));
+      } else if (lo < hi) {
+        // elements outside the chunk's valid range read as 0: no dy, so
+        // they add nothing to the column sums
+        f2 xv[NP], dv[NP], ov[NP];
+        stripe_pairs<T>(lds128(slot(j, 0)), lo, hi, 0.f, xv);
+        stripe_pairs<T>(lds128(slot(j, 1)), lo, hi, 0.f, dv);
+        stripe_dx<kLN, NP>(xv, dv, gam[0], coef[j], want, ov, accg, accb);
+        T *dst = dx + L.off[j] + dc;
+        if (lo == 0 && hi == E) {
+          stg_stream(dst, pairs_to_chunk<T>(ov));
+        } else {
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
-          const bool on = j + u < j1;
-          const int jj = on ? j + u : j;
-          ch[u] = stripe_chunk<E>(L.off[jj], on ? L.len[jj] : 0, c, from, W, tid);
-          xr[u] = dr[u] = make_uint4(0u, 0u, 0u, 0u);
-          if (ch[u].lo < ch[u].hi) {
-            xr[u] = stripe_load<T>(x + ch[u].elem, ch[u].whole, ch[u].lo, ch[u].hi);
-            dr[u] = stripe_load<T>(dy + ch[u].elem, ch[u].whole, ch[u].lo, ch[u].hi);
-          }
-        }
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-          if (ch[u].lo >= ch[u].hi) continue;
-          const float4 cf = coef[j + u];
-          const f2 C0 = f2_bcast(cf.x), C1 = f2_bcast(cf.y), NA_ = f2_bcast(cf.z),
-                   NB = f2_bcast(cf.w);
-          // elements outside the chunk's valid range read as 0: no dy, so
-          // they add nothing to the column sums
-          f2 xv[NP], dv[NP], o[NP];
-          stripe_pairs<T>(xr[u], ch[u].lo, ch[u].hi, 0.f, xv);
-          stripe_pairs<T>(dr[u], ch[u].lo, ch[u].hi, 0.f, dv);
-#pragma unroll
-          for (int i = 0; i < NP; ++i) {
-            const f2 xh = f2_fma(xv[i], C0, C1);
-            const f2 t = f2_mul(dv[i], gam[0][i]);
-            o[i] = f2_fma(t, C0, f2_fma(xh, NB, NA_));
-            if (want) {
-              accg[i] = f2_fma(dv[i], xh, accg[i]);
-              if constexpr (kLN) accb[i] = f2_add(accb[i], dv[i]);
-            }
-          }
-          if (ch[u].lo == 0 && ch[u].hi == E) {
-            stg_stream(dx + ch[u].elem, pairs_to_chunk<T>(o));
-          } else {
-#pragma unroll
-            for (int e = 0; e < E; ++e)
-              if (e >= ch[u].lo && e < ch[u].hi) dx[ch[u].elem + e] = from_f32<T>(pair_elem(o, e));
-          }
+          for (int e = 0; e < E; ++e)
+            if (e >= lo && e < hi) dst[e] = from_f32<T>(pair_elem(ov, e));
         }
       }
-      if (want) {  // the class's sums into the partial row, at their columns
-#pragma unroll
-        for (int e = 0; e < E; ++e) {
-          const int local = E * tid + e - c;
-          if (local >= 0 && local < W) {
-            const int q = stripe_pad(local);
-            spart[0][q] = __fadd_rn(spart[0][q], pair_elem(accg, e));
-            if constexpr (kLN) spart[NA - 1][q] = __fadd_rn(spart[NA - 1][q], pair_elem(accb, e));
-          }
-        }
-#pragma unroll
-        for (int i = 0; i < NP; ++i) accg[i] = accb[i] = f2_bcast(0.f);
-      }
-      __syncthreads();
     }
+    cp_async_wait<0>();
+    if (cur >= 0) flush(cur);  // ends with a barrier: L and coef may be rewritten
   }
   if (!waited) asm volatile("griddepcontrol.wait;" ::: "memory");
   if (!want) return;
   __syncthreads();
-  const int64_t ncols = lim - from;
+  const int ncols = lim - from;
   for (int a = 0; a < NA; ++a) {
     float *prow = p.part + (g * NA + a) * p.max_len + from;
     for (int i = tid; i < ncols; i += NT) prow[i] = spart[a][stripe_pad(i)];
+  }
+}
+
+// dgamma[j] (dbeta[j]) = the sum over the dx kernel's group partial rows
+// q = 0, 1, ... of part[q][0 (1)][j], for j < cols.  A block of 256 threads
+// takes 64 columns: warp w adds, for column half w & 1, the partials
+// q = w >> 1, (w >> 1) + 4, ... in that order, eight loads ahead; the four
+// slices are then added in slice order.  Launched as a programmatic
+// dependent of the dx kernel.
+constexpr int kStripeFinThreads = 256;
+template <typename T>
+__global__ void __launch_bounds__(kStripeFinThreads) bwd_stripe_finalize_kernel(
+    const float *part, int64_t nparts, int64_t cols, int nacc, T *dgamma, T *dbeta) {
+  __shared__ float sums[4][64];
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const int lane = threadIdx.x & 31;
+  const int w = threadIdx.x >> 5;
+  const int a = blockIdx.y;
+  T *out = a == 0 ? dgamma : dbeta;
+  if (out == nullptr) return;  // uniform over the block
+  const int col = 32 * (w & 1) + lane;
+  const int slice = w >> 1;
+  const int64_t j = static_cast<int64_t>(blockIdx.x) * 64 + col;
+  float sum = 0.f;
+  if (j < cols) {
+    constexpr int U = 8;
+    for (int64_t q0 = slice; q0 < nparts; q0 += 4 * U) {
+      float v[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int64_t q = q0 + 4 * u;
+        v[u] = q < nparts ? __ldcs(part + (q * nacc + a) * cols + j) : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (q0 + 4 * u < nparts) sum = __fadd_rn(sum, v[u]);
+    }
+  }
+  sums[slice][col] = sum;
+  __syncthreads();
+  if (w < 2 && j < cols) {
+    float t = sums[0][col];
+#pragma unroll
+    for (int q = 1; q < 4; ++q) t = __fadd_rn(t, sums[q][col]);
+    out[j] = from_f32<T>(t);
   }
 }
 

@@ -70,4 +70,20 @@ inline cudaError_t prepare_kernel(const void *kernel, const DeviceInfo &d, bool 
   return cudaSuccess;
 }
 
+// A kernel's dynamic shared-memory limit raised to `bytes` (for kernels
+// that also hold static shared memory), once per kernel and device.
+inline cudaError_t reserve_dynamic_smem(const void *kernel, const DeviceInfo &d, size_t bytes) {
+  static std::mutex mu;
+  static std::map<std::pair<const void *, int>, size_t> done;
+  std::lock_guard<std::mutex> lk(mu);
+  const auto key = std::make_pair(kernel, d.device);
+  auto it = done.find(key);
+  if (it != done.end() && it->second >= bytes) return cudaSuccess;
+  const cudaError_t e =
+      cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
+  if (e != cudaSuccess) return e;
+  done[key] = bytes;
+  return cudaSuccess;
+}
+
 }  // namespace rowop
