@@ -214,15 +214,26 @@ ROWOP_API int rowop_logsoftmax_backward_ragged(const void *y, const void *dy, vo
  * row of that length.  dgamma[j] (and, for LayerNorm, dbeta[j]) for
  * j < max_len sums dy_j xhat_j (dy_j) over the rows longer than j: max_len
  * elements of dtype each, or NULL when not wanted; rows == 0 sets them to
- * zero.  Rows are read and written element by element, at any alignment.
+ * zero.  Rows may start at any element.
+ *
+ * Two designs, chosen per call (each with its own summation order):
+ *   * x, dy and dx at the same offset past a 16-byte boundary and
+ *     max_len >= 2048: column stripes.  A first kernel writes each row's
+ *     sums over each stripe of 4088 (bf16 / fp16) or 2044 (fp32) columns.
+ *     A second adds them into the row statistics, writes dx and sums
+ *     dgamma / dbeta into one float32 partial row per group of rows; a
+ *     finalize adds the groups in index order.  x and dy are read twice.
+ *     LayerNorm's variance is taken about each row's first element.
+ *   * otherwise: the forward's classify plan, one launch per row bucket,
+ *     and one float32 partial row per CTA for each bucket, added in index
+ *     order, the buckets in order (SMALL, MEDIUM, LARGE).
+ * Either way nothing is atomic: the result is reproducible bit for bit on
+ * one device.
  *
  * ws: device, 256-byte aligned, at least
  * rowop_{layernorm,rmsnorm}_backward_ragged_workspace_size(rows, max_len,
- * dtype) bytes on the current device: the classify plan, then one float32
- * partial row per CTA for each row bucket, covering that bucket's longest
- * row.  The partials of each bucket are added in index order, the buckets in
- * order (SMALL, MEDIUM, LARGE), so the result is reproducible bit for bit on
- * one device.  The workspace must not be shared by concurrent calls.
+ * dtype) bytes on the current device (enough for either design).  The
+ * workspace must not be shared by concurrent calls.
  *
  * max_len <= ROWOP_BWD_MAX_COLS_NORM_RAGGED (else ROWOP_ERR_TOO_LONG); rows longer
  * than max_len or with decreasing offsets are skipped and flagged as in the
