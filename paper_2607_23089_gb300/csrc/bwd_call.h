@@ -84,12 +84,12 @@ inline int64_t stripe_dx_width(int esize) {
   return static_cast<int64_t>(16 / esize) * (kDxThreads - 1);
 }
 
-// Workspace of the striped design, all 256-byte aligned: each row's first
-// element (LayerNorm's shift), the per-stripe row sums [rows][ns1] float4,
-// and the dgamma / dbeta partial rows [ng2][nacc][max_len] float32.
+// Workspace of the striped design, both parts 256-byte aligned: the
+// per-stripe row statistics [rows][ns1] float4, and the dgamma / dbeta
+// partial rows [ng2][nacc][max_len] float32.
 struct StripeLayout {
   int64_t ns1, ng1, ns2, ng2, g2;  // stripes and row groups of the two kernels
-  size_t shift, psum, part, total;
+  size_t psum, part, total;
 };
 
 inline StripeLayout stripe_layout(int64_t rows, int64_t max_len, int esize, int nacc) {
@@ -102,8 +102,7 @@ inline StripeLayout stripe_layout(int64_t rows, int64_t max_len, int esize, int 
       1, std::min<int64_t>((rows + kDxMinGroupRows - 1) / kDxMinGroupRows, kDxMaxGroups));
   L.g2 = (rows + L.ng2 - 1) / L.ng2;
   const size_t r = static_cast<size_t>(std::max<int64_t>(rows, 0));
-  L.shift = 0;
-  L.psum = up(r * sizeof(float));
+  L.psum = 0;
   L.part = L.psum + up(r * static_cast<size_t>(L.ns1) * 16u);
   L.total = L.part + up(static_cast<size_t>(L.ng2) * static_cast<size_t>(nacc) *
                         static_cast<size_t>(max_len) * sizeof(float));

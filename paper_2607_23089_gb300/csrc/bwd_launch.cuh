@@ -312,7 +312,6 @@ bool try_bwd_stripe(const BwdRaggedCall &c, const DeviceInfo &d, int mode, cudaE
   p.max_len = c.max_len;
   p.eps = c.eps;
   p.hb = static_cast<int>((reinterpret_cast<uintptr_t>(c.a) & 15u) / SZ);
-  p.shift = reinterpret_cast<float *>(ws + L.shift);
   p.psum = reinterpret_cast<float4 *>(ws + L.psum);
   p.part = want_params ? reinterpret_cast<float *>(ws + L.part) : nullptr;
   p.ns1 = L.ns1;

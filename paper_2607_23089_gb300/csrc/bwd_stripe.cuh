@@ -2,15 +2,15 @@
 // (the derivatives of §2.1's row-wise norms, as in bwd_row.cuh, on the ragged
 // layout), by column stripes, for x, dy and dx congruent modulo 16 bytes.
 //
-// Two kernels, then bwd_param_finalize_kernel:
+// Two kernels, then bwd_stripe_finalize_kernel:
 //   * bwd_stripe_stats_kernel: CTA (s, g) takes rows [64 g, 64 g + 64) and
-//     their columns [s W1, (s+1) W1).  For each row it writes the sums over
-//     those columns (LayerNorm: sum (x - k), sum (x - k)^2, sum t and
-//     sum t (x - k), with t = dy gamma and k the row's first element;
-//     RMSNorm: sum x^2 and sum t x): one float4 per row and stripe;
+//     their columns [s W1, (s+1) W1).  For each row it writes the statistics
+//     of those columns (LayerNorm: mean, sum of squares about it, sum t and
+//     sum t (x - mean), with t = dy gamma; RMSNorm: sum x^2 and sum t x): one
+//     float4 per row and stripe;
 //   * bwd_stripe_dx_kernel: CTA (s, g) takes the rows of group g and their
-//     columns [s W2, (s+1) W2).  It adds each row's stripe sums in stripe
-//     order into the row statistics, writes dx over its columns, and sums
+//     columns [s W2, (s+1) W2).  It merges each row's stripe statistics in
+//     stripe order into the row's, writes dx over its columns, and sums
 //     dy xhat (and dy) over its rows into group g's partial row;
 //   * the finalize adds the groups' partial rows in index order.
 // x and dy are read twice (10 bytes an element of a 16-bit type against the
@@ -30,10 +30,13 @@
 // that crosses a stripe edge is read whole when it lies inside the row and
 // written element by element.
 //
-// LayerNorm's mean and variance come from the sums about k, the shifted-data
-// formula: var = mean((x - k)^2) - mean(x - k)^2, whose cancellation grows
-// only with (mean - k)^2 / var.  Nothing is atomic, and every sum has a
-// fixed order given the offsets, so the result is bitwise reproducible.
+// LayerNorm's statistics are formed about local means: each warp takes the
+// mean of its elements of a row, then the sums about that mean from the same
+// registers, and the warps' and then the stripes' statistics are merged
+// pairwise (count, mean, M2, sum t, sum t (x - mean)), so no cancellation
+// grows with the distance of the values from zero or from one another.
+// Nothing is atomic, and every sum and merge has a fixed order given the
+// offsets, so the result is bitwise reproducible.
 #pragma once
 
 #include "bwd_call.h"
@@ -50,8 +53,7 @@ struct StripeParams {
   int64_t rows, max_len;
   float eps;
   int hb;        // element offset of x (dy, dx) past a 16-byte boundary
-  float *shift;  // [rows] LayerNorm: each row's first element
-  float4 *psum;  // [rows][ns1] the stats kernel's row sums per stripe
+  float4 *psum;  // [rows][ns1] the stats kernel's row statistics per stripe
   float *part;   // [ng2][nacc][max_len] dgamma (dbeta) partial rows; NULL = not wanted
   int64_t ns1, ng1, ng2, g2;
   unsigned int *status;
@@ -71,13 +73,10 @@ struct StripeRows {
 
 // Rows [r0, r0 + n), one a thread (n <= NT): those that reach column `from`
 // (valid, 0 <= length <= max_len, and longer than `from`) are listed in L by
-// head class, then by row.  With `first` given, the thread of a listed row
-// also stores the row's first element in first_out[position].  Returns
-// whether the thread's row is invalid.
+// head class, then by row.  Returns whether the thread's row is invalid.
 template <typename T, int NT, int N>
 __device__ __forceinline__ bool stripe_sort(StripeRows<N> &L, const int64_t *offsets, int64_t r0,
-                                            int n, int64_t from, int64_t max_len, int hb,
-                                            const T *first, float *first_out) {
+                                            int n, int64_t from, int64_t max_len, int hb) {
   constexpr int E = Elem<T>::kPerChunk;
   constexpr int NW = NT / 32;
   static_assert(N <= NT && NW <= kDxThreads / 32, "one row a thread");
@@ -88,17 +87,13 @@ __device__ __forceinline__ bool stripe_sort(StripeRows<N> &L, const int64_t *off
   int len = 0;
   int64_t o = 0;
   bool bad = false;
-  float k = 0.f;
   if (tid < n) {
     o = offsets[r0 + tid];
     const int64_t l = offsets[r0 + tid + 1] - o;
     bad = l < 0 || l > max_len;
     if (!bad) {
       len = static_cast<int>(l);
-      if (l > from) {
-        key = static_cast<int>((o + hb) & (E - 1));
-        if (first) k = load_elem(first + o);
-      }
+      if (l > from) key = static_cast<int>((o + hb) & (E - 1));
     }
   }
   unsigned mine = 0;
@@ -124,7 +119,6 @@ __device__ __forceinline__ bool stripe_sort(StripeRows<N> &L, const int64_t *off
     L.len[pos] = len;
     L.row[pos] = static_cast<int>(r0 + tid);
     L.cls[pos] = key;
-    if (first) first_out[pos] = k;
   }
   __syncthreads();
   return bad;
@@ -231,49 +225,98 @@ __device__ __forceinline__ float warp_reduce_scatter(float (&v)[NV], int lane) {
   return t;
 }
 
-// A lane's sums over its M chunks of one row (raw, from the ring): LayerNorm
-// sum (x - k), sum (x - k)^2, sum t, sum t (x - k) (t = dy gamma); RMSNorm
-// sum x^2, sum t x.  MASK: elements outside a chunk's valid range [lo, hi)
-// read as k (x) and 0 (dy).
+// Row statistics of a set of a row's elements, about their own mean:
+// count n, mean m, M2 = sum (x - m)^2, St = sum t and Stx = sum t (x - m)
+// (t = dy gamma).  stat_merge folds b into a (Chan, Golub and LeVeque's
+// pairwise update, with sum t (x - m) carried to the merged mean); the
+// order of merges is fixed by the caller.
+struct RowStat {
+  float n, m, M2, St, Stx;
+};
+__device__ __forceinline__ void stat_merge(RowStat &a, const RowStat &b) {
+  if (b.n == 0.f) return;
+  if (a.n == 0.f) {
+    a = b;
+    return;
+  }
+  const float nn = __fadd_rn(a.n, b.n);
+  const float d = __fsub_rn(b.m, a.m);
+  const float fb = __fdividef(b.n, nn);  // the share of b
+  const float fa = __fdividef(a.n, nn);
+  a.M2 = __fadd_rn(__fadd_rn(a.M2, b.M2), __fmul_rn(__fmul_rn(d, d), __fmul_rn(a.n, fb)));
+  a.Stx = __fadd_rn(__fadd_rn(a.Stx, b.Stx),
+                    __fmul_rn(d, __fsub_rn(__fmul_rn(b.St, fa), __fmul_rn(a.St, fb))));
+  a.St = __fadd_rn(a.St, b.St);
+  a.m = __fadd_rn(a.m, __fmul_rn(d, fb));
+  a.n = nn;
+}
+
+// A warp's statistics of one row over its lanes' M chunks (pairs, elements
+// outside [lo, hi) zero when MASK).  LayerNorm: the warp's sum (a
+// butterfly) over its n_w elements (n_w > 0, from the row's geometry) gives
+// its mean m_w, then the sums about m_w from the same registers are reduced
+// by recursive halving: lanes 0, 8 and 16 return M2, St and Stx.  m_w is
+// the quotient rounded once more; it stands as the shift of those sums, and
+// a shift off the mean by a rounding error changes M2 by n_w times its
+// square.  RMSNorm: sum x^2 and sum t x, in lanes 0 and 16.
 template <typename T, bool kLN, int M, bool MASK>
-__device__ __forceinline__ void stat_sums(const uint4 (&xr)[M], const uint4 (&dr)[M],
-                                          const int (&lo)[M], const int (&hi)[M], float k,
-                                          const f2 (&gam)[M][Elem<T>::kPerChunk / 2],
-                                          float (&v)[kLN ? 4 : 2]) {
-  constexpr int NP = Elem<T>::kPerChunk / 2;
-  const f2 nk = f2_bcast(-k);
-  f2 s1 = f2_bcast(0.f), s2 = f2_bcast(0.f), s3 = f2_bcast(0.f), s4 = f2_bcast(0.f);
-#pragma unroll
-  for (int m = 0; m < M; ++m) {
-    f2 xv[NP], dv[NP];
-    if constexpr (MASK) {
-      stripe_pairs<T>(xr[m], lo[m], hi[m], k, xv);
-      stripe_pairs<T>(dr[m], lo[m], hi[m], 0.f, dv);
-    } else {
-      chunk_to_pairs<T>(xr[m], xv);
-      chunk_to_pairs<T>(dr[m], dv);
-    }
-#pragma unroll
-    for (int i = 0; i < NP; ++i) {
-      const f2 xs = kLN ? f2_add(xv[i], nk) : xv[i];
-      const f2 t = f2_mul(dv[i], gam[m][i]);
-      if constexpr (kLN) {
-        s1 = f2_add(s1, xs);
-        s3 = f2_add(s3, t);
-      }
-      s2 = f2_fma(xs, xs, s2);
-      s4 = f2_fma(t, xs, s4);
-    }
-  }
+__device__ __forceinline__ float warp_row_stats(const f2 (&xv)[M][Elem<T>::kPerChunk / 2],
+                                                const f2 (&dv)[M][Elem<T>::kPerChunk / 2],
+                                                const int (&lo)[M], const int (&hi)[M],
+                                                const f2 (&gam)[M][Elem<T>::kPerChunk / 2],
+                                                int lane, float n_w, float &m_w) {
+  constexpr int E = Elem<T>::kPerChunk;
+  constexpr int NP = E / 2;
   if constexpr (kLN) {
-    v[0] = f2_total(s1);
-    v[1] = f2_total(s2);
-    v[2] = f2_total(s3);
-    v[3] = f2_total(s4);
+    f2 sx = f2_bcast(0.f);
+#pragma unroll
+    for (int m = 0; m < M; ++m)
+#pragma unroll
+      for (int i = 0; i < NP; ++i) sx = f2_add(sx, xv[m][i]);
+    float t = f2_total(sx);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t = __fadd_rn(t, __shfl_xor_sync(kFullMask, t, o));
+    m_w = __fdividef(t, n_w);
+    const f2 nm = f2_bcast(-m_w);
+    f2 s2 = f2_bcast(0.f), s3 = f2_bcast(0.f), s4 = f2_bcast(0.f);
+#pragma unroll
+    for (int m = 0; m < M; ++m)
+#pragma unroll
+      for (int i = 0; i < NP; ++i) {
+        f2 xc = f2_add(xv[m][i], nm);
+        if (MASK)
+          xc = f2_select(xc, 2 * i >= lo[m] && 2 * i < hi[m], 2 * i + 1 >= lo[m] && 2 * i + 1 < hi[m],
+                         0.f);
+        const f2 tt = f2_mul(dv[m][i], gam[m][i]);
+        s2 = f2_fma(xc, xc, s2);
+        s3 = f2_add(s3, tt);
+        s4 = f2_fma(tt, xc, s4);
+      }
+    float v[4] = {f2_total(s2), f2_total(s3), f2_total(s4), 0.f};
+    return warp_reduce_scatter<4>(v, lane);
   } else {
-    v[0] = f2_total(s2);
-    v[1] = f2_total(s4);
+    f2 s2 = f2_bcast(0.f), s4 = f2_bcast(0.f);
+#pragma unroll
+    for (int m = 0; m < M; ++m)
+#pragma unroll
+      for (int i = 0; i < NP; ++i) {
+        const f2 tt = f2_mul(dv[m][i], gam[m][i]);
+        s2 = f2_fma(xv[m][i], xv[m][i], s2);
+        s4 = f2_fma(tt, xv[m][i], s4);
+      }
+    float v[2] = {f2_total(s2), f2_total(s4)};
+    m_w = 0.f;
+    return warp_reduce_scatter<2>(v, lane);
   }
+}
+
+// The number of a row's elements in warp w's chunks [64 w, 64 w + 64) of
+// the stats kernel's stripe at column `from`: columns [from + 64 E w - c,
+// + 64 E) within [from, rl), rl = min(stripe end, row length).
+template <int E>
+__device__ __forceinline__ int stat_warp_count(int from, int rl, int c, int w) {
+  const int cs = from + 64 * E * w - c;
+  return max(0, min(rl, cs + 64 * E) - max(from, cs));
 }
 
 // Bytes of a lane's chunk that starting at column dc lie before the end of a
@@ -284,15 +327,16 @@ __device__ __forceinline__ uint32_t stripe_bytes(int dc, int len) {
 }
 
 // ---------------------------------------------------------------------------
-// Row sums per stripe.  Warp w owns the stripe's window chunks
+// Row statistics per stripe.  Warp w owns the stripe's window chunks
 // [64 w, 64 w + 64), lane l chunks 64 w + l and 64 w + l + 32.  The lanes
 // walk the CTA's sorted rows with their chunks of x and dy of the next
 // kStatDepth - 1 rows in flight (cp.async into the lane's own slots of a
-// shared-memory ring); per row the warp's four (LayerNorm) or two (RMSNorm)
-// sums are reduced by recursive halving into shared memory, and the warps
-// are added in warp order at the end.  A row whose chunks in the warp are
-// all whole and inside the stripe takes a path without masks; a warp with
-// no element of the row skips it (its sums stay zero).
+// shared-memory ring).  Per row each warp forms its statistics about its
+// own mean (LayerNorm: count, mean, M2, sum t, sum t (x - mean); RMSNorm:
+// sum x^2, sum t x) into shared memory; at the end they are merged (added)
+// in warp order, one RowStat (two sums) per row and stripe.  A row whose
+// chunks in the warp are all whole and inside the stripe takes a path
+// without masks; a warp with no element of the row skips it (count zero).
 // ---------------------------------------------------------------------------
 constexpr int kStatDepth = 4;
 constexpr size_t kStatRingBytes = static_cast<size_t>(kStatDepth) * kStatChunks * 2 * kStatThreads * 16;
@@ -310,10 +354,11 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
   constexpr int D = kStatDepth;
   constexpr int W = E * (NT * M - 1);
   constexpr bool kLN = OP == kLayerNorm;
-  constexpr int NV = kLN ? 4 : 2;  // sums of a row
   __shared__ StripeRows<kStatRows> L;
-  __shared__ float kfirst[kStatRows];
-  __shared__ float4 wsum[kStatRows][NW];
+  // per row and warp: {mean, M2, St, Stx} (LayerNorm; the warp's count
+  // follows from the row's length and head class), {-, sum x^2, -, sum t x}
+  // (RMSNorm)
+  __shared__ float4 wsa[kStatRows][NW];
   extern __shared__ __align__(16) unsigned char ring[];
   // the dx kernel may be scheduled once every CTA of this one has started;
   // it waits for this grid's completion before it reads what this one writes
@@ -338,13 +383,11 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
   int q[M];
 #pragma unroll
   for (int m = 0; m < M; ++m) q[m] = 64 * w + lane + 32 * m;
-  for (int i = tid; i < kStatRows * NW; i += NT) (&wsum[0][0])[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int i = tid; i < kStatRows * NW; i += NT) (&wsa[0][0])[i] = make_float4(0.f, 0.f, 0.f, 0.f);
 
-  const bool bad = stripe_sort<T, NT>(L, p.offsets, r0, n, from, p.max_len, p.hb,
-                                      kLN ? x : nullptr, kfirst);
+  const bool bad = stripe_sort<T, NT>(L, p.offsets, r0, n, from, p.max_len, p.hb);
   if (s == 0) {  // uniform over the CTA
     if (__syncthreads_or(bad) && tid == 0) atomicOr(p.status, kStatusBadOffsets);
-    if (kLN && tid < L.seg[E]) p.shift[L.row[tid]] = kfirst[tid];
   }
   const int cnt = L.seg[E];
   // list entry j's chunks into the ring (a group per entry, empty or not)
@@ -385,7 +428,6 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
       stripe_gamma<T, M>(gam, gamma, from, lim, dc);
     }
     const int rl = min(lim, L.len[j]);
-    const float k = kLN ? kfirst[j] : 0.f;
     int hi[M];
     bool full = true, any = false;
 #pragma unroll
@@ -395,52 +437,67 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
       any = any || hi[m] > lo[m];
     }
     cp_async_wait<D - 1>();  // entry j's copies have landed
-    float v[NV];
-    uint4 xr[M], dr[M];
+    f2 xv[M][NP], dv[M][NP];
+    const float n_w = static_cast<float>(stat_warp_count<E>(from, rl, c, w));
+    float t, m_w;
     if (__all_sync(kFullMask, full)) {
 #pragma unroll
       for (int m = 0; m < M; ++m) {
-        xr[m] = lds128(slot(j, m, 0));
-        dr[m] = lds128(slot(j, m, 1));
+        chunk_to_pairs<T>(lds128(slot(j, m, 0)), xv[m]);
+        chunk_to_pairs<T>(lds128(slot(j, m, 1)), dv[m]);
       }
-      stat_sums<T, kLN, M, false>(xr, dr, lo, hi, k, gam, v);
+      t = warp_row_stats<T, kLN, M, false>(xv, dv, lo, hi, gam, lane, n_w, m_w);
     } else if (__any_sync(kFullMask, any)) {
+      // elements outside a chunk's valid range read as 0
 #pragma unroll
       for (int m = 0; m < M; ++m) {
-        xr[m] = dr[m] = make_uint4(0u, 0u, 0u, 0u);
-        if (lo[m] < hi[m]) {
-          xr[m] = lds128(slot(j, m, 0));
-          dr[m] = lds128(slot(j, m, 1));
-        }
+        const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+        stripe_pairs<T>(lo[m] < hi[m] ? lds128(slot(j, m, 0)) : z, lo[m], hi[m], 0.f, xv[m]);
+        stripe_pairs<T>(lo[m] < hi[m] ? lds128(slot(j, m, 1)) : z, lo[m], hi[m], 0.f, dv[m]);
       }
-      stat_sums<T, kLN, M, true>(xr, dr, lo, hi, k, gam, v);
+      t = warp_row_stats<T, kLN, M, true>(xv, dv, lo, hi, gam, lane, n_w, m_w);
     } else {
       continue;  // no element of the row in this warp's chunks
     }
-    const float t = warp_reduce_scatter<NV>(v, lane);
-    constexpr int kStride = 32 / NV;
-    if ((lane & (kStride - 1)) == 0) {
-      const int i = lane / kStride;                   // value index
-      const int comp = kLN ? i : 1 + 2 * i;           // RMSNorm: .y, .w
-      reinterpret_cast<float *>(&wsum[j][w])[comp] = t;
+    if constexpr (kLN) {
+      if (lane == 0) {
+        wsa[j][w].x = m_w;
+        wsa[j][w].y = t;
+      }
+      if (lane == 8) wsa[j][w].z = t;
+      if (lane == 16) wsa[j][w].w = t;
+    } else {
+      if (lane == 0) wsa[j][w].y = t;
+      if (lane == 16) wsa[j][w].w = t;
     }
   }
   cp_async_wait<0>();
   __syncthreads();
   for (int j = tid; j < cnt; j += NT) {
-    float4 t = wsum[j][0];
+    float4 out;
+    if constexpr (kLN) {
+      // warp qq's elements: columns [from + 64 E qq - c, + 64 E) of the row
+      // within [from, min(lim, len))
+      const int c = L.cls[j];
+      const int rl = min(lim, L.len[j]);
+      RowStat a = {0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-    for (int qq = 1; qq < NW; ++qq) {
-      const float4 u = wsum[j][qq];
-      t.y = __fadd_rn(t.y, u.y);
-      t.w = __fadd_rn(t.w, u.w);
-      if constexpr (kLN) {
-        t.x = __fadd_rn(t.x, u.x);
-        t.z = __fadd_rn(t.z, u.z);
+      for (int qq = 0; qq < NW; ++qq) {
+        const float4 u = wsa[j][qq];
+        stat_merge(a, RowStat{static_cast<float>(stat_warp_count<E>(from, rl, c, qq)), u.x, u.y,
+                              u.z, u.w});
       }
+      out = make_float4(a.m, a.M2, a.St, a.Stx);
+    } else {
+      float s2 = wsa[j][0].y, s4 = wsa[j][0].w;
+#pragma unroll
+      for (int qq = 1; qq < NW; ++qq) {
+        s2 = __fadd_rn(s2, wsa[j][qq].y);
+        s4 = __fadd_rn(s4, wsa[j][qq].w);
+      }
+      out = make_float4(0.f, s2, 0.f, s4);
     }
-    if constexpr (!kLN) t.x = t.z = 0.f;
-    p.psum[static_cast<int64_t>(L.row[j]) * p.ns1 + s] = t;
+    p.psum[static_cast<int64_t>(L.row[j]) * p.ns1 + s] = out;
   }
 }
 
@@ -448,17 +505,19 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
 // word of padding every 32, so that lanes E columns apart hit distinct banks.
 __device__ __forceinline__ int stripe_pad(int local) { return local + (local >> 5); }
 
-// dx of one chunk from its pairs and the row's coefficients {rstd,
-// -mean rstd, -mean(t) rstd, -mean(t xhat) rstd} (t = dy gamma), adding
-// dy xhat (and dy) to the lane's column sums when wanted.
+// dx of one chunk from its pairs and the row's coefficients {rstd, -mean,
+// -mean(t) rstd, -mean(t xhat) rstd} (t = dy gamma), adding dy xhat (and
+// dy) to the lane's column sums when wanted.  xhat = (x - mean) rstd: x -
+// mean is exact near the mean, where x rstd - mean rstd would carry the
+// rounding of mean rstd.
 template <bool kLN, int NP>
 __device__ __forceinline__ void stripe_dx(const f2 (&xv)[NP], const f2 (&dv)[NP],
                                           const f2 (&gam)[NP], const float4 &cf, bool want,
                                           f2 (&o)[NP], f2 (&accg)[NP], f2 (&accb)[NP]) {
-  const f2 C0 = f2_bcast(cf.x), C1 = f2_bcast(cf.y), NA = f2_bcast(cf.z), NB = f2_bcast(cf.w);
+  const f2 C0 = f2_bcast(cf.x), NMU = f2_bcast(cf.y), NA = f2_bcast(cf.z), NB = f2_bcast(cf.w);
 #pragma unroll
   for (int i = 0; i < NP; ++i) {
-    const f2 xh = f2_fma(xv[i], C0, C1);
+    const f2 xh = kLN ? f2_mul(f2_add(xv[i], NMU), C0) : f2_mul(xv[i], C0);
     const f2 t = f2_mul(dv[i], gam[i]);
     o[i] = f2_fma(t, C0, f2_fma(xh, NB, NA));
     if (want) {
@@ -543,8 +602,7 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
   bool waited = false;
   for (int64_t r0 = gr0; r0 < gr1; r0 += kDxBatch) {
     const int n = static_cast<int>(min(static_cast<int64_t>(kDxBatch), gr1 - r0));
-    (void)stripe_sort<T, NT>(L, p.offsets, r0, n, from, p.max_len, p.hb,
-                             static_cast<const T *>(nullptr), nullptr);
+    (void)stripe_sort<T, NT>(L, p.offsets, r0, n, from, p.max_len, p.hb);
     if (!waited) {
       // launched as a programmatic dependent of the stats kernel: its sums
       // are read, and dx (which may be x or dy) written, only past this
@@ -571,33 +629,36 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
 #pragma unroll
     for (int j = 0; j < D - 1; ++j) issue(j);
     if (tid < cnt) {
+      // the row's statistics: its stripes' in stripe order (stripe q holds
+      // min(W1, len - q W1) of the row's elements)
       const int64_t r = L.row[tid];
       const int len = L.len[tid];
       const int nst = (len + W1 - 1) / W1;
       const float4 *ps = p.psum + r * p.ns1;
-      float4 t = ps[0];
-#pragma unroll 4
-      for (int qq = 1; qq < nst; ++qq) {
-        const float4 u = ps[qq];
-        t.x = __fadd_rn(t.x, u.x);
-        t.y = __fadd_rn(t.y, u.y);
-        t.z = __fadd_rn(t.z, u.z);
-        t.w = __fadd_rn(t.w, u.w);
-      }
       const float inv_n = __frcp_rn(static_cast<float>(len));
       float4 cf;
       if constexpr (kLN) {
-        const float m1 = __fmul_rn(t.x, inv_n);  // mean - k
-        const float var = fmaxf(__fsub_rn(__fmul_rn(t.y, inv_n), __fmul_rn(m1, m1)), 0.f);
-        const float c0 = rsqrtf(__fadd_rn(var, p.eps));        // rstd
-        const float mu = __fadd_rn(p.shift[r], m1);            // mean
-        const float a = __fmul_rn(t.z, inv_n);                 // mean(t)
-        const float b = __fmul_rn(c0, __fsub_rn(__fmul_rn(t.w, inv_n), __fmul_rn(m1, a)));
-        cf = make_float4(c0, -__fmul_rn(mu, c0), -__fmul_rn(a, c0), -__fmul_rn(b, c0));
+        RowStat a = {0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
+        for (int qq = 0; qq < nst; ++qq) {
+          const float4 u = ps[qq];
+          stat_merge(a, RowStat{static_cast<float>(min(W1, len - qq * W1)), u.x, u.y, u.z, u.w});
+        }
+        const float c0 = rsqrtf(__fadd_rn(__fmul_rn(a.M2, inv_n), p.eps));  // rstd
+        const float am = __fmul_rn(a.St, inv_n);                           // mean(t)
+        const float bm = __fmul_rn(__fmul_rn(a.Stx, c0), inv_n);           // mean(t xhat)
+        cf = make_float4(c0, -a.m, -__fmul_rn(am, c0), -__fmul_rn(bm, c0));
       } else {
-        const float c0 = rsqrtf(__fmaf_rn(t.y, inv_n, p.eps));  // rstd
-        const float b = __fmul_rn(__fmul_rn(t.w, c0), inv_n);   // mean(t xhat)
-        cf = make_float4(c0, 0.f, 0.f, -__fmul_rn(b, c0));
+        float s2 = 0.f, s4 = 0.f;
+#pragma unroll 4
+        for (int qq = 0; qq < nst; ++qq) {
+          const float4 u = ps[qq];
+          s2 = __fadd_rn(s2, u.y);
+          s4 = __fadd_rn(s4, u.w);
+        }
+        const float c0 = rsqrtf(__fmaf_rn(s2, inv_n, p.eps));   // rstd
+        const float bm = __fmul_rn(__fmul_rn(s4, c0), inv_n);   // mean(t xhat)
+        cf = make_float4(c0, 0.f, 0.f, -__fmul_rn(bm, c0));
       }
       coef[tid] = cf;
     }

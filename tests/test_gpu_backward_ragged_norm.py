@@ -398,3 +398,47 @@ def test_ragged_norm_backward_stripe_congruent(rw, monkeypatch, op):
                f"congruent {op} shift {shift}")
         assert is_canary(dxb[:G]).all() and is_canary(dxb[G + int(off[-1]):]).all()
 
+
+@pytest.mark.parametrize("design", ["team", "stripe"])
+def test_ragged_layernorm_backward_far_from_zero(rw, monkeypatch, design):
+    """fp32 ragged LayerNorm backward of rows whose mean is 100 times their
+    spread, in both designs: the stripe design's variance about each row's
+    first element and its xhat = (x - mean) rstd keep the full tolerance."""
+    monkeypatch.setenv("ROWOP_BWD_STRIPE", "0" if design == "team" else "2")
+    dtype = torch.float32
+    lens = np.array([1, 2, 9, 700, 3000, 5000, 8191, 4096, 17], dtype=np.int64)
+    max_len = int(lens.max())
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    g = torch.Generator("cpu").manual_seed(31)
+    x = (50.0 + 0.5 * torch.randn(int(off[-1]), generator=g, dtype=torch.float64)).float()
+    dy = torch.randn(int(off[-1]), generator=g)
+    gam = 1.0 + 0.2 * torch.randn(max_len, generator=g)
+    st, dxb, dgb, dbb = call(rw, "layernorm", dtype, x, dy, gam, off, max_len)
+    assert st == 0 and rw.check_status() == 0
+    dx_rows, params, ps = reference("layernorm", x, dy, gam, off, max_len)
+    verify("layernorm", dtype, dx_rows, params, ps, off, dxb, dgb, dbb, max_len,
+           f"far from zero {design}")
+
+
+@pytest.mark.parametrize("design", ["team", "stripe"])
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16], ids=["f32", "bf16"])
+def test_ragged_layernorm_backward_outliers(rw, monkeypatch, design, dtype):
+    """Rows whose first element (or one in the middle) is an outlier 10^4
+    times the spread of the rest, in both designs: statistics formed about a
+    shift far from the mean would lose the variance to cancellation."""
+    monkeypatch.setenv("ROWOP_BWD_STRIPE", "0" if design == "team" else "2")
+    lens = np.array([5000, 3, 4096, 9000, 700, 12000], dtype=np.int64)
+    max_len = int(lens.max())
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    g = torch.Generator("cpu").manual_seed(32)
+    x = torch.randn(int(off[-1]), generator=g, dtype=torch.float64)
+    for i, pos in enumerate((0, 0, 0, 4500, 0, 11000)):
+        x[int(off[i]) + pos] = 1.0e4 if i % 2 == 0 else -3.0e3
+    x, dy = x.to(dtype), torch.randn(int(off[-1]), generator=g).to(dtype)
+    gam = (1.0 + 0.2 * torch.randn(max_len, generator=g)).to(dtype)
+    st, dxb, dgb, dbb = call(rw, "layernorm", dtype, x, dy, gam, off, max_len)
+    assert st == 0 and rw.check_status() == 0
+    dx_rows, params, ps = reference("layernorm", x, dy, gam, off, max_len)
+    verify("layernorm", dtype, dx_rows, params, ps, off, dxb, dgb, dbb, max_len,
+           f"outliers {design} {dtype}")
+
