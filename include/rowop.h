@@ -219,11 +219,12 @@ ROWOP_API int rowop_logsoftmax_backward_ragged(const void *y, const void *dy, vo
  * Two designs, chosen per call (each with its own summation order):
  *   * x, dy and dx at the same offset past a 16-byte boundary and
  *     max_len >= 2048: column stripes.  A first kernel writes each row's
- *     sums over each stripe of 4088 (bf16 / fp16) or 2044 (fp32) columns.
+ *     statistics over each stripe of 512 16-byte chunks (4096 bf16 / fp16
+ *     or 2048 fp32 elements, counted from the 16-byte boundary at or
+ *     before the row's first element).
  *     A second adds them into the row statistics, writes dx and sums
  *     dgamma / dbeta into one float32 partial row per group of rows; a
  *     finalize adds the groups in index order.  x and dy are read twice.
- *     LayerNorm's variance is taken about each row's first element.
  *   * otherwise: the forward's classify plan, one launch per row bucket,
  *     and one float32 partial row per CTA for each bucket, added in index
  *     order, the buckets in order (SMALL, MEDIUM, LARGE).

@@ -62,10 +62,9 @@ inline size_t bwd_ragged_layout(int64_t rows, int64_t max_len, int esize, int na
   return off;
 }
 
-// The striped ragged norm backward (bwd_stripe.cuh): column stripes of
-// each kernel, in elements of esize bytes.  A stripe is one 16-byte window
-// chunk narrower than the chunk slots of the kernel's CTA, so the stripe of
-// a row that starts mid-chunk still fits.
+// The striped ragged norm backward (bwd_stripe.cuh): each kernel's stripe
+// is a range of 16-byte window chunks (one per chunk slot of its CTA), so a
+// stripe's columns move with the row's head offset.
 constexpr int kStatThreads = 256;  // threads of a stats CTA
 constexpr int kStatChunks = 2;     // window chunks a stats lane holds per row
 constexpr int kStatRows = 64;      // rows of a stats CTA
@@ -78,15 +77,15 @@ constexpr int kDxMinGroupRows = 32;
 constexpr int64_t kStripeMinCols = 2048;
 
 inline int64_t stripe_stat_width(int esize) {
-  return static_cast<int64_t>(16 / esize) * (kStatThreads * kStatChunks - 1);
+  return static_cast<int64_t>(16 / esize) * kStatThreads * kStatChunks;
 }
-inline int64_t stripe_dx_width(int esize) {
-  return static_cast<int64_t>(16 / esize) * (kDxThreads - 1);
-}
+inline int64_t stripe_dx_width(int esize) { return static_cast<int64_t>(16 / esize) * kDxThreads; }
 
 // Workspace of the striped design, both parts 256-byte aligned: the
 // per-stripe row statistics [rows][ns1] float4, and the dgamma / dbeta
-// partial rows [ng2][nacc][max_len] float32.
+// partial rows [ng2][ns2][nacc][W2 + E] float32 (a dx stripe's columns
+// under every head offset).  ns = stripes covering window positions up to
+// max_len + E - 1.
 struct StripeLayout {
   int64_t ns1, ng1, ns2, ng2, g2;  // stripes and row groups of the two kernels
   size_t psum, part, total;
@@ -95,8 +94,9 @@ struct StripeLayout {
 inline StripeLayout stripe_layout(int64_t rows, int64_t max_len, int esize, int nacc) {
   StripeLayout L = {};
   const auto up = [](size_t v) { return (v + 255) & ~static_cast<size_t>(255); };
-  L.ns1 = max_len > 0 ? (max_len + stripe_stat_width(esize) - 1) / stripe_stat_width(esize) : 0;
-  L.ns2 = max_len > 0 ? (max_len + stripe_dx_width(esize) - 1) / stripe_dx_width(esize) : 0;
+  const int64_t span = max_len > 0 ? max_len + 16 / esize - 1 : 0;
+  L.ns1 = (span + stripe_stat_width(esize) - 1) / stripe_stat_width(esize);
+  L.ns2 = (span + stripe_dx_width(esize) - 1) / stripe_dx_width(esize);
   L.ng1 = (rows + kStatRows - 1) / kStatRows;
   L.ng2 = std::max<int64_t>(
       1, std::min<int64_t>((rows + kDxMinGroupRows - 1) / kDxMinGroupRows, kDxMaxGroups));
@@ -104,8 +104,9 @@ inline StripeLayout stripe_layout(int64_t rows, int64_t max_len, int esize, int 
   const size_t r = static_cast<size_t>(std::max<int64_t>(rows, 0));
   L.psum = 0;
   L.part = L.psum + up(r * static_cast<size_t>(L.ns1) * 16u);
-  L.total = L.part + up(static_cast<size_t>(L.ng2) * static_cast<size_t>(nacc) *
-                        static_cast<size_t>(max_len) * sizeof(float));
+  L.total = L.part + up(static_cast<size_t>(L.ng2) * static_cast<size_t>(L.ns2) *
+                        static_cast<size_t>(nacc) *
+                        static_cast<size_t>(stripe_dx_width(esize) + 16 / esize) * sizeof(float));
   return L;
 }
 

@@ -316,6 +316,7 @@ bool try_bwd_stripe(const BwdRaggedCall &c, const DeviceInfo &d, int mode, cudaE
   p.part = want_params ? reinterpret_cast<float *>(ws + L.part) : nullptr;
   p.ns1 = L.ns1;
   p.ng1 = L.ng1;
+  p.ns2 = L.ns2;
   p.ng2 = L.ng2;
   p.g2 = L.g2;
   p.status = d.status;
@@ -357,8 +358,8 @@ bool try_bwd_stripe(const BwdRaggedCall &c, const DeviceInfo &d, int mode, cudaE
     cfg.blockDim = dim3(kStripeFinThreads, 1, 1);
     cfg.stream = c.stream;
     e = cudaLaunchKernelEx(&cfg, bwd_stripe_finalize_kernel<T>, static_cast<const float *>(p.part),
-                           L.ng2, c.max_len, nacc, static_cast<T *>(c.dgamma),
-                           static_cast<T *>(c.dbeta));
+                           L.ng2, L.ns2, static_cast<int>(stripe_dx_width(SZ)), 16 / SZ,
+                           c.max_len, nacc, static_cast<T *>(c.dgamma), static_cast<T *>(c.dbeta));
     if (e == cudaSuccess) e = cudaGetLastError();
   }
   *err = e;

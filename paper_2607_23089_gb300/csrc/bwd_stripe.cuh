@@ -4,12 +4,14 @@
 //
 // Two kernels, then bwd_stripe_finalize_kernel:
 //   * bwd_stripe_stats_kernel: CTA (s, g) takes rows [64 g, 64 g + 64) and
-//     their columns [s W1, (s+1) W1).  For each row it writes the statistics
+//     their window chunks [512 s, 512 s + 512).  For each row it writes the
+//     statistics
 //     of those columns (LayerNorm: mean, sum of squares about it, sum t and
 //     sum t (x - mean), with t = dy gamma; RMSNorm: sum x^2 and sum t x): one
 //     float4 per row and stripe;
 //   * bwd_stripe_dx_kernel: CTA (s, g) takes the rows of group g and their
-//     columns [s W2, (s+1) W2).  It merges each row's stripe statistics in
+//     window chunks [256 s, 256 s + 256).  It merges each row's stripe
+//     statistics in
 //     stripe order into the row's, writes dx over its columns, and sums
 //     dy xhat (and dy) over its rows into group g's partial row;
 //   * the finalize adds the groups' partial rows in index order.
@@ -18,17 +20,18 @@
 // length keep many loads in flight on every SM, and a lane's dgamma / dbeta
 // sums sit in registers at fixed columns.
 //
-// Alignment.  Lane t of a CTA owns window chunks t, t + NT, ... of the
-// stripe.  Window chunks are the 16-byte chunks counted from the boundary
-// at or before the row's first element, so every whole-chunk load and store
-// is aligned.  A row that starts h elements past a boundary (head class h)
-// puts its column j at window position j + h.  Each CTA sorts its rows by
-// head class (stably, by row index).  Per class it loads gamma at its
-// lanes' columns once; the dx kernel also adds its lanes' sums into the
-// CTA's partial row in shared memory when the class ends.  A chunk that
-// crosses a row's end is read and written element by element.  A chunk
-// that crosses a stripe edge is read whole when it lies inside the row and
-// written element by element.
+// Alignment.  Window chunks are the 16-byte chunks counted from the
+// boundary at or before the row's first element, so every whole-chunk load
+// and store is aligned; a row that starts h elements past a boundary (head
+// class h) puts its column j at window position j + h.  Stripes are ranges
+// of window chunks, so no chunk crosses a stripe edge and a stripe's columns
+// move with the head class.  Lane t of a CTA owns window chunks t, t + NT,
+// ... of its stripe.  Each CTA sorts its rows by head class (stably, by row
+// index).  Per class it loads gamma at its lanes' columns once; the dx
+// kernel also adds its lanes' sums into the CTA's partial row (its stripe's
+// columns under every head class: E columns of halo before the stripe) in
+// shared memory when the class ends.  Only a row's first and last chunks can
+// be partial: those are read and written element by element.
 //
 // LayerNorm's statistics are formed about local means: each warp takes the
 // mean of its elements of a row, then the sums about that mean from the same
@@ -55,7 +58,7 @@ struct StripeParams {
   int hb;        // element offset of x (dy, dx) past a 16-byte boundary
   float4 *psum;  // [rows][ns1] the stats kernel's row statistics per stripe
   float *part;   // [ng2][nacc][max_len] dgamma (dbeta) partial rows; NULL = not wanted
-  int64_t ns1, ng1, ng2, g2;
+  int64_t ns1, ng1, ns2, ng2, g2;
   unsigned int *status;
 };
 
@@ -71,9 +74,10 @@ struct StripeRows {
   int wcnt[9][kDxThreads / 32];
 };
 
-// Rows [r0, r0 + n), one a thread (n <= NT): those that reach column `from`
-// (valid, 0 <= length <= max_len, and longer than `from`) are listed in L by
-// head class, then by row.  Returns whether the thread's row is invalid.
+// Rows [r0, r0 + n), one a thread (n <= NT): those that reach window
+// position `from` (valid, 0 < length <= max_len, and head class + length >
+// from) are listed in L by head class, then by row.  Returns whether the
+// thread's row is invalid.
 template <typename T, int NT, int N>
 __device__ __forceinline__ bool stripe_sort(StripeRows<N> &L, const int64_t *offsets, int64_t r0,
                                             int n, int64_t from, int64_t max_len, int hb) {
@@ -93,7 +97,8 @@ __device__ __forceinline__ bool stripe_sort(StripeRows<N> &L, const int64_t *off
     bad = l < 0 || l > max_len;
     if (!bad) {
       len = static_cast<int>(l);
-      if (l > from) key = static_cast<int>((o + hb) & (E - 1));
+      const int c = static_cast<int>((o + hb) & (E - 1));
+      if (l > 0 && l + c > from) key = c;
     }
   }
   unsigned mine = 0;
@@ -183,7 +188,7 @@ __device__ __forceinline__ uint4 lds128(uint32_t addr) {
 }
 
 // gamma at the columns of a lane's M window chunks for head class h: the
-// lane's chunk m starts at column dc[m] (window chunk q: from + E q - h);
+// lane's chunk m starts at column dc[m] (window position p: p - h);
 // columns outside [from, lim) read as 1 (their data is masked out).
 template <typename T, int M>
 __device__ __forceinline__ void stripe_gamma(f2 (&gam)[M][Elem<T>::kPerChunk / 2], const T *gamma,
@@ -311,12 +316,12 @@ __device__ __forceinline__ float warp_row_stats(const f2 (&xv)[M][Elem<T>::kPerC
 }
 
 // The number of a row's elements in warp w's chunks [64 w, 64 w + 64) of
-// the stats kernel's stripe at column `from`: columns [from + 64 E w - c,
-// + 64 E) within [from, rl), rl = min(stripe end, row length).
+// the stats kernel's stripe at window position `from`: columns
+// [from + 64 E w - c, + 64 E) within [0, len).
 template <int E>
-__device__ __forceinline__ int stat_warp_count(int from, int rl, int c, int w) {
+__device__ __forceinline__ int stat_warp_count(int from, int len, int c, int w) {
   const int cs = from + 64 * E * w - c;
-  return max(0, min(rl, cs + 64 * E) - max(from, cs));
+  return max(0, min(len, cs + 64 * E) - max(0, cs));
 }
 
 // Bytes of a lane's chunk that starting at column dc lie before the end of a
@@ -352,7 +357,7 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
   constexpr int NT = kStatThreads;
   constexpr int NW = NT / 32;
   constexpr int D = kStatDepth;
-  constexpr int W = E * (NT * M - 1);
+  constexpr int W = E * NT * M;  // window positions of a stripe
   constexpr bool kLN = OP == kLayerNorm;
   __shared__ StripeRows<kStatRows> L;
   // per row and warp: {mean, M2, St, Stx} (LayerNorm; the warp's count
@@ -370,8 +375,8 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
   const int64_t g = static_cast<int64_t>(blockIdx.x) % p.ng1;
   const int64_t r0 = g * kStatRows;
   const int n = static_cast<int>(min(static_cast<int64_t>(kStatRows), p.rows - r0));
-  const int from = static_cast<int>(s) * W;
-  const int lim = static_cast<int>(min(static_cast<int64_t>(from) + W, p.max_len));
+  const int from = static_cast<int>(s) * W;  // the stripe's first window position
+  const int cols = static_cast<int>(p.max_len);
   const T *x = static_cast<const T *>(p.x);
   const T *dy = static_cast<const T *>(p.dy);
   const T *gamma = static_cast<const T *>(p.gamma);
@@ -396,12 +401,11 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
       const int c = L.cls[j];
       const int len = L.len[j];
       const int64_t o = L.off[j];
-      const int rl = min(lim, len);
 #pragma unroll
       for (int m = 0; m < M; ++m) {
         const int dc = from + E * q[m] - c;
-        const int lo = q[m] == 0 ? c : 0;
-        if (lo < min(E, rl - dc)) {
+        const int lo = max(0, -dc);
+        if (lo < min(E, len - dc)) {
           const uint32_t nb = stripe_bytes<SZ>(dc, len);
           cp_async16(slot(j, m, 0), x + o + dc, nb);
           cp_async16(slot(j, m, 1), dy + o + dc, nb);
@@ -423,11 +427,11 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
 #pragma unroll
       for (int m = 0; m < M; ++m) {
         dc[m] = from + E * q[m] - c;
-        lo[m] = q[m] == 0 ? c : 0;
+        lo[m] = max(0, -dc[m]);
       }
-      stripe_gamma<T, M>(gam, gamma, from, lim, dc);
+      stripe_gamma<T, M>(gam, gamma, 0, cols, dc);
     }
-    const int rl = min(lim, L.len[j]);
+    const int rl = L.len[j];
     int hi[M];
     bool full = true, any = false;
 #pragma unroll
@@ -477,9 +481,9 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
     float4 out;
     if constexpr (kLN) {
       // warp qq's elements: columns [from + 64 E qq - c, + 64 E) of the row
-      // within [from, min(lim, len))
+      // within [0, len)
       const int c = L.cls[j];
-      const int rl = min(lim, L.len[j]);
+      const int rl = L.len[j];
       RowStat a = {0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int qq = 0; qq < NW; ++qq) {
@@ -535,10 +539,11 @@ __device__ __forceinline__ void stripe_dx(const f2 (&xv)[NP], const f2 (&dv)[NP]
 // kDxDepth - 1 rows in flight (cp.async into the lane's own ring slots): the
 // lane writes its dx chunk and adds dy xhat (and dy) to its register sums.
 // When the head class changes the lane adds those sums into the CTA's
-// partial row in shared memory at their columns.  A row whose chunks in the
-// warp are all whole and inside the stripe takes a path without masks; a
-// warp with no element of the row skips it.  The CTA writes its partial row
-// (its stripe of group g's row) at the end.
+// partial row in shared memory at their columns: the stripe's columns under
+// every head class, [from - E, from + W2) for the stripe at window position
+// `from`.  A row whose chunks in the warp are all whole takes a path without
+// masks; a warp with no element of the row skips it.  The CTA writes its
+// partial row to part[g][s] at the end.
 // ---------------------------------------------------------------------------
 constexpr int kDxDepth = 5;
 constexpr size_t kDxRingBytes = static_cast<size_t>(kDxDepth) * 2 * kDxThreads * 16;
@@ -551,11 +556,12 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
   constexpr int NP = E / 2;
   constexpr int NT = kDxThreads;
   constexpr int D = kDxDepth;
-  constexpr int W = E * (NT - 1);
-  constexpr int W1 = E * (kStatThreads * kStatChunks - 1);
+  constexpr int W = E * NT;                             // window positions of a stripe
+  constexpr int W1 = E * kStatThreads * kStatChunks;    // ... of a stats stripe
   constexpr bool kLN = OP == kLayerNorm;
   constexpr int NA = kLN ? 2 : 1;
-  constexpr int kPadW = W + W / 32 + 1;
+  constexpr int kSeg = W + E;  // the partial row: E columns of halo, then the stripe's W
+  constexpr int kPadW = kSeg + kSeg / 32 + 1;
   __shared__ StripeRows<kDxBatch> L;
   __shared__ float4 coef[kDxBatch];
   __shared__ float spart[NA][kPadW];
@@ -563,8 +569,8 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
   const int tid = threadIdx.x;
   const int64_t s = static_cast<int64_t>(blockIdx.x) / p.ng2;  // heavy stripes first
   const int64_t g = static_cast<int64_t>(blockIdx.x) % p.ng2;
-  const int from = static_cast<int>(s) * W;
-  const int lim = static_cast<int>(min(static_cast<int64_t>(from) + W, p.max_len));
+  const int from = static_cast<int>(s) * W;  // the stripe's first window position
+  const int cols = static_cast<int>(p.max_len);
   const T *x = static_cast<const T *>(p.x);
   const T *dy = static_cast<const T *>(p.dy);
   T *dx = static_cast<T *>(p.dx);
@@ -580,17 +586,15 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
   f2 accg[NP], accb[NP];
 #pragma unroll
   for (int i = 0; i < NP; ++i) accg[i] = accb[i] = f2_bcast(0.f);
-  // the class's sums into the partial row at their columns (class c)
+  // the class's sums into the partial row at their columns (class c):
+  // entry E t + e - c + E is column from - E + E t + e - c
   const auto flush = [&](int c) {
     if (want) {
 #pragma unroll
       for (int e = 0; e < E; ++e) {
-        const int local = E * tid + e - c;
-        if (local >= 0 && local < W) {
-          const int qq = stripe_pad(local);
-          spart[0][qq] = __fadd_rn(spart[0][qq], pair_elem(accg, e));
-          if constexpr (kLN) spart[NA - 1][qq] = __fadd_rn(spart[NA - 1][qq], pair_elem(accb, e));
-        }
+        const int qq = stripe_pad(E * tid + e - c + E);
+        spart[0][qq] = __fadd_rn(spart[0][qq], pair_elem(accg, e));
+        if constexpr (kLN) spart[NA - 1][qq] = __fadd_rn(spart[NA - 1][qq], pair_elem(accb, e));
       }
 #pragma unroll
       for (int i = 0; i < NP; ++i) accg[i] = accb[i] = f2_bcast(0.f);
@@ -616,8 +620,8 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
         const int c = L.cls[j];
         const int len = L.len[j];
         const int dc = from + E * tid - c;
-        const int lo = tid == 0 ? c : 0;
-        if (lo < min(E, min(lim, len) - dc)) {
+        const int lo = max(0, -dc);
+        if (lo < min(E, len - dc)) {
           const int64_t o = L.off[j];
           const uint32_t nb = stripe_bytes<SZ>(dc, len);
           cp_async16(slot(j, 0), x + o + dc, nb);
@@ -629,11 +633,12 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
 #pragma unroll
     for (int j = 0; j < D - 1; ++j) issue(j);
     if (tid < cnt) {
-      // the row's statistics: its stripes' in stripe order (stripe q holds
-      // min(W1, len - q W1) of the row's elements)
+      // the row's statistics: its stripes' in stripe order (stats stripe q
+      // holds its columns [W1 q - c, W1 (q + 1) - c) within [0, len))
       const int64_t r = L.row[tid];
       const int len = L.len[tid];
-      const int nst = (len + W1 - 1) / W1;
+      const int cr = L.cls[tid];
+      const int nst = (len + cr + W1 - 1) / W1;
       const float4 *ps = p.psum + r * p.ns1;
       const float inv_n = __frcp_rn(static_cast<float>(len));
       float4 cf;
@@ -642,7 +647,8 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
 #pragma unroll 4
         for (int qq = 0; qq < nst; ++qq) {
           const float4 u = ps[qq];
-          stat_merge(a, RowStat{static_cast<float>(min(W1, len - qq * W1)), u.x, u.y, u.z, u.w});
+          const int nq = min(len, W1 * (qq + 1) - cr) - max(0, W1 * qq - cr);
+          stat_merge(a, RowStat{static_cast<float>(nq), u.x, u.y, u.z, u.w});
         }
         const float c0 = rsqrtf(__fadd_rn(__fmul_rn(a.M2, inv_n), p.eps));  // rstd
         const float am = __fmul_rn(a.St, inv_n);                           // mean(t)
@@ -672,12 +678,12 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
         if (cur >= 0) flush(cur);
         cur = c;
         dc = from + E * tid - c;
-        lo = tid == 0 ? c : 0;
+        lo = max(0, -dc);
         const int dc1[1] = {dc};
-        stripe_gamma<T, 1>(gam, gamma, from, lim, dc1);
+        stripe_gamma<T, 1>(gam, gamma, 0, cols, dc1);
       }
       const int len = L.len[j];
-      const int hi = min(E, min(lim, len) - dc);
+      const int hi = min(E, len - dc);
       const bool full = hi == E && lo == 0;
       cp_async_wait<D - 1>();  // entry j's copies have landed
       if (__all_sync(kFullMask, full)) {
@@ -709,23 +715,26 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
   if (!waited) asm volatile("griddepcontrol.wait;" ::: "memory");
   if (!want) return;
   __syncthreads();
-  const int ncols = lim - from;
   for (int a = 0; a < NA; ++a) {
-    float *prow = p.part + (g * NA + a) * p.max_len + from;
-    for (int i = tid; i < ncols; i += NT) prow[i] = spart[a][stripe_pad(i)];
+    float *prow = p.part + ((g * p.ns2 + s) * NA + a) * kSeg;
+    for (int i = tid; i < kSeg; i += NT) prow[i] = spart[a][stripe_pad(i)];
   }
 }
 
-// dgamma[j] (dbeta[j]) = the sum over the dx kernel's group partial rows
-// q = 0, 1, ... of part[q][0 (1)][j], for j < cols.  A block of 256 threads
-// takes 64 columns: warp w adds, for column half w & 1, the partials
-// q = w >> 1, (w >> 1) + 4, ... in that order, eight loads ahead; the four
-// slices are then added in slice order.  Launched as a programmatic
-// dependent of the dx kernel.
+// dgamma[j] (dbeta[j]) for j < cols: the sum over the dx kernel's groups
+// g = 0, 1, ... of that group's partial rows at column j.  Partial row
+// part[g][s][a] holds columns [W2 s - E, W2 s + W2) at entries [0, W2 + E),
+// so column j lies in stripe j / W2 and, for the last E columns of that
+// stripe, in the halo of the next: a group's two entries are added first,
+// then the groups in order.  A block of 256 threads takes 64 columns: warp w
+// adds, for column half w & 1, the groups w >> 1, (w >> 1) + 4, ..., eight
+// loads ahead; the four slices are then added in slice order.  Launched as
+// a programmatic dependent of the dx kernel.
 constexpr int kStripeFinThreads = 256;
 template <typename T>
 __global__ void __launch_bounds__(kStripeFinThreads) bwd_stripe_finalize_kernel(
-    const float *part, int64_t nparts, int64_t cols, int nacc, T *dgamma, T *dbeta) {
+    const float *part, int64_t ngroups, int64_t nstripes, int w2, int e_halo, int64_t cols,
+    int nacc, T *dgamma, T *dbeta) {
   __shared__ float sums[4][64];
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int lane = threadIdx.x & 31;
@@ -735,20 +744,28 @@ __global__ void __launch_bounds__(kStripeFinThreads) bwd_stripe_finalize_kernel(
   if (out == nullptr) return;  // uniform over the block
   const int col = 32 * (w & 1) + lane;
   const int slice = w >> 1;
-  const int64_t j = static_cast<int64_t>(blockIdx.x) * 64 + col;
+  const int j = blockIdx.x * 64 + col;  // cols <= 2^31
+  const int64_t seg = w2 + e_halo;
   float sum = 0.f;
   if (j < cols) {
+    const int sa = j / w2;
+    const int ia = j - sa * w2 + e_halo;  // entry in stripe sa
+    const int ib = ia - w2;               // entry in stripe sa + 1 (its halo)
+    const bool twob = sa + 1 < nstripes && ib >= 0;
     constexpr int U = 8;
-    for (int64_t q0 = slice; q0 < nparts; q0 += 4 * U) {
-      float v[U];
+    for (int64_t g0 = slice; g0 < ngroups; g0 += 4 * U) {
+      float va[U], vb[U];
 #pragma unroll
       for (int u = 0; u < U; ++u) {
-        const int64_t q = q0 + 4 * u;
-        v[u] = q < nparts ? __ldcs(part + (q * nacc + a) * cols + j) : 0.f;
+        const int64_t gg = g0 + 4 * u;
+        const bool ok = gg < ngroups;
+        const float *pa = part + ((min(gg, ngroups - 1) * nstripes + sa) * nacc + a) * seg;
+        va[u] = ok ? __ldcs(pa + ia) : 0.f;
+        vb[u] = (ok && twob) ? __ldcs(pa + nacc * seg + ib) : 0.f;
       }
 #pragma unroll
       for (int u = 0; u < U; ++u)
-        if (q0 + 4 * u < nparts) sum = __fadd_rn(sum, v[u]);
+        if (g0 + 4 * u < ngroups) sum = __fadd_rn(sum, twob ? __fadd_rn(va[u], vb[u]) : va[u]);
     }
   }
   sums[slice][col] = sum;

@@ -303,10 +303,11 @@ def test_workload_ragged_norm_backward(rw, op):
 
 
 def _stripe_widths(dtype):
-    """Columns of a stripe of the stats and dx kernels: 511 and 255 window
-    chunks of 16 bytes."""
+    """Window positions of a stripe of the stats and dx kernels: 512 and 256
+    chunks of 16 bytes (a stripe's columns move with the row's head
+    offset)."""
     e = 16 // ESIZE[dtype]
-    return e * 511, e * 255
+    return e * 512, e * 256
 
 
 @pytest.mark.parametrize("dtype", DTYPES, ids=DTYPE_IDS)
@@ -320,8 +321,8 @@ def test_ragged_norm_backward_stripe_edges(rw, monkeypatch, op, dtype, base_off)
     oracle, with nothing outside the outputs written."""
     monkeypatch.setenv("ROWOP_BWD_STRIPE", "2")
     w1, w2 = _stripe_widths(dtype)
-    base = [0, 1, 2, 3, 5, 7, 8, 9, 15, 17, w2 - 1, w2, w2 + 1, 2 * w2 + 3, w1 - 1, w1,
-            w1 + 1, w1 + w2, 2 * w1 + 5]
+    base = [0, 1, 2, 3, 5, 7, 8, 9, 15, 17, w2 - 7, w2 - 1, w2, w2 + 1, w2 + 7, 2 * w2 + 3,
+            w1 - 7, w1 - 1, w1, w1 + 1, w1 + 7, w1 + w2, 2 * w1 + 5]
     lens = np.array(base * 3, dtype=np.int64)
     np.random.default_rng(base_off).shuffle(lens)
     max_len = int(lens.max()) + 11
