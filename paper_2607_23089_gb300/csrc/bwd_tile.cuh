@@ -17,8 +17,11 @@
 //     partial row; bwd_param_finalize_kernel sums the partial rows in index
 //     order.
 // Row sums: per lane in packed pairs, a butterfly over the warp, then the NW
-// warp sums in warp order through shared memory (one named barrier per
-// round; LayerNorm takes two rounds: the mean, then the sums about it).
+// warps' values in warp order through shared memory at one named barrier
+// per row.  LayerNorm: each warp first takes the mean of its own 512
+// elements (a butterfly) and forms its sums about it from the registers;
+// the warps' statistics are then merged (equal counts: the mean of the
+// means, M2 plus 512 times the squared offsets of the means).
 // Nothing is atomic and the order of every sum is fixed by the shape, so the
 // result is bitwise reproducible.
 #pragma once
@@ -108,6 +111,8 @@ __global__ void __launch_bounds__(NW * 32, MINB) bwd_tile_kernel(const BwdTilePa
   constexpr int NS = 2 * R;
   constexpr uint32_t kRowBytes = NW * R * kTileBytes;
   constexpr bool kLN = OP == kLayerNorm;
+  constexpr int kWarpElems = NS * Elem<T>::kPerChunk * 32;  // elements a warp holds: 512
+  static_assert((kWarpElems & (kWarpElems - 1)) == 0 && (NW & (NW - 1)) == 0, "exact scalings");
   extern __shared__ __align__(1024) unsigned char smem[];
   const BwdTileSmem L(p.stage_bytes, p.stages, NW);
   const int S = p.stages;
@@ -200,19 +205,69 @@ __global__ void __launch_bounds__(NW * 32, MINB) bwd_tile_kernel(const BwdTilePa
 #pragma unroll
         for (int i = 0; i < NP; ++i) x[k][i] = d[k][i] = f2_bcast(0.f);
     }
-    // ---- the first round of row sums; past its barrier every warp holds
-    // its chunks of row r, so the stage is refilled ----
-    float c0, c1, c2 = 0.f, mu = 0.f;
+    // ---- the row's sums, one round through shared memory; past its
+    // barrier every warp holds its chunks of row r, so the stage is
+    // refilled ----
+    float c0, c1, c2 = 0.f, sh = 0.f;
     bool stop;
+    float4 *redj = red + NW * static_cast<int>(j & 1);
     if constexpr (kLN) {
+      // each warp holds kWarpElems of the row: its own mean (a butterfly),
+      // then its sums about that mean from the registers: sum (x - m_w)^2,
+      // sum g, sum g (x - m_w), g = dy gamma
       f2 sx = f2_bcast(0.f);
 #pragma unroll
       for (int k = 0; k < NS; ++k)
 #pragma unroll
         for (int i = 0; i < NP; ++i) sx = f2_add(sx, x[k][i]);
-      float v[1] = {f2_total(sx)};
-      stop = bwd_cta_sum<1, NW>(v, red, w, lane, bad);
-      mu = __fmul_rn(v[0], inv_n);
+      float t = f2_total(sx);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) t = __fadd_rn(t, __shfl_xor_sync(kFullMask, t, o));
+      const float mw = __fmul_rn(t, 1.f / kWarpElems);  // a power of two: exact
+      const f2 nmw = f2_bcast(-mw);
+      f2 sdd = f2_bcast(0.f), sg = f2_bcast(0.f), sgd = f2_bcast(0.f);
+#pragma unroll
+      for (int k = 0; k < NS; ++k)
+#pragma unroll
+        for (int i = 0; i < NP; ++i) {
+          x[k][i] = f2_add(x[k][i], nmw);  // x - m_w from here on
+          const f2 gg = f2_mul(d[k][i], gam[k][i]);
+          sdd = f2_fma(x[k][i], x[k][i], sdd);
+          sg = f2_add(sg, gg);
+          sgd = f2_fma(gg, x[k][i], sgd);
+        }
+      float v[3] = {f2_total(sdd), f2_total(sg), f2_total(sgd)};
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+        for (int q = 0; q < 3; ++q) v[q] = __fadd_rn(v[q], __shfl_xor_sync(kFullMask, v[q], o));
+      }
+      if (lane == 0) redj[w] = make_float4(mw, v[0], v[1], v[2]);
+      stop = named_sync_or(kBwdTileBar, NW * 32, bad);
+      if (!stop) {
+        // the warps' statistics merged (equal counts), in warp order: the
+        // mean of the means, M2 = sum M2_w + n_w sum (m_w - mean)^2,
+        // sum g (x - mean) = sum (sum g (x - m_w) + sum g (m_w - mean))
+        float sm = redj[0].x;
+#pragma unroll 4
+        for (int q = 1; q < NW; ++q) sm = __fadd_rn(sm, redj[q].x);
+        const float mean = __fmul_rn(sm, 1.f / NW);  // a power of two: exact
+        float m2 = 0.f, dd = 0.f, st = 0.f, stx = 0.f;
+#pragma unroll 2
+        for (int q = 0; q < NW; ++q) {
+          const float4 u = redj[q];
+          const float dm = __fsub_rn(u.x, mean);
+          m2 = __fadd_rn(m2, u.y);
+          dd = __fmaf_rn(dm, dm, dd);
+          st = __fadd_rn(st, u.z);
+          stx = __fadd_rn(stx, __fmaf_rn(u.z, dm, u.w));
+        }
+        m2 = __fmaf_rn(static_cast<float>(kWarpElems), dd, m2);
+        c0 = rsqrtf(__fmaf_rn(m2, inv_n, p.eps));     // rstd
+        c1 = __fmul_rn(st, inv_n);                    // mean(g)
+        c2 = __fmul_rn(__fmul_rn(stx, c0), inv_n);    // mean(g xhat)
+        sh = __fmul_rn(__fsub_rn(mw, mean), c0);      // (m_w - mean) rstd
+      }
     } else {
       f2 sxx = f2_bcast(0.f), sgx = f2_bcast(0.f);
 #pragma unroll
@@ -223,7 +278,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) bwd_tile_kernel(const BwdTilePa
           sgx = f2_fma(f2_mul(d[k][i], gam[k][i]), x[k][i], sgx);
         }
       float v[2] = {f2_total(sxx), f2_total(sgx)};
-      stop = bwd_cta_sum<2, NW>(v, red + NW * static_cast<int>(j & 1), w, lane, bad);
+      stop = bwd_cta_sum<2, NW>(v, redj, w, lane, bad);
       c0 = rsqrtf(__fmaf_rn(v[0], inv_n, p.eps));  // rstd
       c1 = __fmul_rn(__fmul_rn(v[1], c0), inv_n);  // mean(g xhat)
     }
@@ -247,36 +302,17 @@ __global__ void __launch_bounds__(NW * 32, MINB) bwd_tile_kernel(const BwdTilePa
       s = 0;
       par ^= 1u;
     }
-    if constexpr (kLN) {
-      // the sums about the mean: sum (x - mu)^2, sum g, sum g (x - mu), g = dy gamma
-      const f2 nmu = f2_bcast(-mu);
-      f2 sdd = f2_bcast(0.f), sg = f2_bcast(0.f), sgd = f2_bcast(0.f);
-#pragma unroll
-      for (int k = 0; k < NS; ++k)
-#pragma unroll
-        for (int i = 0; i < NP; ++i) {
-          x[k][i] = f2_add(x[k][i], nmu);  // x - mu from here on
-          const f2 gg = f2_mul(d[k][i], gam[k][i]);
-          sdd = f2_fma(x[k][i], x[k][i], sdd);
-          sg = f2_add(sg, gg);
-          sgd = f2_fma(gg, x[k][i], sgd);
-        }
-      float v[3] = {f2_total(sdd), f2_total(sg), f2_total(sgd)};
-      (void)bwd_cta_sum<3, NW>(v, red + NW, w, lane, false);
-      c0 = rsqrtf(__fadd_rn(__fmul_rn(v[0], inv_n), p.eps));  // rstd
-      c1 = __fmul_rn(v[1], inv_n);                            // mean(g)
-      c2 = __fmul_rn(__fmul_rn(v[2], c0), inv_n);             // mean(g xhat)
-    }
     // ---- dx = rstd (g - mean(g) - xhat mean(g xhat)), and the lane's
     // dgamma (dy xhat) and dbeta (dy) sums ----
-    const f2 C0 = f2_bcast(c0), NC1 = f2_bcast(-c1), NC2 = f2_bcast(-c2);
+    const f2 C0 = f2_bcast(c0), NC1 = f2_bcast(-c1), NC2 = f2_bcast(-c2), SH = f2_bcast(sh);
     char *dxrow = dxbase + r * row_bytes;
 #pragma unroll
     for (int k = 0; k < NS; ++k) {
       f2 o[NP];
 #pragma unroll
       for (int i = 0; i < NP; ++i) {
-        const f2 xh = f2_mul(x[k][i], C0);
+        // LayerNorm: x holds x - m_w; xhat = (x - m_w) rstd + (m_w - mean) rstd
+        const f2 xh = kLN ? f2_fma(x[k][i], C0, SH) : f2_mul(x[k][i], C0);
         f2 t = kLN ? f2_fma(d[k][i], gam[k][i], NC1) : f2_mul(d[k][i], gam[k][i]);
         t = f2_fma(xh, kLN ? NC2 : NC1, t);
         o[i] = f2_mul(C0, t);
