@@ -319,7 +319,7 @@ __device__ __forceinline__ float warp_row_stats(const f2 (&xv)[M][Elem<T>::kPerC
 // the stats kernel's stripe at window position `from`: columns
 // [from + 64 E w - c, + 64 E) within [0, len).
 template <int E>
-__device__ __forceinline__ int stat_warp_count(int from, int len, int c, int w) {
+__host__ __device__ __forceinline__ int stat_warp_count(int from, int len, int c, int w) {
   const int cs = from + 64 * E * w - c;
   return max(0, min(len, cs + 64 * E) - max(0, cs));
 }

@@ -1,7 +1,8 @@
 // host_rules.cu -- the launch code's host-side rules, checked exhaustively on
 // the CPU (no device is touched): the backward team shapes, the ragged
 // workspace offsets, the ragged norm backward's bucket covers and partial-row
-// segments, and the longest ragged norm row.  Built and run by
+// segments, the longest ragged norm row, and the stripe design's stripes,
+// element counts, partial-row columns and workspace.  Built and run by
 // tests/test_host_rules.py; prints "ok" and exits 0 when every check holds.
 #include <cstdio>
 #include <initializer_list>
@@ -157,7 +158,79 @@ static void check_forward_rules() {
     }
 }
 
+// Stripe design of the ragged norm backward: for every head class c and
+// row length, the stats stripes cover the row's window positions and their
+// element counts (the stats kernel's per-warp counts, the dx kernel's
+// per-stripe counts) add up to the row; every column a dx stripe of any
+// head class writes lands at an entry the finalize reads, and no other
+// stripe writes it; the workspace parts are aligned, disjoint and large
+// enough, and within the size the call asks for.
+static void check_stripe_layout() {
+  for (int es : {2, 4}) {
+    const int e = 16 / es;
+    const int64_t w1 = stripe_stat_width(es), w2 = stripe_dx_width(es);
+    CHECK(w1 == static_cast<int64_t>(e) * kStatThreads * kStatChunks && w2 == static_cast<int64_t>(e) * kDxThreads,
+          "es %d", es);
+    for (int64_t max_len : {1LL, 7LL, 8LL, 2047LL, 2048LL, 4095LL, 4096LL, 4097LL, 32768LL,
+                            70000LL, 131072LL}) {
+      const StripeLayout L = stripe_layout(1000, max_len, es, 2);
+      for (int c = 0; c < e; ++c) {
+        for (int64_t len : std::initializer_list<int64_t>{1, 2, e - 1, e, e + 1, w2 - 1, w2,
+                                                          w2 + 1, w1 - 1, w1, w1 + 1,
+                                                          2 * w1 + 3, max_len - 1, max_len}) {
+          if (len < 1 || len > max_len) continue;
+          const int n = static_cast<int>(len);
+          const int64_t nst = (len + c + w1 - 1) / w1;
+          CHECK(nst <= L.ns1, "es %d c %d len %lld nst %lld ns1 %lld", es, c, (long long)len,
+                (long long)nst, (long long)L.ns1);
+          int64_t total = 0;
+          for (int64_t q = 0; q < nst; ++q) {
+            const int nq = static_cast<int>(std::min<int64_t>(len, w1 * (q + 1) - c) -
+                                            std::max<int64_t>(0, w1 * q - c));
+            int warps = 0;
+            for (int w = 0; w < kStatThreads / 32; ++w)
+              warps += e == 8 ? stat_warp_count<8>(static_cast<int>(w1 * q), n, c, w)
+                              : stat_warp_count<4>(static_cast<int>(w1 * q), n, c, w);
+            CHECK(nq > 0 && nq == warps, "es %d c %d len %lld stripe %lld: %d vs %d", es, c,
+                  (long long)len, (long long)q, nq, warps);
+            total += nq;
+          }
+          CHECK(total == len, "es %d c %d len %lld", es, c, (long long)len);
+          CHECK((len + c + w2 - 1) / w2 <= L.ns2, "es %d c %d len %lld", es, c, (long long)len);
+        }
+        // a column j of head class c is in dx stripe (j + c) / w2, at entry
+        // j - (w2 s - e); the finalize reads stripe j / w2 at j - w2 sa + e
+        // and, when that entry is at least w2, stripe sa + 1 at that minus w2
+        for (int64_t j = 0; j < std::min<int64_t>(max_len, 3 * w2 + 17); ++j) {
+          const int64_t s = (j + c) / w2, l = j - (w2 * s - e);
+          const int64_t sa = j / w2, ia = j - w2 * sa + e, ib = ia - w2;
+          CHECK(s < L.ns2 && l >= 0 && l < w2 + e, "es %d c %d j %lld", es, c, (long long)j);
+          const bool read = (s == sa && l == ia) || (s == sa + 1 && sa + 1 < L.ns2 && ib >= 0 && l == ib);
+          CHECK(read, "es %d c %d column %lld (stripe %lld entry %lld) not read", es, c,
+                (long long)j, (long long)s, (long long)l);
+        }
+      }
+      for (int64_t rows : {1LL, 31LL, 32LL, 33LL, 4095LL, 16384LL, 33000LL, 1000000LL})
+        for (int nacc : {1, 2}) {
+          const StripeLayout R = stripe_layout(rows, max_len, es, nacc);
+          CHECK(R.ng2 >= 1 && R.ng2 <= kDxMaxGroups && R.g2 >= 1 && R.ng2 * R.g2 >= rows,
+                "rows %lld ng2 %lld g2 %lld", (long long)rows, (long long)R.ng2, (long long)R.g2);
+          CHECK(R.ng1 * kStatRows >= rows && (R.ng1 - 1) * kStatRows < rows, "rows %lld",
+                (long long)rows);
+          CHECK(R.psum % 256 == 0 && R.part % 256 == 0 &&
+                    R.part >= R.psum + static_cast<size_t>(rows) * R.ns1 * 16,
+                "rows %lld", (long long)rows);
+          CHECK(R.total >= R.part + static_cast<size_t>(R.ng2) * R.ns2 * nacc * (w2 + e) * 4,
+                "rows %lld", (long long)rows);
+          CHECK(bwd_ragged_norm_ws(rows, max_len, es, nacc, 152) >= R.total, "rows %lld",
+                (long long)rows);
+        }
+    }
+  }
+}
+
 int main() {
+  check_stripe_layout();
   check_forward_rules();
   check_shapes();
   check_ragged_workspace();
