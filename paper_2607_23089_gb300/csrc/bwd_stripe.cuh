@@ -57,8 +57,9 @@ struct StripeParams {
   float eps;
   int hb;        // element offset of x (dy, dx) past a 16-byte boundary
   float4 *psum;  // [rows][ns1] the stats kernel's row statistics per stripe
-  float *part;   // [ng2][nacc][max_len] dgamma (dbeta) partial rows; NULL = not wanted
-  int64_t ns1, ng1, ns2, ng2, g2;
+  float *part;   // [ng2][ns2][nacc][W2 + E] dgamma (dbeta) partial rows; NULL = not wanted
+  int64_t ns1, ng1;      // stats kernel: stripes, groups of kStatRows rows
+  int64_t ns2, ng2, g2;  // dx kernel: stripes, groups, rows a group
   unsigned int *status;
 };
 
@@ -534,7 +535,7 @@ __device__ __forceinline__ void stripe_dx(const f2 (&xv)[NP], const f2 (&dv)[NP]
 // ---------------------------------------------------------------------------
 // dx and the column sums.  Lane t owns window chunk t of the stripe.  Per
 // batch of up to 256 rows of the group: sort, then each listed row's
-// statistics from the stats kernel's stripe sums (in stripe order), then the
+// statistics, merged from the stats kernel's stripes in stripe order, then the
 // rows in list order with the lane's chunks of x and dy of the next
 // kDxDepth - 1 rows in flight (cp.async into the lane's own ring slots): the
 // lane writes its dx chunk and adds dy xhat (and dy) to its register sums.
