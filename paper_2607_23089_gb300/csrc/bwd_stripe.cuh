@@ -546,7 +546,7 @@ __device__ __forceinline__ void stripe_dx(const f2 (&xv)[NP], const f2 (&dv)[NP]
 // masks; a warp with no element of the row skips it.  The CTA writes its
 // partial row to part[g][s] at the end.
 // ---------------------------------------------------------------------------
-constexpr int kDxDepth = 5;
+constexpr int kDxDepth = 6;
 constexpr size_t kDxRingBytes = static_cast<size_t>(kDxDepth) * 2 * kDxThreads * 16;
 
 template <int OP, typename T>
