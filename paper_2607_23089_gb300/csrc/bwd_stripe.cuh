@@ -382,9 +382,11 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
   const T *dy = static_cast<const T *>(p.dy);
   const T *gamma = static_cast<const T *>(p.gamma);
   const uint32_t rbase = smem_addr(ring) + 16u * tid;
-  // the lane's slot of chunk m of tensor t (0 x, 1 dy) for list entry j
-  const auto slot = [&](int j, int m, int t) -> uint32_t {
-    return rbase + static_cast<uint32_t>((((j % D) * M + m) * 2 + t) * NT * 16);
+  // the lane's bytes of chunk m of tensor t (0 x, 1 dy) in ring slot sl
+  // (list entry j takes slot j mod D, counted as the list is walked)
+  const auto slot = [&](int sl, int m, int t) -> uint32_t {
+    return rbase + static_cast<uint32_t>(sl) * (M * 2 * NT * 16) +
+           static_cast<uint32_t>((m * 2 + t) * NT * 16);
   };
   int q[M];
 #pragma unroll
@@ -397,7 +399,7 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
   }
   const int cnt = L.seg[E];
   // list entry j's chunks into the ring (a group per entry, empty or not)
-  const auto issue = [&](int j) {
+  const auto issue = [&](int j, int sl) {
     if (j < cnt) {
       const int c = L.cls[j];
       const int len = L.len[j];
@@ -408,20 +410,22 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
         const int lo = max(0, -dc);
         if (lo < min(E, len - dc)) {
           const uint32_t nb = stripe_bytes<SZ>(dc, len);
-          cp_async16(slot(j, m, 0), x + o + dc, nb);
-          cp_async16(slot(j, m, 1), dy + o + dc, nb);
+          cp_async16(slot(sl, m, 0), x + o + dc, nb);
+          cp_async16(slot(sl, m, 1), dy + o + dc, nb);
         }
       }
     }
     cp_async_commit();
   };
 #pragma unroll
-  for (int j = 0; j < D - 1; ++j) issue(j);
+  for (int j = 0; j < D - 1; ++j) issue(j, j);
   int cur = -1;
   int dc[M], lo[M];
   f2 gam[M][NP];
-  for (int j = 0; j < cnt; ++j) {
-    issue(j + D - 1);
+  // sc: entry j's slot; si: the slot entry j + D - 1 is issued into
+  for (int j = 0, sc = 0, si = D - 1; j < cnt;
+       ++j, sc = sc + 1 == D ? 0 : sc + 1, si = si + 1 == D ? 0 : si + 1) {
+    issue(j + D - 1, si);
     const int c = L.cls[j];
     if (c != cur) {  // a new head class: the lane's columns and gamma there
       cur = c;
@@ -448,8 +452,8 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
     if (__all_sync(kFullMask, full)) {
 #pragma unroll
       for (int m = 0; m < M; ++m) {
-        chunk_to_pairs<T>(lds128(slot(j, m, 0)), xv[m]);
-        chunk_to_pairs<T>(lds128(slot(j, m, 1)), dv[m]);
+        chunk_to_pairs<T>(lds128(slot(sc, m, 0)), xv[m]);
+        chunk_to_pairs<T>(lds128(slot(sc, m, 1)), dv[m]);
       }
       t = warp_row_stats<T, kLN, M, false>(xv, dv, lo, hi, gam, lane, n_w, m_w);
     } else if (__any_sync(kFullMask, any)) {
@@ -457,8 +461,8 @@ __global__ void __launch_bounds__(kStatThreads, 3) bwd_stripe_stats_kernel(const
 #pragma unroll
       for (int m = 0; m < M; ++m) {
         const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-        stripe_pairs<T>(lo[m] < hi[m] ? lds128(slot(j, m, 0)) : z, lo[m], hi[m], 0.f, xv[m]);
-        stripe_pairs<T>(lo[m] < hi[m] ? lds128(slot(j, m, 1)) : z, lo[m], hi[m], 0.f, dv[m]);
+        stripe_pairs<T>(lo[m] < hi[m] ? lds128(slot(sc, m, 0)) : z, lo[m], hi[m], 0.f, xv[m]);
+        stripe_pairs<T>(lo[m] < hi[m] ? lds128(slot(sc, m, 1)) : z, lo[m], hi[m], 0.f, dv[m]);
       }
       t = warp_row_stats<T, kLN, M, true>(xv, dv, lo, hi, gam, lane, n_w, m_w);
     } else {
@@ -578,9 +582,10 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
   const T *gamma = static_cast<const T *>(p.gamma);
   const bool want = p.part != nullptr;
   const uint32_t rbase = smem_addr(ring) + 16u * tid;
-  // the lane's slot of tensor t (0 x, 1 dy) for list entry j
-  const auto slot = [&](int j, int t) -> uint32_t {
-    return rbase + static_cast<uint32_t>(((j % D) * 2 + t) * NT * 16);
+  // the lane's bytes of tensor t (0 x, 1 dy) in ring slot sl (list entry j
+  // takes slot j mod D, counted as the list is walked)
+  const auto slot = [&](int sl, int t) -> uint32_t {
+    return rbase + static_cast<uint32_t>(sl) * (2 * NT * 16) + static_cast<uint32_t>(t * NT * 16);
   };
   for (int i = tid; i < NA * kPadW; i += NT) (&spart[0][0])[i] = 0.f;
 
@@ -616,7 +621,7 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
     }
     const int cnt = L.seg[E];
     // list entry j's chunk into the ring (a group per entry, empty or not)
-    const auto issue = [&](int j) {
+    const auto issue = [&](int j, int sl) {
       if (j < cnt) {
         const int c = L.cls[j];
         const int len = L.len[j];
@@ -625,14 +630,14 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
         if (lo < min(E, len - dc)) {
           const int64_t o = L.off[j];
           const uint32_t nb = stripe_bytes<SZ>(dc, len);
-          cp_async16(slot(j, 0), x + o + dc, nb);
-          cp_async16(slot(j, 1), dy + o + dc, nb);
+          cp_async16(slot(sl, 0), x + o + dc, nb);
+          cp_async16(slot(sl, 1), dy + o + dc, nb);
         }
       }
       cp_async_commit();
     };
 #pragma unroll
-    for (int j = 0; j < D - 1; ++j) issue(j);
+    for (int j = 0; j < D - 1; ++j) issue(j, j);
     if (tid < cnt) {
       // the row's statistics: its stripes' in stripe order (stats stripe q
       // holds its columns [W1 q - c, W1 (q + 1) - c) within [0, len))
@@ -672,8 +677,10 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
     __syncthreads();
     int cur = -1, dc = 0, lo = 0;
     f2 gam[1][NP];
-    for (int j = 0; j < cnt; ++j) {
-      issue(j + D - 1);
+    // sc: entry j's slot; si: the slot entry j + D - 1 is issued into
+    for (int j = 0, sc = 0, si = D - 1; j < cnt;
+         ++j, sc = sc + 1 == D ? 0 : sc + 1, si = si + 1 == D ? 0 : si + 1) {
+      issue(j + D - 1, si);
       const int c = L.cls[j];
       if (c != cur) {  // a new head class: the lane's columns and gamma there
         if (cur >= 0) flush(cur);
@@ -689,16 +696,16 @@ __global__ void __launch_bounds__(kDxThreads, 3) bwd_stripe_dx_kernel(const Stri
       cp_async_wait<D - 1>();  // entry j's copies have landed
       if (__all_sync(kFullMask, full)) {
         f2 xv[NP], dv[NP], ov[NP];
-        chunk_to_pairs<T>(lds128(slot(j, 0)), xv);
-        chunk_to_pairs<T>(lds128(slot(j, 1)), dv);
+        chunk_to_pairs<T>(lds128(slot(sc, 0)), xv);
+        chunk_to_pairs<T>(lds128(slot(sc, 1)), dv);
         stripe_dx<kLN, NP>(xv, dv, gam[0], coef[j], want, ov, accg, accb);
         stg_stream(dx + L.off[j] + dc, pairs_to_chunk<T>(ov));
       } else if (lo < hi) {
         // elements outside the chunk's valid range read as 0: no dy, so
         // they add nothing to the column sums
         f2 xv[NP], dv[NP], ov[NP];
-        stripe_pairs<T>(lds128(slot(j, 0)), lo, hi, 0.f, xv);
-        stripe_pairs<T>(lds128(slot(j, 1)), lo, hi, 0.f, dv);
+        stripe_pairs<T>(lds128(slot(sc, 0)), lo, hi, 0.f, xv);
+        stripe_pairs<T>(lds128(slot(sc, 1)), lo, hi, 0.f, dv);
         stripe_dx<kLN, NP>(xv, dv, gam[0], coef[j], want, ov, accg, accb);
         T *dst = dx + L.off[j] + dc;
         if (lo == 0 && hi == E) {
